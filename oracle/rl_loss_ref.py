@@ -1,0 +1,379 @@
+"""Float64 CPU oracle of the per-token RL loss over the vocabulary.
+
+TEST INFRASTRUCTURE ONLY: imported by ``tests/``, ``__graft_entry__.smoke()``
+and the CPU-baseline leg of ``bench.py``; never by the library.
+
+Every function is the plain definition, written in numpy float64 in the order
+the method states it, with no fusion, blocking or reordering beyond chunking
+rows (which changes no arithmetic of any row). Inputs in bf16 or fp32 are
+widened exactly to float64 first.
+
+What the paper fixes (Miles v0.1, arxiv 2609.08368):
+  * the importance ratio r = exp(log pi_train - log pi_rollout)      (Sec. 3.4)
+  * GRPO: a trajectory is scored against the other trajectories of the same
+    prompt, i.e. rewards are centred within their group                (Sec. 2, Sec. 9.1)
+  * a group whose attempts all got the same reward carries no signal  (Sec. 2.2, Table 2)
+  * tokens the model did not generate are loss-masked                 (Sec. 2.4)
+  * truncated importance sampling (TIS): clamp the ratio to an interval,
+    default [0, 2], and use it as a per-token weight on the PG loss;
+    clip-or-pop: weight 0 outside the interval, the unclipped ratio inside;
+    reported metrics: pre-clamp ratio, clipped fraction, mean |r - 1|  (Sec. 3.4)
+  * OPD shaping: subtract coef * (log pi_student - log pi_teacher) of the
+    sampled token from each token's advantage; both are fixed inputs   (Sec. 5.2)
+
+What the paper leaves unwritten, and the reading taken here (each is listed
+with its reason in the design notes): the PPO clipped surrogate with asymmetric
+clip and dual clip (PPO, Schulman et al. 2017, cited in Sec. 3.4), the k3 KL
+estimator exp(d) - d - 1 with d = log pi_ref - log pi, an entropy bonus, a
+temperature dividing the logits, sample (n-1) standard deviation with a floor
+max(sigma, floor), one global masked token-mean, strict inequalities at every
+clip threshold.
+
+Parity status: every function here is pinned by the CPU tests in
+``tests/test_oracle_pins.py`` (closed forms, invariants, library special
+cases, finite differences, brute force); the paper prints no worked example.
+"""
+
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import numpy as np
+
+CORRECTIONS = ("none", "tis", "clip_or_pop")
+
+
+@dataclass(frozen=True)
+class LossParams:
+    """Scalar knobs of the loss (one set per call)."""
+
+    temperature: float = 1.0
+    eps_lo: float = 0.2
+    eps_hi: float = 0.2
+    dual_clip_c: float = 0.0      # 0 = off, else > 1
+    kl_coef: float = 0.0          # beta
+    entropy_coef: float = 0.0     # gamma: loss -= gamma * H
+    std_floor: float = 1e-6
+    normalize_std: bool = True    # GRPO divides by the group std
+    unbiased_std: bool = True     # Bessel (n - 1)
+    correction: str = "none"      # "none" | "tis" | "clip_or_pop"   (Sec. 3.4)
+    corr_lo: float = 0.0
+    corr_hi: float = 2.0
+    opd_coef: float = 0.0         # lambda of Sec. 5.2
+
+
+# --------------------------------------------------------------------------
+# input widening
+# --------------------------------------------------------------------------
+
+def widen_bf16(bits: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns (uint16) -> exact float64 values.
+
+    A bf16 number is the upper half of the fp32 number with the same bits, so
+    shifting the 16 bits into the top of a 32-bit word gives the fp32 value
+    exactly, and fp32 -> fp64 is exact.
+    """
+    b = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)
+    return b.view(np.float32).astype(np.float64)
+
+
+def _widen(z: np.ndarray) -> np.ndarray:
+    if z.dtype == np.uint16:
+        return widen_bf16(z)
+    return np.asarray(z, dtype=np.float64)
+
+
+# --------------------------------------------------------------------------
+# (a2) log-softmax, gathered log-prob and entropy of each row
+# --------------------------------------------------------------------------
+
+def row_log_softmax(z: np.ndarray, y: np.ndarray, temperature: float):
+    """Tempered log-softmax of each row, the sampled token's log-prob and the
+    entropy of the row's distribution.
+
+    s_j = z_j / T;  lse = log sum_j exp(s_j) (taken as M + log sum exp(s - M)
+    with M = max s, the textbook stable form);  log p_j = s_j - lse;
+    logp = log p_y;  H = -sum_j p_j log p_j.
+
+    The ratio of Sec. 3.4 needs log pi_train of the sampled token; the
+    trainer computes it for the same tokens the rollout sampled (Sec. 9.2).
+    Returns (logp [r], H [r], lse [r]) in float64.
+    """
+    s = _widen(z) / float(temperature)
+    m = s.max(axis=1, keepdims=True)
+    lse = m[:, 0] + np.log(np.exp(s - m).sum(axis=1))
+    logp_all = s - lse[:, None]
+    p = np.exp(logp_all)
+    rows = np.arange(s.shape[0])
+    logp = logp_all[rows, np.asarray(y, dtype=np.int64)]
+    H = -(p * logp_all).sum(axis=1)
+    return logp, H, lse
+
+
+# --------------------------------------------------------------------------
+# (a1) GRPO group-relative advantages
+# --------------------------------------------------------------------------
+
+def group_advantages(w: np.ndarray, gid: np.ndarray, n_groups: int, p: LossParams):
+    """Per-trajectory GRPO advantages.
+
+    Each trajectory is scored against the other trajectories for the same
+    prompt (Sec. 2): with the members i of group g,
+        mu = mean(w_i),  sigma = std(w_i) (n-1 if unbiased, n otherwise),
+        A_i = (w_i - mu) / max(sigma, floor)      if normalize_std
+        A_i =  w_i - mu                           otherwise.
+    A group whose members all received the same reward carries no advantage
+    signal (Sec. 2.2, Table 2): its A_i are exactly 0. A one-member group is
+    such a group.
+    Returns (A [n_traj] float64, n_g [n_groups] int64).
+    """
+    w = np.asarray(w, dtype=np.float64)
+    gid = np.asarray(gid, dtype=np.int64)
+    A = np.zeros(w.shape[0], dtype=np.float64)
+    n_g = np.zeros(n_groups, dtype=np.int64)
+    for g in range(n_groups):
+        idx = np.nonzero(gid == g)[0]
+        n_g[g] = idx.size
+        if idx.size == 0:
+            continue
+        wg = w[idx]
+        if wg.max() == wg.min():
+            continue  # equal rewards: no signal, A stays exactly 0
+        mu = wg.mean()
+        if not p.normalize_std:
+            A[idx] = wg - mu
+            continue
+        ddof = 1 if p.unbiased_std else 0
+        sigma = float(np.sqrt(((wg - mu) ** 2).sum() / (idx.size - ddof)))
+        A[idx] = (wg - mu) / max(sigma, p.std_floor)
+    return A, n_g
+
+
+def row_advantages(A_traj: np.ndarray, cu_seqlens: np.ndarray, n_rows: int) -> np.ndarray:
+    """Broadcast each trajectory's advantage to its rows.
+
+    Trajectory i owns rows [cu[i], cu[i+1]) of the packed layout; an outcome
+    reward gives every token of the trajectory the same advantage.
+    """
+    cu = np.asarray(cu_seqlens, dtype=np.int64)
+    A_row = np.zeros(n_rows, dtype=np.float64)
+    for i in range(cu.shape[0] - 1):
+        A_row[cu[i]:cu[i + 1]] = A_traj[i]
+    return A_row
+
+
+def shape_advantages_opd(A_row: np.ndarray, student_lp: np.ndarray,
+                         teacher_lp: np.ndarray, coef: float) -> np.ndarray:
+    """On-policy distillation shaping (Sec. 5.2): after the estimator, each
+    token's advantage loses coef * (log pi_student(x_t) - log pi_teacher(x_t)).
+    Both log-probs are fixed inputs (recorded at rollout / by a teacher pass);
+    the student's is the rollout-recorded one."""
+    return np.asarray(A_row, np.float64) - coef * (
+        np.asarray(student_lp, np.float64) - np.asarray(teacher_lp, np.float64))
+
+
+# --------------------------------------------------------------------------
+# (a3) per-token objective
+# --------------------------------------------------------------------------
+
+def token_objective(logp, rho, q, A_row, H, p: LossParams, old=None):
+    """Per-token loss terms and the derivative of the token loss w.r.t. logp.
+
+    ratio (Sec. 3.4):  r = exp(logp - base), base = old if given else rho.
+    PPO clip:          u = -A r;  c = -A clip(r, 1-eps_lo, 1+eps_hi);
+                       pg = max(u, c); clipped iff c > u (strict);
+                       clip_hi iff clipped and r > 1+eps_hi; clip_lo iff
+                       clipped and r < 1-eps_lo.
+    dual clip:         if c_dual > 0 and A < 0: d = -A c_dual; if d < pg
+                       (strict) then pg = d and the token is dual-clipped.
+    correction (Sec. 3.4), needs ``old``: rc = exp(old - rho) is the
+                       train/rollout ratio, a constant weight:
+                       TIS wt = min(max(rc, lo), hi);
+                       clip-or-pop wt = rc if lo <= rc <= hi else 0;
+                       pg <- wt * pg.
+    k3 KL:             dlt = q - logp; k3 = exp(dlt) - dlt - 1.
+    token loss:        l = pg + beta k3 - gamma H.
+    G = dl/dlogp:      wt * (-A r if neither clipped nor dual-clipped else 0)
+                       + beta (1 - exp(dlt)).
+    """
+    logp = np.asarray(logp, np.float64)
+    rho = np.asarray(rho, np.float64)
+    A = np.asarray(A_row, np.float64)
+    H = np.asarray(H, np.float64)
+    base = rho if old is None else np.asarray(old, np.float64)
+    r = np.exp(logp - base)
+    u = -A * r
+    c = -A * np.clip(r, 1.0 - p.eps_lo, 1.0 + p.eps_hi)
+    pg = np.maximum(u, c)
+    clipped = c > u
+    clip_hi = clipped & (r > 1.0 + p.eps_hi)
+    clip_lo = clipped & (r < 1.0 - p.eps_lo)
+    dual = np.zeros_like(clipped)
+    if p.dual_clip_c > 0.0:
+        d = -A * p.dual_clip_c
+        dual = (A < 0.0) & (d < pg)
+        pg = np.where(dual, d, pg)
+    g_pg = np.where(clipped | dual, 0.0, -A * r)
+
+    wt = np.ones_like(r)
+    rc = np.ones_like(r)
+    corr_clip = np.zeros_like(clipped)
+    if p.correction != "none":
+        if p.correction not in CORRECTIONS:
+            raise ValueError(p.correction)
+        if old is None:
+            raise ValueError("a ratio correction needs old log-probs")
+        rc = np.exp(np.asarray(old, np.float64) - rho)
+        outside = (rc < p.corr_lo) | (rc > p.corr_hi)
+        corr_clip = outside
+        if p.correction == "tis":
+            wt = np.minimum(np.maximum(rc, p.corr_lo), p.corr_hi)
+        else:
+            wt = np.where(outside, 0.0, rc)
+        pg = wt * pg
+        g_pg = wt * g_pg
+
+    if q is None:
+        dlt = np.zeros_like(logp)
+        k3 = np.zeros_like(logp)
+        g_kl = np.zeros_like(logp)
+    else:
+        dlt = np.asarray(q, np.float64) - logp
+        k3 = np.exp(dlt) - dlt - 1.0
+        g_kl = 1.0 - np.exp(dlt)
+    ell = pg + p.kl_coef * k3 - p.entropy_coef * H
+    G = g_pg + p.kl_coef * g_kl
+    return dict(r=r, pg=pg, k3=k3, ell=ell, G=G, clip_hi=clip_hi, clip_lo=clip_lo,
+                dual=dual, wt=wt, rc=rc, corr_clip=corr_clip)
+
+
+# --------------------------------------------------------------------------
+# (a4) masked token-mean and the reported metrics
+# --------------------------------------------------------------------------
+
+def masked_token_mean(ell: np.ndarray, mask: np.ndarray):
+    """One global token mean over the tokens that train: L = sum m l / N,
+    N = sum m (L = 0 when N = 0). Returns (L, N)."""
+    m = np.asarray(mask).astype(bool)
+    N = int(m.sum())
+    if N == 0:
+        return 0.0, 0
+    return float(np.asarray(ell, np.float64)[m].sum() / N), N
+
+
+def loss_stats(obj: dict, logp, rho, H, mask) -> dict:
+    """Metrics over the tokens that train (m = 1): means of r, |r - 1|,
+    |logp - rho| (the train/rollout divergence of Sec. 9.2), k3, H and the PG
+    term; min / max of r; counts of clip_hi / clip_lo / dual-clipped tokens;
+    for a correction (Sec. 3.4) the mean pre-clamp ratio rc, the number of
+    tokens whose weight was changed, and mean |rc - 1|. All zero when N = 0."""
+    m = np.asarray(mask).astype(bool)
+    N = int(m.sum())
+    L, _ = masked_token_mean(obj["ell"], m)
+    out = dict(loss=L, n_tokens=N,
+               n_clip_hi=int(obj["clip_hi"][m].sum()),
+               n_clip_lo=int(obj["clip_lo"][m].sum()),
+               n_dual_clip=int(obj["dual"][m].sum()),
+               n_corr_clip=int(obj["corr_clip"][m].sum()))
+    if N == 0:
+        out.update(pg_loss_mean=0.0, kl_mean=0.0, entropy_mean=0.0, ratio_mean=0.0,
+                   ratio_absdev_mean=0.0, logprob_absdiff_mean=0.0, ratio_min=0.0,
+                   ratio_max=0.0, corr_ratio_mean=0.0, corr_absdev_mean=0.0)
+        return out
+    r = obj["r"][m]
+    out.update(
+        pg_loss_mean=float(obj["pg"][m].sum() / N),
+        kl_mean=float(obj["k3"][m].sum() / N),
+        entropy_mean=float(np.asarray(H, np.float64)[m].sum() / N),
+        ratio_mean=float(r.sum() / N),
+        ratio_absdev_mean=float(np.abs(r - 1.0).sum() / N),
+        logprob_absdiff_mean=float(np.abs(np.asarray(logp, np.float64)[m]
+                                          - np.asarray(rho, np.float64)[m]).sum() / N),
+        ratio_min=float(r.min()),
+        ratio_max=float(r.max()),
+        corr_ratio_mean=float(obj["rc"][m].sum() / N),
+        corr_absdev_mean=float(np.abs(obj["rc"][m] - 1.0).sum() / N),
+    )
+    return out
+
+
+# --------------------------------------------------------------------------
+# (a5) dLogits
+# --------------------------------------------------------------------------
+
+def dlogits_rows(z, y, temperature, lse, H, G, mask, N, grad_loss, entropy_coef):
+    """Gradient of g * L with respect to the logits of the given rows.
+
+    With p_j = exp(s_j - lse), d logp / d s_j = 1[j = y] - p_j and
+    d H / d s_j = -p_j (log p_j + H); the chain rule through l = pg + beta k3
+    - gamma H and L = sum m l / N gives
+        dZ_j = g (m / N) (1 / T) [ G (1[j = y] - p_j) + gamma p_j (log p_j + H) ].
+    """
+    s = _widen(z) / float(temperature)
+    logp_all = s - np.asarray(lse, np.float64)[:, None]
+    pj = np.exp(logp_all)
+    onehot = np.zeros_like(s)
+    onehot[np.arange(s.shape[0]), np.asarray(y, np.int64)] = 1.0
+    m = np.asarray(mask).astype(np.float64)
+    scale = (grad_loss * m / N / float(temperature)) if N > 0 else np.zeros_like(m)
+    Gc = np.asarray(G, np.float64)[:, None]
+    Hc = np.asarray(H, np.float64)[:, None]
+    return scale[:, None] * (Gc * (onehot - pj) + entropy_coef * pj * (logp_all + Hc))
+
+
+# --------------------------------------------------------------------------
+# whole pipeline
+# --------------------------------------------------------------------------
+
+def rl_loss_rows(z, y, rho, q, A_row, mask, N, p: LossParams, grad_loss=1.0,
+                 old=None, want_dlogits=True):
+    """Every per-row output for a set of rows, given the call-wide values
+    (their advantages and the masked count N of the whole call)."""
+    logp, H, lse = row_log_softmax(z, y, p.temperature)
+    obj = token_objective(logp, rho, q, A_row, H, p, old=old)
+    out = dict(logp=logp, H=H, lse=lse, **obj)
+    if want_dlogits:
+        out["dlogits"] = dlogits_rows(z, y, p.temperature, lse, H, obj["G"], mask, N,
+                                      grad_loss, p.entropy_coef)
+    return out
+
+
+def rl_loss(z, y, rho, q, w, gid, cu_seqlens, n_groups, mask, p: LossParams,
+            grad_loss=1.0, old=None, teacher=None, want_dlogits=True, chunk=256):
+    """The whole loss for one call: advantages, per-row outputs, the masked
+    token-mean, the metrics, and (optionally) dLogits as a float64 array.
+
+    Rows are processed in chunks of ``chunk`` rows; each row's arithmetic is
+    independent of the chunking."""
+    R = int(np.asarray(y).shape[0])
+    A_traj, n_g = group_advantages(w, gid, n_groups, p)
+    A_row = row_advantages(A_traj, cu_seqlens, R)
+    if p.opd_coef != 0.0:
+        A_row = shape_advantages_opd(A_row, rho, teacher, p.opd_coef)
+    m = np.asarray(mask).astype(bool)
+    N = int(m.sum())
+    keys = ("logp", "H", "lse", "r", "pg", "k3", "ell", "G", "clip_hi", "clip_lo",
+            "dual", "wt", "rc", "corr_clip")
+    parts = {k: [] for k in keys}
+    dz = [] if want_dlogits else None
+    for lo in range(0, R, chunk):
+        hi = min(R, lo + chunk)
+        o = rl_loss_rows(z[lo:hi], np.asarray(y)[lo:hi], np.asarray(rho)[lo:hi],
+                         None if q is None else np.asarray(q)[lo:hi], A_row[lo:hi],
+                         m[lo:hi], N, p, grad_loss,
+                         old=None if old is None else np.asarray(old)[lo:hi],
+                         want_dlogits=want_dlogits)
+        for k in keys:
+            parts[k].append(o[k])
+        if want_dlogits:
+            dz.append(o["dlogits"])
+    cat = {k: (np.concatenate(v) if v else np.zeros(0)) for k, v in parts.items()}
+    for k in ("clip_hi", "clip_lo", "dual", "corr_clip"):
+        cat[k] = cat[k].astype(bool)
+    stats = loss_stats(cat, cat["logp"], rho, cat["H"], m)
+    out = dict(cat, A_traj=A_traj, group_sizes=n_g, A_row=A_row, N=N, stats=stats,
+               loss=stats["loss"])
+    if want_dlogits:
+        V = np.asarray(z).shape[1] if R else 0
+        out["dlogits"] = np.concatenate(dz) if dz else np.zeros((0, V))
+    return out

@@ -1,0 +1,377 @@
+"""Pins of the float64 oracle against facts that do not come from the oracle:
+hand-derived closed forms, invariants, library routines that compute the same
+quantity (torch.log_softmax, torch.nn.functional.cross_entropy, torch.std,
+Categorical entropy), arbitrary-precision brute force (mpmath), and central
+finite differences of the loss. CPU only.
+"""
+
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from oracle import LossParams
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+
+
+def _ev(x):
+    return float(eval(x, {"math": math})) if isinstance(x, str) else float(x)
+
+
+def _golden():
+    with open(os.path.join(HERE, "golden", "hand_cases.json")) as f:
+        return {c["name"]: c for c in json.load(f)["cases"]}
+
+
+# ---------------------------------------------------------------- log-softmax
+
+@pytest.mark.parametrize("name", ["two_point_row", "tempered_row"])
+def test_row_golden(name):
+    c = _golden()[name]
+    z = np.array([[_ev(v) for v in row] for row in c["z"]])
+    logp, H, lse = oracle.row_log_softmax(z, np.array(c["y"]), _ev(c["T"]))
+    for key, got in (("logp", logp), ("lse", lse), ("H", H)):
+        want = np.array([_ev(v) for v in c["expect"][key]])
+        np.testing.assert_allclose(got, want, rtol=0, atol=1e-14)
+
+
+def test_log_softmax_matches_torch_library():
+    rng = np.random.default_rng(1)
+    z = rng.normal(0, 3, size=(17, 301))
+    y = rng.integers(0, 301, size=17)
+    for T in (1.0, 0.7, 1.9):
+        logp, H, lse = oracle.row_log_softmax(z, y, T)
+        zt = torch.from_numpy(z) / T
+        ref = torch.log_softmax(zt, dim=1)
+        np.testing.assert_allclose(logp, ref[torch.arange(17), torch.from_numpy(y)].numpy(),
+                                   atol=1e-12, rtol=0)
+        np.testing.assert_allclose(lse, torch.logsumexp(zt, dim=1).numpy(), atol=1e-12, rtol=0)
+        ent = torch.distributions.Categorical(logits=zt).entropy().numpy()
+        np.testing.assert_allclose(H, ent, atol=1e-12, rtol=0)
+
+
+def test_probabilities_sum_to_one_and_shift_invariance():
+    rng = np.random.default_rng(2)
+    z = rng.normal(0, 5, size=(9, 1000))
+    y = rng.integers(0, 1000, size=9)
+    logp, H, lse = oracle.row_log_softmax(z, y, 1.0)
+    assert np.all(np.abs(np.exp(z - lse[:, None]).sum(1) - 1.0) < 1e-12)
+    # adding a constant to a row changes nothing but lse
+    logp2, H2, lse2 = oracle.row_log_softmax(z + 1000.0, y, 1.0)
+    np.testing.assert_allclose(logp2, logp, atol=1e-9)
+    np.testing.assert_allclose(H2, H, atol=1e-9)
+    np.testing.assert_allclose(lse2 - lse, 1000.0, atol=1e-9)
+
+
+def test_entropy_extremes():
+    for V in (1, 2, 7, 4096):
+        z = np.zeros((1, V))
+        logp, H, _ = oracle.row_log_softmax(z, np.array([0]), 1.0)
+        assert abs(H[0] - math.log(V)) < 1e-12
+        assert abs(logp[0] + math.log(V)) < 1e-12
+    z = np.zeros((1, 50))
+    z[0, 3] = 200.0
+    logp, H, _ = oracle.row_log_softmax(z, np.array([3]), 1.0)
+    assert H[0] < 1e-80 and abs(logp[0]) < 1e-80
+
+
+def test_log_softmax_mpmath_brute_force():
+    mpmath = pytest.importorskip("mpmath")
+    mpmath.mp.dps = 50
+    rng = np.random.default_rng(3)
+    for V in (2, 3, 5, 8):
+        z = rng.normal(0, 4, size=(4, V))
+        y = rng.integers(0, V, size=4)
+        T = 0.8
+        logp, H, lse = oracle.row_log_softmax(z, y, T)
+        for i in range(4):
+            s = [mpmath.mpf(float(v)) / mpmath.mpf(T) for v in z[i]]
+            L = mpmath.log(mpmath.fsum(mpmath.exp(v) for v in s))
+            ps = [mpmath.exp(v - L) for v in s]
+            Hm = -mpmath.fsum(p * mpmath.log(p) for p in ps)
+            assert abs(float(L) - lse[i]) < 1e-13
+            assert abs(float(s[y[i]] - L) - logp[i]) < 1e-13
+            assert abs(float(Hm) - H[i]) < 1e-13
+
+
+def test_widen_bf16_exact():
+    x = torch.tensor([1.0, -2.5, 3.140625, 1e-30, 65504.0, -0.0], dtype=torch.bfloat16)
+    bits = x.view(torch.int16).numpy().view(np.uint16)
+    np.testing.assert_array_equal(oracle.widen_bf16(bits), x.double().numpy())
+
+
+# ---------------------------------------------------------------- advantages
+
+@pytest.mark.parametrize("name", ["grpo_two_members", "grpo_three_members"])
+def test_group_advantages_golden(name):
+    c = _golden()[name]
+    w = np.array([_ev(v) for v in c["w"]])
+    gid = np.array(c["gid"])
+    A, n = oracle.group_advantages(w, gid, c["n_groups"], LossParams())
+    np.testing.assert_allclose(A, [_ev(v) for v in c["expect_unbiased"]], atol=1e-15, rtol=0)
+    A, _ = oracle.group_advantages(w, gid, c["n_groups"], LossParams(unbiased_std=False))
+    np.testing.assert_allclose(A, [_ev(v) for v in c["expect_population"]], atol=1e-15, rtol=0)
+    assert n.tolist() == [len(w)]
+
+
+def test_group_advantages_match_torch_std_and_sum_to_zero():
+    rng = np.random.default_rng(4)
+    n_groups, gsz = 11, 7
+    w = rng.random(n_groups * gsz)
+    gid = rng.permutation(np.repeat(np.arange(n_groups), gsz))  # scattered members
+    A, n = oracle.group_advantages(w, gid, n_groups, LossParams())
+    assert n.tolist() == [gsz] * n_groups
+    for g in range(n_groups):
+        idx = gid == g
+        wt = torch.from_numpy(w[idx])
+        ref = ((wt - wt.mean()) / wt.std()).numpy()  # torch.std is the n-1 std
+        np.testing.assert_allclose(A[idx], ref, atol=1e-13, rtol=0)
+        assert abs(A[idx].sum()) < 1e-12 * gsz
+    A0, _ = oracle.group_advantages(w, gid, n_groups, LossParams(normalize_std=False))
+    for g in range(n_groups):
+        idx = gid == g
+        np.testing.assert_allclose(A0[idx], w[idx] - w[idx].mean(), atol=1e-15)
+
+
+def test_group_advantages_equal_rewards_floor_and_empty_groups():
+    p = LossParams(std_floor=1e-6)
+    w = np.array([0.5, 0.5, 0.5, 0.0, 1e-9, 3.0])
+    gid = np.array([0, 0, 0, 1, 1, 3])  # group 2 empty, group 3 single member
+    A, n = oracle.group_advantages(w, gid, 4, p)
+    assert A[0] == 0.0 and A[1] == 0.0 and A[2] == 0.0  # equal rewards: exactly 0
+    assert A[5] == 0.0
+    assert n.tolist() == [3, 2, 0, 1]
+    # sigma = 1e-9/sqrt(2) < floor -> divide by the floor
+    np.testing.assert_allclose(A[3:5], [-0.5e-9 / 1e-6, 0.5e-9 / 1e-6], rtol=1e-12)
+
+
+def test_row_advantages_and_opd_shaping():
+    A = np.array([1.0, -2.0, 3.0])
+    cu = np.array([0, 2, 2, 5])
+    np.testing.assert_array_equal(oracle.row_advantages(A, cu, 5), [1, 1, 3, 3, 3])
+    s = oracle.shape_advantages_opd(np.array([1.0, 1.0]), np.array([-1.0, -3.0]),
+                                    np.array([-2.0, -1.0]), 0.5)
+    # student favoured token 0 more than the teacher (+1) -> penalised;
+    # teacher favoured token 1 more (-2) -> encouraged
+    np.testing.assert_allclose(s, [0.5, 2.0], atol=1e-15)
+
+
+# ---------------------------------------------------------------- objective
+
+def test_ppo_tokens_golden():
+    c = _golden()["ppo_tokens"]
+    A = np.array([_ev(v) for v in c["A"]])
+    logp = np.array([_ev(v) for v in c["log_r"]])
+    o = oracle.token_objective(logp, np.zeros_like(logp), None, A, np.zeros_like(A),
+                               LossParams(**c["params"]))
+    np.testing.assert_allclose(o["pg"], [_ev(v) for v in c["expect"]["pg"]], atol=1e-14)
+    np.testing.assert_allclose(o["G"], [_ev(v) for v in c["expect"]["G"]], atol=1e-14)
+    for k in ("clip_hi", "clip_lo", "dual"):
+        assert o[k].astype(int).tolist() == c["expect"][k]
+
+
+def test_k3_golden():
+    c = _golden()["k3_token"]
+    logp = np.array([_ev(v) for v in c["logp"]])
+    q = np.array([_ev(v) for v in c["q"]])
+    o = oracle.token_objective(logp, logp, q, np.array([0.0]), np.zeros(1),
+                               LossParams(kl_coef=c["kl_coef"]))
+    for k in ("k3", "ell", "G"):
+        np.testing.assert_allclose(o[k], [_ev(v) for v in c["expect"][k]], atol=1e-15)
+    # q == logp: k3 and its gradient vanish
+    o = oracle.token_objective(logp, logp, logp, np.array([0.0]), np.zeros(1),
+                               LossParams(kl_coef=1.0))
+    assert o["k3"][0] == 0.0 and o["G"][0] == 0.0
+
+
+def _threshold_probe(approx):
+    """A float64 d, the ratio t = exp(d) it gives (the threshold), and the
+    neighbouring doubles d_up / d_dn whose exp lies strictly above / below t."""
+    d = math.log(approx)
+    t = math.exp(d)
+    up = np.nextafter(d, math.inf)
+    while math.exp(up) <= t:
+        up = np.nextafter(up, math.inf)
+    dn = np.nextafter(d, -math.inf)
+    while math.exp(dn) >= t:
+        dn = np.nextafter(dn, -math.inf)
+    return d, t, up, dn
+
+
+def test_clip_engages_exactly_past_the_threshold():
+    d_hi, t_hi, up_hi, _ = _threshold_probe(1.25)
+    d_lo, t_lo, _, dn_lo = _threshold_probe(0.75)
+    d_c, t_c, up_c, _ = _threshold_probe(3.0)
+    # eps chosen so that 1 + eps_hi == t_hi and 1 - eps_lo == t_lo exactly
+    # (Sterbenz: t - 1 and 1 - t are exact for t in [0.5, 2])
+    p = LossParams(eps_lo=1.0 - t_lo, eps_hi=t_hi - 1.0, dual_clip_c=t_c)
+    assert 1.0 + p.eps_hi == t_hi and 1.0 - p.eps_lo == t_lo
+    logp = np.array([d_hi, up_hi, d_lo, dn_lo, d_c, up_c])
+    A = np.array([1.0, 1.0, -1.0, -1.0, -1.0, -1.0])
+    o = oracle.token_objective(logp, np.zeros(6), None, A, np.zeros(6), p)
+    assert o["r"][0] == t_hi and o["r"][2] == t_lo and o["r"][4] == t_c
+    assert o["clip_hi"].tolist() == [False, True, False, False, False, False]
+    assert o["clip_lo"].tolist() == [False, False, False, True, False, False]
+    assert o["dual"].tolist() == [False, False, False, False, False, True]
+    # at the threshold the gradient flows through the unclipped branch
+    assert o["G"][0] == -t_hi and o["G"][2] == t_lo and o["G"][4] == t_c
+    assert o["G"][1] == 0.0 and o["G"][3] == 0.0 and o["G"][5] == 0.0
+
+
+def test_ratio_one_gives_minus_mean_advantage():
+    rng = np.random.default_rng(5)
+    R = 64
+    logp = -rng.random(R) * 5
+    A = rng.normal(size=R)
+    m = rng.random(R) < 0.6
+    o = oracle.token_objective(logp, logp.copy(), None, A, np.zeros(R),
+                               LossParams(dual_clip_c=3.0))
+    assert np.all(o["r"] == 1.0)
+    L, N = oracle.masked_token_mean(o["ell"], m)
+    assert N == int(m.sum())
+    assert abs(L - (-(A[m]).sum() / N)) < 1e-14
+    assert not o["clip_hi"].any() and not o["clip_lo"].any() and not o["dual"].any()
+
+
+def test_corrections_tis_and_clip_or_pop():
+    rho = np.zeros(5)
+    old = np.log(np.array([3.0, 0.5, 2.0, 1.0, 2.5]))
+    logp = old.copy()                 # PPO ratio against old is exactly 1
+    A = np.ones(5)
+    base = oracle.token_objective(logp, rho, None, A, np.zeros(5), LossParams(), old=old)
+    tis = oracle.token_objective(logp, rho, None, A, np.zeros(5),
+                                 LossParams(correction="tis", corr_lo=0.0, corr_hi=2.0), old=old)
+    pop = oracle.token_objective(logp, rho, None, A, np.zeros(5),
+                                 LossParams(correction="clip_or_pop", corr_lo=0.0, corr_hi=2.0),
+                                 old=old)
+    rc = np.exp(old - rho)
+    np.testing.assert_allclose(tis["wt"], [2.0, 0.5, rc[2], 1.0, 2.0], rtol=1e-15)
+    np.testing.assert_allclose(pop["wt"], [0.0, 0.5, rc[2], 1.0, 0.0], rtol=1e-15)
+    assert tis["corr_clip"].tolist() == [True, False, False, False, True]
+    assert pop["corr_clip"].tolist() == [True, False, False, False, True]
+    np.testing.assert_allclose(tis["pg"], tis["wt"] * base["pg"], rtol=1e-15)
+    np.testing.assert_allclose(pop["G"], pop["wt"] * base["G"], rtol=1e-15)
+    with pytest.raises(ValueError):
+        oracle.token_objective(logp, rho, None, A, np.zeros(5), LossParams(correction="tis"))
+
+
+def test_masked_mean_edge_cases():
+    assert oracle.masked_token_mean(np.array([1.0, 2.0]), np.array([0, 0])) == (0.0, 0)
+    L, N = oracle.masked_token_mean(np.array([1.0, 2.0, 4.0]), np.array([1, 0, 1]))
+    assert N == 2 and L == 2.5
+
+
+# ---------------------------------------------------------------- gradient
+
+@pytest.mark.parametrize("name", ["full_two_tokens"])
+def test_full_pipeline_golden(name):
+    c = _golden()[name]
+    z = np.array([[_ev(v) for v in row] for row in c["z"]])
+    out = oracle.rl_loss(z, np.array(c["y"]), np.array([_ev(v) for v in c["rho"]]), None,
+                         np.array([_ev(v) for v in c["w"]]), np.array(c["gid"]),
+                         np.array(c["cu"]), c["n_groups"], np.array(c["mask"]), LossParams())
+    assert abs(out["loss"] - _ev(c["expect"]["loss"])) < 1e-14
+    want = np.array([[_ev(v) for v in row] for row in c["expect"]["dlogits"]])
+    np.testing.assert_allclose(out["dlogits"], want, atol=1e-14, rtol=0)
+
+
+def test_cross_entropy_special_case():
+    """A = 1, rho = logp, beta = gamma = 0, T = 1, all tokens train: r = 1,
+    L = -1 and dZ = (p - onehot)/N, the gradient of the mean cross-entropy."""
+    rng = np.random.default_rng(6)
+    R, V = 12, 37
+    z = rng.normal(0, 2, size=(R, V))
+    y = rng.integers(0, V, size=R)
+    logp, H, lse = oracle.row_log_softmax(z, y, 1.0)
+    o = oracle.rl_loss_rows(z, y, logp, None, np.ones(R), np.ones(R, bool), R, LossParams())
+    assert np.all(o["r"] == 1.0) and abs(o["ell"].mean() + 1.0) < 1e-15
+    zt = torch.from_numpy(z).requires_grad_(True)
+    torch.nn.functional.cross_entropy(zt, torch.from_numpy(y), reduction="mean").backward()
+    np.testing.assert_allclose(o["dlogits"], zt.grad.numpy(), atol=1e-15, rtol=0)
+
+
+def _near_kink(out, p, guard=1e-4):
+    r = out["r"]
+    th = [1 - p.eps_lo, 1 + p.eps_hi] + ([p.dual_clip_c] if p.dual_clip_c else [])
+    if p.correction != "none":
+        th += [p.corr_lo, p.corr_hi]
+        r = np.concatenate([r, out["rc"]])
+    return any(np.any(np.abs(r - t) < guard * max(1.0, t)) for t in th)
+
+
+@pytest.mark.parametrize("V", [2, 3, 5, 8])
+@pytest.mark.parametrize("variant", ["ppo_dual_kl_ent_T", "tis", "clip_or_pop", "opd"])
+def test_dlogits_central_finite_differences(V, variant):
+    rng = np.random.default_rng(100 + V)
+    n_traj, L_ = 4, 2
+    R = n_traj * L_
+    p = LossParams(temperature=0.8, eps_lo=0.15, eps_hi=0.25, dual_clip_c=2.5,
+                   kl_coef=0.3, entropy_coef=0.07)
+    if variant in ("tis", "clip_or_pop"):
+        p = LossParams(temperature=1.3, eps_lo=0.2, eps_hi=0.2, kl_coef=0.1,
+                       entropy_coef=0.02, correction=variant, corr_lo=0.5, corr_hi=1.5)
+    if variant == "opd":
+        p = LossParams(temperature=1.0, eps_lo=0.2, eps_hi=0.2, opd_coef=0.7)
+    for attempt in range(50):
+        z = rng.normal(0, 1.5, size=(R, V))
+        y = rng.integers(0, V, size=R)
+        logp, _, _ = oracle.row_log_softmax(z, y, p.temperature)
+        rho = logp + rng.normal(0, 0.6, size=R)
+        q = logp + rng.normal(0, 0.5, size=R)
+        old = logp + rng.normal(0, 0.3, size=R) if p.correction != "none" else None
+        teacher = logp + rng.normal(0, 0.5, size=R)
+        w = rng.random(n_traj)
+        gid = np.array([0, 0, 1, 1])
+        cu = np.arange(n_traj + 1) * L_
+        m = np.array([1, 1, 0, 1, 1, 1, 1, 0], dtype=bool)
+        args = (y, rho, q, w, gid, cu, 2, m, p)
+        out = oracle.rl_loss(z, *args, grad_loss=1.7, old=old, teacher=teacher)
+        if not _near_kink(out, p):
+            break
+    else:
+        pytest.fail("no draw away from the kinks")
+    if variant == "ppo_dual_kl_ent_T":
+        assert out["clip_hi"].any() or out["clip_lo"].any() or out["dual"].any()
+    h = 1e-6
+    num = np.zeros_like(z)
+    for i in range(R):
+        for j in range(V):
+            zp = z.copy(); zp[i, j] += h
+            zm = z.copy(); zm[i, j] -= h
+            lp = oracle.rl_loss(zp, *args, old=old, teacher=teacher, want_dlogits=False)["loss"]
+            lm = oracle.rl_loss(zm, *args, old=old, teacher=teacher, want_dlogits=False)["loss"]
+            num[i, j] = 1.7 * (lp - lm) / (2 * h)
+    scale = np.abs(out["dlogits"]).max()
+    np.testing.assert_allclose(out["dlogits"], num, atol=1e-6 * max(scale, 1e-3), rtol=1e-6)
+    assert np.all(out["dlogits"][~m] == 0.0)
+
+
+def test_chunking_changes_nothing():
+    rng = np.random.default_rng(7)
+    R, V = 40, 33
+    z = rng.normal(0, 2, size=(R, V))
+    y = rng.integers(0, V, size=R)
+    rho = rng.normal(-3, 0.1, size=R)
+    w = rng.random(8)
+    gid = np.repeat(np.arange(2), 4)
+    cu = np.arange(9) * 5
+    m = rng.random(R) < 0.7
+    p = LossParams(dual_clip_c=3.0)
+    a = oracle.rl_loss(z, y, rho, None, w, gid, cu, 2, m, p, chunk=1)
+    b = oracle.rl_loss(z, y, rho, None, w, gid, cu, 2, m, p, chunk=256)
+    assert a["loss"] == b["loss"]
+    np.testing.assert_array_equal(a["dlogits"], b["dlogits"])
+
+
+def test_no_training_tokens():
+    z = np.zeros((3, 4))
+    out = oracle.rl_loss(z, np.array([0, 1, 2]), np.zeros(3), None, np.array([0.0, 1.0]),
+                         np.array([0, 0]), np.array([0, 2, 3]), 1, np.zeros(3), LossParams())
+    assert out["loss"] == 0.0 and out["N"] == 0
+    assert np.all(out["dlogits"] == 0.0)
+    assert out["stats"]["ratio_mean"] == 0.0
