@@ -1,0 +1,418 @@
+#!/usr/bin/env python
+"""Throughput of the fused RL-loss forward+backward on GB300.
+
+One step = one rl_loss_fwd_bwd call (advantage kernel, fused vocabulary
+sweep, statistics kernel) over one synthetic batch shaped like the paper's
+long agentic sessions: 65,536 rows (64 trajectories x 1,024 tokens, groups
+of 16) x vocabulary 154,880, bf16 logits -> bf16 dLogits, dual clip 3, k3
+KL 0.01 (the "glm" recipe of paper_2609_08368_gb300.workloads).
+
+Prints one JSON line (rank 0). Under torchrun every rank runs its own
+independent batch (weak scaling; the loss has no exchange between
+replicas). ``--impl reference`` times the float64 CPU oracle instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import shutil
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "RL-loss fwd+bwd tokens/sec at vocab 154,880 bf16; achieved HBM GB/s vs 8 TB/s"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "sweep_kernel_glm.md")
+SWEEP_SOURCES = ["k_sweep.cu", "common.cuh", "kernels.h"]
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="glm")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--cpu-sample-rows", type=int, default=512)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------- plumbing
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend=backend)
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(local)
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+class ClockSampler:
+    """nvidia-smi samples of the SM clock and throttle reasons while the
+    timed region runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    REASONS = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, device_index: int, period_ms: int = 50):
+        self.proc = None
+        self.path = None
+        exe = shutil.which("nvidia-smi")
+        if exe is None:
+            return
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        self.cmd = [exe, "-i", str(device_index), f"--query-gpu={self.FIELDS}",
+                    "--format=csv,noheader,nounits", "-lms", str(period_ms)]
+
+    def start(self):
+        if self.path is None:
+            return
+        self.fh = open(self.path, "w")
+        self.proc = subprocess.Popen(self.cmd, stdout=self.fh, stderr=subprocess.DEVNULL)
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.1)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.fh.close()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) != 8:
+                continue
+            try:
+                rows.append((float(parts[0]), float(parts[1]), parts[2], parts[4:]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [r[0] for r in rows]
+        reasons = sorted({self.REASONS[i] for r in rows for i, v in enumerate(r[3])
+                          if v.lower() == "active"})
+        try:
+            power = max(float(r[2]) for r in rows)
+        except ValueError:
+            power = None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(r[1] for r in rows),
+                "sm_mhz_min": min(sm), "samples": len(rows), "power_w_max": power,
+                "reasons": reasons}
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            return json.load(f), "measured"
+    return {"hbm_gbs": FALLBACK_HBM_GBS}, "fallback"
+
+
+def sweep_source_hash() -> str:
+    h = hashlib.sha256()
+    for name in SWEEP_SOURCES:
+        with open(os.path.join(ROOT, "paper_2609_08368_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(rows_now: int):
+    """DRAM bytes of one sweep launch from the committed ncu summary, if it
+    was taken on the current kernel source; scaled by rows if captured on a
+    smaller case of the same vocabulary."""
+    if not os.path.exists(PROFILE_SUMMARY):
+        return None
+    text = open(PROFILE_SUMMARY).read()
+    src = re.search(r"source_sha256:\s*([0-9a-f]+)", text)
+    tb = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    rows = re.search(r"rows_per_launch:\s*([0-9]+)", text)
+    if not (src and tb and rows) or src.group(1) != sweep_source_hash():
+        return None
+    return float(tb.group(1)) * rows_now / int(rows.group(1))
+
+
+def algorithmic_bytes_per_row(w, dl_dtype) -> int:
+    """Logits read once + dLogits written once + the per-row inputs and
+    outputs (target, rollout log-prob, optional ref / old / teacher
+    log-probs, mask byte, log-prob and entropy out)."""
+    es_in = w.logits.element_size()
+    es_out = torch.tensor([], dtype=dl_dtype).element_size()
+    small = 4 + 4 + 1 + 4 + 4
+    for t in (w.ref_logprobs, w.old_logprobs, w.teacher_logprobs):
+        if t is not None:
+            small += 4
+    return w.vocab * (es_in + es_out) + small
+
+
+# ---------------------------------------------------------------- CPU oracle
+
+def oracle_sample(w, n_rows: int, seed: int = 7):
+    """Times the float64 CPU oracle on ``n_rows`` rows of the workload (every
+    per-row output and dLogits of those rows, with the call-wide advantages
+    and token count of the whole batch). Returns (rows/s, seconds, rows)."""
+    import oracle
+
+    p = oracle.LossParams(**w.params)
+    rng = np.random.default_rng(seed)
+    rows = np.sort(rng.choice(w.n_rows, size=min(n_rows, w.n_rows), replace=False))
+    idx = torch.from_numpy(rows).to(w.logits.device)
+    z = w.logits[idx, :w.vocab].cpu()
+    z = z.view(torch.int16).numpy().view(np.uint16) if z.dtype == torch.bfloat16 else z.numpy()
+
+    def host(t):
+        return None if t is None else t.cpu().numpy()
+
+    mask = host(w.loss_mask)
+    y, rho = host(w.targets)[rows], host(w.rollout_logprobs)[rows]
+    q = None if w.ref_logprobs is None else host(w.ref_logprobs)[rows]
+    t0 = time.perf_counter()
+    A, _ = oracle.group_advantages(host(w.rewards), host(w.group_id), w.n_groups, p)
+    A_row = oracle.row_advantages(A, host(w.cu_seqlens), w.n_rows)
+    N = int(mask.astype(bool).sum())
+    for lo in range(0, len(rows), 128):
+        hi = min(len(rows), lo + 128)
+        oracle.rl_loss_rows(z[lo:hi], y[lo:hi], rho[lo:hi], None if q is None else q[lo:hi],
+                            A_row[rows[lo:hi]], mask[rows[lo:hi]].astype(bool), N, p)
+    dt = time.perf_counter() - t0
+    return len(rows) / dt, dt, len(rows)
+
+
+def run_reference(args, rank, world):
+    """The reference arm: the float64 CPU oracle as it stands, on the host
+    cores, on bounded samples of the same workload."""
+    if rank != 0:
+        return
+    from paper_2609_08368_gb300 import workloads as wl
+
+    rec = wl.RECIPES[args.workload]
+    w = wl.make(rec, "cuda" if torch.cuda.is_available() else "cpu")
+    rows_per_step = 128
+    for _ in range(args.warmup):
+        oracle_sample(w, rows_per_step, seed=1)
+    times = []
+    for k in range(args.steps):
+        _, dt, n = oracle_sample(w, rows_per_step, seed=100 + k)
+        times.append(dt)
+    total = sum(times)
+    value = rows_per_step * args.steps / total
+    sample = (f"{rows_per_step} random rows of the {rec.n_rows} x {rec.vocab} batch per step "
+              f"(all per-row outputs and dLogits; call-wide advantages and N)")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * total / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": f"{args.workload}: {rec.n_rows} rows x vocab {rec.vocab}",
+                       "rows": rec.n_rows, "vocab": rec.vocab},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------- GPU arm
+
+def _pinned_copy(w):
+    """The workload's tensors copied into pinned host memory."""
+    from paper_2609_08368_gb300 import workloads as wl
+
+    def pin(t):
+        if t is None:
+            return None
+        h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+        h.copy_(t)
+        return h
+    return wl.Workload(w.recipe, pin(w.logits), pin(w.targets), pin(w.rollout_logprobs),
+                       pin(w.ref_logprobs), pin(w.old_logprobs), pin(w.teacher_logprobs),
+                       pin(w.rewards), pin(w.group_id), pin(w.cu_seqlens), pin(w.loss_mask),
+                       w.n_groups, dict(w.params))
+
+
+def run_ours(args, rank, world, local):
+    from paper_2609_08368_gb300 import api, milesloss as ml, workloads as wl
+
+    ml.load()
+    dev = torch.device("cuda", local)
+    rec = wl.RECIPES[args.workload]
+    rec = wl.shrink(rec, seed=rec.seed + 1000 * rank)  # each replica has its own batch
+    w = wl.make(rec, dev)
+    R, V = w.n_rows, w.vocab
+    dl_dtype = w.logits.dtype
+    buf = api.alloc(R, int(w.rewards.shape[0]), w.n_groups, dev, vocab=V, dlogits_dtype=dl_dtype)
+    stream = torch.cuda.current_stream()
+
+    for _ in range(max(3, args.warmup)):
+        api.fwd_bwd(w, buf)
+    torch.cuda.synchronize()
+    err = ml.rl_loss_check_device_error(buf.workspace)
+    if err:
+        raise RuntimeError(f"device error during warm-up: {ml.status_string(err)}")
+
+    K = args.steps
+    ev_sweep = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                for _ in range(K)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    clocks.start()
+    barrier(world)
+    torch.cuda.synchronize()
+    start.record(stream)
+    for i in range(K):
+        ml.rl_set_sweep_events(*ev_sweep[i])
+        api.fwd_bwd(w, buf)
+    stop.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    ml.rl_set_sweep_events(None, None)
+    clk = clocks.stop()
+    ms_total = start.elapsed_time(stop)
+    ms_total = max_over_ranks(ms_total, world)
+    ms_step = ms_total / K
+    sweep_ms = [b.elapsed_time(e) for b, e in ev_sweep]
+    err = ml.rl_loss_check_device_error(buf.workspace)
+    if err:
+        raise RuntimeError(f"device error: {ml.status_string(err)}")
+    stats = buf.read_stats()
+    rows_all = sum_over_ranks(float(R), world)
+    value = rows_all * K / (ms_total / 1e3)
+
+    bpr = algorithmic_bytes_per_row(w, dl_dtype)
+    launch_bytes = bpr * R
+    sweep_avg = statistics.fmean(sweep_ms)
+    peaks, peak_kind = measured_peaks()
+    peak = float(peaks["hbm_gbs"])
+    achieved = launch_bytes / (sweep_avg / 1e3) / 1e9
+    step_gbs = launch_bytes / (ms_step / 1e3) / 1e9
+
+    # end to end through host buffers (pinned), one call per step
+    e2e = None
+    if not args.no_e2e and args.e2e_steps > 0:
+        host_w = _pinned_copy(w)
+        call = api.HostCall(host_w, dev, dev_w=w, buf=buf)
+        call()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier(world)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(args.e2e_steps):
+            call()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier(world)
+        ms_e2e = max_over_ranks(e0.elapsed_time(e1), world) / args.e2e_steps
+        e2e = {"value": rows_all / (ms_e2e / 1e3), "unit": "tokens/s",
+               "ms_per_step": ms_e2e, "steps": args.e2e_steps,
+               "h2d_bytes_per_step": call.bytes_in(), "d2h_bytes_per_step": call.bytes_out()}
+        del call, host_w
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rps, secs, n = oracle_sample(w, args.cpu_sample_rows)
+        cpu = {"value": rps, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+               "sample": f"{n} random rows of the {R} x {V} batch (every per-row output and "
+                         f"dLogits of those rows; call-wide advantages and N), {secs:.1f} s"}
+
+    traffic = profiled_traffic(R)
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
+        "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"{args.workload}: {R} rows ({rec.n_traj} traj x {rec.traj_len} "
+                               f"tokens, groups of {rec.group_size}) x vocab {V}, "
+                               f"{'bf16' if w.logits.dtype == torch.bfloat16 else 'f32'} logits "
+                               f"-> dLogits",
+                   "rows": R, "vocab": V, "parallelism": f"replicas x{world}",
+                   "l2": "inputs larger than L2 (20+ GB per step), no flush"},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "kernel": "k_sweep (fused fwd+bwd vocabulary sweep)",
+                     "bytes_per_launch": launch_bytes, "sweep_ms": sweep_avg,
+                     "peak_kind": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"
+                     if peak_kind == "measured" else "fallback 6.8 TB/s",
+                     "frac_of_8tbs": achieved / NOMINAL_HBM_GBS},
+        "step_hbm_gbs": step_gbs,
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": 3 * K,
+        "clocks": clk,
+        "loss": stats["loss"],
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    rank, world, local = dist_setup()
+    try:
+        if args.impl == "reference":
+            run_reference(args, rank, world)
+        else:
+            run_ours(args, rank, world, local)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

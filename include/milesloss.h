@@ -1,0 +1,223 @@
+/*
+ * libmilesloss: the per-token RL loss over the vocabulary, forward and
+ * backward, on one GB300 GPU (sm_103a).
+ *
+ * The trainer side of an RL post-training loop ("Miles v0.1: Production-Level
+ * Post-Training", arxiv 2609.08368) computes, for every token a policy sampled,
+ * the trainer's log-prob of that token, the importance ratio against the log-
+ * prob the rollout engine reported, r = exp(log pi_train - log pi_rollout)
+ * (Sec. 3.4), a group-relative advantage (GRPO, Sec. 2 and Sec. 9.1), and a
+ * loss whose gradient updates the policy (Sec. 1.1). This library evaluates
+ * that loss from the policy's logits over the full vocabulary and writes
+ * dLogits, without ever materialising the softmax.
+ *
+ * Per token t (row t of the logits), with s = z / T:
+ *   logp_t = s_y - logsumexp(s),  H_t = -sum_j p_j log p_j      (entropy)
+ *   r_t    = exp(logp_t - base_t), base = old log-probs if given, else the
+ *            rollout log-probs                                       (Sec. 3.4)
+ *   pg_t   = max(-A r, -A clip(r, 1-eps_lo, 1+eps_hi)), then for A < 0 capped
+ *            at -A c by the dual clip                               (PPO)
+ *   optional TIS / clip-or-pop weight on pg_t                      (Sec. 3.4)
+ *   k3_t   = exp(q - logp) - (q - logp) - 1 against reference log-probs q
+ *   l_t    = pg_t + kl_coef k3_t - entropy_coef H_t
+ *   loss   = sum_t m_t l_t / sum_t m_t  (m = loss mask, Sec. 2.4)
+ * A is the GRPO advantage of the token's trajectory: rewards centred (and by
+ * default scaled by the sample std, floored) within the trajectory's group;
+ * a group whose rewards are all equal gets A = 0 (Sec. 2.2, Table 2). With
+ * on-policy distillation, A_t -= opd_coef (rollout_logprob_t -
+ * teacher_logprob_t) (Sec. 5.2).
+ *
+ * Conventions shared by every call below.
+ *  - Every array pointer is DEVICE memory owned by the caller. The library
+ *    never allocates, frees or synchronises; each call only enqueues work on
+ *    `stream` and returns. The library keeps no state between calls except
+ *    per-device kernel attributes set once.
+ *  - Calls on different streams are safe given distinct workspaces and
+ *    outputs. A workspace written by rl_loss_fwd must not be reused before
+ *    the matching rl_loss_bwd has run.
+ *  - Host-side argument errors return a status before anything is enqueued.
+ *  - Data-dependent errors (a target outside [0, vocab), a group id outside
+ *    [0, n_groups), cu_seqlens not non-decreasing from 0 to n_rows, a wait
+ *    inside a kernel that ran out of time) never trap: the kernels finish,
+ *    write zeros for the affected rows, and record the error in the
+ *    workspace; read it with rl_loss_check_device_error after the stream is
+ *    synchronised.
+ *  - Outputs are defined for every row, trained or not; rows with mask 0 get
+ *    their log-prob and entropy and a zero dLogits row.
+ *  - n_rows == 0 is a valid no-op apart from zeroed statistics.
+ */
+#ifndef MILESLOSS_H
+#define MILESLOSS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st* rl_stream;
+
+typedef enum {
+  RL_OK = 0,
+  RL_ERR_INVALID_ARG = 1,         /* a pointer, size or parameter is invalid   */
+  RL_ERR_UNSUPPORTED = 2,         /* valid but not implemented (see message)   */
+  RL_ERR_WORKSPACE_TOO_SMALL = 3, /* workspace_bytes < rl_loss_workspace_size  */
+  RL_ERR_CUDA = 4,                /* a CUDA runtime call failed                */
+  RL_ERR_TARGET_OUT_OF_RANGE = 5, /* device: a target id not in [0, vocab)     */
+  RL_ERR_GROUP_OUT_OF_RANGE = 6,  /* device: a group id not in [0, n_groups)   */
+  RL_ERR_BAD_SEQLENS = 7,         /* device: cu_seqlens not 0 <= ... <= n_rows,
+                                     non-decreasing, ending at n_rows          */
+  RL_ERR_DEVICE_TIMEOUT = 8       /* device: a bounded wait gave up            */
+} rl_status;
+
+typedef enum { RL_BF16 = 0, RL_F32 = 1 } rl_dtype;
+
+/* Ratio corrections of Sec. 3.4. Both need old_logprobs: the PPO ratio is
+ * then exp(logp - old) and the correction ratio rc = exp(old - rollout) is a
+ * constant per-token weight on the policy-gradient term:
+ *   RL_CORR_TIS          weight = min(max(rc, corr_lo), corr_hi)
+ *   RL_CORR_CLIP_OR_POP  weight = rc if corr_lo <= rc <= corr_hi, else 0 */
+typedef enum { RL_CORR_NONE = 0, RL_CORR_TIS = 1, RL_CORR_CLIP_OR_POP = 2 } rl_correction;
+
+typedef struct {
+  float temperature;   /* T > 0: logits are divided by T before the softmax      */
+  float eps_lo;        /* >= 0: lower clip at 1 - eps_lo                          */
+  float eps_hi;        /* >= 0: upper clip at 1 + eps_hi                          */
+  float dual_clip_c;   /* 0 = off, else > 1: for A < 0 the PG term is capped at -A c */
+  float kl_coef;       /* beta >= 0; ref_logprobs must be given when beta > 0     */
+  float entropy_coef;  /* gamma >= 0: the token loss gets -gamma * H              */
+  float std_floor;     /* > 0: GRPO divides by max(std, std_floor)                */
+  int32_t normalize_std; /* 1: divide by the group std (GRPO); 0: centre only   */
+  int32_t unbiased_std;  /* 1: sample std (n - 1); 0: population std (n)        */
+  int32_t correction;    /* rl_correction                                       */
+  float corr_lo;       /* correction interval [corr_lo, corr_hi], default [0, 2] */
+  float corr_hi;
+  float opd_coef;      /* on-policy distillation coefficient; 0 = off (Sec. 5.2) */
+} rl_loss_params;
+
+/* Call-wide statistics, written to DEVICE memory by the stream. Means are
+ * over the tokens that train (mask 1); all fields are 0 when there are none.
+ * The integers are exact counts. */
+typedef struct {
+  double loss;                 /* sum m l / N                                      */
+  double pg_loss_mean;         /* mean PG term (after any correction weight)       */
+  double kl_mean;              /* mean k3 (0 without ref_logprobs)                 */
+  double entropy_mean;         /* mean H                                           */
+  double ratio_mean;           /* mean r                                           */
+  double ratio_absdev_mean;    /* mean |r - 1|                                     */
+  double logprob_absdiff_mean; /* mean |logp - rollout logp| (train/rollout divergence, Sec. 9.2) */
+  double corr_ratio_mean;      /* mean pre-clamp correction ratio rc (1 without)   */
+  double corr_absdev_mean;     /* mean |rc - 1|                                    */
+  float ratio_min;
+  float ratio_max;
+  int64_t n_tokens;            /* N = sum m                                        */
+  int64_t n_clip_hi;           /* PPO clip engaged above 1 + eps_hi               */
+  int64_t n_clip_lo;           /* PPO clip engaged below 1 - eps_lo               */
+  int64_t n_dual_clip;         /* dual clip engaged                                */
+  int64_t n_corr_clip;         /* correction weight differs from rc (Sec. 3.4 clipped fraction) */
+} rl_loss_stats;
+
+/* Bytes of device workspace that one call with these sizes needs (the same
+ * value serves rl_loss_fwd, rl_loss_bwd and rl_loss_fwd_bwd). The workspace
+ * is caller-owned, 256-byte aligned, needs no initialisation, and carries the
+ * per-row state from rl_loss_fwd to rl_loss_bwd. */
+rl_status rl_loss_workspace_size(int64_t n_rows, int32_t n_traj, int32_t n_groups,
+                                 size_t* bytes);
+
+/* Forward: log-probs, entropy, advantages, the loss and its statistics.
+ *
+ *  logits            [n_rows, ld] of `logits_dtype` (bf16 or fp32); row t
+ *                    holds the logits that scored targets[t] (already shifted
+ *                    by the caller); only the first `vocab` columns are read.
+ *                    Rows whose start is 16-byte aligned (ld * element size a
+ *                    multiple of 16 and a 16-byte aligned base) take the
+ *                    fast bulk-copy path; any other layout is still correct.
+ *  targets           [n_rows] int32 sampled token ids, in [0, vocab)
+ *  rollout_logprobs  [n_rows] fp32 log-probs the rollout engine reported
+ *  ref_logprobs      [n_rows] fp32 reference-policy log-probs, or NULL
+ *                    (required when kl_coef > 0)
+ *  old_logprobs      [n_rows] fp32 log-probs of the policy before this update,
+ *                    or NULL (then the PPO ratio is taken against the rollout
+ *                    log-probs); required when a correction is set
+ *  teacher_logprobs  [n_rows] fp32 teacher log-probs for OPD, or NULL
+ *                    (required when opd_coef != 0)
+ *  rewards           [n_traj] fp32, one outcome reward per trajectory
+ *  group_id          [n_traj] int32 in [0, n_groups): the prompt of each
+ *                    trajectory; members of a group may be anywhere
+ *  cu_seqlens        [n_traj + 1] int32 row offsets: trajectory i owns rows
+ *                    [cu[i], cu[i+1]); cu[0] = 0, cu[n_traj] = n_rows
+ *  loss_mask         [n_rows] uint8, nonzero = the token trains (model-
+ *                    generated; tool output and prompts are masked, Sec. 2.4)
+ *  params            host pointer, read during the call only
+ *  token_logprobs    [n_rows] fp32 out, or NULL
+ *  entropy           [n_rows] fp32 out, or NULL
+ *  advantages        [n_traj] fp32 out (before OPD shaping), or NULL
+ *  group_sizes       [n_groups] int32 out, or NULL
+ *  stats             one rl_loss_stats out (device), or NULL
+ *  workspace         device, >= rl_loss_workspace_size bytes
+ */
+rl_status rl_loss_fwd(const void* logits, rl_dtype logits_dtype, int64_t n_rows,
+                      int64_t vocab, int64_t ld, const int32_t* targets,
+                      const float* rollout_logprobs, const float* ref_logprobs,
+                      const float* old_logprobs, const float* teacher_logprobs,
+                      const float* rewards, const int32_t* group_id,
+                      const int32_t* cu_seqlens, int32_t n_traj, int32_t n_groups,
+                      const uint8_t* loss_mask, const rl_loss_params* params,
+                      float* token_logprobs, float* entropy, float* advantages,
+                      int32_t* group_sizes, rl_loss_stats* stats, void* workspace,
+                      size_t workspace_bytes, rl_stream stream);
+
+/* Backward from the state rl_loss_fwd left in `workspace`: dLogits of
+ * g * loss with g = grad_loss * (*grad_loss_device if non-NULL), i.e.
+ *   dZ_tj = g (m_t / N) (1/T) [G_t (1[j = y_t] - p_j) + gamma p_j (log p_j + H_t)]
+ * with G_t = d l_t / d logp_t. Re-reads the logits once. The logits, targets,
+ * mask and params must be the ones given to rl_loss_fwd.
+ *  dlogits  [n_rows, ld_out] of `dlogits_dtype` (bf16 rounded to nearest
+ *           even, or fp32); columns >= vocab are not written. */
+rl_status rl_loss_bwd(const void* logits, rl_dtype logits_dtype, int64_t n_rows,
+                      int64_t vocab, int64_t ld, const int32_t* targets,
+                      const uint8_t* loss_mask, const rl_loss_params* params,
+                      float grad_loss, const float* grad_loss_device,
+                      const void* workspace, size_t workspace_bytes, void* dlogits,
+                      rl_dtype dlogits_dtype, int64_t ld_out, rl_stream stream);
+
+/* Forward and backward in one pass that reads each logit row from HBM once:
+ * every output of rl_loss_fwd plus dLogits as in rl_loss_bwd. */
+rl_status rl_loss_fwd_bwd(const void* logits, rl_dtype logits_dtype, int64_t n_rows,
+                          int64_t vocab, int64_t ld, const int32_t* targets,
+                          const float* rollout_logprobs, const float* ref_logprobs,
+                          const float* old_logprobs, const float* teacher_logprobs,
+                          const float* rewards, const int32_t* group_id,
+                          const int32_t* cu_seqlens, int32_t n_traj, int32_t n_groups,
+                          const uint8_t* loss_mask, const rl_loss_params* params,
+                          float* token_logprobs, float* entropy, float* advantages,
+                          int32_t* group_sizes, rl_loss_stats* stats,
+                          float grad_loss, const float* grad_loss_device, void* dlogits,
+                          rl_dtype dlogits_dtype, int64_t ld_out, void* workspace,
+                          size_t workspace_bytes, rl_stream stream);
+
+/* After the stream that ran a call on `workspace` has been synchronised:
+ * RL_OK, or the data-dependent error the kernels recorded (when several
+ * kinds occurred, the lowest code). Performs one small blocking
+ * device-to-host copy on the legacy default stream. */
+rl_status rl_loss_check_device_error(const void* workspace);
+
+/* Static text for a status code; never NULL. */
+const char* rl_status_string(rl_status status);
+
+/* Optional timing hook for the calling host thread: when both are non-NULL,
+ * later calls on this thread record `begin` / `end` (cudaEvent_t) on their
+ * stream immediately before and after the main vocabulary-sweep kernel.
+ * Pass NULLs to turn it off. */
+rl_status rl_set_sweep_events(void* begin_event, void* end_event);
+
+/* Version of this interface, e.g. 100 for 1.0. */
+int32_t rl_loss_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MILESLOSS_H */

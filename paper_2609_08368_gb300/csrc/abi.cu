@@ -1,0 +1,473 @@
+// The C ABI of libmilesloss: argument validation, workspace layout, launch
+// planning and kernel launches. Nothing here allocates, frees or
+// synchronises; every call enqueues its kernels on the caller's stream.
+//
+// rl_loss_fwd_bwd = advantage kernel -> fused sweep -> statistics kernel
+// rl_loss_fwd     = advantage kernel -> forward-only sweep -> statistics kernel
+// rl_loss_bwd     = gradient sweep from the saved per-row state
+#include <climits>
+#include <cmath>
+#include <cstdlib>
+#include <map>
+#include <mutex>
+#include <tuple>
+
+#include "kernels.h"
+
+using namespace milesloss;
+
+namespace {
+
+thread_local cudaEvent_t t_ev_begin = nullptr;
+thread_local cudaEvent_t t_ev_end = nullptr;
+
+std::mutex g_mu;
+std::map<std::pair<int, const void*>, int> g_smem_set;               // (device, fn) -> bytes
+std::map<std::tuple<int, const void*, int, int>, int> g_occupancy;   // (dev, fn, C, smem) -> clusters
+
+bool finite(float x) { return std::isfinite(x); }
+
+rl_status cuda_fail(cudaError_t e) { return e == cudaSuccess ? RL_OK : RL_ERR_CUDA; }
+
+int env_int(const char* name, int dflt) {
+  const char* v = std::getenv(name);
+  if (!v || !*v) return dflt;
+  return std::atoi(v);
+}
+
+rl_status set_smem(const void* fn, int dev, int bytes) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  auto key = std::make_pair(dev, fn);
+  auto it = g_smem_set.find(key);
+  if (it != g_smem_set.end() && it->second >= bytes) return RL_OK;
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e != cudaSuccess) return RL_ERR_CUDA;
+  g_smem_set[key] = bytes;
+  return RL_OK;
+}
+
+// Number of clusters of C CTAs that can be resident at once.
+rl_status resident_clusters(const void* fn, int dev, int C, int smem, int threads, int* out) {
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    auto it = g_occupancy.find(std::make_tuple(dev, fn, C, smem));
+    if (it != g_occupancy.end()) { *out = it->second; return RL_OK; }
+  }
+  int n = 0;
+  if (C == 1) {
+    int per_sm = 0, sms = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, threads, smem) != cudaSuccess)
+      return RL_ERR_CUDA;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return RL_ERR_CUDA;
+    n = per_sm * sms;
+  } else {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(C);
+    cfg.blockDim = dim3(threads);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = C;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess) return RL_ERR_CUDA;
+  }
+  if (n <= 0) return RL_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_occupancy[std::make_tuple(dev, fn, C, smem)] = n;
+  *out = n;
+  return RL_OK;
+}
+
+rl_status launch(const void* fn, dim3 grid, dim3 block, int smem, int cluster, cudaStream_t s,
+                 void* arg) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  if (cluster > 1) {
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = cluster;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+  }
+  void* args[1] = {arg};
+  return cuda_fail(cudaLaunchKernelExC(&cfg, fn, args));
+}
+
+size_t elem_size(rl_dtype d) { return d == RL_BF16 ? 2 : 4; }
+bool dtype_ok(int d) { return d == RL_BF16 || d == RL_F32; }
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+rl_status check_params(const rl_loss_params* p) {
+  if (!p) return RL_ERR_INVALID_ARG;
+  if (!finite(p->temperature) || !(p->temperature > 0.0f)) return RL_ERR_INVALID_ARG;
+  if (!finite(p->eps_lo) || !finite(p->eps_hi) || p->eps_lo < 0.0f || p->eps_hi < 0.0f)
+    return RL_ERR_INVALID_ARG;
+  if (!finite(p->dual_clip_c) || p->dual_clip_c < 0.0f ||
+      (p->dual_clip_c > 0.0f && p->dual_clip_c <= 1.0f))
+    return RL_ERR_INVALID_ARG;
+  if (!finite(p->kl_coef) || p->kl_coef < 0.0f) return RL_ERR_INVALID_ARG;
+  if (!finite(p->entropy_coef) || p->entropy_coef < 0.0f) return RL_ERR_INVALID_ARG;
+  if (!finite(p->std_floor) || !(p->std_floor > 0.0f)) return RL_ERR_INVALID_ARG;
+  if ((p->normalize_std != 0 && p->normalize_std != 1) ||
+      (p->unbiased_std != 0 && p->unbiased_std != 1))
+    return RL_ERR_INVALID_ARG;
+  if (p->correction < RL_CORR_NONE || p->correction > RL_CORR_CLIP_OR_POP)
+    return RL_ERR_INVALID_ARG;
+  if (p->correction != RL_CORR_NONE &&
+      (!finite(p->corr_lo) || !finite(p->corr_hi) || p->corr_lo < 0.0f || p->corr_lo > p->corr_hi))
+    return RL_ERR_INVALID_ARG;
+  if (!finite(p->opd_coef)) return RL_ERR_INVALID_ARG;
+  return RL_OK;
+}
+
+LossScalars scalars(const rl_loss_params* p) {
+  LossScalars s;
+  s.invT = 1.0f / p->temperature;
+  s.k = 1.4426950408889634f / p->temperature;
+  s.eps_lo = p->eps_lo;
+  s.eps_hi = p->eps_hi;
+  s.dual_c = p->dual_clip_c;
+  s.beta = p->kl_coef;
+  s.gamma = p->entropy_coef;
+  s.corr_lo = p->corr_lo;
+  s.corr_hi = p->corr_hi;
+  s.corr = p->correction;
+  return s;
+}
+
+struct SweepPlan {
+  int C, S, slice, stage_bytes, smem;
+};
+
+// Smallest cluster whose per-CTA slice fits two stages in shared memory;
+// as many stages as fit, up to kMaxStages. Overridable for tuning through
+// MILESLOSS_SWEEP_CLUSTER / MILESLOSS_SWEEP_STAGES.
+rl_status plan_sweep(rl_dtype dt, long long V, int dev, SweepPlan* out) {
+  int optin = 0;
+  if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+    return RL_ERR_CUDA;
+  const int budget = optin - kSweepSmemExtra;
+  const int es = static_cast<int>(elem_size(dt));
+  const int vec = 16 / es;
+  const int forced_c = env_int("MILESLOSS_SWEEP_CLUSTER", 0);
+  const int forced_s = env_int("MILESLOSS_SWEEP_STAGES", 0);
+  for (int C = 1; C <= 8; C *= 2) {
+    if (forced_c && C != forced_c) continue;
+    long long slice = (V + C - 1) / C;
+    slice = (slice + vec - 1) / vec * vec;
+    if (C > 1 && slice * (C - 1) >= V) continue;  // every CTA must own columns
+    const long long stage = (slice * es + 127) / 128 * 128;
+    if (2 * stage > budget) continue;
+    int S = static_cast<int>(budget / stage);
+    if (S > kMaxStages) S = kMaxStages;
+    if (forced_s) {
+      if (forced_s < 1 || forced_s > kMaxStages || forced_s * stage > budget) return RL_ERR_UNSUPPORTED;
+      S = forced_s;
+    }
+    out->C = C;
+    out->S = S;
+    out->slice = static_cast<int>(slice);
+    out->stage_bytes = static_cast<int>(stage);
+    out->smem = static_cast<int>(S * stage) + kSweepSmemExtra;
+    return RL_OK;
+  }
+  return RL_ERR_UNSUPPORTED;  // vocabulary too large for an 8-CTA cluster
+}
+
+struct Common {
+  const void* logits;
+  rl_dtype dt;
+  long long R, V, ld;
+  const int32_t* targets;
+  const uint8_t* mask;
+  const rl_loss_params* p;
+};
+
+rl_status check_common(const Common& c) {
+  if (!dtype_ok(c.dt)) return RL_ERR_INVALID_ARG;
+  if (c.R < 0 || c.V < 1 || c.V > INT_MAX / 8 || c.ld < c.V) return RL_ERR_INVALID_ARG;
+  if (c.R > 0 && (!c.logits || !c.targets || !c.mask)) return RL_ERR_INVALID_ARG;
+  return check_params(c.p);
+}
+
+struct FwdIn {
+  Common c;
+  const float *rho, *q, *old, *teacher, *rewards;
+  const int32_t *gid, *cu;
+  int n_traj, n_groups;
+  float *out_logp, *out_H, *out_adv;
+  int32_t* out_gsize;
+  rl_loss_stats* stats;
+  void* ws;
+  size_t ws_bytes;
+};
+
+rl_status check_fwd(const FwdIn& f) {
+  rl_status st = check_common(f.c);
+  if (st != RL_OK) return st;
+  const rl_loss_params* p = f.c.p;
+  if (f.n_traj < 0 || f.n_groups < 0) return RL_ERR_INVALID_ARG;
+  if (f.n_traj > 0 && (f.n_groups < 1 || !f.rewards || !f.gid)) return RL_ERR_INVALID_ARG;
+  if (!f.cu) return RL_ERR_INVALID_ARG;
+  if (f.c.R > 0 && !f.rho) return RL_ERR_INVALID_ARG;
+  if (f.c.R > 0 && p->kl_coef > 0.0f && !f.q) return RL_ERR_INVALID_ARG;
+  if (f.c.R > 0 && p->correction != RL_CORR_NONE && !f.old) return RL_ERR_INVALID_ARG;
+  if (f.c.R > 0 && p->opd_coef != 0.0f && !f.teacher) return RL_ERR_INVALID_ARG;
+  if (!f.ws || (reinterpret_cast<uintptr_t>(f.ws) & 255u)) return RL_ERR_INVALID_ARG;
+  size_t need = 0;
+  rl_loss_workspace_size(f.c.R, f.n_traj, f.n_groups, &need);
+  if (f.ws_bytes < need) return RL_ERR_WORKSPACE_TOO_SMALL;
+  return RL_OK;
+}
+
+struct GradOut {
+  float g;
+  const float* g_dev;
+  void* dl;
+  rl_dtype dt;
+  long long ld_out;
+};
+
+rl_status check_grad(const Common& c, const GradOut& o) {
+  if (!finite(o.g)) return RL_ERR_INVALID_ARG;
+  if (!dtype_ok(o.dt)) return RL_ERR_INVALID_ARG;
+  if (o.ld_out < c.V) return RL_ERR_INVALID_ARG;
+  if (c.R > 0 && !o.dl) return RL_ERR_INVALID_ARG;
+  return RL_OK;
+}
+
+void record(cudaEvent_t ev, cudaStream_t s) {
+  if (ev && t_ev_begin && t_ev_end) cudaEventRecord(ev, s);
+}
+
+rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return RL_ERR_CUDA;
+  const Common& c = f.c;
+  const WsLayout L = WsLayout::make(c.R, f.n_traj, f.n_groups);
+  const WsPtrs ws = WsPtrs::at(f.ws, L);
+
+  // advantages, N, validation
+  AdvArgs aa;
+  aa.R = c.R;
+  aa.n_traj = f.n_traj;
+  aa.n_groups = f.n_groups;
+  aa.rewards = f.rewards;
+  aa.gid = f.gid;
+  aa.cu = f.cu;
+  aa.mask = c.mask;
+  aa.rho = f.rho;
+  aa.teacher = (c.p->opd_coef != 0.0f) ? f.teacher : nullptr;
+  aa.opd_coef = c.p->opd_coef;
+  aa.normalize_std = c.p->normalize_std;
+  aa.unbiased_std = c.p->unbiased_std;
+  aa.std_floor = c.p->std_floor;
+  aa.advantages = f.out_adv;
+  aa.group_sizes = f.out_gsize;
+  aa.ws = ws;
+  rl_status st = launch(adv_kernel(), dim3(1), dim3(kAdvThreads), 0, 1, s, &aa);
+  if (st != RL_OK) return st;
+
+  if (c.R > 0) {
+    const bool grad = go != nullptr;
+    SweepPlan pl;
+    st = plan_sweep(c.dt, c.V, dev, &pl);
+    if (st != RL_OK) return st;
+    const void* fn = sweep_kernel(c.dt, grad ? go->dt : c.dt, grad);
+    st = set_smem(fn, dev, pl.smem);
+    if (st != RL_OK) return st;
+    int clusters = 0;
+    st = resident_clusters(fn, dev, pl.C, pl.smem, kSweepThreads, &clusters);
+    if (st != RL_OK) return st;
+    const long long n_cl = std::min<long long>(clusters, c.R);
+
+    SweepArgs sa;
+    sa.logits = c.logits;
+    sa.ld = c.ld;
+    sa.R = c.R;
+    sa.V = static_cast<int>(c.V);
+    sa.slice = pl.slice;
+    sa.stages = pl.S;
+    sa.stage_bytes = pl.stage_bytes;
+    const size_t es = elem_size(c.dt);
+    sa.in_bulk = aligned16(c.logits) && ((c.ld * es) % 16 == 0);
+    sa.out_vec = grad && aligned16(go->dl) && ((go->ld_out * elem_size(go->dt)) % 16 == 0);
+    sa.targets = c.targets;
+    sa.rho = f.rho;
+    sa.q = f.q;
+    sa.old = f.old;
+    sa.mask = c.mask;
+    sa.out_logp = f.out_logp;
+    sa.out_H = f.out_H;
+    sa.dlogits = grad ? go->dl : nullptr;
+    sa.ld_out = grad ? go->ld_out : 0;
+    sa.grad_loss = grad ? go->g : 0.0f;
+    sa.grad_loss_dev = grad ? go->g_dev : nullptr;
+    sa.s = scalars(c.p);
+    sa.ws = ws;
+    record(t_ev_begin, s);
+    st = launch(fn, dim3(static_cast<unsigned>(n_cl * pl.C)), dim3(kSweepThreads), pl.smem, pl.C,
+                s, &sa);
+    record(t_ev_end, s);
+    if (st != RL_OK) return st;
+  }
+
+  if (f.stats) {
+    StatArgs ta;
+    ta.R = c.R;
+    ta.mask = c.mask;
+    ta.rho = f.rho;
+    ta.out = f.stats;
+    ta.ws = ws;
+    long long blocks = (c.R + kStatThreads * 4 - 1) / (kStatThreads * 4);
+    blocks = std::max<long long>(1, std::min<long long>(blocks, kMaxStatBlocks));
+    st = launch(stats_kernel(), dim3(static_cast<unsigned>(blocks)), dim3(kStatThreads), 0, 1, s,
+                &ta);
+    if (st != RL_OK) return st;
+  }
+  return RL_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+rl_status rl_loss_workspace_size(int64_t n_rows, int32_t n_traj, int32_t n_groups, size_t* bytes) {
+  if (!bytes || n_rows < 0 || n_traj < 0 || n_groups < 0) return RL_ERR_INVALID_ARG;
+  *bytes = WsLayout::make(n_rows, n_traj, n_groups).total;
+  return RL_OK;
+}
+
+rl_status rl_loss_fwd(const void* logits, rl_dtype logits_dtype, int64_t n_rows, int64_t vocab,
+                      int64_t ld, const int32_t* targets, const float* rollout_logprobs,
+                      const float* ref_logprobs, const float* old_logprobs,
+                      const float* teacher_logprobs, const float* rewards,
+                      const int32_t* group_id, const int32_t* cu_seqlens, int32_t n_traj,
+                      int32_t n_groups, const uint8_t* loss_mask, const rl_loss_params* params,
+                      float* token_logprobs, float* entropy, float* advantages,
+                      int32_t* group_sizes, rl_loss_stats* stats, void* workspace,
+                      size_t workspace_bytes, rl_stream stream) {
+  FwdIn f{{logits, logits_dtype, n_rows, vocab, ld, targets, loss_mask, params},
+          rollout_logprobs, ref_logprobs, old_logprobs, teacher_logprobs, rewards,
+          group_id, cu_seqlens, n_traj, n_groups, token_logprobs, entropy, advantages,
+          group_sizes, stats, workspace, workspace_bytes};
+  rl_status st = check_fwd(f);
+  if (st != RL_OK) return st;
+  return run_fwd(f, nullptr, reinterpret_cast<cudaStream_t>(stream));
+}
+
+rl_status rl_loss_fwd_bwd(const void* logits, rl_dtype logits_dtype, int64_t n_rows,
+                          int64_t vocab, int64_t ld, const int32_t* targets,
+                          const float* rollout_logprobs, const float* ref_logprobs,
+                          const float* old_logprobs, const float* teacher_logprobs,
+                          const float* rewards, const int32_t* group_id,
+                          const int32_t* cu_seqlens, int32_t n_traj, int32_t n_groups,
+                          const uint8_t* loss_mask, const rl_loss_params* params,
+                          float* token_logprobs, float* entropy, float* advantages,
+                          int32_t* group_sizes, rl_loss_stats* stats, float grad_loss,
+                          const float* grad_loss_device, void* dlogits, rl_dtype dlogits_dtype,
+                          int64_t ld_out, void* workspace, size_t workspace_bytes,
+                          rl_stream stream) {
+  FwdIn f{{logits, logits_dtype, n_rows, vocab, ld, targets, loss_mask, params},
+          rollout_logprobs, ref_logprobs, old_logprobs, teacher_logprobs, rewards,
+          group_id, cu_seqlens, n_traj, n_groups, token_logprobs, entropy, advantages,
+          group_sizes, stats, workspace, workspace_bytes};
+  rl_status st = check_fwd(f);
+  if (st != RL_OK) return st;
+  GradOut go{grad_loss, grad_loss_device, dlogits, dlogits_dtype, ld_out};
+  st = check_grad(f.c, go);
+  if (st != RL_OK) return st;
+  return run_fwd(f, &go, reinterpret_cast<cudaStream_t>(stream));
+}
+
+rl_status rl_loss_bwd(const void* logits, rl_dtype logits_dtype, int64_t n_rows, int64_t vocab,
+                      int64_t ld, const int32_t* targets, const uint8_t* loss_mask,
+                      const rl_loss_params* params, float grad_loss,
+                      const float* grad_loss_device, const void* workspace,
+                      size_t workspace_bytes, void* dlogits, rl_dtype dlogits_dtype,
+                      int64_t ld_out, rl_stream stream) {
+  Common c{logits, logits_dtype, n_rows, vocab, ld, targets, loss_mask, params};
+  rl_status st = check_common(c);
+  if (st != RL_OK) return st;
+  GradOut go{grad_loss, grad_loss_device, dlogits, dlogits_dtype, ld_out};
+  st = check_grad(c, go);
+  if (st != RL_OK) return st;
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return RL_ERR_INVALID_ARG;
+  const WsLayout L = WsLayout::make(n_rows, 0, 0);
+  if (workspace_bytes < L.total) return RL_ERR_WORKSPACE_TOO_SMALL;
+  if (n_rows == 0) return RL_OK;
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return RL_ERR_CUDA;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return RL_ERR_CUDA;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  BwdArgs b;
+  b.logits = logits;
+  b.ld = ld;
+  b.R = n_rows;
+  b.V = static_cast<int>(vocab);
+  b.tiles_per_row = static_cast<int>((vocab + kBwdTile - 1) / kBwdTile);
+  b.n_tiles = n_rows * b.tiles_per_row;
+  b.in_vec = aligned16(logits) && ((ld * elem_size(logits_dtype)) % 16 == 0);
+  b.out_vec = aligned16(dlogits) && ((ld_out * elem_size(dlogits_dtype)) % 16 == 0);
+  b.targets = targets;
+  b.mask = loss_mask;
+  b.dlogits = dlogits;
+  b.ld_out = ld_out;
+  b.grad_loss = grad_loss;
+  b.grad_loss_dev = grad_loss_device;
+  b.invT = 1.0f / params->temperature;
+  b.k = 1.4426950408889634f / params->temperature;
+  b.gamma = params->entropy_coef;
+  b.ws = WsPtrs::at(const_cast<void*>(workspace), L);
+  const long long grid = std::min<long long>(b.n_tiles, static_cast<long long>(sms) * 8);
+  record(t_ev_begin, s);
+  st = launch(bwd_kernel(logits_dtype, dlogits_dtype), dim3(static_cast<unsigned>(grid)),
+              dim3(kBwdThreads), 0, 1, s, &b);
+  record(t_ev_end, s);
+  return st;
+}
+
+rl_status rl_loss_check_device_error(const void* workspace) {
+  if (!workspace) return RL_ERR_INVALID_ARG;
+  uint32_t bits = 0;
+  if (cudaMemcpy(&bits, workspace, sizeof(bits), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return RL_ERR_CUDA;
+  for (int code = RL_ERR_TARGET_OUT_OF_RANGE; code <= RL_ERR_DEVICE_TIMEOUT; ++code)
+    if (bits & (1u << code)) return static_cast<rl_status>(code);
+  return RL_OK;
+}
+
+const char* rl_status_string(rl_status status) {
+  switch (status) {
+    case RL_OK: return "ok";
+    case RL_ERR_INVALID_ARG: return "invalid argument";
+    case RL_ERR_UNSUPPORTED: return "unsupported configuration";
+    case RL_ERR_WORKSPACE_TOO_SMALL: return "workspace too small";
+    case RL_ERR_CUDA: return "CUDA runtime error";
+    case RL_ERR_TARGET_OUT_OF_RANGE: return "target id outside [0, vocab)";
+    case RL_ERR_GROUP_OUT_OF_RANGE: return "group id outside [0, n_groups)";
+    case RL_ERR_BAD_SEQLENS: return "cu_seqlens not non-decreasing from 0 to n_rows";
+    case RL_ERR_DEVICE_TIMEOUT: return "a bounded wait inside a kernel timed out";
+  }
+  return "unknown status";
+}
+
+rl_status rl_set_sweep_events(void* begin_event, void* end_event) {
+  t_ev_begin = static_cast<cudaEvent_t>(begin_event);
+  t_ev_end = static_cast<cudaEvent_t>(end_event);
+  return RL_OK;
+}
+
+int32_t rl_loss_abi_version(void) { return 100; }
+
+}  // extern "C"

@@ -1,0 +1,391 @@
+// Device helpers and the workspace layout shared by the kernels of
+// libmilesloss. sm_103a only: inline PTX for mbarrier, bulk async copies
+// (cp.async.bulk, non-multicast), thread-block-cluster barriers and
+// distributed shared memory.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "milesloss.h"
+
+namespace milesloss {
+
+// ------------------------------------------------------------------ errors
+// Data-dependent errors are recorded as bits (1 << status code) in the
+// workspace header; the host reports the lowest set code.
+enum : uint32_t {
+  kErrTarget = 1u << RL_ERR_TARGET_OUT_OF_RANGE,
+  kErrGroup = 1u << RL_ERR_GROUP_OUT_OF_RANGE,
+  kErrSeqlens = 1u << RL_ERR_BAD_SEQLENS,
+  kErrTimeout = 1u << RL_ERR_DEVICE_TIMEOUT,
+};
+
+// Per-row flag bits kept in the workspace.
+enum : uint8_t {
+  kFlagClipHi = 1, kFlagClipLo = 2, kFlagDual = 4, kFlagCorrClip = 8, kFlagBad = 16,
+};
+
+// --------------------------------------------------------------- workspace
+struct WsHeader {
+  uint32_t err_bits;   // OR of kErr* bits
+  uint32_t ticket;     // last-block counter of the statistics reduction
+  long long n_tokens;  // N = sum of the loss mask, written by the advantage kernel
+  uint32_t pad[60];
+};
+static_assert(sizeof(WsHeader) == 256, "header is one 256-byte segment");
+
+// Partial sums of one block of the statistics reduction.
+struct StatPart {
+  double s_ell, s_pg, s_k3, s_H, s_r, s_rabs, s_lpabs, s_rc, s_rcabs;
+  float rmin, rmax;
+  unsigned long long n, n_hi, n_lo, n_dual, n_corr;
+};
+
+constexpr int kStatThreads = 256;
+constexpr int kMaxStatBlocks = 256;  // one partial per thread of the final block
+
+struct WsLayout {
+  size_t hdr, g_mu, g_den, g_flag, a_traj, a_row;
+  size_t r_logp, r_H, r_lse, r_G, r_ell, r_pg, r_k3, r_r, r_rc, r_flags;
+  size_t parts, total;
+
+  __host__ __device__ static size_t up(size_t x) { return (x + 255) & ~size_t(255); }
+
+  // Per-row state first: its offsets depend on the row count only, so the
+  // backward call (which does not know the trajectory and group counts)
+  // finds it.
+  __host__ __device__ static WsLayout make(long long R, int n_traj, int n_groups) {
+    WsLayout L;
+    size_t o = 0;
+    L.hdr = o; o += up(sizeof(WsHeader));
+    L.a_row = o; o += up(sizeof(float) * (size_t)R);
+    size_t* rows[] = {&L.r_logp, &L.r_H, &L.r_lse, &L.r_G, &L.r_ell,
+                      &L.r_pg, &L.r_k3, &L.r_r, &L.r_rc};
+    for (size_t* p : rows) { *p = o; o += up(sizeof(float) * (size_t)R); }
+    L.r_flags = o; o += up((size_t)R);
+    L.parts = o; o += up(sizeof(StatPart) * kMaxStatBlocks);
+    L.g_mu = o; o += up(sizeof(double) * (size_t)n_groups);
+    L.g_den = o; o += up(sizeof(double) * (size_t)n_groups);
+    L.g_flag = o; o += up(sizeof(int) * (size_t)n_groups);
+    L.a_traj = o; o += up(sizeof(float) * (size_t)n_traj);
+    L.total = o;
+    return L;
+  }
+};
+
+// Pointers into one workspace.
+struct WsPtrs {
+  WsHeader* hdr;
+  double* g_mu;
+  double* g_den;
+  int* g_flag;
+  float* a_traj;
+  float* a_row;
+  float *logp, *H, *lse, *G, *ell, *pg, *k3, *r, *rc;
+  uint8_t* flags;
+  StatPart* parts;
+
+  static WsPtrs at(void* base, const WsLayout& L) {
+    char* b = static_cast<char*>(base);
+    WsPtrs p;
+    p.hdr = reinterpret_cast<WsHeader*>(b + L.hdr);
+    p.g_mu = reinterpret_cast<double*>(b + L.g_mu);
+    p.g_den = reinterpret_cast<double*>(b + L.g_den);
+    p.g_flag = reinterpret_cast<int*>(b + L.g_flag);
+    p.a_traj = reinterpret_cast<float*>(b + L.a_traj);
+    p.a_row = reinterpret_cast<float*>(b + L.a_row);
+    p.logp = reinterpret_cast<float*>(b + L.r_logp);
+    p.H = reinterpret_cast<float*>(b + L.r_H);
+    p.lse = reinterpret_cast<float*>(b + L.r_lse);
+    p.G = reinterpret_cast<float*>(b + L.r_G);
+    p.ell = reinterpret_cast<float*>(b + L.r_ell);
+    p.pg = reinterpret_cast<float*>(b + L.r_pg);
+    p.k3 = reinterpret_cast<float*>(b + L.r_k3);
+    p.r = reinterpret_cast<float*>(b + L.r_r);
+    p.rc = reinterpret_cast<float*>(b + L.r_rc);
+    p.flags = reinterpret_cast<uint8_t*>(b + L.r_flags);
+    p.parts = reinterpret_cast<StatPart*>(b + L.parts);
+    return p;
+  }
+};
+
+// Scalar parameters as the kernels use them.
+struct LossScalars {
+  float invT;      // 1 / T
+  float k;         // log2(e) / T: logits -> base-2 exponent units
+  float eps_lo, eps_hi, dual_c, beta, gamma, corr_lo, corr_hi;
+  int corr;        // rl_correction
+};
+
+// ------------------------------------------------------------------ PTX
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ float ex2(float x) {  // 2^x, flush-to-zero
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Waits for the phase with the given parity; gives up after ~limit_ns.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
+                                                  uint64_t limit_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t n = 1;; ++n) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((n & 63u) == 0 && globaltimer_ns() - t0 > limit_ns) return false;
+  }
+}
+
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+// Global -> own shared memory bulk copy (no multicast); completion is
+// signalled on the mbarrier as transaction bytes. dst, src 16-byte aligned;
+// bytes a multiple of 16.
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes,
+                                         uint32_t bar, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1], %2, [%3], %4;" ::"r"(dst),
+      "l"(src), "r"(bytes), "r"(bar), "l"(policy)
+      : "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ uint32_t cluster_nctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+
+__device__ __forceinline__ float4 ld_dsmem_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
+
+// Streaming 16-byte global load that does not allocate in L1.
+__device__ __forceinline__ uint4 ld_stream_u4(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+// Streaming (evict-first) stores.
+__device__ __forceinline__ void st_stream_u4(void* p, uint4 v) {
+  asm volatile("st.global.cs.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y),
+               "r"(v.z), "r"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ void st_stream_u2(void* p, uint2 v) {
+  asm volatile("st.global.cs.v2.u32 [%0], {%1, %2};" ::"l"(p), "r"(v.x), "r"(v.y) : "memory");
+}
+
+// ------------------------------------------------------------ dtype traits
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+struct InBf16 {
+  using storage = uint16_t;
+  static constexpr int kVec = 8;  // elements per 16 bytes
+  __device__ static __forceinline__ void unpack(uint4 w, float* f) {
+    f[0] = bf16_lo(w.x); f[1] = bf16_hi(w.x); f[2] = bf16_lo(w.y); f[3] = bf16_hi(w.y);
+    f[4] = bf16_lo(w.z); f[5] = bf16_hi(w.z); f[6] = bf16_lo(w.w); f[7] = bf16_hi(w.w);
+  }
+  __device__ static __forceinline__ float vmax(uint4 w) {
+    __nv_bfloat162 a = __hmax2(*reinterpret_cast<__nv_bfloat162*>(&w.x),
+                               *reinterpret_cast<__nv_bfloat162*>(&w.y));
+    __nv_bfloat162 b = __hmax2(*reinterpret_cast<__nv_bfloat162*>(&w.z),
+                               *reinterpret_cast<__nv_bfloat162*>(&w.w));
+    __nv_bfloat162 c = __hmax2(a, b);
+    uint32_t u = *reinterpret_cast<uint32_t*>(&c);
+    return fmaxf(bf16_lo(u), bf16_hi(u));
+  }
+  __device__ static __forceinline__ float load1(const void* base, long long i) {
+    uint16_t h = static_cast<const uint16_t*>(base)[i];
+    return __uint_as_float(static_cast<uint32_t>(h) << 16);
+  }
+};
+
+struct InF32 {
+  using storage = float;
+  static constexpr int kVec = 4;
+  __device__ static __forceinline__ void unpack(uint4 w, float* f) {
+    f[0] = __uint_as_float(w.x); f[1] = __uint_as_float(w.y);
+    f[2] = __uint_as_float(w.z); f[3] = __uint_as_float(w.w);
+  }
+  __device__ static __forceinline__ float vmax(uint4 w) {
+    return fmaxf(fmaxf(__uint_as_float(w.x), __uint_as_float(w.y)),
+                 fmaxf(__uint_as_float(w.z), __uint_as_float(w.w)));
+  }
+  __device__ static __forceinline__ float load1(const void* base, long long i) {
+    return static_cast<const float*>(base)[i];
+  }
+};
+
+struct OutBf16 {
+  static constexpr size_t kSize = 2;
+  __device__ static __forceinline__ void store1(void* base, long long i, float v) {
+    __nv_bfloat16 h = __float2bfloat16_rn(v);
+    static_cast<__nv_bfloat16*>(base)[i] = h;
+  }
+  // n = 8 or 4 values starting at an element offset aligned to n * 2 bytes;
+  // `sign` is XORed into every packed sign bit (0 or 0x80008000).
+  template <int n>
+  __device__ static __forceinline__ void storev(void* p, const float* f, uint32_t sign) {
+    if constexpr (n == 8) {
+      uint4 v = make_uint4(pack_bf16x2(f[0], f[1]) ^ sign, pack_bf16x2(f[2], f[3]) ^ sign,
+                           pack_bf16x2(f[4], f[5]) ^ sign, pack_bf16x2(f[6], f[7]) ^ sign);
+      st_stream_u4(p, v);
+    } else {
+      uint2 v = make_uint2(pack_bf16x2(f[0], f[1]) ^ sign, pack_bf16x2(f[2], f[3]) ^ sign);
+      st_stream_u2(p, v);
+    }
+  }
+  static constexpr uint32_t kSignMask = 0x80008000u;
+};
+
+struct OutF32 {
+  static constexpr size_t kSize = 4;
+  __device__ static __forceinline__ void store1(void* base, long long i, float v) {
+    static_cast<float*>(base)[i] = v;
+  }
+  template <int n>
+  __device__ static __forceinline__ void storev(void* p, const float* f, uint32_t sign) {
+    uint4 a = make_uint4(__float_as_uint(f[0]) ^ sign, __float_as_uint(f[1]) ^ sign,
+                         __float_as_uint(f[2]) ^ sign, __float_as_uint(f[3]) ^ sign);
+    st_stream_u4(p, a);
+    if constexpr (n == 8) {
+      uint4 b = make_uint4(__float_as_uint(f[4]) ^ sign, __float_as_uint(f[5]) ^ sign,
+                           __float_as_uint(f[6]) ^ sign, __float_as_uint(f[7]) ^ sign);
+      st_stream_u4(static_cast<char*>(p) + 16, b);
+    }
+  }
+  static constexpr uint32_t kSignMask = 0x80000000u;
+};
+
+// ------------------------------------------------- per-token objective
+// The per-row epilogue shared by the fused and forward-only sweeps: from
+// the row's log-prob and entropy, the token loss terms and G = dl/dlogp.
+struct TokenTerms {
+  float r, pg, k3, ell, G, rc;
+  uint8_t flags;
+};
+
+__device__ __forceinline__ TokenTerms token_terms(float logp, float H, float rho, float q,
+                                                  bool has_q, float old, bool has_old,
+                                                  float A, const LossScalars& s) {
+  TokenTerms t;
+  const float base = has_old ? old : rho;
+  const float r = expf(logp - base);
+  const float u = -A * r;
+  const float cl = fminf(fmaxf(r, 1.0f - s.eps_lo), 1.0f + s.eps_hi);
+  const float c = -A * cl;
+  const bool clipped = c > u;
+  float pg = clipped ? c : u;
+  uint8_t fl = 0;
+  if (clipped && r > 1.0f + s.eps_hi) fl |= kFlagClipHi;
+  if (clipped && r < 1.0f - s.eps_lo) fl |= kFlagClipLo;
+  bool dual = false;
+  if (s.dual_c > 0.0f && A < 0.0f) {
+    const float d = -A * s.dual_c;
+    if (d < pg) { pg = d; dual = true; fl |= kFlagDual; }
+  }
+  float gpg = (clipped || dual) ? 0.0f : -A * r;
+  float rc = 1.0f;
+  if (s.corr != RL_CORR_NONE) {
+    rc = expf(old - rho);
+    const bool outside = (rc < s.corr_lo) || (rc > s.corr_hi);
+    const float wt = (s.corr == RL_CORR_TIS) ? fminf(fmaxf(rc, s.corr_lo), s.corr_hi)
+                                             : (outside ? 0.0f : rc);
+    if (outside) fl |= kFlagCorrClip;
+    pg *= wt;
+    gpg *= wt;
+  }
+  float k3 = 0.0f, gkl = 0.0f;
+  if (has_q) {
+    const float dlt = q - logp;
+    const float ed = expf(dlt);
+    k3 = ed - dlt - 1.0f;
+    gkl = 1.0f - ed;
+  }
+  t.r = r;
+  t.pg = pg;
+  t.k3 = k3;
+  t.ell = pg + s.beta * k3 - s.gamma * H;
+  t.G = gpg + s.beta * gkl;
+  t.rc = rc;
+  t.flags = fl;
+  return t;
+}
+
+}  // namespace milesloss

@@ -1,0 +1,84 @@
+// dLogits from the per-row state a forward call saved (split forward /
+// backward path): the logits are read once more, row statistics come from
+// the workspace.
+//   dZ_tj = g (m_t / N) (1/T) [G_t (1[j = y_t] - p_j) + gamma p_j (log p_j + H_t)]
+// A tile is a contiguous run of kBwdTile columns of one row; blocks stride
+// over tiles. Loads are 16-byte streaming loads that skip L1, stores are
+// 16-byte streaming stores when the rows are aligned.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace milesloss {
+
+namespace {
+
+template <class In, class Out>
+__global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
+  constexpr int V8 = In::kVec;
+  using St = typename In::storage;
+  WsPtrs ws = a.ws;
+  const long long N = ws.hdr->n_tokens;
+  float g = a.grad_loss;
+  if (a.grad_loss_dev) g *= *a.grad_loss_dev;
+  const float cscale = (N > 0) ? g / static_cast<float>(N) * a.invT : 0.0f;
+
+  for (long long tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x) {
+    const long long row = tile / a.tiles_per_row;
+    const int j0 = static_cast<int>(tile % a.tiles_per_row) * kBwdTile;
+    const int j1 = min(a.V, j0 + kBwdTile);
+    const bool bad = (ws.flags[row] & kFlagBad) != 0;
+    const float cc = (a.mask[row] && !bad) ? cscale : 0.0f;
+    const float G = ws.G[row], H = ws.H[row], lse = ws.lse[row];
+    const float ca = cc * (-G + a.gamma * (H - lse));
+    const float cb = cc * a.gamma * a.invT;
+    const float L2 = lse * 1.4426950408889634f;
+    const char* zrow = static_cast<const char*>(a.logits) + row * a.ld * static_cast<long long>(sizeof(St));
+    char* drow = static_cast<char*>(a.dlogits) + row * a.ld_out * static_cast<long long>(Out::kSize);
+    const int y = a.targets[row];
+    const float add = cc * G;
+    auto value = [&](float z, int j) {
+      float x = (cc == 0.0f) ? 0.0f : ex2(fmaf(z, a.k, -L2)) * fmaf(cb, z, ca);
+      if (j == y) x += add;
+      return x;
+    };
+    if (a.in_vec && a.out_vec) {
+      // j0 is a multiple of V8 (kBwdTile is), so every vector is aligned.
+      const int nv = (j1 - j0) / V8;
+      for (int v = threadIdx.x; v < nv; v += kBwdThreads) {
+        const int jb = j0 + v * V8;
+        float f[V8];
+        In::unpack(ld_stream_u4(zrow + static_cast<size_t>(jb) * sizeof(St)), f);
+        if (cc == 0.0f) {
+#pragma unroll
+          for (int e = 0; e < V8; ++e) f[e] = 0.0f;
+        } else {
+#pragma unroll
+          for (int e = 0; e < V8; ++e) f[e] = ex2(fmaf(f[e], a.k, -L2)) * fmaf(cb, f[e], ca);
+          if (static_cast<unsigned>(y - jb) < static_cast<unsigned>(V8)) {
+#pragma unroll
+            for (int e = 0; e < V8; ++e)
+              if (jb + e == y) f[e] += add;
+          }
+        }
+        Out::template storev<V8>(drow + static_cast<size_t>(jb) * Out::kSize, f, 0u);
+      }
+      for (int j = j0 + nv * V8 + threadIdx.x; j < j1; j += kBwdThreads)
+        Out::store1(drow, j, value(In::load1(zrow, j), j));
+    } else {
+      for (int j = j0 + threadIdx.x; j < j1; j += kBwdThreads)
+        Out::store1(drow, j, value(In::load1(zrow, j), j));
+    }
+  }
+}
+
+}  // namespace
+
+const void* bwd_kernel(rl_dtype in, rl_dtype out) {
+  if (in == RL_BF16)
+    return out == RL_BF16 ? reinterpret_cast<const void*>(&k_bwd<InBf16, OutBf16>)
+                          : reinterpret_cast<const void*>(&k_bwd<InBf16, OutF32>);
+  return out == RL_BF16 ? reinterpret_cast<const void*>(&k_bwd<InF32, OutBf16>)
+                        : reinterpret_cast<const void*>(&k_bwd<InF32, OutF32>);
+}
+
+}  // namespace milesloss

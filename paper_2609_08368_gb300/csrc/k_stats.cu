@@ -1,0 +1,148 @@
+// The masked token-mean of the loss and the reported metrics: means over
+// training tokens of the PG term, k3, entropy, ratio, |r - 1|, |logp -
+// rollout logp| (the train/rollout divergence of Sec. 9.2) and the
+// correction ratio (Sec. 3.4), min / max ratio, and exact clip counts.
+//
+// Each block reduces a fixed strided set of rows into double-precision
+// partial sums (butterfly merges in a fixed order), stores them in the
+// workspace, and the last block to finish (an atomic ticket, no waiting)
+// merges the partials in block order. The grid size depends only on the row
+// count, so the scalar loss is bit-for-bit reproducible.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace milesloss {
+
+namespace {
+
+struct Part {
+  double v[9];  // ell, pg, k3, H, r, |r-1|, |logp-rho|, rc, |rc-1|
+  float rmin, rmax;
+  unsigned long long c[5];  // n, clip_hi, clip_lo, dual, corr_clip
+};
+
+__device__ __forceinline__ void part_zero(Part& p) {
+#pragma unroll
+  for (int i = 0; i < 9; ++i) p.v[i] = 0.0;
+  p.rmin = INFINITY;
+  p.rmax = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < 5; ++i) p.c[i] = 0ull;
+}
+
+__device__ __forceinline__ void part_merge_shfl(Part& p, int o) {
+#pragma unroll
+  for (int i = 0; i < 9; ++i) p.v[i] += __shfl_xor_sync(0xffffffffu, p.v[i], o);
+  p.rmin = fminf(p.rmin, __shfl_xor_sync(0xffffffffu, p.rmin, o));
+  p.rmax = fmaxf(p.rmax, __shfl_xor_sync(0xffffffffu, p.rmax, o));
+#pragma unroll
+  for (int i = 0; i < 5; ++i) p.c[i] += __shfl_xor_sync(0xffffffffu, p.c[i], o);
+}
+
+// Block reduction in a fixed order; the result is valid in thread 0.
+__device__ void block_reduce(Part& p, Part* sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  constexpr int kWarps = kStatThreads / 32;
+#pragma unroll 1
+  for (int o = 16; o > 0; o >>= 1) part_merge_shfl(p, o);
+  if (lane == 0) sh[warp] = p;
+  __syncthreads();
+  if (warp == 0) {
+    if (lane < kWarps) p = sh[lane]; else part_zero(p);
+#pragma unroll 1
+    for (int o = 16; o > 0; o >>= 1) part_merge_shfl(p, o);
+  }
+}
+
+__device__ __forceinline__ void to_stat(const Part& p, StatPart& s) {
+  s.s_ell = p.v[0]; s.s_pg = p.v[1]; s.s_k3 = p.v[2]; s.s_H = p.v[3]; s.s_r = p.v[4];
+  s.s_rabs = p.v[5]; s.s_lpabs = p.v[6]; s.s_rc = p.v[7]; s.s_rcabs = p.v[8];
+  s.rmin = p.rmin; s.rmax = p.rmax;
+  s.n = p.c[0]; s.n_hi = p.c[1]; s.n_lo = p.c[2]; s.n_dual = p.c[3]; s.n_corr = p.c[4];
+}
+
+__device__ __forceinline__ void from_stat(const StatPart* sp, Part& p) {
+  const double* d = reinterpret_cast<const double*>(sp);
+#pragma unroll
+  for (int i = 0; i < 9; ++i) p.v[i] = __ldcg(d + i);
+  p.rmin = __ldcg(&sp->rmin);
+  p.rmax = __ldcg(&sp->rmax);
+  const unsigned long long* c = &sp->n;
+#pragma unroll
+  for (int i = 0; i < 5; ++i) p.c[i] = __ldcg(c + i);
+}
+
+__global__ void __launch_bounds__(kStatThreads) k_stats(const StatArgs a) {
+  __shared__ Part sh[kStatThreads / 32];
+  __shared__ int s_last;
+  WsPtrs ws = a.ws;
+  Part p;
+  part_zero(p);
+  const long long stride = static_cast<long long>(gridDim.x) * kStatThreads;
+  for (long long t = blockIdx.x * static_cast<long long>(kStatThreads) + threadIdx.x; t < a.R;
+       t += stride) {
+    if (!a.mask[t]) continue;
+    const uint8_t f = ws.flags[t];
+    const float r = ws.r[t], rc = ws.rc[t];
+    p.v[0] += ws.ell[t];
+    p.v[1] += ws.pg[t];
+    p.v[2] += ws.k3[t];
+    p.v[3] += ws.H[t];
+    p.v[4] += r;
+    p.v[5] += fabs(static_cast<double>(r) - 1.0);
+    p.v[6] += fabs(static_cast<double>(ws.logp[t]) - static_cast<double>(a.rho[t]));
+    p.v[7] += rc;
+    p.v[8] += fabs(static_cast<double>(rc) - 1.0);
+    p.rmin = fminf(p.rmin, r);
+    p.rmax = fmaxf(p.rmax, r);
+    p.c[0] += 1;
+    p.c[1] += (f & kFlagClipHi) ? 1 : 0;
+    p.c[2] += (f & kFlagClipLo) ? 1 : 0;
+    p.c[3] += (f & kFlagDual) ? 1 : 0;
+    p.c[4] += (f & kFlagCorrClip) ? 1 : 0;
+  }
+  block_reduce(p, sh);
+  if (threadIdx.x == 0) {
+    to_stat(p, ws.parts[blockIdx.x]);
+    __threadfence();
+    const unsigned int ticket = atomicAdd(&ws.hdr->ticket, 1u);
+    s_last = (ticket == gridDim.x - 1) ? 1 : 0;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+
+  // Last block: merge the partials in block order.
+  if (static_cast<int>(threadIdx.x) < static_cast<int>(gridDim.x)) from_stat(&ws.parts[threadIdx.x], p);
+  else part_zero(p);
+  block_reduce(p, sh);
+  if (threadIdx.x == 0) {
+    rl_loss_stats o;
+    const unsigned long long n = p.c[0];
+    const double inv = n ? 1.0 / static_cast<double>(n) : 0.0;
+    o.loss = p.v[0] * inv;
+    o.pg_loss_mean = p.v[1] * inv;
+    o.kl_mean = p.v[2] * inv;
+    o.entropy_mean = p.v[3] * inv;
+    o.ratio_mean = p.v[4] * inv;
+    o.ratio_absdev_mean = p.v[5] * inv;
+    o.logprob_absdiff_mean = p.v[6] * inv;
+    o.corr_ratio_mean = p.v[7] * inv;
+    o.corr_absdev_mean = p.v[8] * inv;
+    o.ratio_min = n ? p.rmin : 0.0f;
+    o.ratio_max = n ? p.rmax : 0.0f;
+    o.n_tokens = static_cast<int64_t>(n);
+    o.n_clip_hi = static_cast<int64_t>(p.c[1]);
+    o.n_clip_lo = static_cast<int64_t>(p.c[2]);
+    o.n_dual_clip = static_cast<int64_t>(p.c[3]);
+    o.n_corr_clip = static_cast<int64_t>(p.c[4]);
+    *a.out = o;
+    ws.hdr->ticket = 0;
+  }
+}
+
+}  // namespace
+
+const void* stats_kernel() { return reinterpret_cast<const void*>(&k_stats); }
+
+}  // namespace milesloss

@@ -1,0 +1,89 @@
+// Internal interface between the C-ABI layer (abi.cu) and the kernels.
+#pragma once
+
+#include "common.cuh"
+
+namespace milesloss {
+
+constexpr int kSweepThreads = 512;
+constexpr int kMaxStages = 4;
+constexpr uint32_t kBulkChunk = 16384;    // bytes per cp.async.bulk
+constexpr int kSweepSmemExtra = 1024;     // mbarriers + exchange + reduction scratch
+constexpr int kAdvThreads = 1024;
+constexpr int kBwdThreads = 256;
+
+struct SweepArgs {
+  const void* logits;
+  long long ld, R;
+  int V;
+  int slice;        // columns per CTA (multiple of 16 bytes of input)
+  int stages;       // ring depth S
+  int stage_bytes;  // bytes per stage (multiple of 128)
+  int in_bulk;      // rows are 16-byte aligned: bulk-copy path
+  int out_vec;      // dLogits rows are 16-byte aligned: vector stores
+  const int* targets;
+  const float* rho;
+  const float* q;
+  const float* old;
+  const uint8_t* mask;
+  float* out_logp;
+  float* out_H;
+  void* dlogits;
+  long long ld_out;
+  float grad_loss;
+  const float* grad_loss_dev;
+  LossScalars s;
+  WsPtrs ws;
+};
+
+struct AdvArgs {
+  long long R;
+  int n_traj, n_groups;
+  const float* rewards;
+  const int* gid;
+  const int* cu;
+  const uint8_t* mask;
+  const float* rho;
+  const float* teacher;
+  float opd_coef;
+  int normalize_std, unbiased_std;
+  float std_floor;
+  float* advantages;   // may be null
+  int* group_sizes;    // may be null
+  WsPtrs ws;
+};
+
+struct StatArgs {
+  long long R;
+  const uint8_t* mask;
+  const float* rho;
+  rl_loss_stats* out;
+  WsPtrs ws;
+};
+
+struct BwdArgs {
+  const void* logits;
+  long long ld, R;
+  int V;
+  int tiles_per_row;
+  long long n_tiles;
+  int in_vec, out_vec;
+  const int* targets;
+  const uint8_t* mask;
+  void* dlogits;
+  long long ld_out;
+  float grad_loss;
+  const float* grad_loss_dev;
+  float invT, k, gamma;
+  WsPtrs ws;
+};
+
+constexpr int kBwdTile = kBwdThreads * 8 * 4;  // elements of one row per tile
+
+// Kernel entry points (device function pointers usable with cudaLaunchKernelEx).
+const void* sweep_kernel(rl_dtype in, rl_dtype out, bool grad);
+const void* bwd_kernel(rl_dtype in, rl_dtype out);
+const void* adv_kernel();
+const void* stats_kernel();
+
+}  // namespace milesloss

@@ -1,0 +1,202 @@
+"""Thin Python binding of libmilesloss (ctypes).
+
+Argument marshalling only: every step of the loss runs in the CUDA library.
+torch.Tensors go in by ``data_ptr()`` and calls are enqueued on the current
+torch CUDA stream. There is no fallback: if the library is missing the
+import of this module's functions fails loudly.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import struct
+
+from . import build as _build
+
+RL_OK = 0
+RL_BF16, RL_F32 = 0, 1
+CORRECTIONS = {"none": 0, "tis": 1, "clip_or_pop": 2}
+STATS_BYTES = 128
+
+
+class RlLossParams(ctypes.Structure):
+    _fields_ = [
+        ("temperature", ctypes.c_float),
+        ("eps_lo", ctypes.c_float),
+        ("eps_hi", ctypes.c_float),
+        ("dual_clip_c", ctypes.c_float),
+        ("kl_coef", ctypes.c_float),
+        ("entropy_coef", ctypes.c_float),
+        ("std_floor", ctypes.c_float),
+        ("normalize_std", ctypes.c_int32),
+        ("unbiased_std", ctypes.c_int32),
+        ("correction", ctypes.c_int32),
+        ("corr_lo", ctypes.c_float),
+        ("corr_hi", ctypes.c_float),
+        ("opd_coef", ctypes.c_float),
+    ]
+
+
+def make_params(temperature=1.0, eps_lo=0.2, eps_hi=0.2, dual_clip_c=0.0, kl_coef=0.0,
+                entropy_coef=0.0, std_floor=1e-6, normalize_std=True, unbiased_std=True,
+                correction="none", corr_lo=0.0, corr_hi=2.0, opd_coef=0.0) -> RlLossParams:
+    return RlLossParams(temperature, eps_lo, eps_hi, dual_clip_c, kl_coef, entropy_coef,
+                        std_floor, int(bool(normalize_std)), int(bool(unbiased_std)),
+                        CORRECTIONS[correction] if isinstance(correction, str) else int(correction),
+                        corr_lo, corr_hi, opd_coef)
+
+
+class MilesLossError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        super().__init__(f"{where}: {status_string(status)} (status {status})")
+        self.status = status
+
+
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = True) -> ctypes.CDLL:
+    """Load libmilesloss.so (building it first if it is missing)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.LIB
+    if not os.path.exists(path):
+        if not build_if_missing:
+            raise RuntimeError(f"libmilesloss is not built ({path}); run build()")
+        _build.build()
+    lib = ctypes.CDLL(path)
+    P, I64, I32, F32, SZ = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_float,
+                            ctypes.c_size_t)
+    PP = ctypes.POINTER(RlLossParams)
+    lib.rl_loss_workspace_size.argtypes = [I64, I32, I32, ctypes.POINTER(SZ)]
+    fwd_common = [P, I32, I64, I64, I64, P, P, P, P, P, P, P, P, I32, I32, P, PP, P, P, P, P, P]
+    lib.rl_loss_fwd.argtypes = fwd_common + [P, SZ, P]
+    lib.rl_loss_fwd_bwd.argtypes = fwd_common + [F32, P, P, I32, I64, P, SZ, P]
+    lib.rl_loss_bwd.argtypes = [P, I32, I64, I64, I64, P, P, PP, F32, P, P, SZ, P, I32, I64, P]
+    lib.rl_loss_check_device_error.argtypes = [P]
+    lib.rl_status_string.argtypes = [I32]
+    lib.rl_status_string.restype = ctypes.c_char_p
+    lib.rl_set_sweep_events.argtypes = [P, P]
+    for name in ("rl_loss_workspace_size", "rl_loss_fwd", "rl_loss_fwd_bwd", "rl_loss_bwd",
+                 "rl_loss_check_device_error", "rl_set_sweep_events", "rl_loss_abi_version"):
+        getattr(lib, name).restype = ctypes.c_int32
+    _lib = lib
+    return lib
+
+
+def status_string(status: int) -> str:
+    return load().rl_status_string(int(status)).decode()
+
+
+def _check(status: int, where: str):
+    if status != RL_OK:
+        raise MilesLossError(status, where)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _dtype_code(t) -> int:
+    import torch
+    if t.dtype == torch.bfloat16:
+        return RL_BF16
+    if t.dtype == torch.float32:
+        return RL_F32
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _stream(stream):
+    import torch
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def rl_loss_workspace_size(n_rows: int, n_traj: int, n_groups: int) -> int:
+    out = ctypes.c_size_t(0)
+    _check(load().rl_loss_workspace_size(n_rows, n_traj, n_groups, ctypes.byref(out)),
+           "rl_loss_workspace_size")
+    return int(out.value)
+
+
+def _params(p) -> RlLossParams:
+    if isinstance(p, RlLossParams):
+        return p
+    return make_params(**(p or {}))
+
+
+def _fwd_args(logits, vocab, targets, rollout_logprobs, ref_logprobs, old_logprobs,
+              teacher_logprobs, rewards, group_id, cu_seqlens, n_groups, loss_mask, params,
+              token_logprobs, entropy, advantages, group_sizes, stats):
+    n_rows = int(logits.shape[0])
+    V = int(logits.shape[1]) if vocab is None else int(vocab)
+    n_traj = int(rewards.shape[0]) if rewards is not None else 0
+    return [_ptr(logits), _dtype_code(logits), n_rows, V, int(logits.stride(0)), _ptr(targets),
+            _ptr(rollout_logprobs), _ptr(ref_logprobs), _ptr(old_logprobs),
+            _ptr(teacher_logprobs), _ptr(rewards), _ptr(group_id), _ptr(cu_seqlens), n_traj,
+            int(n_groups), _ptr(loss_mask), ctypes.byref(_params(params)), _ptr(token_logprobs),
+            _ptr(entropy), _ptr(advantages), _ptr(group_sizes), _ptr(stats)]
+
+
+def rl_loss_fwd(logits, targets, rollout_logprobs, ref_logprobs, old_logprobs, teacher_logprobs,
+                rewards, group_id, cu_seqlens, n_groups, loss_mask, params, token_logprobs,
+                entropy, advantages, group_sizes, stats, workspace, vocab=None, stream=None):
+    args = _fwd_args(logits, vocab, targets, rollout_logprobs, ref_logprobs, old_logprobs,
+                     teacher_logprobs, rewards, group_id, cu_seqlens, n_groups, loss_mask, params,
+                     token_logprobs, entropy, advantages, group_sizes, stats)
+    _check(load().rl_loss_fwd(*args, _ptr(workspace), workspace.numel() * workspace.element_size(),
+                              _stream(stream)), "rl_loss_fwd")
+
+
+def rl_loss_fwd_bwd(logits, targets, rollout_logprobs, ref_logprobs, old_logprobs,
+                    teacher_logprobs, rewards, group_id, cu_seqlens, n_groups, loss_mask, params,
+                    token_logprobs, entropy, advantages, group_sizes, stats, dlogits, workspace,
+                    grad_loss=1.0, grad_loss_device=None, vocab=None, stream=None):
+    args = _fwd_args(logits, vocab, targets, rollout_logprobs, ref_logprobs, old_logprobs,
+                     teacher_logprobs, rewards, group_id, cu_seqlens, n_groups, loss_mask, params,
+                     token_logprobs, entropy, advantages, group_sizes, stats)
+    _check(load().rl_loss_fwd_bwd(*args, float(grad_loss), _ptr(grad_loss_device), _ptr(dlogits),
+                                  _dtype_code(dlogits), int(dlogits.stride(0)), _ptr(workspace),
+                                  workspace.numel() * workspace.element_size(), _stream(stream)),
+           "rl_loss_fwd_bwd")
+
+
+def rl_loss_bwd(logits, targets, loss_mask, params, workspace, dlogits, grad_loss=1.0,
+                grad_loss_device=None, vocab=None, stream=None):
+    V = int(logits.shape[1]) if vocab is None else int(vocab)
+    _check(load().rl_loss_bwd(_ptr(logits), _dtype_code(logits), int(logits.shape[0]), V,
+                              int(logits.stride(0)), _ptr(targets), _ptr(loss_mask),
+                              ctypes.byref(_params(params)), float(grad_loss),
+                              _ptr(grad_loss_device), _ptr(workspace),
+                              workspace.numel() * workspace.element_size(), _ptr(dlogits),
+                              _dtype_code(dlogits), int(dlogits.stride(0)), _stream(stream)),
+           "rl_loss_bwd")
+
+
+def rl_loss_check_device_error(workspace) -> int:
+    return int(load().rl_loss_check_device_error(_ptr(workspace)))
+
+
+def rl_set_sweep_events(begin=None, end=None):
+    _check(load().rl_set_sweep_events(None if begin is None else ctypes.c_void_p(begin.cuda_event),
+                                      None if end is None else ctypes.c_void_p(end.cuda_event)),
+           "rl_set_sweep_events")
+
+
+_STATS_FMT = "<9d2f5q"
+STATS_FIELDS = ("loss", "pg_loss_mean", "kl_mean", "entropy_mean", "ratio_mean",
+                "ratio_absdev_mean", "logprob_absdiff_mean", "corr_ratio_mean",
+                "corr_absdev_mean", "ratio_min", "ratio_max", "n_tokens", "n_clip_hi",
+                "n_clip_lo", "n_dual_clip", "n_corr_clip")
+assert struct.calcsize(_STATS_FMT) == 120
+
+
+def parse_stats(raw: bytes) -> dict:
+    """Decode one rl_loss_stats (bytes copied back from the device)."""
+    return dict(zip(STATS_FIELDS, struct.unpack(_STATS_FMT, bytes(raw)[:120])))

@@ -1,0 +1,143 @@
+"""Helpers of the GPU parity tests: run the CUDA library on a seeded
+workload, run the float64 oracle on the same inputs (copied to the host),
+and compare with the tolerances of the target:
+  token log-probs / entropy   2e-3 absolute for bf16 logits, 1e-5 for fp32
+  scalar loss                 1e-4 relative
+  dLogits                     1e-2 relative or 1e-5 absolute
+  integer outputs             exact (clip counts: exact outside a 1e-5
+                              relative guard band around each threshold)
+"""
+
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle
+from paper_2609_08368_gb300 import api
+from paper_2609_08368_gb300 import milesloss as ml
+
+GUARD = 1e-5
+
+
+def oracle_params(params: dict) -> oracle.LossParams:
+    return oracle.LossParams(**params)
+
+
+def host_logits(w, rows=None) -> np.ndarray:
+    z = w.logits[:, :w.vocab] if rows is None else w.logits[rows, :w.vocab]
+    z = z.cpu()
+    if z.dtype == torch.bfloat16:
+        return z.contiguous().view(torch.int16).numpy().view(np.uint16)
+    return z.numpy()
+
+
+def np_(t):
+    return None if t is None else t.cpu().numpy()
+
+
+def run_gpu(w, mode="fused", dl_dtype=None, grad_loss=1.0, ld_out=None, params=None):
+    """mode: 'fused' (rl_loss_fwd_bwd), 'split' (rl_loss_fwd then rl_loss_bwd)
+    or 'fwd' (rl_loss_fwd only)."""
+    R, n_traj = w.n_rows, int(w.rewards.shape[0])
+    if dl_dtype is None:
+        dl_dtype = w.logits.dtype
+    buf = api.alloc(R, n_traj, w.n_groups, w.logits.device, vocab=w.vocab,
+                    dlogits_dtype=None if mode == "fwd" else dl_dtype, ld_out=ld_out,
+                    fill_nan=True)
+    if mode == "fused":
+        api.fwd_bwd(w, buf, params=params, grad_loss=grad_loss)
+    else:
+        api.fwd(w, buf, params=params)
+        if mode == "split":
+            api.bwd(w, buf, params=params, grad_loss=grad_loss)
+    torch.cuda.synchronize()
+    out = dict(logp=np_(buf.token_logprobs), H=np_(buf.entropy), A=np_(buf.advantages),
+               group_sizes=np_(buf.group_sizes), stats=buf.read_stats(),
+               err=ml.rl_loss_check_device_error(buf.workspace), buf=buf)
+    if buf.dlogits is not None:
+        out["dlogits_t"] = buf.dlogits
+    return out
+
+
+def run_oracle(w, grad_loss=1.0, want_dlogits=True, params=None):
+    p = oracle_params(params if params is not None else w.params)
+    return oracle.rl_loss(host_logits(w), np_(w.targets), np_(w.rollout_logprobs),
+                          np_(w.ref_logprobs), np_(w.rewards), np_(w.group_id),
+                          np_(w.cu_seqlens), w.n_groups, np_(w.loss_mask), p,
+                          grad_loss=grad_loss, old=np_(w.old_logprobs),
+                          teacher=np_(w.teacher_logprobs), want_dlogits=want_dlogits)
+
+
+def logp_tol(w) -> float:
+    return 2e-3 if w.logits.dtype == torch.bfloat16 else 1e-5
+
+
+def assert_dlogits_close(got: np.ndarray, ref: np.ndarray, rel=1e-2, abs_=1e-5):
+    got = got.astype(np.float64)
+    err = np.abs(got - ref)
+    bound = np.maximum(rel * np.abs(ref), abs_)
+    bad = err > bound
+    assert np.isfinite(got).all(), "non-finite dLogits"
+    if bad.any():
+        i = np.argwhere(bad)[0]
+        raise AssertionError(f"dLogits mismatch at {tuple(i)}: got {got[tuple(i)]!r} "
+                             f"ref {ref[tuple(i)]!r} ({int(bad.sum())} entries)")
+
+
+def assert_rel_on_large(got: np.ndarray, ref: np.ndarray, floor=1e-6, rel=1e-2):
+    """Relative error on every entry with |ref| >= floor (entries of O(p))."""
+    got = got.astype(np.float64)
+    sel = np.abs(ref) >= floor
+    err = np.abs(got[sel] - ref[sel]) / np.abs(ref[sel])
+    assert sel.any()
+    assert err.max() <= rel, f"max rel err {err.max():.3g} on {int(sel.sum())} entries"
+
+
+def clip_counts(p: oracle.LossParams, logp, rho, q, A_row, H, mask, old=None):
+    """Clip counts of the oracle's decision rule applied to given log-probs,
+    and the number of training tokens within the guard band of a threshold."""
+    o = oracle.token_objective(logp, rho, q, A_row, H, p, old=old)
+    m = np.asarray(mask).astype(bool)
+    th = [1 - p.eps_lo, 1 + p.eps_hi] + ([p.dual_clip_c] if p.dual_clip_c else [])
+    near = np.zeros_like(m)
+    for t in th:
+        near |= np.abs(o["r"] - t) <= GUARD * t
+    if p.correction != "none":
+        for t in (p.corr_lo, p.corr_hi):
+            near |= np.abs(o["rc"] - t) <= GUARD * max(t, 1e-30)
+    counts = dict(n_clip_hi=int(o["clip_hi"][m].sum()), n_clip_lo=int(o["clip_lo"][m].sum()),
+                  n_dual_clip=int(o["dual"][m].sum()), n_corr_clip=int(o["corr_clip"][m].sum()))
+    return counts, int((near & m).sum())
+
+
+def compare_forward(w, g, o, params=None):
+    """Per-row outputs, advantages, group sizes, counts and the loss."""
+    p = oracle_params(params if params is not None else w.params)
+    tol = logp_tol(w)
+    np.testing.assert_allclose(g["logp"], o["logp"], atol=tol, rtol=0)
+    np.testing.assert_allclose(g["H"], o["H"], atol=tol, rtol=0)
+    np.testing.assert_allclose(g["A"], o["A_traj"], rtol=1e-6, atol=1e-6)
+    np.testing.assert_array_equal(g["group_sizes"], o["group_sizes"])
+    st = g["stats"]
+    assert st["n_tokens"] == o["N"]
+    # clip counts: the oracle's rule on the GPU's own log-probs reproduces the
+    # GPU counts exactly (up to tokens in the guard band); against the
+    # oracle's float64 log-probs they differ only inside the band.
+    old = np_(w.old_logprobs)
+    c_gpu, band_g = clip_counts(p, g["logp"].astype(np.float64), np_(w.rollout_logprobs),
+                                np_(w.ref_logprobs), o["A_row"], g["H"], np_(w.loss_mask), old)
+    c_ora, band_o = clip_counts(p, o["logp"], np_(w.rollout_logprobs), np_(w.ref_logprobs),
+                                o["A_row"], o["H"], np_(w.loss_mask), old)
+    for k in c_gpu:
+        assert abs(st[k] - c_gpu[k]) <= band_g, (k, st[k], c_gpu[k], band_g)
+        assert abs(st[k] - c_ora[k]) <= band_g + band_o, (k, st[k], c_ora[k])
+    os_ = o["stats"]
+    scale = max(abs(os_["loss"]), float(np.abs(o["ell"][np_(w.loss_mask).astype(bool)]).mean())
+                if o["N"] else 0.0)
+    assert abs(st["loss"] - os_["loss"]) <= 1e-4 * max(scale, 1e-30), (st["loss"], os_["loss"])
+    for k in ("ratio_mean", "ratio_absdev_mean", "logprob_absdiff_mean", "entropy_mean",
+              "kl_mean", "pg_loss_mean", "corr_ratio_mean", "corr_absdev_mean"):
+        assert abs(st[k] - os_[k]) <= 1e-4 * max(abs(os_[k]), 1e-3), (k, st[k], os_[k])
+    for k in ("ratio_min", "ratio_max"):
+        assert abs(st[k] - os_[k]) <= 1e-4 * max(abs(os_[k]), 1e-3), (k, st[k], os_[k])

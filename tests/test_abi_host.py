@@ -1,0 +1,164 @@
+"""Host-side checks of the C ABI that need no GPU: the library builds for
+sm_103a and loads, exports every entry point include/milesloss.h declares,
+sizes workspaces, names its status codes, and rejects every invalid
+argument before enqueuing anything."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2609_08368_gb300 import milesloss as ml
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "milesloss.h")
+
+RL_ERR_INVALID_ARG = 1
+RL_ERR_WORKSPACE_TOO_SMALL = 3
+
+
+@pytest.fixture(scope="module")
+def lib():
+    return ml.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(rl_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for want in ("rl_loss_fwd", "rl_loss_bwd", "rl_loss_fwd_bwd", "rl_loss_workspace_size",
+                 "rl_loss_check_device_error", "rl_status_string"):
+        assert want in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_abi_version_and_status_strings(lib):
+    assert lib.rl_loss_abi_version() == 100
+    seen = set()
+    for code in range(0, 9):
+        s = ml.status_string(code)
+        assert s and s != "unknown status"
+        seen.add(s)
+    assert len(seen) == 9
+    assert ml.status_string(99) == "unknown status"
+
+
+def test_workspace_size(lib):
+    a = ml.rl_loss_workspace_size(0, 0, 0)
+    b = ml.rl_loss_workspace_size(65536, 64, 4)
+    c = ml.rl_loss_workspace_size(131072, 64, 4)
+    assert 0 < a < b < c
+    assert b % 256 == 0
+    # roughly 41 bytes of per-row state
+    assert 40 * 65536 < b - a < 48 * 65536
+    out = ctypes.c_size_t()
+    assert lib.rl_loss_workspace_size(-1, 0, 0, ctypes.byref(out)) == RL_ERR_INVALID_ARG
+    assert lib.rl_loss_workspace_size(1, 0, 0, None) == RL_ERR_INVALID_ARG
+
+
+FAKE = 1 << 20  # never dereferenced: every case below fails validation first
+
+
+def _fwd_bwd_args(**over):
+    p = ml.make_params(**over.pop("params", {}))
+    a = dict(logits=FAKE, dt=ml.RL_BF16, R=16, V=64, ld=64, targets=FAKE, rho=FAKE, q=None,
+             old=None, teacher=None, rewards=FAKE, gid=FAKE, cu=FAKE, n_traj=2, n_groups=1,
+             mask=FAKE, params=p, logp=FAKE, H=FAKE, adv=FAKE, gs=FAKE, stats=FAKE, g=1.0,
+             gdev=None, dl=FAKE, dl_dt=ml.RL_BF16, ld_out=64, ws=FAKE * 2, ws_bytes=1 << 30)
+    a.update(over)
+    return a
+
+
+def _call_fwd_bwd(lib, a):
+    v = ctypes.c_void_p
+    return lib.rl_loss_fwd_bwd(
+        v(a["logits"]), a["dt"], a["R"], a["V"], a["ld"], v(a["targets"]), v(a["rho"]),
+        v(a["q"]), v(a["old"]), v(a["teacher"]), v(a["rewards"]), v(a["gid"]), v(a["cu"]),
+        a["n_traj"], a["n_groups"], v(a["mask"]), ctypes.byref(a["params"]), v(a["logp"]),
+        v(a["H"]), v(a["adv"]), v(a["gs"]), v(a["stats"]), a["g"], v(a["gdev"]), v(a["dl"]),
+        a["dl_dt"], a["ld_out"], v(a["ws"]), a["ws_bytes"], None)
+
+
+INVALID = [
+    dict(logits=None),
+    dict(targets=None),
+    dict(rho=None),
+    dict(mask=None),
+    dict(cu=None),
+    dict(rewards=None),
+    dict(gid=None),
+    dict(dl=None),
+    dict(dt=7),
+    dict(dl_dt=5),
+    dict(V=0),
+    dict(R=-1),
+    dict(ld=63),
+    dict(ld_out=10),
+    dict(n_traj=-1),
+    dict(n_groups=0),
+    dict(g=float("inf")),
+    dict(ws=FAKE * 2 + 8),
+    dict(ws=None),
+    dict(params=dict(temperature=0.0)),
+    dict(params=dict(temperature=float("nan"))),
+    dict(params=dict(eps_lo=-0.1)),
+    dict(params=dict(eps_hi=float("inf"))),
+    dict(params=dict(dual_clip_c=1.0)),
+    dict(params=dict(dual_clip_c=-2.0)),
+    dict(params=dict(kl_coef=0.1)),                    # no ref log-probs
+    dict(params=dict(kl_coef=-0.1), q=FAKE),
+    dict(params=dict(entropy_coef=-1.0)),
+    dict(params=dict(std_floor=0.0)),
+    dict(params=dict(correction="tis")),               # no old log-probs
+    dict(params=dict(correction="tis", corr_lo=3.0, corr_hi=2.0), old=FAKE),
+    dict(params=dict(correction=5), old=FAKE),
+    dict(params=dict(opd_coef=0.5)),                   # no teacher log-probs
+    dict(params=dict(opd_coef=float("nan")), teacher=FAKE),
+]
+
+
+@pytest.mark.parametrize("over", INVALID, ids=[str(i) for i in range(len(INVALID))])
+def test_invalid_arguments_are_rejected_on_the_host(lib, over):
+    params = over.pop("params", None)
+    a = _fwd_bwd_args(**({"params": params} if params else {}), **over)
+    assert _call_fwd_bwd(lib, a) == RL_ERR_INVALID_ARG
+
+
+def test_workspace_too_small_is_rejected(lib):
+    need = ml.rl_loss_workspace_size(16, 2, 1)
+    a = _fwd_bwd_args(ws_bytes=need - 1)
+    assert _call_fwd_bwd(lib, a) == RL_ERR_WORKSPACE_TOO_SMALL
+
+
+def test_bwd_and_fwd_validate_too(lib):
+    v = ctypes.c_void_p
+    p = ml.make_params()
+    # ld < vocab
+    assert lib.rl_loss_bwd(v(FAKE), 0, 4, 64, 32, v(FAKE), v(FAKE), ctypes.byref(p), 1.0, None,
+                           v(FAKE * 2), 1 << 30, v(FAKE), 0, 64, None) == RL_ERR_INVALID_ARG
+    # workspace too small for the rows
+    assert lib.rl_loss_bwd(v(FAKE), 0, 4096, 64, 64, v(FAKE), v(FAKE), ctypes.byref(p), 1.0, None,
+                           v(FAKE * 2), 1024, v(FAKE), 0, 64, None) == RL_ERR_WORKSPACE_TOO_SMALL
+    # fwd without rollout log-probs
+    assert lib.rl_loss_fwd(v(FAKE), 0, 4, 64, 64, v(FAKE), None, None, None, None, v(FAKE),
+                           v(FAKE), v(FAKE), 1, 1, v(FAKE), ctypes.byref(p), None, None, None,
+                           None, None, v(FAKE * 2), 1 << 30, None) == RL_ERR_INVALID_ARG
+
+
+def test_params_struct_layout_matches_header():
+    assert ctypes.sizeof(ml.RlLossParams) == 52
+    text = open(HEADER).read()
+    body = text[text.index("typedef struct {", text.index("rl_correction;")):
+                text.index("} rl_loss_params;")]
+    fields = re.findall(r"\b(?:float|int32_t)\s+([a-z_0-9]+(?:\s*,\s*[a-z_0-9]+)*)\s*;", body)
+    names = [n.strip() for group in fields for n in group.split(",")]
+    assert names == [f[0] for f in ml.RlLossParams._fields_]

@@ -1,0 +1,276 @@
+"""GPU parity: the CUDA library against the float64 oracle, element by
+element, on seeded workloads at sizes the oracle finishes in seconds (many
+rows, every cluster size, ragged tails), plus edge cases, error paths,
+determinism and batch invariance. All calls go through the C ABI."""
+
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import _parity as P
+from paper_2609_08368_gb300 import api, workloads as wl
+from paper_2609_08368_gb300 import milesloss as ml
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda"
+
+SHRUNK = {
+    "tiny": wl.RECIPES["tiny"],
+    "qwen": wl.shrink(wl.RECIPES["qwen"], n_prompts=2, traj_len=16),
+    "glm": wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=48),
+    "agentic": wl.shrink(wl.RECIPES["agentic"], traj_len=2048, vocab=8192),
+    "fp32": wl.shrink(wl.RECIPES["fp32"], n_prompts=8, traj_len=32),
+    # wide rollout noise: many tokens past every clip threshold
+    "glm_noisy": wl.shrink(wl.RECIPES["glm"], n_prompts=2, group_size=4, traj_len=64,
+                           vocab=20480, rho_noise=0.35, ref_noise=0.3),
+    "fp32_noisy": wl.shrink(wl.RECIPES["fp32"], n_prompts=4, traj_len=64, vocab=12288,
+                            rho_noise=0.4),
+}
+
+
+@pytest.fixture(autouse=True)
+def _no_overrides(monkeypatch):
+    monkeypatch.delenv("MILESLOSS_SWEEP_CLUSTER", raising=False)
+    monkeypatch.delenv("MILESLOSS_SWEEP_STAGES", raising=False)
+
+
+def _full_check(w, mode="fused", dl_dtype=None, params=None):
+    g = P.run_gpu(w, mode=mode, dl_dtype=dl_dtype, params=params)
+    assert g["err"] == 0, ml.status_string(g["err"])
+    o = P.run_oracle(w, params=params)
+    P.compare_forward(w, g, o, params=params)
+    if mode != "fwd":
+        P.assert_dlogits_close(g["dlogits_t"][:, :w.vocab].float().cpu().numpy(), o["dlogits"])
+    return g, o
+
+
+@pytest.mark.parametrize("name", list(SHRUNK))
+def test_parity_fused(name):
+    _full_check(wl.make(SHRUNK[name], DEV))
+
+
+@pytest.mark.parametrize("name", ["tiny", "fp32", "glm_noisy"])
+def test_parity_split_fwd_then_bwd(name):
+    _full_check(wl.make(SHRUNK[name], DEV), mode="split")
+
+
+def test_clip_decisions_are_exercised():
+    w = wl.make(SHRUNK["glm_noisy"], DEV)
+    g, _ = _full_check(w)
+    st = g["stats"]
+    assert st["n_clip_hi"] > 0 and st["n_clip_lo"] > 0 and st["n_dual_clip"] > 0
+
+
+def test_dlogits_relative_error_on_order_p_entries():
+    """With grad_loss = N the entries are O(p), so the relative bound is
+    checked on every entry of magnitude >= 1e-6."""
+    for name in ("tiny", "fp32_noisy"):
+        w = wl.make(SHRUNK[name], DEV)
+        N = int(w.loss_mask.sum())
+        g = P.run_gpu(w, grad_loss=float(N), dl_dtype=torch.float32)
+        o = P.run_oracle(w, grad_loss=float(N))
+        got = g["dlogits_t"].cpu().numpy()
+        P.assert_rel_on_large(got, o["dlogits"], floor=1e-6, rel=1e-3)
+        P.assert_dlogits_close(got, o["dlogits"])
+
+
+@pytest.mark.parametrize("cluster", [1, 2, 4, 8])
+def test_every_cluster_size(monkeypatch, cluster):
+    monkeypatch.setenv("MILESLOSS_SWEEP_CLUSTER", str(cluster))
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=24, vocab=20000 + 24)
+    _full_check(wl.make(rec, DEV))
+
+
+@pytest.mark.parametrize("stages", [1, 2, 3, 4])
+def test_every_ring_depth(monkeypatch, stages):
+    monkeypatch.setenv("MILESLOSS_SWEEP_CLUSTER", "2")
+    monkeypatch.setenv("MILESLOSS_SWEEP_STAGES", str(stages))
+    rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=1, group_size=4, traj_len=40, vocab=6144)
+    _full_check(wl.make(rec, DEV))
+
+
+@pytest.mark.parametrize("vocab", [1, 2, 7, 9, 4097, 12345])
+def test_ragged_vocab(vocab):
+    rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=1, group_size=3, traj_len=5, vocab=vocab,
+                    mask="none")
+    _full_check(wl.make(rec, DEV))
+
+
+def test_padded_and_misaligned_rows():
+    rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=1, group_size=2, traj_len=24, vocab=1000)
+    # ld = 1003 bf16 elements: rows are not 16-byte aligned (scalar path)
+    w = wl.make(rec, DEV, ld=1003)
+    g, o = _full_check(w)
+    # padded, aligned rows; the dLogits padding must stay untouched (NaN)
+    w = wl.make(rec, DEV, ld=1024)
+    g = P.run_gpu(w, ld_out=1032)
+    assert torch.isnan(g["dlogits_t"][:, 1000:]).all()
+    o = P.run_oracle(w)
+    P.assert_dlogits_close(g["dlogits_t"][:, :1000].float().cpu().numpy(), o["dlogits"])
+
+
+@pytest.mark.parametrize("logit_dtype,dl_dtype", [("bf16", torch.float32), ("f32", torch.bfloat16)])
+def test_mixed_dtypes(logit_dtype, dl_dtype):
+    rec = wl.shrink(wl.RECIPES["fp32" if logit_dtype == "f32" else "tiny"], n_prompts=2,
+                    group_size=4, traj_len=16, vocab=5000)
+    _full_check(wl.make(rec, DEV), dl_dtype=dl_dtype)
+
+
+def test_temperature_entropy_kl_correction_opd():
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=2, group_size=4, traj_len=32, vocab=9000,
+                    rho_noise=0.25, ref_noise=0.2, old_noise=0.1, teacher_noise=0.3)
+    for params in (dict(temperature=0.7, eps_lo=0.2, eps_hi=0.28, dual_clip_c=3.0, kl_coef=0.05,
+                        entropy_coef=0.01),
+                   dict(temperature=1.3, correction="tis", corr_lo=0.0, corr_hi=1.1, kl_coef=0.1),
+                   dict(correction="clip_or_pop", corr_lo=0.9, corr_hi=1.1, dual_clip_c=2.0),
+                   dict(opd_coef=0.5, entropy_coef=0.002),
+                   dict(normalize_std=False, unbiased_std=False)):
+        w = wl.make(rec, DEV)
+        _full_check(w, params=params)
+        _full_check(w, mode="split", params=params)
+
+
+def test_no_training_tokens_and_empty_call():
+    rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=1, group_size=2, traj_len=8, vocab=300)
+    w = wl.make(rec, DEV)
+    w.loss_mask.zero_()
+    g = P.run_gpu(w)
+    assert g["err"] == 0
+    assert g["stats"]["n_tokens"] == 0 and g["stats"]["loss"] == 0.0
+    assert (g["dlogits_t"] == 0).all()
+    o = P.run_oracle(w)
+    np.testing.assert_allclose(g["logp"], o["logp"], atol=2e-3)
+    # zero rows: advantages still computed, statistics all zero
+    buf = api.alloc(0, 2, 1, DEV, vocab=300, dlogits_dtype=torch.bfloat16)
+    empty = torch.empty(0, dtype=torch.bfloat16, device=DEV)
+    ml.rl_loss_fwd_bwd(empty.view(0, 300), torch.empty(0, dtype=torch.int32, device=DEV),
+                       torch.empty(0, device=DEV), None, None, None,
+                       torch.tensor([0.0, 1.0], device=DEV),
+                       torch.zeros(2, dtype=torch.int32, device=DEV),
+                       torch.zeros(3, dtype=torch.int32, device=DEV), 1,
+                       torch.empty(0, dtype=torch.uint8, device=DEV), {}, buf.token_logprobs,
+                       buf.entropy, buf.advantages, buf.group_sizes, buf.stats, buf.dlogits,
+                       buf.workspace, vocab=300)
+    torch.cuda.synchronize()
+    st = buf.read_stats()
+    assert st["n_tokens"] == 0 and st["loss"] == 0.0
+    assert buf.group_sizes.tolist() == [2]
+    np.testing.assert_allclose(buf.advantages.cpu().numpy(), [-2 ** -0.5, 2 ** -0.5], rtol=1e-6)
+
+
+def test_device_errors_are_reported_not_trapped():
+    rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=2, group_size=2, traj_len=8, vocab=256)
+    w = wl.make(rec, DEV)
+    w.targets[3] = 256                     # outside [0, vocab)
+    g = P.run_gpu(w)
+    assert g["err"] == 5                   # RL_ERR_TARGET_OUT_OF_RANGE
+    assert g["logp"][3] == 0.0 and (g["dlogits_t"][3] == 0).all()
+    assert np.isfinite(g["logp"]).all()
+    w = wl.make(rec, DEV)
+    w.group_id[1] = 9
+    assert P.run_gpu(w)["err"] == 6        # RL_ERR_GROUP_OUT_OF_RANGE
+    w = wl.make(rec, DEV)
+    w.cu_seqlens[2] = 3                    # not non-decreasing
+    assert P.run_gpu(w)["err"] == 7        # RL_ERR_BAD_SEQLENS
+    w = wl.make(rec, DEV)
+    assert P.run_gpu(w)["err"] == 0        # the error word resets on the next call
+
+
+def test_bitwise_reproducible_and_fwd_matches_fused():
+    w = wl.make(SHRUNK["glm_noisy"], DEV)
+    a = P.run_gpu(w)
+    b = P.run_gpu(w)
+    c = P.run_gpu(w, mode="fwd")
+    assert torch.equal(a["dlogits_t"], b["dlogits_t"])
+    np.testing.assert_array_equal(a["logp"], b["logp"])
+    assert a["stats"] == b["stats"]
+    np.testing.assert_array_equal(a["logp"], c["logp"])
+    np.testing.assert_array_equal(a["H"], c["H"])
+    assert a["stats"] == c["stats"]
+
+
+def test_batch_invariance_of_row_outputs():
+    """A row's log-prob and entropy do not depend on where it sits or on how
+    many other rows share the call."""
+    rec = wl.shrink(wl.RECIPES["qwen"], n_prompts=2, group_size=4, traj_len=32, vocab=30000)
+    w = wl.make(rec, DEV)
+    full = P.run_gpu(w, mode="fwd")
+    perm = torch.randperm(w.n_rows, generator=torch.Generator().manual_seed(0)).to(DEV)
+    sub = perm[:37]
+    w2 = wl.Workload(rec, w.logits[sub].contiguous(), w.targets[sub].contiguous(),
+                     w.rollout_logprobs[sub].contiguous(), None, None, None,
+                     torch.tensor([0.0], device=DEV), torch.zeros(1, dtype=torch.int32, device=DEV),
+                     torch.tensor([0, 37], dtype=torch.int32, device=DEV),
+                     w.loss_mask[sub].contiguous(), 1, dict(w.params))
+    part = P.run_gpu(w2, mode="fwd")
+    idx = sub.cpu().numpy()
+    np.testing.assert_array_equal(part["logp"], full["logp"][idx])
+    np.testing.assert_array_equal(part["H"], full["H"][idx])
+
+
+def test_grad_loss_device_scalar():
+    w = wl.make(SHRUNK["tiny"], DEV)
+    a = P.run_gpu(w, grad_loss=3.0, dl_dtype=torch.float32)
+    buf = api.alloc(w.n_rows, int(w.rewards.shape[0]), w.n_groups, DEV, vocab=w.vocab,
+                    dlogits_dtype=torch.float32)
+    api.fwd_bwd(w, buf, grad_loss=1.5, grad_loss_device=torch.tensor([2.0], device=DEV))
+    torch.cuda.synchronize()
+    assert torch.equal(buf.dlogits, a["dlogits_t"])
+
+
+# ---------------------------------------------------------------- full sizes
+
+FULL = ["qwen", "glm", "agentic", "fp32"]
+
+
+def _sampled_rows(w, n=24, seed=0):
+    rng = np.random.default_rng(seed)
+    R = w.n_rows
+    return np.unique(np.concatenate([[0, R - 1], rng.integers(0, R, size=n)]))
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("name", FULL)
+def test_full_size_sampled_rows(name):
+    """Full-size workloads in the launch configuration the benchmark times:
+    sampled rows against the oracle one by one, and the loss against the
+    oracle's per-token rule applied to the GPU's own log-probs."""
+    rec = wl.RECIPES[name]
+    w = wl.make(rec, DEV)
+    g = P.run_gpu(w)
+    assert g["err"] == 0
+    p = P.oracle_params(w.params)
+    import oracle
+    A_traj, n_g = oracle.group_advantages(P.np_(w.rewards), P.np_(w.group_id), w.n_groups, p)
+    np.testing.assert_allclose(g["A"], A_traj, rtol=1e-6, atol=1e-6)
+    np.testing.assert_array_equal(g["group_sizes"], n_g)
+    A_row = oracle.row_advantages(A_traj, P.np_(w.cu_seqlens), w.n_rows)
+    mask = P.np_(w.loss_mask)
+    N = int(mask.astype(bool).sum())
+    assert g["stats"]["n_tokens"] == N
+    rows = _sampled_rows(w)
+    o = oracle.rl_loss_rows(P.host_logits(w, torch.from_numpy(rows).to(DEV)),
+                            P.np_(w.targets)[rows], P.np_(w.rollout_logprobs)[rows],
+                            None if w.ref_logprobs is None else P.np_(w.ref_logprobs)[rows],
+                            A_row[rows], mask[rows].astype(bool), N, p)
+    tol = P.logp_tol(w)
+    np.testing.assert_allclose(g["logp"][rows], o["logp"], atol=tol, rtol=0)
+    np.testing.assert_allclose(g["H"][rows], o["H"], atol=tol, rtol=0)
+    dl = g["dlogits_t"][torch.from_numpy(rows).to(DEV), :w.vocab].float().cpu().numpy()
+    P.assert_dlogits_close(dl, o["dlogits"])
+    # loss and counts: the oracle's per-token rule on the GPU's log-probs
+    obj = oracle.token_objective(g["logp"].astype(np.float64), P.np_(w.rollout_logprobs),
+                                 P.np_(w.ref_logprobs), A_row, g["H"].astype(np.float64), p)
+    L, _ = oracle.masked_token_mean(obj["ell"], mask)
+    m = mask.astype(bool)
+    scale = np.abs(obj["ell"][m]).mean()
+    assert abs(g["stats"]["loss"] - L) <= 1e-4 * scale
+    counts, band = P.clip_counts(p, g["logp"].astype(np.float64), P.np_(w.rollout_logprobs),
+                                 P.np_(w.ref_logprobs), A_row, g["H"], mask)
+    for k, v in counts.items():
+        assert abs(g["stats"][k] - v) <= band, (k, g["stats"][k], v, band)
+    del g, w
+    torch.cuda.empty_cache()
