@@ -50,6 +50,10 @@ def parse_args():
     ap.add_argument("--cpu-sample-rows", type=int, default=512)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--n-prompts", type=int, default=None,
+                    help="fewer groups (a smaller case of the same workload, for profiling)")
+    ap.add_argument("--traj-len", type=int, default=None,
+                    help="shorter trajectories (a smaller case, for profiling)")
     return ap.parse_args()
 
 
@@ -292,7 +296,8 @@ def run_ours(args, rank, world, local):
     ml.load()
     dev = torch.device("cuda", local)
     rec = wl.RECIPES[args.workload]
-    rec = wl.shrink(rec, seed=rec.seed + 1000 * rank)  # each replica has its own batch
+    rec = wl.shrink(rec, n_prompts=args.n_prompts, traj_len=args.traj_len,
+                    seed=rec.seed + 1000 * rank)  # each replica has its own batch
     w = wl.make(rec, dev)
     R, V = w.n_rows, w.vocab
     dl_dtype = w.logits.dtype
@@ -309,6 +314,9 @@ def run_ours(args, rank, world, local):
     K = args.steps
     ev_sweep = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                 for _ in range(K)]
+    for b, e in ev_sweep:  # torch creates the CUDA event handles on first record
+        b.record(stream)
+        e.record(stream)
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(local)
     clocks.start()

@@ -145,40 +145,61 @@ LossScalars scalars(const rl_loss_params* p) {
 }
 
 struct SweepPlan {
-  int C, S, slice, stage_bytes, smem;
+  int C, S, slice, stage_bytes, smem, threads, variant;
 };
 
-// Smallest cluster whose per-CTA slice fits two stages in shared memory;
-// as many stages as fit, up to kMaxStages. Overridable for tuning through
-// MILESLOSS_SWEEP_CLUSTER / MILESLOSS_SWEEP_STAGES.
+// Several CTAs per SM hide each other's per-row synchronisation, so the
+// plan aims at five CTAs of 256 threads per SM: the smallest cluster whose
+// per-CTA slice fits a fifth of the SM's shared memory, then as many ring
+// stages as still fit; if no cluster size fits, one CTA per SM.
+// Overridable for tuning through MILESLOSS_SWEEP_CLUSTER / _STAGES /
+// _THREADS / _CTAS_PER_SM.
 rl_status plan_sweep(rl_dtype dt, long long V, int dev, SweepPlan* out) {
-  int optin = 0;
-  if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+  int optin = 0, per_sm = 0, reserved = 0;
+  if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) !=
+          cudaSuccess ||
+      cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev) !=
+          cudaSuccess)
     return RL_ERR_CUDA;
-  const int budget = optin - kSweepSmemExtra;
+  // Block shapes compiled: 256 threads for 5 or 4 CTAs per SM (48 or 64
+  // registers), 512 threads for 2 CTAs per SM.
+  const int threads = env_int("MILESLOSS_SWEEP_THREADS", 256);
+  const int target = env_int("MILESLOSS_SWEEP_CTAS_PER_SM", threads == 256 ? 5 : 2);
+  if (!((threads == 256 && (target == 4 || target == 5)) || (threads == 512 && target == 2)))
+    return RL_ERR_UNSUPPORTED;
+  const int variant = threads == 512 ? 512 : (target == 5 ? 255 : 256);
   const int es = static_cast<int>(elem_size(dt));
   const int vec = 16 / es;
   const int forced_c = env_int("MILESLOSS_SWEEP_CLUSTER", 0);
   const int forced_s = env_int("MILESLOSS_SWEEP_STAGES", 0);
-  for (int C = 1; C <= 8; C *= 2) {
-    if (forced_c && C != forced_c) continue;
-    long long slice = (V + C - 1) / C;
-    slice = (slice + vec - 1) / vec * vec;
-    if (C > 1 && slice * (C - 1) >= V) continue;  // every CTA must own columns
-    const long long stage = (slice * es + 127) / 128 * 128;
-    if (2 * stage > budget) continue;
-    int S = static_cast<int>(budget / stage);
-    if (S > kMaxStages) S = kMaxStages;
-    if (forced_s) {
-      if (forced_s < 1 || forced_s > kMaxStages || forced_s * stage > budget) return RL_ERR_UNSUPPORTED;
-      S = forced_s;
+  const int hard = optin - kSweepSmemExtra;                            // one CTA per SM
+  const int share = per_sm / target - reserved - kSweepSmemExtra;      // `target` per SM
+  for (int pass = 0; pass < 2; ++pass) {
+    const int budget = pass == 0 ? share : hard;
+    for (int C = 1; C <= kMaxCluster; C *= 2) {
+      if (forced_c && C != forced_c) continue;
+      long long slice = (V + C - 1) / C;
+      slice = (slice + vec - 1) / vec * vec;
+      if (C > 1 && slice * (C - 1) >= V) continue;  // every CTA must own columns
+      const long long stage = (slice * es + 127) / 128 * 128;
+      if (stage > budget) continue;
+      int S = static_cast<int>(budget / stage);
+      if (S > kMaxStages) S = kMaxStages;
+      if (forced_s) {
+        if (forced_s < 1 || forced_s > kMaxStages || forced_s * stage > hard)
+          return RL_ERR_UNSUPPORTED;
+        S = forced_s;
+      }
+      out->C = C;
+      out->S = S;
+      out->slice = static_cast<int>(slice);
+      out->stage_bytes = static_cast<int>(stage);
+      out->smem = static_cast<int>(S * stage) + kSweepSmemExtra;
+      out->threads = threads;
+      out->variant = variant;
+      return RL_OK;
     }
-    out->C = C;
-    out->S = S;
-    out->slice = static_cast<int>(slice);
-    out->stage_bytes = static_cast<int>(stage);
-    out->smem = static_cast<int>(S * stage) + kSweepSmemExtra;
-    return RL_OK;
   }
   return RL_ERR_UNSUPPORTED;  // vocabulary too large for an 8-CTA cluster
 }
@@ -282,11 +303,11 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s) {
     SweepPlan pl;
     st = plan_sweep(c.dt, c.V, dev, &pl);
     if (st != RL_OK) return st;
-    const void* fn = sweep_kernel(c.dt, grad ? go->dt : c.dt, grad);
+    const void* fn = sweep_kernel(c.dt, grad ? go->dt : c.dt, grad, pl.variant);
     st = set_smem(fn, dev, pl.smem);
     if (st != RL_OK) return st;
     int clusters = 0;
-    st = resident_clusters(fn, dev, pl.C, pl.smem, kSweepThreads, &clusters);
+    st = resident_clusters(fn, dev, pl.C, pl.smem, pl.threads, &clusters);
     if (st != RL_OK) return st;
     const long long n_cl = std::min<long long>(clusters, c.R);
 
@@ -315,7 +336,7 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s) {
     sa.s = scalars(c.p);
     sa.ws = ws;
     record(t_ev_begin, s);
-    st = launch(fn, dim3(static_cast<unsigned>(n_cl * pl.C)), dim3(kSweepThreads), pl.smem, pl.C,
+    st = launch(fn, dim3(static_cast<unsigned>(n_cl * pl.C)), dim3(pl.threads), pl.smem, pl.C,
                 s, &sa);
     record(t_ev_end, s);
     if (st != RL_OK) return st;

@@ -226,6 +226,45 @@ __device__ __forceinline__ float4 ld_dsmem_f4(uint32_t addr) {
   return v;
 }
 
+// Asynchronous 16-byte store into the shared memory of a CTA of the cluster
+// (possibly another SM); the bytes are counted as transactions on the
+// destination CTA's mbarrier. Both addresses come from mapa.
+__device__ __forceinline__ void st_async_f4(uint32_t remote_addr, float4 v, uint32_t remote_bar) {
+  asm volatile(
+      "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];"
+      ::"r"(remote_addr), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(remote_bar)
+      : "memory");
+}
+
+// Packed pairs of fp32 (sm_100+ f32x2 instructions: two IEEE operations,
+// each rounded to nearest, per instruction).
+__device__ __forceinline__ unsigned long long f2_bits(float2 v) {
+  unsigned long long r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(v.x), "f"(v.y));
+  return r;
+}
+__device__ __forceinline__ float2 bits_f2(unsigned long long r) {
+  float2 v;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(v.x), "=f"(v.y) : "l"(r));
+  return v;
+}
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  unsigned long long d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(f2_bits(a)), "l"(f2_bits(b)), "l"(f2_bits(c)));
+  return bits_f2(d);
+}
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
+  unsigned long long d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(f2_bits(a)), "l"(f2_bits(b)));
+  return bits_f2(d);
+}
+__device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
+  unsigned long long d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(f2_bits(a)), "l"(f2_bits(b)));
+  return bits_f2(d);
+}
+__device__ __forceinline__ float2 ex2x2(float2 t) { return make_float2(ex2(t.x), ex2(t.y)); }
+
 // Streaming 16-byte global load that does not allocate in L1.
 __device__ __forceinline__ uint4 ld_stream_u4(const void* p) {
   uint4 v;
@@ -261,6 +300,27 @@ struct InBf16 {
     f[0] = bf16_lo(w.x); f[1] = bf16_hi(w.x); f[2] = bf16_lo(w.y); f[3] = bf16_hi(w.y);
     f[4] = bf16_lo(w.z); f[5] = bf16_hi(w.z); f[6] = bf16_lo(w.w); f[7] = bf16_hi(w.w);
   }
+  // the 16 bytes as kVec / 2 pairs
+  __device__ static __forceinline__ void unpack2(uint4 w, float2* f) {
+    f[0] = make_float2(bf16_lo(w.x), bf16_hi(w.x));
+    f[1] = make_float2(bf16_lo(w.y), bf16_hi(w.y));
+    f[2] = make_float2(bf16_lo(w.z), bf16_hi(w.z));
+    f[3] = make_float2(bf16_lo(w.w), bf16_hi(w.w));
+  }
+  // running maximum kept as a packed pair (bf16x2 for bf16 input)
+  using MaxAcc = uint32_t;
+  static constexpr uint32_t kMaxInit = 0xff80ff80u;  // (-inf, -inf)
+  __device__ static __forceinline__ uint32_t max_acc(uint32_t m, uint4 w) {
+    __nv_bfloat162 a = __hmax2(*reinterpret_cast<__nv_bfloat162*>(&w.x),
+                               *reinterpret_cast<__nv_bfloat162*>(&w.y));
+    __nv_bfloat162 b = __hmax2(*reinterpret_cast<__nv_bfloat162*>(&w.z),
+                               *reinterpret_cast<__nv_bfloat162*>(&w.w));
+    __nv_bfloat162 c = __hmax2(__hmax2(a, b), *reinterpret_cast<__nv_bfloat162*>(&m));
+    return *reinterpret_cast<uint32_t*>(&c);
+  }
+  __device__ static __forceinline__ float max_val(uint32_t m) {
+    return fmaxf(bf16_lo(m), bf16_hi(m));
+  }
   __device__ static __forceinline__ float vmax(uint4 w) {
     __nv_bfloat162 a = __hmax2(*reinterpret_cast<__nv_bfloat162*>(&w.x),
                                *reinterpret_cast<__nv_bfloat162*>(&w.y));
@@ -283,6 +343,17 @@ struct InF32 {
     f[0] = __uint_as_float(w.x); f[1] = __uint_as_float(w.y);
     f[2] = __uint_as_float(w.z); f[3] = __uint_as_float(w.w);
   }
+  __device__ static __forceinline__ void unpack2(uint4 w, float2* f) {
+    f[0] = make_float2(__uint_as_float(w.x), __uint_as_float(w.y));
+    f[1] = make_float2(__uint_as_float(w.z), __uint_as_float(w.w));
+  }
+  using MaxAcc = float;
+  static constexpr float kMaxInit = -INFINITY;
+  __device__ static __forceinline__ float max_acc(float m, uint4 w) {
+    return fmaxf(fmaxf(fmaxf(__uint_as_float(w.x), __uint_as_float(w.y)),
+                       fmaxf(__uint_as_float(w.z), __uint_as_float(w.w))), m);
+  }
+  __device__ static __forceinline__ float max_val(float m) { return m; }
   __device__ static __forceinline__ float vmax(uint4 w) {
     return fmaxf(fmaxf(__uint_as_float(w.x), __uint_as_float(w.y)),
                  fmaxf(__uint_as_float(w.z), __uint_as_float(w.w)));
@@ -373,10 +444,11 @@ __device__ __forceinline__ TokenTerms token_terms(float logp, float H, float rho
   }
   float k3 = 0.0f, gkl = 0.0f;
   if (has_q) {
+    // expm1 keeps both terms accurate when q is close to logp
     const float dlt = q - logp;
-    const float ed = expf(dlt);
-    k3 = ed - dlt - 1.0f;
-    gkl = 1.0f - ed;
+    const float em1 = expm1f(dlt);
+    k3 = em1 - dlt;
+    gkl = -em1;
   }
   t.r = r;
   t.pg = pg;

@@ -35,11 +35,13 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
     const char* zrow = static_cast<const char*>(a.logits) + row * a.ld * static_cast<long long>(sizeof(St));
     char* drow = static_cast<char*>(a.dlogits) + row * a.ld_out * static_cast<long long>(Out::kSize);
     const int y = a.targets[row];
-    const float add = cc * G;
+    // The sampled token's entry: cc [G (1 - p_y) + gamma p_y (log p_y + H)]
+    // with 1 - p_y = -expm1(logp), accurate when p_y is close to 1.
+    const float logp = ws.logp[row];
+    const float dzy = cc * (G * -expm1f(logp) + a.gamma * expf(logp) * (logp + H));
     auto value = [&](float z, int j) {
-      float x = (cc == 0.0f) ? 0.0f : ex2(fmaf(z, a.k, -L2)) * fmaf(cb, z, ca);
-      if (j == y) x += add;
-      return x;
+      if (j == y) return dzy;
+      return (cc == 0.0f) ? 0.0f : ex2(fmaf(z, a.k, -L2)) * fmaf(cb, z, ca);
     };
     if (a.in_vec && a.out_vec) {
       // j0 is a multiple of V8 (kBwdTile is), so every vector is aligned.
@@ -57,7 +59,7 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
           if (static_cast<unsigned>(y - jb) < static_cast<unsigned>(V8)) {
 #pragma unroll
             for (int e = 0; e < V8; ++e)
-              if (jb + e == y) f[e] += add;
+              if (jb + e == y) f[e] = dzy;
           }
         }
         Out::template storev<V8>(drow + static_cast<size_t>(jb) * Out::kSize, f, 0u);

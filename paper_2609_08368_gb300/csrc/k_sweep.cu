@@ -7,20 +7,26 @@
 // every row the cluster visits (rows cluster_id, cluster_id + n_clusters,
 // ...). Each CTA streams its slices into an S-stage shared-memory ring with
 // bulk async copies (cp.async.bulk, completion counted on an mbarrier per
-// stage), so the copies of the next S-1 rows are in flight while the current
-// one is processed. Per row:
-//   pass A  every thread folds its elements into an online (max m, sum S of
-//           2^(t - m k), sum U of 2^(t - m k) (t - m k)) with t = z log2(e)/T;
-//           warp shuffles, then one warp, combine the threads in a fixed
-//           order; CTAs exchange their triples through distributed shared
-//           memory and every CTA combines the C triples in rank order, so all
-//           CTAs of the cluster hold bit-identical row statistics;
-//   epilogue one thread evaluates the per-token objective (ratio, clips, k3,
-//           entropy term) and the coefficients of the gradient;
+// stage). Several CTAs share an SM, so one CTA's per-row synchronisation
+// overlaps the others' arithmetic. Per row:
+//   pass M  every thread takes the maximum m of its own elements;
+//   pass A  it sums S = sum 2^(t - m k) and U = sum 2^(t - m k) (t - m k),
+//           t = z log2(e)/T, two lanes per instruction (f32x2);
+//           warp shuffles, then one warp, merge the threads' (m, S, U) in a
+//           fixed order;
+//   exchange thread 0 pushes the CTA's (m, S, U, z_y) into every peer's
+//           shared memory with st.async, counted on the peer's mbarrier,
+//           and merges the C triples in rank order once they have all
+//           arrived, so every CTA of the cluster holds bit-identical row
+//           statistics;
+//   epilogue thread 0 evaluates the per-token objective and the gradient
+//           coefficients;
 //   pass B  (kGrad) the slice is swept again from shared memory and dLogits
 //           is written with 16-byte streaming stores.
 // Definitions: Sec. 3.4 (ratio), Sec. 2 / 9.1 (group-relative advantage),
 // Sec. 2.4 (loss mask); the gradient is the chain rule through them.
+#include <type_traits>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -28,45 +34,36 @@ namespace milesloss {
 
 namespace {
 
-constexpr int kThreads = kSweepThreads;
-constexpr int kWarps = kThreads / 32;
-constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s per bulk-copy wait
+constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s per bounded wait
 constexpr float kLn2 = 0.69314718055994531f;
 
 struct Tri {
   float m, s, u;  // max of z; sum of 2^(t - m k); sum of 2^(t - m k) (t - m k)
 };
 
-// Merge two triples (k = log2(e)/T). Commutative bit-for-bit, so butterfly
-// reductions leave every lane with the same value.
-__device__ __forceinline__ Tri merge(Tri a, Tri b, float k) {
-  if (b.s == 0.0f) return a;
-  if (a.s == 0.0f) return b;
-  const float m = fmaxf(a.m, b.m);
-  const float da = (a.m - m) * k, db = (b.m - m) * k;
-  const float fa = ex2(da), fb = ex2(db);
-  Tri r;
-  r.m = m;
-  r.s = fa * a.s + fb * b.s;
-  r.u = fa * fmaf(da, a.s, a.u) + fb * fmaf(db, b.s, b.u);
-  return r;
-}
-
-__device__ __forceinline__ Tri shfl_xor(Tri t, int o) {
-  Tri r;
-  r.m = __shfl_xor_sync(0xffffffffu, t.m, o);
-  r.s = __shfl_xor_sync(0xffffffffu, t.s, o);
-  r.u = __shfl_xor_sync(0xffffffffu, t.u, o);
-  return r;
-}
-
+// Warp-wide merge in a fixed order: the maximum first, then every lane
+// rescales its sums once to that maximum, then plain butterfly sums.
+// Every lane ends with the same triple.
 __device__ __forceinline__ Tri warp_merge(Tri t, float k) {
+  float M = t.m;
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) t = merge(t, shfl_xor(t, o), k);
-  return t;
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  float s = 0.0f, u = 0.0f;
+  if (t.s > 0.0f) {
+    const float d = (t.m - M) * k, f = ex2(d);
+    s = f * t.s;
+    u = f * fmaf(d, t.s, t.u);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    s += __shfl_xor_sync(0xffffffffu, s, o);
+    u += __shfl_xor_sync(0xffffffffu, u, o);
+  }
+  return Tri{M, s, u};
 }
 
 // Block-wide merge; the result is valid in warp 0. Contains a __syncthreads.
+template <int kWarps>
 __device__ __forceinline__ Tri block_merge(Tri t, float k, float4* red) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   t = warp_merge(t, k);
@@ -83,44 +80,64 @@ __device__ __forceinline__ Tri block_merge(Tri t, float k, float4* red) {
   return t;
 }
 
-// Fold one value into a thread's running triple (two interleaved sums).
-struct Acc {
-  float m = -INFINITY, mt = -INFINITY, s0 = 0.0f, s1 = 0.0f, u0 = 0.0f, u1 = 0.0f;
-
-  __device__ __forceinline__ void raise(float vm, float k) {
-    if (vm > m) {
-      if (s0 + s1 > 0.0f) {
-        const float d = (m - vm) * k, f = ex2(d);
-        u0 = f * fmaf(d, s0, u0);
-        u1 = f * fmaf(d, s1, u1);
-        s0 *= f;
-        s1 *= f;
+// Sum of 2^(t - mt) and of 2^(t - mt) (t - mt) over the thread's vectors,
+// t = z k, for a fixed mt (the thread's own maximum times k). kSafe skips
+// -inf logits exactly (0 * -inf would otherwise give NaN); it runs only
+// when the fast pass produced a NaN.
+template <class In, int kThreads, bool kSafe>
+__device__ __forceinline__ void sum_pass(const uint4* sv, int n_vec, float k, float mt,
+                                         float& s_out, float& u_out) {
+  constexpr int P = In::kVec / 2;  // pairs per 16 bytes
+  const float2 k2 = make_float2(k, k);
+  const float2 nm2 = make_float2(-mt, -mt);
+  float2 s0 = make_float2(0.0f, 0.0f), s1 = s0, u0 = s0, u1 = s0;
+  int v = threadIdx.x;
+  for (; v + kThreads < n_vec; v += 2 * kThreads) {
+    float2 fa[P], fb[P];
+    In::unpack2(sv[v], fa);
+    In::unpack2(sv[v + kThreads], fb);
+#pragma unroll
+    for (int e = 0; e < P; ++e) {
+      float2 ta = ffma2(fa[e], k2, nm2), tb = ffma2(fb[e], k2, nm2);
+      if (kSafe) {
+        if (fa[e].x == -INFINITY) ta.x = -127.0f;
+        if (fa[e].y == -INFINITY) ta.y = -127.0f;
+        if (fb[e].x == -INFINITY) tb.x = -127.0f;
+        if (fb[e].y == -INFINITY) tb.y = -127.0f;
       }
-      m = vm;
-      mt = vm * k;
+      const float2 xa = ex2x2(ta), xb = ex2x2(tb);
+      s0 = fadd2(s0, xa);
+      s1 = fadd2(s1, xb);
+      u0 = ffma2(xa, ta, u0);
+      u1 = ffma2(xb, tb, u1);
     }
   }
-  // t below -127 contributes 0 either way; the clamp keeps -inf logits
-  // from producing 0 * -inf.
-  __device__ __forceinline__ void add0(float z, float k) {
-    const float t = fmaxf(fmaf(z, k, -mt), -127.0f);
-    const float x = ex2(t);
-    s0 += x;
-    u0 = fmaf(x, t, u0);
+  if (v < n_vec) {
+    float2 fa[P];
+    In::unpack2(sv[v], fa);
+#pragma unroll
+    for (int e = 0; e < P; ++e) {
+      float2 ta = ffma2(fa[e], k2, nm2);
+      if (kSafe) {
+        if (fa[e].x == -INFINITY) ta.x = -127.0f;
+        if (fa[e].y == -INFINITY) ta.y = -127.0f;
+      }
+      const float2 xa = ex2x2(ta);
+      s0 = fadd2(s0, xa);
+      u0 = ffma2(xa, ta, u0);
+    }
   }
-  __device__ __forceinline__ void add1(float z, float k) {
-    const float t = fmaxf(fmaf(z, k, -mt), -127.0f);
-    const float x = ex2(t);
-    s1 += x;
-    u1 = fmaf(x, t, u1);
-  }
-  __device__ __forceinline__ Tri tri() const { return Tri{m, s0 + s1, u0 + u1}; }
-};
+  const float2 s = fadd2(s0, s1), u = fadd2(u0, u1);
+  s_out = s.x + s.y;
+  u_out = u.x + u.y;
+}
 
-template <class In, class Out, bool kGrad>
-__global__ void __launch_bounds__(kThreads, 1) k_sweep(const SweepArgs a) {
+template <class In, class Out, bool kGrad, int kThreads, int kMinBlocks>
+__global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs a) {
   using St = typename In::storage;
   constexpr int V8 = In::kVec;
+  constexpr int P = V8 / 2;
+  constexpr int kWarps = kThreads / 32;
   extern __shared__ __align__(128) unsigned char smem[];
   const int tid = threadIdx.x;
   const int C = static_cast<int>(cluster_nctarank());
@@ -138,10 +155,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_sweep(const SweepArgs a) {
 
   unsigned char* stages = smem;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(S) * a.stage_bytes);
-  float4* xch = reinterpret_cast<float4*>(bars + kMaxStages);  // [2]
-  float4* red = xch + 2;                                        // [kWarps]
-  float4* bc = red + kWarps;                                    // [1]
-  int4* bci = reinterpret_cast<int4*>(bc + 1);                  // [1]
+  uint64_t* xbar = bars + kMaxStages;                          // [2] exchange barriers
+  float4* xch = reinterpret_cast<float4*>(xbar + 2);           // [2][kMaxCluster]
+  float4* red = xch + 2 * kMaxCluster;                         // [kWarps]
+  float4* bc = red + kWarps;                                   // [2]
+  int4* bci = reinterpret_cast<int4*>(bc + 2);                 // [1]
 
   WsPtrs ws = a.ws;
   const long long N = ws.hdr->n_tokens;
@@ -151,9 +169,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_sweep(const SweepArgs a) {
 
   if (tid == 0) {
     for (int s = 0; s < S; ++s) mbar_init(smem_u32(&bars[s]), 1);
+    mbar_init(smem_u32(&xbar[0]), 1);
+    mbar_init(smem_u32(&xbar[1]), 1);
     fence_mbar_init();
   }
-  __syncthreads();
+  // Peers push into this CTA's exchange slots: all barriers must be
+  // initialised cluster-wide first.
+  if (C > 1) cluster_sync_all(); else __syncthreads();
 
   const uint64_t pol = l2_policy_evict_first();
   const char* lg = static_cast<const char*>(a.logits);
@@ -189,8 +211,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_sweep(const SweepArgs a) {
     const uint32_t parity = static_cast<uint32_t>((it / S) & 1);
     const unsigned char* sb = stages + static_cast<size_t>(s) * a.stage_bytes;
     const char* grow = row_src(row);
+    const uint4* sv = reinterpret_cast<const uint4*>(sb);
 
-    // Row scalars for the epilogue; their latency hides behind pass A.
+    // Row scalars for the epilogue; their latency hides behind the passes.
     int y = 0;
     float rho = 0.0f, q = 0.0f, old = 0.0f, A = 0.0f;
     uint8_t msk = 0;
@@ -210,29 +233,32 @@ __global__ void __launch_bounds__(kThreads, 1) k_sweep(const SweepArgs a) {
       }
     }
 
-    // ---------------- pass A
-    Acc acc;
-    const uint4* sv = reinterpret_cast<const uint4*>(sb);
-#pragma unroll 2
-    for (int v = tid; v < n_vec; v += kThreads) {
-      const uint4 w = sv[v];
-      acc.raise(In::vmax(w), k);
-      float f[V8];
-      In::unpack(w, f);
-#pragma unroll
-      for (int e = 0; e < V8; e += 2) {
-        acc.add0(f[e], k);
-        acc.add1(f[e + 1], k);
-      }
-    }
-    for (int j = vec_elems + tid; j < cnt; j += kThreads) {
-      const float z = In::load1(grow, j);
-      acc.raise(z, k);
-      acc.add0(z, k);
-    }
-    Tri t = block_merge(acc.tri(), k, red);
+    // ---------------- pass M: the thread's own maximum
+    typename In::MaxAcc macc = In::kMaxInit;
+    for (int v = tid; v < n_vec; v += kThreads) macc = In::max_acc(macc, sv[v]);
+    float mz = In::max_val(macc);
+    for (int j = vec_elems + tid; j < cnt; j += kThreads) mz = fmaxf(mz, In::load1(grow, j));
 
-    // ---------------- cluster exchange and epilogue
+    // ---------------- pass A: sums at the fixed maximum
+    Tri t{mz, 0.0f, 0.0f};
+    if (mz != -INFINITY) {
+      const float mt = mz * k;
+      float su, uu;
+      sum_pass<In, kThreads, false>(sv, n_vec, k, mt, su, uu);
+      if (__isnanf(uu) || __isnanf(su)) sum_pass<In, kThreads, true>(sv, n_vec, k, mt, su, uu);
+      for (int j = vec_elems + tid; j < cnt; j += kThreads) {
+        const float z = In::load1(grow, j);
+        if (z == -INFINITY) continue;
+        const float tt = fmaf(z, k, -mt), x = ex2(tt);
+        su += x;
+        uu = fmaf(x, tt, uu);
+      }
+      t.s = su;
+      t.u = uu;
+    }
+    t = block_merge<kWarps>(t, k, red);
+
+    // ---------------- exchange and epilogue (thread 0)
     const bool yok = (tid == 0) && (y >= 0) && (y < a.V);
     const int owner = yok ? y / slice : -1;
     if (tid == 0) {
@@ -241,28 +267,41 @@ __global__ void __launch_bounds__(kThreads, 1) k_sweep(const SweepArgs a) {
         const int jl = y - lo;
         zy = (jl < vec_elems) ? In::load1(sb, jl) : In::load1(grow, jl);
       }
-      xch[it & 1] = make_float4(t.m, t.s, t.u, zy);
-    }
-    if (C > 1) {
-      cluster_sync_all();
-    } else {
-      __syncthreads();
-    }
-    if (tid == 0) {
-      Tri tot{-INFINITY, 0.0f, 0.0f};
-      float zy = 0.0f;
-      const uint32_t mine = smem_u32(&xch[it & 1]);
-      for (int r = 0; r < C; ++r) {
-        const float4 e = (C > 1) ? ld_dsmem_f4(mapa_shared(mine, r)) : xch[it & 1];
-        tot = merge(tot, Tri{e.x, e.y, e.z}, k);
-        if (r == owner) zy = e.w;
+      const int slot = static_cast<int>(it & 1);
+      const float4 mine = make_float4(t.m, t.s, t.u, zy);
+      Tri tot = Tri{t.m, t.s, t.u};
+      float zy_all = zy;
+      if (C > 1) {
+        float4* xs = xch + slot * kMaxCluster;
+        xs[crank] = mine;
+        const uint32_t xaddr = smem_u32(&xs[crank]);
+        const uint32_t xb = smem_u32(&xbar[slot]);
+        for (int r = 0; r < C; ++r)
+          if (r != crank) st_async_f4(mapa_shared(xaddr, r), mine, mapa_shared(xb, r));
+        mbar_arrive_expect_tx(xb, static_cast<uint32_t>(C - 1) * 16u);
+        if (!dead && !mbar_wait_bounded(xb, static_cast<uint32_t>((it >> 1) & 1), kWaitLimitNs)) {
+          dead = true;
+          atomicOr(&ws.hdr->err_bits, kErrTimeout);
+        }
+        float M = -INFINITY;
+        for (int r = 0; r < C; ++r) M = fmaxf(M, xs[r].x);
+        tot = Tri{M, 0.0f, 0.0f};
+        for (int r = 0; r < C; ++r) {
+          const float4 e = xs[r];
+          if (e.y > 0.0f) {
+            const float d = (e.x - M) * k, f = ex2(d);
+            tot.s += f * e.y;
+            tot.u += f * fmaf(d, e.y, e.z);
+          }
+          if (r == owner) zy_all = e.w;
+        }
       }
       const bool bad = !yok;
       if (bad) atomicOr(&ws.hdr->err_bits, kErrTarget);
       const float lnS = logf(tot.s);
       const float lse = tot.m * a.s.invT + lnS;
       float H = lnS - tot.u * kLn2 / tot.s;
-      float logp = zy * a.s.invT - lse;
+      float logp = zy_all * a.s.invT - lse;
       if (bad) { logp = 0.0f; H = 0.0f; }
       TokenTerms tt = token_terms(logp, H, rho, q, a.q != nullptr, old, a.old != nullptr, A, a.s);
       if (bad) tt = TokenTerms{0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, kFlagBad};
@@ -281,17 +320,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_sweep(const SweepArgs a) {
         ws.flags[row] = tt.flags;
       }
       if (kGrad) {
-        // dZ_j = p_j (ca + cb z_j) + add 1[j = y],  p_j = 2^(z_j k - L2)
+        // dZ_j = p_j (ca + cb z_j) + cc G 1[j = y],  p_j = 2^(z_j k - L2)
         const float cc = (msk && !bad) ? cscale : 0.0f;
         const float ca = cc * (-tt.G + a.s.gamma * (H - lse));
         const float cb = cc * a.s.gamma * a.s.invT;
-        const float add = cc * tt.G;
         const float L2 = tot.m * k + __log2f(tot.s);
         const bool zero = (cc == 0.0f) || (ca == 0.0f && cb == 0.0f);
         const bool fold = !zero && (cb == 0.0f);
         // fold: p_j ca = sign(ca) 2^(z_j k - L2 + log2|ca|)
         const float off = fold ? (__log2f(fabsf(ca)) - L2) : -L2;
-        bc[0] = make_float4(off, ca, cb, add);
+        bc[0] = make_float4(off, ca, cb, 0.0f);
+        bc[1] = make_float4(logp, H, cc, tt.G);
         bci[0] = make_int4(zero, fold, (fold && ca < 0.0f) ? 1 : 0,
                            (owner == crank && !zero) ? y - lo : -1);
       }
@@ -306,6 +345,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_sweep(const SweepArgs a) {
                    (row * a.ld_out + lo) * static_cast<long long>(Out::kSize);
       const int nvo = a.out_vec ? n_vec : 0;
       const int vo_elems = nvo * V8;
+      const float2 k2 = make_float2(k, k);
+      const float2 off2 = make_float2(c.x, c.x);
       if (ci.x) {
         float zf[V8];
 #pragma unroll
@@ -314,28 +355,40 @@ __global__ void __launch_bounds__(kThreads, 1) k_sweep(const SweepArgs a) {
           Out::template storev<V8>(drow + static_cast<size_t>(v) * V8 * Out::kSize, zf, 0u);
         for (int j = vo_elems + tid; j < cnt; j += kThreads) Out::store1(drow, j, 0.0f);
       } else if (ci.y) {
-        const uint32_t sgn = ci.z ? Out::kSignMask : 0u;
+        // p_j ca with |ca| folded into the exponent; the sign is applied
+        // when packing (a negated operand costs no instruction).
+        auto fold_loop = [&](auto neg) {
+          constexpr bool kNeg = decltype(neg)::value;
 #pragma unroll 2
-        for (int v = tid; v < nvo; v += kThreads) {
-          float f[V8];
-          In::unpack(sv[v], f);
+          for (int v = tid; v < nvo; v += kThreads) {
+            float2 f[P];
+            In::unpack2(sv[v], f);
 #pragma unroll
-          for (int e = 0; e < V8; ++e) f[e] = ex2(fmaf(f[e], k, c.x));
-          Out::template storev<V8>(drow + static_cast<size_t>(v) * V8 * Out::kSize, f, sgn);
-        }
+            for (int e = 0; e < P; ++e) {
+              f[e] = ex2x2(ffma2(f[e], k2, off2));
+              if (kNeg) f[e] = make_float2(-f[e].x, -f[e].y);
+            }
+            Out::template storev<V8>(drow + static_cast<size_t>(v) * V8 * Out::kSize,
+                                     reinterpret_cast<const float*>(f), 0u);
+          }
+        };
+        if (ci.z) fold_loop(std::true_type{}); else fold_loop(std::false_type{});
         for (int j = vo_elems + tid; j < cnt; j += kThreads) {
           const float z = (j < vec_elems) ? In::load1(sb, j) : In::load1(grow, j);
           const float x = ex2(fmaf(z, k, c.x));
           Out::store1(drow, j, ci.z ? -x : x);
         }
       } else {
+        const float2 ca2 = make_float2(c.y, c.y), cb2 = make_float2(c.z, c.z);
 #pragma unroll 2
         for (int v = tid; v < nvo; v += kThreads) {
-          float f[V8];
-          In::unpack(sv[v], f);
+          float2 f[P];
+          In::unpack2(sv[v], f);
 #pragma unroll
-          for (int e = 0; e < V8; ++e) f[e] = ex2(fmaf(f[e], k, c.x)) * fmaf(c.z, f[e], c.y);
-          Out::template storev<V8>(drow + static_cast<size_t>(v) * V8 * Out::kSize, f, 0u);
+          for (int e = 0; e < P; ++e)
+            f[e] = fmul2(ex2x2(ffma2(f[e], k2, off2)), ffma2(cb2, f[e], ca2));
+          Out::template storev<V8>(drow + static_cast<size_t>(v) * V8 * Out::kSize,
+                                   reinterpret_cast<const float*>(f), 0u);
         }
         for (int j = vo_elems + tid; j < cnt; j += kThreads) {
           const float z = (j < vec_elems) ? In::load1(sb, j) : In::load1(grow, j);
@@ -344,17 +397,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_sweep(const SweepArgs a) {
       }
       __syncthreads();
       if (tid == 0 && ci.w >= 0) {
-        // the sampled token's entry gets + cc G (the one-hot term)
-        const int jl = ci.w;
-        const float z = (jl < vec_elems) ? In::load1(sb, jl) : In::load1(grow, jl);
-        float x;
-        if (ci.y) {
-          x = ex2(fmaf(z, k, c.x));
-          if (ci.z) x = -x;
-        } else {
-          x = ex2(fmaf(z, k, c.x)) * fmaf(c.z, z, c.y);
-        }
-        Out::store1(drow, jl, x + c.w);
+        // The sampled token's entry: cc [G (1 - p_y) + gamma p_y (log p_y + H)],
+        // with 1 - p_y = -expm1(logp) so that p_y close to 1 keeps its
+        // relative accuracy.
+        const float4 ex = bc[1];  // logp, H, cc, G
+        const float py = expf(ex.x);
+        const float x = ex.z * (ex.w * -expm1f(ex.x) + a.s.gamma * py * (ex.x + ex.y));
+        Out::store1(drow, ci.w, x);
       }
     }
 
@@ -375,23 +424,27 @@ __global__ void __launch_bounds__(kThreads, 1) k_sweep(const SweepArgs a) {
       if (iss_any & (1u << s))
         mbar_wait_bounded(smem_u32(&bars[s]), ((iss_par >> s) & 1u) ^ 1u, kWaitLimitNs);
   }
-  // No CTA may leave while a peer can still read its exchange slot.
+  // No CTA leaves while a peer's last exchange store into it may be in flight.
   if (C > 1) cluster_sync_all();
+}
+
+template <class In, class Out, bool kGrad>
+const void* pick(int threads) {
+  switch (threads) {
+    case 256: return reinterpret_cast<const void*>(&k_sweep<In, Out, kGrad, 256, 4>);
+    case 255: return reinterpret_cast<const void*>(&k_sweep<In, Out, kGrad, 256, 5>);  // 5 per SM
+    default: return reinterpret_cast<const void*>(&k_sweep<In, Out, kGrad, 512, 2>);
+  }
 }
 
 }  // namespace
 
-template <class In, class Out, bool kGrad>
-static const void* sweep_fn() {
-  return reinterpret_cast<const void*>(&k_sweep<In, Out, kGrad>);
-}
-
-const void* sweep_kernel(rl_dtype in, rl_dtype out, bool grad) {
-  if (!grad) return in == RL_BF16 ? sweep_fn<InBf16, OutBf16, false>()
-                                  : sweep_fn<InF32, OutF32, false>();
-  if (in == RL_BF16) return out == RL_BF16 ? sweep_fn<InBf16, OutBf16, true>()
-                                           : sweep_fn<InBf16, OutF32, true>();
-  return out == RL_BF16 ? sweep_fn<InF32, OutBf16, true>() : sweep_fn<InF32, OutF32, true>();
+const void* sweep_kernel(rl_dtype in, rl_dtype out, bool grad, int threads) {
+  if (!grad) return in == RL_BF16 ? pick<InBf16, OutBf16, false>(threads)
+                                  : pick<InF32, OutF32, false>(threads);
+  if (in == RL_BF16) return out == RL_BF16 ? pick<InBf16, OutBf16, true>(threads)
+                                           : pick<InBf16, OutF32, true>(threads);
+  return out == RL_BF16 ? pick<InF32, OutBf16, true>(threads) : pick<InF32, OutF32, true>(threads);
 }
 
 }  // namespace milesloss

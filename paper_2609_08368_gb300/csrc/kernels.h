@@ -5,8 +5,8 @@
 
 namespace milesloss {
 
-constexpr int kSweepThreads = 512;
 constexpr int kMaxStages = 4;
+constexpr int kMaxCluster = 8;
 constexpr uint32_t kBulkChunk = 16384;    // bytes per cp.async.bulk
 constexpr int kSweepSmemExtra = 1024;     // mbarriers + exchange + reduction scratch
 constexpr int kAdvThreads = 1024;
@@ -81,7 +81,7 @@ struct BwdArgs {
 constexpr int kBwdTile = kBwdThreads * 8 * 4;  // elements of one row per tile
 
 // Kernel entry points (device function pointers usable with cudaLaunchKernelEx).
-const void* sweep_kernel(rl_dtype in, rl_dtype out, bool grad);
+const void* sweep_kernel(rl_dtype in, rl_dtype out, bool grad, int threads);
 const void* bwd_kernel(rl_dtype in, rl_dtype out);
 const void* adv_kernel();
 const void* stats_kernel();
