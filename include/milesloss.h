@@ -198,6 +198,35 @@ rl_status rl_loss_fwd_bwd(const void* logits, rl_dtype logits_dtype, int64_t n_r
                           rl_dtype dlogits_dtype, int64_t ld_out, void* workspace,
                           size_t workspace_bytes, rl_stream stream);
 
+/* rl_loss_fwd_bwd for callers that cannot allocate device memory at call
+ * time (the paper has no counterpart; this is a deployment convenience).
+ * Frameworks that reserve nearly all of HBM for their own pool, plain-C
+ * hosts and plugins without access to the process's allocator, and code
+ * whose memory footprint must stay fixed after start-up cannot provide a
+ * workspace; this call takes every other argument of rl_loss_fwd_bwd and
+ * uses an 8 MiB array compiled into the library instead (about 200,000 rows
+ * at small trajectory and group counts). Larger calls return
+ * RL_ERR_WORKSPACE_TOO_SMALL before anything is enqueued. Each device on
+ * which the library's code is loaded keeps the array until the process
+ * exits. The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress, with that device current): make it before any
+ * stream capture. No call allocates or frees memory. All calls on a device
+ * share the array: calls that overlap on the GPU race and must be
+ * serialised by the caller; what must start at zero is reset by every
+ * call. The device-side error word is kept in the array and cannot be read
+ * back; rows with a bad target still get zeros. */
+rl_status rl_loss_fwd_bwd_noalloc(const void* logits, rl_dtype logits_dtype, int64_t n_rows,
+                                  int64_t vocab, int64_t ld, const int32_t* targets,
+                                  const float* rollout_logprobs, const float* ref_logprobs,
+                                  const float* old_logprobs, const float* teacher_logprobs,
+                                  const float* rewards, const int32_t* group_id,
+                                  const int32_t* cu_seqlens, int32_t n_traj, int32_t n_groups,
+                                  const uint8_t* loss_mask, const rl_loss_params* params,
+                                  float* token_logprobs, float* entropy, float* advantages,
+                                  int32_t* group_sizes, rl_loss_stats* stats, float grad_loss,
+                                  const float* grad_loss_device, void* dlogits,
+                                  rl_dtype dlogits_dtype, int64_t ld_out, rl_stream stream);
+
 /* After the stream that ran a call on `workspace` has been synchronised:
  * RL_OK, or the data-dependent error the kernels recorded (when several
  * kinds occurred, the lowest code). Performs one small blocking
