@@ -35,8 +35,8 @@ sys.path.insert(0, ROOT)
 METRIC = "RL-loss fwd+bwd tokens/sec at vocab 154,880 bf16; achieved HBM GB/s vs 8 TB/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
-PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "sweep_kernel_glm.md")
-SWEEP_SOURCES = ["k_sweep.cu", "common.cuh", "kernels.h"]
+PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "stream_kernel_glm.md")
+SWEEP_SOURCES = ["k_stream.cu", "common.cuh", "kernels.h", "abi.cu"]
 
 
 def parse_args():
@@ -392,7 +392,7 @@ def run_ours(args, rank, world, local):
                    "l2": "inputs larger than L2 (20+ GB per step), no flush"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
-                     "kernel": "k_sweep (fused fwd+bwd vocabulary sweep)",
+                     "kernel": "k_stream (fused fwd+bwd vocabulary sweep, one CTA per row)",
                      "bytes_per_launch": launch_bytes, "sweep_ms": sweep_avg,
                      "peak_kind": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"
                      if peak_kind == "measured" else "fallback 6.8 TB/s",

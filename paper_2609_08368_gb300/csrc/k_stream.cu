@@ -1,0 +1,468 @@
+// The vocabulary sweep for long rows, one CTA per row: the same per-row
+// results as k_sweep (log-softmax statistics, log-prob, entropy, per-token
+// objective, dLogits), with no exchange between CTAs.
+//
+// A CTA is warp-specialised. One producer warp streams the row in chunks
+// (bulk async copies, non-multicast) into a ring of shared-memory slots,
+// each slot with a "full" mbarrier (transaction bytes) and an "empty"
+// mbarrier (one arrival per consumer warp). The producer walks the task list
+// row by row: the chunks of the row for pass A, then the same chunks again
+// for pass B. Pass A's copies are marked evict-last in L2 and pass B's
+// evict-first: with one CTA per SM only ~one row per SM is live (~46 MB on
+// the headline workload, against a 126 MB L2), so the second read of a row
+// is served by L2 and HBM sees each logit once (checked with the DRAM byte
+// counters). The sixteen consumer warps:
+//   pass A  per chunk, each thread folds its vectors into an online
+//           (max, S, U) in packed f32x2 (rescaling when its maximum grows),
+//           then releases the slot;
+//   merge   butterfly merges, maximum first, in a fixed order;
+//   epilogue one thread evaluates the per-token objective and the gradient
+//           coefficients;
+//   pass B  per chunk, dLogits from the re-read chunk, 16-byte streaming
+//           stores; the sampled token's entry is rewritten during the next
+//           row's epilogue (after a barrier that orders every store before it).
+// Definitions: Sec. 3.4 (ratio), Sec. 2 / 9.1 (advantage), Sec. 2.4 (mask).
+#include <type_traits>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace milesloss {
+
+namespace {
+
+constexpr int kCons = kStreamConsumers;   // consumer threads
+constexpr int kConsWarps = kCons / 32;
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+constexpr float kLn2f = 0.69314718055994531f;
+
+__device__ __forceinline__ void cons_sync() {
+  asm volatile("bar.sync 1, %0;" ::"r"(kCons) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+struct Tri {
+  float m, s, u;
+};
+
+__device__ __forceinline__ Tri warp_merge(Tri t, float k) {
+  float M = t.m;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  float s = 0.0f, u = 0.0f;
+  if (t.s > 0.0f) {
+    const float d = (t.m - M) * k, f = ex2(d);
+    s = f * t.s;
+    u = f * fmaf(d, t.s, t.u);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    s += __shfl_xor_sync(0xffffffffu, s, o);
+    u += __shfl_xor_sync(0xffffffffu, u, o);
+  }
+  return Tri{M, s, u};
+}
+
+// Running (max, sums) of one thread over the chunks of a row.
+struct Run {
+  float m = -INFINITY, mt = -INFINITY;
+  float2 s0 = {0.0f, 0.0f}, s1 = {0.0f, 0.0f}, u0 = {0.0f, 0.0f}, u1 = {0.0f, 0.0f};
+
+  __device__ __forceinline__ void raise(float cm, float k) {
+    if (!(cm > m)) return;
+    if (m != -INFINITY) {
+      const float d = (m - cm) * k, f = ex2(d);
+      const float2 f2 = make_float2(f, f), d2 = make_float2(d, d);
+      u0 = fmul2(f2, ffma2(d2, s0, u0));
+      u1 = fmul2(f2, ffma2(d2, s1, u1));
+      s0 = fmul2(f2, s0);
+      s1 = fmul2(f2, s1);
+    }
+    m = cm;
+    mt = cm * k;
+  }
+  template <bool kSafe>
+  __device__ __forceinline__ void add_pair(float2 z, float2 k2, float2& s, float2& u) {
+    float2 t = ffma2(z, k2, make_float2(-mt, -mt));
+    if (kSafe) {
+      if (z.x == -INFINITY) t.x = -127.0f;
+      if (z.y == -INFINITY) t.y = -127.0f;
+    }
+    const float2 x = ex2x2(t);
+    s = fadd2(s, x);
+    u = ffma2(x, t, u);
+  }
+  __device__ __forceinline__ Tri tri() const {
+    const float2 s = fadd2(s0, s1), u = fadd2(u0, u1);
+    return Tri{m, s.x + s.y, u.x + u.y};
+  }
+};
+
+// dLogits of one chunk with vector stores. kMode 0: p ca with |ca| folded
+// into the exponent; 1: the same negated; 2: p (ca + cb z).
+template <class In, class Out, int kMode>
+__device__ __forceinline__ void pass_b_chunk(const uint4* sv, int nv, char* dchunk, float2 k2,
+                                             float2 off2, float2 ca2, float2 cb2) {
+  constexpr int V8 = In::kVec;
+  constexpr int P = V8 / 2;
+#pragma unroll 2
+  for (int v = threadIdx.x; v < nv; v += kCons) {
+    float2 f[P];
+    In::unpack2(sv[v], f);
+#pragma unroll
+    for (int e = 0; e < P; ++e) {
+      if (kMode == 2) {
+        f[e] = fmul2(ex2x2(ffma2(f[e], k2, off2)), ffma2(cb2, f[e], ca2));
+      } else {
+        f[e] = ex2x2(ffma2(f[e], k2, off2));
+        if (kMode == 1) f[e] = make_float2(-f[e].x, -f[e].y);
+      }
+    }
+    Out::template storev<V8>(dchunk + static_cast<size_t>(v) * V8 * Out::kSize,
+                             reinterpret_cast<const float*>(f), 0u);
+  }
+}
+
+template <class In, class Out, bool kGrad>
+__global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const StreamArgs a) {
+  using St = typename In::storage;
+  constexpr int V8 = In::kVec;
+  constexpr int P = V8 / 2;
+  extern __shared__ __align__(128) unsigned char smem[];
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5, lane = tid & 31;
+  const int NS = a.n_slots;
+  const int CB = a.chunk_bytes;
+  const int CV = CB / 16;                        // vectors per full chunk
+  const int row_vec = a.V / V8;                  // whole 16-byte vectors per row
+  const int tail0 = row_vec * V8;                // first element not in a vector
+  const int n_chunks = (row_vec + CV - 1) / CV;
+  const float k = a.s.k;
+
+  unsigned char* ring = smem;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(NS) * CB);
+  uint64_t* empty = full + kMaxSlots;
+  float4* red = reinterpret_cast<float4*>(empty + kMaxSlots);  // [kConsWarps]
+  float4* bc = red + kConsWarps;                                // [2]
+  int4* bci = reinterpret_cast<int4*>(bc + 2);                  // [1]
+
+  if (tid == 0) {
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), kConsWarps);
+    }
+    fence_mbar_init();
+  }
+  __syncthreads();
+
+  WsPtrs ws = a.ws;
+  const char* lg = static_cast<const char*>(a.logits);
+  const long long rows_mine = (a.R > blockIdx.x) ? (a.R - 1 - blockIdx.x) / gridDim.x + 1 : 0;
+
+  if (warp == kConsWarps) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      const uint64_t pol_a = l2_policy_evict_last(), pol_b = l2_policy_evict_first();
+      bool dead = false;
+      long long q = 0;
+      for (long long i = 0; i < rows_mine && !dead; ++i) {
+        const long long row = blockIdx.x + i * gridDim.x;
+        const char* src_row = lg + row * a.ld * static_cast<long long>(sizeof(St));
+        // a row that does not train has an all-zero gradient: no second read
+        const int tasks = (kGrad && a.mask[row]) ? 2 * n_chunks : n_chunks;
+        for (int t = 0; t < tasks; ++t, ++q) {
+          const int c = t % n_chunks;
+          const int s = static_cast<int>(q % NS);
+          if (q >= NS &&
+              !mbar_wait_bounded(smem_u32(&empty[s]), static_cast<uint32_t>(((q / NS) - 1) & 1),
+                                 kWaitLimitNs)) {
+            dead = true;
+            atomicOr(&ws.hdr->err_bits, kErrTimeout);
+            break;
+          }
+          const int v0 = c * CV;
+          const uint32_t bytes = static_cast<uint32_t>(min(CV, row_vec - v0)) * 16u;
+          const uint32_t bar = smem_u32(&full[s]);
+          mbar_arrive_expect_tx(bar, bytes);
+          bulk_g2s(smem_u32(ring + static_cast<size_t>(s) * CB), src_row + static_cast<size_t>(v0) * 16,
+                   bytes, bar, t < n_chunks ? pol_a : pol_b);
+        }
+      }
+      // A timeout leaves copies in flight: wait (bounded) for the last one
+      // issued into each slot before the CTA can exit.
+      if (dead) {
+        for (int s = 0; s < NS; ++s) {
+          if (q > s) {
+            const long long last = q - 1 - ((q - 1 - s) % NS);
+            mbar_wait_bounded(smem_u32(&full[s]), static_cast<uint32_t>((last / NS) & 1),
+                              kWaitLimitNs);
+          }
+        }
+      }
+    }
+    return;
+  }
+
+  // -------------------------------------------------------------- consumers
+  const long long N = ws.hdr->n_tokens;
+  float g = a.grad_loss;
+  if (a.grad_loss_dev) g *= *a.grad_loss_dev;
+  const float cscale = (N > 0) ? g / static_cast<float>(N) * a.s.invT : 0.0f;
+  const float2 k2 = make_float2(k, k);
+  bool dead = false;
+  // the sampled token's dLogit of the previous row, written after the next
+  // barrier (so after every store of that row)
+  char* fix_ptr = nullptr;
+  float fix_val = 0.0f;
+
+  auto wait_slot = [&](long long q) {
+    const int s = static_cast<int>(q % NS);
+    if (!dead &&
+        !mbar_wait_bounded(smem_u32(&full[s]), static_cast<uint32_t>((q / NS) & 1), kWaitLimitNs)) {
+      dead = true;
+      atomicOr(&ws.hdr->err_bits, kErrTimeout);
+    }
+    return reinterpret_cast<const uint4*>(ring + static_cast<size_t>(s) * CB);
+  };
+  auto release_slot = [&](long long q) {
+    __syncwarp();
+    if (lane == 0) mbar_arrive(smem_u32(&empty[q % NS]));
+  };
+
+  long long q0 = 0;  // task number of the row's first chunk (same count as the producer's)
+  for (long long i = 0; i < rows_mine; ++i) {
+    const long long row = blockIdx.x + i * gridDim.x;
+    const char* grow = lg + row * a.ld * static_cast<long long>(sizeof(St));
+    const bool trains = a.mask[row] != 0;
+
+    int y = 0;
+    float rho = 0.0f, q = 0.0f, old = 0.0f, A = 0.0f, zy = 0.0f;
+    uint8_t msk = 0;
+    bool yok = false;
+    if (tid == 0) {
+      y = a.targets[row];
+      rho = a.rho[row];
+      if (a.q) q = a.q[row];
+      if (a.old) old = a.old[row];
+      A = ws.a_row[row];
+      msk = a.mask[row];
+      yok = (y >= 0) && (y < a.V);
+      if (yok && y >= tail0) zy = In::load1(grow, y);
+    }
+    const int yv = yok ? y / V8 : -1;  // thread 0 only
+
+    // ---------------- pass A
+    Run run;
+    for (int c = 0; c < n_chunks; ++c) {
+      const uint4* sv = wait_slot(q0 + c);
+      const int nv = min(CV, row_vec - c * CV);
+      uint4 w[2];
+      int nw = 0;
+      typename In::MaxAcc macc = In::kMaxInit;
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        const int v = tid + r * kCons;
+        if (v < nv) {
+          w[r] = sv[v];
+          macc = In::max_acc(macc, w[r]);
+          nw = r + 1;
+        }
+      }
+      for (int v = tid + 2 * kCons; v < nv; v += kCons) macc = In::max_acc(macc, sv[v]);
+      if (tid == 0 && yv >= c * CV && yv < c * CV + nv) zy = In::load1(sv, y - c * CV * V8);
+      run.raise(In::max_val(macc), k);
+      if (run.m != -INFINITY) {
+        const Run keep = run;
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          if (r < nw) {
+            float2 f[P];
+            In::unpack2(w[r], f);
+#pragma unroll
+            for (int e = 0; e < P; ++e) run.add_pair<false>(f[e], k2, (e & 1) ? run.s1 : run.s0,
+                                                            (e & 1) ? run.u1 : run.u0);
+          }
+        }
+        for (int v = tid + 2 * kCons; v < nv; v += kCons) {
+          float2 f[P];
+          In::unpack2(sv[v], f);
+#pragma unroll
+          for (int e = 0; e < P; ++e) run.add_pair<false>(f[e], k2, run.s0, run.u0);
+        }
+        const Tri cur = run.tri();
+        if (__isnanf(cur.u) || __isnanf(cur.s)) {
+          // -inf logits in this chunk: redo it, skipping them exactly
+          run = keep;
+          for (int v = tid; v < nv; v += kCons) {
+            float2 f[P];
+            In::unpack2(sv[v], f);
+#pragma unroll
+            for (int e = 0; e < P; ++e) run.add_pair<true>(f[e], k2, run.s0, run.u0);
+          }
+        }
+      }
+      release_slot(q0 + c);
+    }
+    Tri t = run.tri();
+    for (int j = tail0 + tid; j < a.V; j += kCons) {
+      const float z = In::load1(grow, j);
+      if (z == -INFINITY) continue;
+      if (z > t.m) {
+        if (t.s > 0.0f) {
+          const float d = (t.m - z) * k, f = ex2(d);
+          t.u = f * fmaf(d, t.s, t.u);
+          t.s *= f;
+        }
+        t.m = z;
+      }
+      const float tt = fmaf(z, k, -t.m * k), x = ex2(tt);
+      t.s += x;
+      t.u = fmaf(x, tt, t.u);
+    }
+
+    // ---------------- merge
+    t = warp_merge(t, k);
+    if (lane == 0) red[warp] = make_float4(t.m, t.s, t.u, 0.0f);
+    cons_sync();
+    if (tid == 0 && fix_ptr) Out::store1(fix_ptr, 0, fix_val);  // previous row's y entry
+    fix_ptr = nullptr;
+    if (warp == 0) {
+      Tri x{-INFINITY, 0.0f, 0.0f};
+      if (lane < kConsWarps) {
+        const float4 v = red[lane];
+        x = Tri{v.x, v.y, v.z};
+      }
+      t = warp_merge(x, k);
+    }
+
+    // ---------------- epilogue (thread 0)
+    char* drow = kGrad ? static_cast<char*>(a.dlogits) +
+                             row * a.ld_out * static_cast<long long>(Out::kSize)
+                       : nullptr;
+    if (tid == 0) {
+      const bool bad = !yok;
+      if (bad) atomicOr(&ws.hdr->err_bits, kErrTarget);
+      const float lnS = logf(t.s);
+      const float lse = t.m * a.s.invT + lnS;
+      float H = lnS - t.u * kLn2f / t.s;
+      float logp = zy * a.s.invT - lse;
+      if (bad) { logp = 0.0f; H = 0.0f; }
+      TokenTerms tt = token_terms(logp, H, rho, q, a.q != nullptr, old, a.old != nullptr, A, a.s);
+      if (bad) tt = TokenTerms{0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, kFlagBad};
+      if (a.out_logp) a.out_logp[row] = logp;
+      if (a.out_H) a.out_H[row] = H;
+      ws.logp[row] = logp;
+      ws.H[row] = H;
+      ws.lse[row] = lse;
+      ws.G[row] = tt.G;
+      ws.ell[row] = tt.ell;
+      ws.pg[row] = tt.pg;
+      ws.k3[row] = tt.k3;
+      ws.r[row] = tt.r;
+      ws.rc[row] = tt.rc;
+      ws.flags[row] = tt.flags;
+      if (kGrad) {
+        const float cc = (msk && !bad) ? cscale : 0.0f;
+        const float ca = cc * (-tt.G + a.s.gamma * (H - lse));
+        const float cb = cc * a.s.gamma * a.s.invT;
+        const float L2 = t.m * k + __log2f(t.s);
+        const bool zero = (cc == 0.0f) || (ca == 0.0f && cb == 0.0f);
+        const bool fold = !zero && (cb == 0.0f);
+        const float off = fold ? (__log2f(fabsf(ca)) - L2) : -L2;
+        bc[0] = make_float4(off, ca, cb, 0.0f);
+        bci[0] = make_int4(zero, fold, (fold && ca < 0.0f) ? 1 : 0, 0);
+        if (!zero) {
+          // cc [G (1 - p_y) + gamma p_y (log p_y + H)], 1 - p_y = -expm1(logp)
+          fix_ptr = drow + static_cast<long long>(y) * Out::kSize;
+          fix_val = cc * (tt.G * -expm1f(logp) + a.s.gamma * expf(logp) * (logp + H));
+        }
+      }
+    }
+    cons_sync();
+
+    // ---------------- pass B
+    if (kGrad) {
+      const float4 cf = bc[0];
+      const int4 ci = bci[0];
+      const float2 off2 = make_float2(cf.x, cf.x);
+      const float2 ca2 = make_float2(cf.y, cf.y), cb2 = make_float2(cf.z, cf.z);
+      const bool vec_out = a.out_vec != 0;
+      for (int c = 0; c < n_chunks; ++c) {
+        const long long qq = q0 + n_chunks + c;
+        const int nv = min(CV, row_vec - c * CV);
+        char* dchunk = drow + static_cast<long long>(c) * CV * V8 * Out::kSize;
+        if (ci.x) {
+          // zero gradient: the chunk's data is not needed; a training row's
+          // chunk was still copied, so its slot is waited on and released to
+          // keep the ring in step with the producer
+          if (trains) wait_slot(qq);
+          float zf[V8];
+#pragma unroll
+          for (int e = 0; e < V8; ++e) zf[e] = 0.0f;
+          for (int v = tid; v < nv; v += kCons) {
+            if (vec_out) Out::template storev<V8>(dchunk + static_cast<size_t>(v) * V8 * Out::kSize, zf, 0u);
+            else for (int e = 0; e < V8; ++e) Out::store1(dchunk, v * V8 + e, 0.0f);
+          }
+          if (trains) release_slot(qq);
+          continue;
+        }
+        const uint4* sv = wait_slot(qq);
+        if (vec_out) {
+          if (!ci.y) pass_b_chunk<In, Out, 2>(sv, nv, dchunk, k2, off2, ca2, cb2);
+          else if (ci.z) pass_b_chunk<In, Out, 1>(sv, nv, dchunk, k2, off2, ca2, cb2);
+          else pass_b_chunk<In, Out, 0>(sv, nv, dchunk, k2, off2, ca2, cb2);
+        } else {
+          for (int v = tid; v < nv; v += kCons) {
+            float2 f[P];
+            In::unpack2(sv[v], f);
+#pragma unroll
+            for (int e = 0; e < P; ++e) {
+              f[e] = ci.y ? ex2x2(ffma2(f[e], k2, off2))
+                          : fmul2(ex2x2(ffma2(f[e], k2, off2)), ffma2(cb2, f[e], ca2));
+              if (ci.y && ci.z) f[e] = make_float2(-f[e].x, -f[e].y);
+            }
+            const float* fv = reinterpret_cast<const float*>(f);
+            for (int e = 0; e < V8; ++e) Out::store1(dchunk, v * V8 + e, fv[e]);
+          }
+        }
+        release_slot(qq);
+      }
+      for (int j = tail0 + tid; j < a.V; j += kCons) {
+        const float z = In::load1(grow, j);
+        float x = 0.0f;
+        if (!ci.x) {
+          x = ci.y ? ex2(fmaf(z, k, cf.x)) : ex2(fmaf(z, k, cf.x)) * fmaf(cf.z, z, cf.y);
+          if (ci.y && ci.z) x = -x;
+        }
+        Out::store1(drow, j, x);
+      }
+    }
+    q0 += (kGrad && trains) ? 2 * n_chunks : n_chunks;
+  }
+  cons_sync();
+  if (tid == 0 && fix_ptr) Out::store1(fix_ptr, 0, fix_val);
+}
+
+template <class In, class Out, bool kGrad>
+const void* fn() {
+  return reinterpret_cast<const void*>(&k_stream<In, Out, kGrad>);
+}
+
+}  // namespace
+
+const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad) {
+  if (!grad) return in == RL_BF16 ? fn<InBf16, OutBf16, false>() : fn<InF32, OutF32, false>();
+  if (in == RL_BF16) return out == RL_BF16 ? fn<InBf16, OutBf16, true>() : fn<InBf16, OutF32, true>();
+  return out == RL_BF16 ? fn<InF32, OutBf16, true>() : fn<InF32, OutF32, true>();
+}
+
+}  // namespace milesloss

@@ -11,6 +11,8 @@ constexpr uint32_t kBulkChunk = 16384;    // bytes per cp.async.bulk
 constexpr int kSweepSmemExtra = 1024;     // mbarriers + exchange + reduction scratch
 constexpr int kAdvThreads = 1024;
 constexpr int kBwdThreads = 256;
+constexpr int kStreamConsumers = 512;     // consumer threads of k_stream (+ one producer warp)
+constexpr int kMaxSlots = 16;             // ring slots of k_stream
 
 struct SweepArgs {
   const void* logits;
@@ -20,6 +22,28 @@ struct SweepArgs {
   int stages;       // ring depth S
   int stage_bytes;  // bytes per stage (multiple of 128)
   int in_bulk;      // rows are 16-byte aligned: bulk-copy path
+  int out_vec;      // dLogits rows are 16-byte aligned: vector stores
+  const int* targets;
+  const float* rho;
+  const float* q;
+  const float* old;
+  const uint8_t* mask;
+  float* out_logp;
+  float* out_H;
+  void* dlogits;
+  long long ld_out;
+  float grad_loss;
+  const float* grad_loss_dev;
+  LossScalars s;
+  WsPtrs ws;
+};
+
+struct StreamArgs {
+  const void* logits;
+  long long ld, R;
+  int V;
+  int chunk_bytes;  // bytes per ring slot (multiple of 128)
+  int n_slots;      // ring depth
   int out_vec;      // dLogits rows are 16-byte aligned: vector stores
   const int* targets;
   const float* rho;
@@ -82,6 +106,7 @@ constexpr int kBwdTile = kBwdThreads * 8 * 4;  // elements of one row per tile
 
 // Kernel entry points (device function pointers usable with cudaLaunchKernelEx).
 const void* sweep_kernel(rl_dtype in, rl_dtype out, bool grad, int threads);
+const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad);
 const void* bwd_kernel(rl_dtype in, rl_dtype out);
 const void* adv_kernel();
 const void* stats_kernel();

@@ -37,6 +37,9 @@ def _no_overrides(monkeypatch):
     monkeypatch.delenv("MILESLOSS_SWEEP_STAGES", raising=False)
     monkeypatch.delenv("MILESLOSS_SWEEP_THREADS", raising=False)
     monkeypatch.delenv("MILESLOSS_SWEEP_CTAS_PER_SM", raising=False)
+    monkeypatch.delenv("MILESLOSS_SWEEP_KIND", raising=False)
+    monkeypatch.delenv("MILESLOSS_STREAM_CHUNK", raising=False)
+    monkeypatch.delenv("MILESLOSS_STREAM_SLOTS", raising=False)
 
 
 def _full_check(w, mode="fused", dl_dtype=None, params=None):
@@ -52,6 +55,31 @@ def _full_check(w, mode="fused", dl_dtype=None, params=None):
 @pytest.mark.parametrize("name", list(SHRUNK))
 def test_parity_fused(name):
     _full_check(wl.make(SHRUNK[name], DEV))
+
+
+@pytest.mark.parametrize("kind", ["cluster", "stream"])
+@pytest.mark.parametrize("name", list(SHRUNK))
+def test_parity_each_sweep_kernel(monkeypatch, kind, name):
+    """Both vocabulary-sweep kernels (cluster exchange, and one CTA per row
+    with an L2-served second read) on every workload."""
+    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+    _full_check(wl.make(SHRUNK[name], DEV))
+    _full_check(wl.make(SHRUNK[name], DEV), mode="split")
+
+
+@pytest.mark.parametrize("chunk,slots", [(16384, 14), (4096, 2), (12288, 3), (1024, 1),
+                                         (65536, 3)])
+def test_stream_ring_shapes(monkeypatch, chunk, slots):
+    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", "stream")
+    monkeypatch.setenv("MILESLOSS_STREAM_CHUNK", str(chunk))
+    monkeypatch.setenv("MILESLOSS_STREAM_SLOTS", str(slots))
+    # ragged rows: 45,003 bf16 columns = 5,625 vectors and a 3-element tail
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=24, vocab=45003,
+                    rho_noise=0.3)
+    _full_check(wl.make(rec, DEV))
+    rec = wl.shrink(wl.RECIPES["fp32"], n_prompts=1, group_size=4, traj_len=16, vocab=20001,
+                    rho_noise=0.3)
+    _full_check(wl.make(rec, DEV))
 
 
 @pytest.mark.parametrize("name", ["tiny", "fp32", "glm_noisy"])
@@ -83,6 +111,7 @@ def test_dlogits_relative_error_on_order_p_entries():
 
 @pytest.mark.parametrize("cluster", [1, 2, 4, 8])
 def test_every_cluster_size(monkeypatch, cluster):
+    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", "cluster")
     monkeypatch.setenv("MILESLOSS_SWEEP_CLUSTER", str(cluster))
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=24, vocab=20000 + 24)
     _full_check(wl.make(rec, DEV))
@@ -90,6 +119,7 @@ def test_every_cluster_size(monkeypatch, cluster):
 
 @pytest.mark.parametrize("threads,per_sm", [(256, 4), (256, 5), (512, 2)])
 def test_every_block_shape(monkeypatch, threads, per_sm):
+    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", "cluster")
     monkeypatch.setenv("MILESLOSS_SWEEP_THREADS", str(threads))
     monkeypatch.setenv("MILESLOSS_SWEEP_CTAS_PER_SM", str(per_sm))
     _full_check(wl.make(SHRUNK["glm_noisy"], DEV))
@@ -97,6 +127,7 @@ def test_every_block_shape(monkeypatch, threads, per_sm):
 
 @pytest.mark.parametrize("stages", [1, 2, 3, 4])
 def test_every_ring_depth(monkeypatch, stages):
+    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", "cluster")
     monkeypatch.setenv("MILESLOSS_SWEEP_CLUSTER", "2")
     monkeypatch.setenv("MILESLOSS_SWEEP_STAGES", str(stages))
     rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=1, group_size=4, traj_len=40, vocab=6144)
@@ -144,7 +175,9 @@ def test_temperature_entropy_kl_correction_opd():
         _full_check(w, mode="split", params=params)
 
 
-def test_no_training_tokens_and_empty_call():
+@pytest.mark.parametrize("kind", ["cluster", "stream"])
+def test_no_training_tokens_and_empty_call(monkeypatch, kind):
+    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
     rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=1, group_size=2, traj_len=8, vocab=300)
     w = wl.make(rec, DEV)
     w.loss_mask.zero_()
@@ -172,7 +205,9 @@ def test_no_training_tokens_and_empty_call():
     np.testing.assert_allclose(buf.advantages.cpu().numpy(), [-2 ** -0.5, 2 ** -0.5], rtol=1e-6)
 
 
-def test_device_errors_are_reported_not_trapped():
+@pytest.mark.parametrize("kind", ["cluster", "stream"])
+def test_device_errors_are_reported_not_trapped(monkeypatch, kind):
+    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
     rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=2, group_size=2, traj_len=8, vocab=256)
     w = wl.make(rec, DEV)
     w.targets[3] = 256                     # outside [0, vocab)
@@ -203,10 +238,11 @@ def test_bitwise_reproducible_and_fwd_matches_fused():
     assert a["stats"] == c["stats"]
 
 
-def test_batch_invariance_of_row_outputs():
+@pytest.mark.parametrize("vocab", [30000, 40000])  # cluster kernel, streaming kernel
+def test_batch_invariance_of_row_outputs(vocab):
     """A row's log-prob and entropy do not depend on where it sits or on how
     many other rows share the call."""
-    rec = wl.shrink(wl.RECIPES["qwen"], n_prompts=2, group_size=4, traj_len=32, vocab=30000)
+    rec = wl.shrink(wl.RECIPES["qwen"], n_prompts=2, group_size=4, traj_len=32, vocab=vocab)
     w = wl.make(rec, DEV)
     full = P.run_gpu(w, mode="fwd")
     perm = torch.randperm(w.n_rows, generator=torch.Generator().manual_seed(0)).to(DEV)
