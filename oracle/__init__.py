@@ -14,6 +14,10 @@ from .rl_loss_ref import (  # noqa: F401
     group_advantages,
     row_advantages,
     shape_advantages_opd,
+    estimator_advantages,
+    training_tokens_per_trajectory,
+    opd_topk_estimate,
+    sequence_objective,
     token_objective,
     masked_token_mean,
     loss_stats,

@@ -41,6 +41,7 @@ from dataclasses import dataclass
 import numpy as np
 
 CORRECTIONS = ("none", "tis", "clip_or_pop")
+ESTIMATORS = ("grpo", "reinforcepp", "reinforcepp_baseline", "gspo")
 
 
 @dataclass(frozen=True)
@@ -60,6 +61,8 @@ class LossParams:
     corr_lo: float = 0.0
     corr_hi: float = 2.0
     opd_coef: float = 0.0         # lambda of Sec. 5.2
+    estimator: str = "grpo"       # "grpo" | "reinforcepp" | "reinforcepp_baseline" | "gspo" (Sec. 3.4)
+    opd_topk: int = 0             # K of the top-K OPD variant (Sec. 5.2), 0 = off
 
 
 # --------------------------------------------------------------------------
@@ -172,6 +175,71 @@ def shape_advantages_opd(A_row: np.ndarray, student_lp: np.ndarray,
         np.asarray(student_lp, np.float64) - np.asarray(teacher_lp, np.float64))
 
 
+def training_tokens_per_trajectory(cu_seqlens, mask) -> np.ndarray:
+    """n_i = number of training tokens (mask 1) in trajectory i."""
+    cu = np.asarray(cu_seqlens, dtype=np.int64)
+    m = np.asarray(mask).astype(bool)
+    return np.array([int(m[cu[i]:cu[i + 1]].sum()) for i in range(cu.shape[0] - 1)],
+                    dtype=np.int64)
+
+
+def estimator_advantages(w, gid, n_groups, cu_seqlens, mask, p: LossParams):
+    """Per-row advantages of the configured estimator (Sec. 3.4 names GRPO,
+    GSPO and REINFORCE++ in plain and baseline-relative forms).
+
+    grpo, gspo: the GRPO advantage of the row's trajectory.
+    reinforcepp: the trajectory's outcome reward is the return of each of its
+        tokens; reinforcepp_baseline: the reward minus its group's mean reward.
+        Either return is then normalised over all training tokens of the
+        batch: A = (b - mu) / max(sigma, floor) with mu, sigma the mean and std
+        (n - 1 if unbiased) of b over the tokens with mask 1 (centred only when
+        normalize_std is off); A = 0 everywhere when those returns are all
+        equal or no token trains.
+    Returns (A_traj [n_traj], A_row [n_rows], group sizes)."""
+    if p.estimator not in ESTIMATORS:
+        raise ValueError(p.estimator)
+    n_rows = int(np.asarray(mask).shape[0])
+    A_grpo, n_g = group_advantages(w, gid, n_groups, p)
+    if p.estimator in ("grpo", "gspo"):
+        return A_grpo, row_advantages(A_grpo, cu_seqlens, n_rows), n_g
+    w = np.asarray(w, np.float64)
+    gid = np.asarray(gid, np.int64)
+    b = w.copy()
+    if p.estimator == "reinforcepp_baseline":
+        for g in range(n_groups):
+            idx = gid == g
+            if idx.any():
+                b[idx] = w[idx] - w[idx].mean()
+    b_row = row_advantages(b, cu_seqlens, n_rows)
+    m = np.asarray(mask).astype(bool)
+    N = int(m.sum())
+    A = np.zeros_like(b)
+    if N > 0 and b_row[m].max() != b_row[m].min():
+        mu = b_row[m].mean()
+        A = b - mu
+        if p.normalize_std:
+            ddof = 1 if p.unbiased_std else 0
+            sigma = float(np.sqrt(((b_row[m] - mu) ** 2).sum() / (N - ddof))) if N > ddof else 0.0
+            A = A / max(sigma, p.std_floor)
+    return A, row_advantages(A, cu_seqlens, n_rows), n_g
+
+
+def opd_topk_estimate(z_rows, temperature, lse, cand_ids, teacher_lp):
+    """Top-K on-policy distillation signal (Sec. 5.2): the teacher scores a
+    candidate set per position; the estimate is the weighted sum, over the
+    set, of log pi_student - log pi_teacher, weighted by the student's
+    probabilities renormalised over the set (the reverse KL restricted to
+    the set). The student's log-probs are the trainer's, from the logits;
+    the estimate is a fixed per-token signal (no gradient flows through it)."""
+    s = _widen(z_rows) / float(temperature)
+    ids = np.asarray(cand_ids, np.int64)
+    rows = np.arange(s.shape[0])[:, None]
+    lps = s[rows, ids] - np.asarray(lse, np.float64)[:, None]
+    ps = np.exp(lps)
+    wts = ps / ps.sum(axis=1, keepdims=True)
+    return (wts * (lps - np.asarray(teacher_lp, np.float64))).sum(axis=1)
+
+
 # --------------------------------------------------------------------------
 # (a3) per-token objective
 # --------------------------------------------------------------------------
@@ -245,6 +313,90 @@ def token_objective(logp, rho, q, A_row, H, p: LossParams, old=None):
     G = g_pg + p.kl_coef * g_kl
     return dict(r=r, pg=pg, k3=k3, ell=ell, G=G, clip_hi=clip_hi, clip_lo=clip_lo,
                 dual=dual, wt=wt, rc=rc, corr_clip=corr_clip)
+
+
+def sequence_objective(logp, rho, q, A_traj, H, cu_seqlens, mask, p: LossParams, old=None):
+    """GSPO (Sec. 3.4 lists it among the estimators; Zheng et al. 2025): the
+    importance ratio of trajectory i is the length-normalised sequence ratio
+        s_i = exp( (1/n_i) sum_{t in i, m_t = 1} (logp_t - base_t) ),
+    clipped at the sequence level with the trajectory's GRPO advantage A_i:
+        pg_i = max(-A_i s_i, -A_i clip(s_i, 1-eps_lo, 1+eps_hi)), dual clip for
+        A_i < 0 as in the token objective;
+    the policy term is the mean of pg_i over the n_seq trajectories that have
+    training tokens, the k3 and entropy terms stay token means. Written per
+    row so that sum m l / N is that loss: a training token of trajectory i
+    carries l_t = (N / (n_seq n_i)) pg_i + beta k3_t - gamma H_t and
+    G_t = dl/dlogp_t = (N / (n_seq n_i)) (-A_i s_i if unclipped else 0)
+    + beta (1 - exp(q_t - logp_t)). A ratio correction (Sec. 3.4) weights each
+    token's share by its constant weight w_t; since s_i depends on every
+    token of the trajectory, the policy part of G_t then carries the mean of
+    w over the trajectory's training tokens. Every row of trajectory i
+    reports r = s_i and the sequence's clip flags."""
+    logp = np.asarray(logp, np.float64)
+    rho = np.asarray(rho, np.float64)
+    H = np.asarray(H, np.float64)
+    base = rho if old is None else np.asarray(old, np.float64)
+    cu = np.asarray(cu_seqlens, np.int64)
+    m = np.asarray(mask).astype(bool)
+    N = int(m.sum())
+    n_i = training_tokens_per_trajectory(cu, m)
+    n_seq = int((n_i > 0).sum())
+    R = logp.shape[0]
+    # ratio correction (Sec. 3.4): a constant weight on each token's share
+    wt = np.ones(R)
+    rc = np.ones(R)
+    corr_clip = np.zeros(R, bool)
+    if p.correction != "none":
+        if old is None:
+            raise ValueError("a ratio correction needs old log-probs")
+        rc = np.exp(np.asarray(old, np.float64) - rho)
+        outside = (rc < p.corr_lo) | (rc > p.corr_hi)
+        corr_clip = outside
+        wt = (np.minimum(np.maximum(rc, p.corr_lo), p.corr_hi) if p.correction == "tis"
+              else np.where(outside, 0.0, rc))
+    r = np.ones(R)
+    pg = np.zeros(R)
+    g_pg = np.zeros(R)
+    clip_hi = np.zeros(R, bool)
+    clip_lo = np.zeros(R, bool)
+    dual = np.zeros(R, bool)
+    for i in range(cu.shape[0] - 1):
+        if n_i[i] == 0:
+            continue
+        rows = slice(cu[i], cu[i + 1])
+        mm = m[rows]
+        s_i = float(np.exp((logp[rows][mm] - base[rows][mm]).sum() / n_i[i]))
+        A = float(A_traj[i])
+        u = -A * s_i
+        c = -A * min(max(s_i, 1.0 - p.eps_lo), 1.0 + p.eps_hi)
+        pgi = max(u, c)
+        clipped = c > u
+        du = False
+        if p.dual_clip_c > 0.0 and A < 0.0:
+            d = -A * p.dual_clip_c
+            if d < pgi:
+                pgi, du = d, True
+        scale = N / (n_seq * n_i[i])
+        r[rows] = s_i
+        pg[rows] = scale * pgi * wt[rows]
+        # every token's logp moves s_i, which every share of the trajectory
+        # carries: the gradient takes the trajectory's mean weight
+        mean_wt = float(wt[rows][mm].mean())
+        g_pg[rows] = 0.0 if (clipped or du) else scale * mean_wt * (-A * s_i)
+        clip_hi[rows] = clipped and s_i > 1.0 + p.eps_hi
+        clip_lo[rows] = clipped and s_i < 1.0 - p.eps_lo
+        dual[rows] = du
+    if q is None:
+        k3 = np.zeros(R)
+        g_kl = np.zeros(R)
+    else:
+        dlt = np.asarray(q, np.float64) - logp
+        k3 = np.exp(dlt) - dlt - 1.0
+        g_kl = 1.0 - np.exp(dlt)
+    ell = pg + p.kl_coef * k3 - p.entropy_coef * H
+    G = g_pg + p.kl_coef * g_kl
+    return dict(r=r, pg=pg, k3=k3, ell=ell, G=G, clip_hi=clip_hi, clip_lo=clip_lo, dual=dual,
+                wt=wt, rc=rc, corr_clip=corr_clip)
 
 
 # --------------------------------------------------------------------------
@@ -339,41 +491,54 @@ def rl_loss_rows(z, y, rho, q, A_row, mask, N, p: LossParams, grad_loss=1.0,
 
 
 def rl_loss(z, y, rho, q, w, gid, cu_seqlens, n_groups, mask, p: LossParams,
-            grad_loss=1.0, old=None, teacher=None, want_dlogits=True, chunk=256):
-    """The whole loss for one call: advantages, per-row outputs, the masked
-    token-mean, the metrics, and (optionally) dLogits as a float64 array.
+            grad_loss=1.0, old=None, teacher=None, want_dlogits=True, chunk=256,
+            topk_ids=None, topk_teacher=None):
+    """The whole loss for one call: advantages, per-row outputs, the loss,
+    the metrics, and (optionally) dLogits as a float64 array.
 
-    Rows are processed in chunks of ``chunk`` rows; each row's arithmetic is
-    independent of the chunking."""
+    Order (Sec. 5.2: the estimator first, then the OPD shaping): estimator
+    advantages; row log-softmax statistics; OPD shaping (one-sample from the
+    rollout / teacher log-probs, or top-K from the candidate sets); the token
+    objective (or GSPO's sequence objective); masked mean and metrics;
+    dLogits. Rows are processed in chunks of ``chunk`` rows; each row's
+    arithmetic is independent of the chunking."""
     R = int(np.asarray(y).shape[0])
-    A_traj, n_g = group_advantages(w, gid, n_groups, p)
-    A_row = row_advantages(A_traj, cu_seqlens, R)
-    if p.opd_coef != 0.0:
-        A_row = shape_advantages_opd(A_row, rho, teacher, p.opd_coef)
     m = np.asarray(mask).astype(bool)
     N = int(m.sum())
-    keys = ("logp", "H", "lse", "r", "pg", "k3", "ell", "G", "clip_hi", "clip_lo",
-            "dual", "wt", "rc", "corr_clip")
-    parts = {k: [] for k in keys}
-    dz = [] if want_dlogits else None
+    A_traj, A_row, n_g = estimator_advantages(w, gid, n_groups, cu_seqlens, m, p)
+    V = np.asarray(z).shape[1] if R else 0
+    logp = np.zeros(R)
+    H = np.zeros(R)
+    lse = np.zeros(R)
     for lo in range(0, R, chunk):
         hi = min(R, lo + chunk)
-        o = rl_loss_rows(z[lo:hi], np.asarray(y)[lo:hi], np.asarray(rho)[lo:hi],
-                         None if q is None else np.asarray(q)[lo:hi], A_row[lo:hi],
-                         m[lo:hi], N, p, grad_loss,
-                         old=None if old is None else np.asarray(old)[lo:hi],
-                         want_dlogits=want_dlogits)
-        for k in keys:
-            parts[k].append(o[k])
-        if want_dlogits:
-            dz.append(o["dlogits"])
-    cat = {k: (np.concatenate(v) if v else np.zeros(0)) for k, v in parts.items()}
-    for k in ("clip_hi", "clip_lo", "dual", "corr_clip"):
-        cat[k] = cat[k].astype(bool)
-    stats = loss_stats(cat, cat["logp"], rho, cat["H"], m)
+        logp[lo:hi], H[lo:hi], lse[lo:hi] = row_log_softmax(z[lo:hi], np.asarray(y)[lo:hi],
+                                                            p.temperature)
+    if p.opd_coef != 0.0:
+        if p.opd_topk > 0:
+            est = np.zeros(R)
+            for lo in range(0, R, chunk):
+                hi = min(R, lo + chunk)
+                est[lo:hi] = opd_topk_estimate(z[lo:hi], p.temperature, lse[lo:hi],
+                                               np.asarray(topk_ids)[lo:hi],
+                                               np.asarray(topk_teacher)[lo:hi])
+            A_row = A_row - p.opd_coef * est
+        else:
+            A_row = shape_advantages_opd(A_row, rho, teacher, p.opd_coef)
+    q_ = None if q is None else np.asarray(q)
+    if p.estimator == "gspo":
+        obj = sequence_objective(logp, rho, q_, A_traj, H, cu_seqlens, m, p, old=old)
+    else:
+        obj = token_objective(logp, rho, q_, A_row, H, p, old=old)
+    cat = dict(obj, logp=logp, H=H, lse=lse)
+    stats = loss_stats(cat, logp, rho, H, m)
     out = dict(cat, A_traj=A_traj, group_sizes=n_g, A_row=A_row, N=N, stats=stats,
                loss=stats["loss"])
     if want_dlogits:
-        V = np.asarray(z).shape[1] if R else 0
+        dz = [dlogits_rows(z[lo:min(R, lo + chunk)], np.asarray(y)[lo:min(R, lo + chunk)],
+                           p.temperature, lse[lo:lo + chunk], H[lo:lo + chunk],
+                           obj["G"][lo:lo + chunk], m[lo:lo + chunk], N, grad_loss,
+                           p.entropy_coef)
+              for lo in range(0, R, chunk)]
         out["dlogits"] = np.concatenate(dz) if dz else np.zeros((0, V))
     return out

@@ -375,3 +375,155 @@ def test_no_training_tokens():
     assert out["loss"] == 0.0 and out["N"] == 0
     assert np.all(out["dlogits"] == 0.0)
     assert out["stats"]["ratio_mean"] == 0.0
+
+
+# ---------------------------------------------------------------- estimators
+
+def test_reinforcepp_golden():
+    c = _golden()["reinforcepp_two_trajectories"]
+    w = np.array([_ev(v) for v in c["w"]])
+    for est in ("reinforcepp", "reinforcepp_baseline"):
+        A, A_row, _ = oracle.estimator_advantages(w, np.array(c["gid"]), c["n_groups"],
+                                                  np.array(c["cu"]), np.array(c["mask"]),
+                                                  LossParams(estimator=est))
+        np.testing.assert_allclose(A, [_ev(v) for v in c["expect"]], atol=1e-15)
+
+
+def test_reinforcepp_global_normalisation_invariants():
+    rng = np.random.default_rng(11)
+    n_traj, n_groups = 12, 3
+    w = rng.normal(size=n_traj)
+    gid = rng.permutation(np.repeat(np.arange(n_groups), 4))
+    lens = rng.integers(1, 9, size=n_traj)
+    cu = np.concatenate([[0], np.cumsum(lens)])
+    mask = rng.random(cu[-1]) < 0.7
+    for est in ("reinforcepp", "reinforcepp_baseline"):
+        p = LossParams(estimator=est)
+        A, A_row, _ = oracle.estimator_advantages(w, gid, n_groups, cu, mask, p)
+        Am = A_row[mask]
+        assert abs(Am.sum()) < 1e-12
+        assert abs((Am ** 2).sum() - (mask.sum() - 1)) < 1e-9
+        # the token-level z-score of the returns, by the library's std
+        b = w.copy()
+        if est == "reinforcepp_baseline":
+            for g in range(n_groups):
+                b[gid == g] -= w[gid == g].mean()
+        bt = torch.from_numpy(oracle.row_advantages(b, cu, cu[-1])[mask])
+        np.testing.assert_allclose(Am, ((bt - bt.mean()) / bt.std()).numpy(), atol=1e-12)
+    # baseline-relative returns ignore a constant added to a group's rewards
+    p = LossParams(estimator="reinforcepp_baseline")
+    w2 = w.copy()
+    w2[gid == 1] += 5.0
+    a1 = oracle.estimator_advantages(w, gid, n_groups, cu, mask, p)[0]
+    a2 = oracle.estimator_advantages(w2, gid, n_groups, cu, mask, p)[0]
+    np.testing.assert_allclose(a1, a2, atol=1e-12)
+    # plain returns: a positive affine map of the rewards changes nothing
+    p = LossParams(estimator="reinforcepp")
+    a3 = oracle.estimator_advantages(3.0 * w - 7.0, gid, n_groups, cu, mask, p)[0]
+    np.testing.assert_allclose(oracle.estimator_advantages(w, gid, n_groups, cu, mask, p)[0],
+                               a3, atol=1e-12)
+    # equal returns: exactly zero
+    z = oracle.estimator_advantages(np.full(n_traj, 0.25), gid, n_groups, cu, mask, p)[0]
+    assert np.all(z == 0.0)
+
+
+def test_opd_topk_estimate_pins():
+    rng = np.random.default_rng(12)
+    R, V = 5, 9
+    z = rng.normal(0, 2, size=(R, V))
+    T = 0.9
+    _, _, lse = oracle.row_log_softmax(z, np.zeros(R, np.int64), T)
+    t_logits = rng.normal(0, 2, size=(R, V))
+    log_t = torch.log_softmax(torch.from_numpy(t_logits), dim=1).numpy()
+    # the full vocabulary as the candidate set: the reverse KL(student || teacher)
+    ids = np.tile(np.arange(V), (R, 1))
+    est = oracle.opd_topk_estimate(z, T, lse, ids, log_t)
+    log_s = torch.log_softmax(torch.from_numpy(z) / T, dim=1)
+    kl = torch.nn.functional.kl_div(torch.from_numpy(log_t), log_s, log_target=True,
+                                    reduction="none").sum(1).numpy()
+    np.testing.assert_allclose(est, kl, atol=1e-12)
+    # one candidate: the one-sample difference at that token
+    c = rng.integers(0, V, size=(R, 1))
+    est1 = oracle.opd_topk_estimate(z, T, lse, c, log_t[np.arange(R)[:, None], c])
+    np.testing.assert_allclose(est1, (log_s.numpy() - log_t)[np.arange(R), c[:, 0]], atol=1e-12)
+
+
+def test_gspo_golden():
+    c = _golden()["gspo_one_trajectory"]
+    lr = np.array([_ev(v) for v in c["log_ratio"]])
+    logp = np.array([-1.0, -2.0])
+    rho = logp - lr
+    o = oracle.sequence_objective(logp, rho, None, np.array([_ev(c["A"])]), np.zeros(2),
+                                  np.array([0, 2]), np.array([1, 1]),
+                                  LossParams(estimator="gspo"))
+    L, _ = oracle.masked_token_mean(o["ell"], np.array([1, 1]))
+    assert abs(L - _ev(c["expect"]["loss"])) < 1e-14
+    np.testing.assert_allclose(o["G"], [_ev(v) for v in c["expect"]["G"]], atol=1e-14)
+    np.testing.assert_allclose(o["r"], _ev(c["expect"]["r"]), atol=1e-15)
+
+
+def test_gspo_on_one_token_trajectories_is_token_ppo():
+    rng = np.random.default_rng(13)
+    R = 16
+    logp = -rng.random(R) * 3
+    rho = logp + rng.normal(0, 0.3, size=R)
+    q = logp + rng.normal(0, 0.2, size=R)
+    A = rng.normal(size=R)
+    H = rng.random(R)
+    cu = np.arange(R + 1)
+    m = np.ones(R, bool)
+    p = LossParams(estimator="gspo", dual_clip_c=2.0, kl_coef=0.1, entropy_coef=0.05)
+    seq = oracle.sequence_objective(logp, rho, q, A, H, cu, m, p)
+    tok = oracle.token_objective(logp, rho, q, A, H, p)
+    for k in ("r", "pg", "ell", "G", "clip_hi", "clip_lo", "dual"):
+        np.testing.assert_allclose(seq[k], tok[k], atol=1e-13)
+
+
+@pytest.mark.parametrize("variant", ["gspo", "gspo_tis", "topk", "reinforcepp_baseline"])
+def test_dlogits_fd_estimators(variant, monkeypatch):
+    rng = np.random.default_rng(200 + len(variant))
+    V, n_traj, L_ = 6, 4, 3
+    R = n_traj * L_
+    base = dict(temperature=0.9, eps_lo=0.2, eps_hi=0.25, kl_coef=0.2, entropy_coef=0.03)
+    extra = dict(gspo=dict(estimator="gspo", dual_clip_c=2.0),
+                 gspo_tis=dict(estimator="gspo", correction="tis", corr_lo=0.5, corr_hi=1.5),
+                 topk=dict(opd_coef=0.6, opd_topk=3),
+                 reinforcepp_baseline=dict(estimator="reinforcepp_baseline"))[variant]
+    p = LossParams(**base, **extra)
+    gid = np.array([0, 0, 1, 1])
+    cu = np.arange(n_traj + 1) * L_
+    m = np.array([1, 1, 0, 1, 1, 1, 0, 1, 1, 1, 1, 1], dtype=bool)
+    for attempt in range(60):
+        z = rng.normal(0, 1.5, size=(R, V))
+        y = rng.integers(0, V, size=R)
+        logp, _, _ = oracle.row_log_softmax(z, y, p.temperature)
+        rho = logp + rng.normal(0, 0.5, size=R)
+        q = logp + rng.normal(0, 0.4, size=R)
+        old = logp + rng.normal(0, 0.3, size=R) if p.correction != "none" else None
+        w = rng.random(n_traj)
+        ids = np.stack([rng.choice(V, 3, replace=False) for _ in range(R)])
+        tlp = np.log(rng.dirichlet(np.ones(V), size=R))[np.arange(R)[:, None], ids]
+        kw = dict(old=old, topk_ids=ids, topk_teacher=tlp)
+        out = oracle.rl_loss(z, y, rho, q, w, gid, cu, 2, m, p, grad_loss=1.3, **kw)
+        if not _near_kink(out, p):
+            break
+    else:
+        pytest.fail("no draw away from the kinks")
+    if variant == "topk":
+        # the top-K signal is a fixed per-token reward: hold it at its value
+        frozen = oracle.opd_topk_estimate(z, p.temperature, out["lse"], ids, tlp)
+        monkeypatch.setattr(oracle.rl_loss_ref, "opd_topk_estimate",
+                            lambda *a, **k: frozen[:a[0].shape[0]] if a[0].shape[0] == R else None)
+    h = 1e-6
+    num = np.zeros_like(z)
+    for i in range(R):
+        for j in range(V):
+            zp = z.copy(); zp[i, j] += h
+            zm = z.copy(); zm[i, j] -= h
+            lp = oracle.rl_loss(zp, y, rho, q, w, gid, cu, 2, m, p, want_dlogits=False,
+                                chunk=R, **kw)["loss"]
+            lm = oracle.rl_loss(zm, y, rho, q, w, gid, cu, 2, m, p, want_dlogits=False,
+                                chunk=R, **kw)["loss"]
+            num[i, j] = 1.3 * (lp - lm) / (2 * h)
+    scale = np.abs(out["dlogits"]).max()
+    np.testing.assert_allclose(out["dlogits"], num, atol=1e-6 * max(scale, 1e-3), rtol=1e-6)
