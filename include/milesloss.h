@@ -81,6 +81,29 @@ typedef enum { RL_BF16 = 0, RL_F32 = 1 } rl_dtype;
  *   RL_CORR_CLIP_OR_POP  weight = rc if corr_lo <= rc <= corr_hi, else 0 */
 typedef enum { RL_CORR_NONE = 0, RL_CORR_TIS = 1, RL_CORR_CLIP_OR_POP = 2 } rl_correction;
 
+/* Advantage estimators of Sec. 3.4.
+ *   RL_EST_GRPO                 rewards centred within the trajectory's group and
+ *                               divided by max(group std, std_floor) (GRPO)
+ *   RL_EST_REINFORCEPP          the outcome reward is every token's return; the
+ *                               returns are normalised over all training tokens
+ *                               of the call (REINFORCE++)
+ *   RL_EST_REINFORCEPP_BASELINE the reward minus its group's mean, then the same
+ *                               normalisation (REINFORCE++ baseline-relative)
+ *   RL_EST_GSPO                 GRPO advantages with a sequence-level ratio:
+ *                               s_i = exp(mean over trajectory i's training tokens
+ *                               of logp - base), clipped per trajectory; the
+ *                               policy term is the mean over trajectories with
+ *                               training tokens (GSPO). Runs as forward sweep,
+ *                               per-trajectory pass and gradient sweep (the
+ *                               gradient of a token depends on its whole
+ *                               trajectory), so it reads the logits twice. */
+typedef enum {
+  RL_EST_GRPO = 0,
+  RL_EST_REINFORCEPP = 1,
+  RL_EST_REINFORCEPP_BASELINE = 2,
+  RL_EST_GSPO = 3
+} rl_estimator;
+
 typedef struct {
   float temperature;   /* T > 0: logits are divided by T before the softmax      */
   float eps_lo;        /* >= 0: lower clip at 1 - eps_lo                          */
@@ -95,6 +118,19 @@ typedef struct {
   float corr_lo;       /* correction interval [corr_lo, corr_hi], default [0, 2] */
   float corr_hi;
   float opd_coef;      /* on-policy distillation coefficient; 0 = off (Sec. 5.2) */
+  int32_t estimator;   /* rl_estimator; RL_EST_GSPO does not combine with opd_coef */
+  int32_t opd_topk;    /* K >= 1 selects the top-K OPD signal (Sec. 5.2), 0 the
+                          one-sample signal from teacher_logprobs; K <= 64     */
+  /* Top-K OPD inputs (DEVICE pointers, read by the kernels; used when
+   * opd_topk > 0 and opd_coef != 0): for row t, K candidate token ids
+   * opd_topk_ids[t*K + k] in [0, vocab) chosen on the serving side (e.g. the
+   * student's K most likely tokens) and the teacher's log-probs of them,
+   * opd_topk_teacher[t*K + k]. The signal is sum_k w_k (log p_k - teacher_k)
+   * with the trainer's probabilities p_k of the candidates renormalised over
+   * the set as weights w_k; it is subtracted, times opd_coef, from the token's
+   * advantage and is not differentiated. */
+  const int32_t* opd_topk_ids;
+  const float* opd_topk_teacher;
 } rl_loss_params;
 
 /* Call-wide statistics, written to DEVICE memory by the stream. Means are
@@ -142,7 +178,7 @@ rl_status rl_loss_workspace_size(int64_t n_rows, int32_t n_traj, int32_t n_group
  *                    or NULL (then the PPO ratio is taken against the rollout
  *                    log-probs); required when a correction is set
  *  teacher_logprobs  [n_rows] fp32 teacher log-probs for OPD, or NULL
- *                    (required when opd_coef != 0)
+ *                    (required when opd_coef != 0 and opd_topk == 0)
  *  rewards           [n_traj] fp32, one outcome reward per trajectory
  *  group_id          [n_traj] int32 in [0, n_groups): the prompt of each
  *                    trajectory; members of a group may be anywhere

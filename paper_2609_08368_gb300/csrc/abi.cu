@@ -127,6 +127,8 @@ rl_status check_params(const rl_loss_params* p) {
       (!finite(p->corr_lo) || !finite(p->corr_hi) || p->corr_lo < 0.0f || p->corr_lo > p->corr_hi))
     return RL_ERR_INVALID_ARG;
   if (!finite(p->opd_coef)) return RL_ERR_INVALID_ARG;
+  if (p->estimator < RL_EST_GRPO || p->estimator > RL_EST_GSPO) return RL_ERR_INVALID_ARG;
+  if (p->opd_topk < 0 || p->opd_topk > kMaxTopK) return RL_ERR_INVALID_ARG;
   return RL_OK;
 }
 
@@ -142,6 +144,11 @@ LossScalars scalars(const rl_loss_params* p) {
   s.corr_lo = p->corr_lo;
   s.corr_hi = p->corr_hi;
   s.corr = p->correction;
+  const bool topk = p->opd_topk > 0 && p->opd_coef != 0.0f;
+  s.topk = topk ? p->opd_topk : 0;
+  s.opd_coef = p->opd_coef;
+  s.topk_ids = topk ? p->opd_topk_ids : nullptr;
+  s.topk_teacher = topk ? p->opd_topk_teacher : nullptr;
   return s;
 }
 
@@ -285,7 +292,13 @@ rl_status check_fwd(const FwdIn& f) {
   if (f.c.R > 0 && !f.rho) return RL_ERR_INVALID_ARG;
   if (f.c.R > 0 && p->kl_coef > 0.0f && !f.q) return RL_ERR_INVALID_ARG;
   if (f.c.R > 0 && p->correction != RL_CORR_NONE && !f.old) return RL_ERR_INVALID_ARG;
-  if (f.c.R > 0 && p->opd_coef != 0.0f && !f.teacher) return RL_ERR_INVALID_ARG;
+  if (f.c.R > 0 && p->opd_coef != 0.0f && p->opd_topk == 0 && !f.teacher)
+    return RL_ERR_INVALID_ARG;
+  if (f.c.R > 0 && p->opd_coef != 0.0f && p->opd_topk > 0 &&
+      (!p->opd_topk_ids || !p->opd_topk_teacher))
+    return RL_ERR_INVALID_ARG;
+  // GSPO scores whole trajectories with one advantage: no per-token shaping
+  if (p->estimator == RL_EST_GSPO && p->opd_coef != 0.0f) return RL_ERR_UNSUPPORTED;
   if (!f.ws || (reinterpret_cast<uintptr_t>(f.ws) & 255u)) return RL_ERR_INVALID_ARG;
   size_t need = 0;
   rl_loss_workspace_size(f.c.R, f.n_traj, f.n_groups, &need);
@@ -313,6 +326,36 @@ void record(cudaEvent_t ev, cudaStream_t s) {
   if (ev && t_ev_begin && t_ev_end) cudaEventRecord(ev, s);
 }
 
+// The gradient sweep from the per-row state in the workspace (lse, H, G).
+rl_status launch_bwd(const Common& c, const GradOut& go, const WsPtrs& ws, cudaStream_t s) {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return RL_ERR_CUDA;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return RL_ERR_CUDA;
+  BwdArgs b;
+  b.logits = c.logits;
+  b.ld = c.ld;
+  b.R = c.R;
+  b.V = static_cast<int>(c.V);
+  b.tiles_per_row = static_cast<int>((c.V + kBwdTile - 1) / kBwdTile);
+  b.n_tiles = c.R * b.tiles_per_row;
+  b.in_vec = aligned16(c.logits) && ((c.ld * elem_size(c.dt)) % 16 == 0);
+  b.out_vec = aligned16(go.dl) && ((go.ld_out * elem_size(go.dt)) % 16 == 0);
+  b.targets = c.targets;
+  b.mask = c.mask;
+  b.dlogits = go.dl;
+  b.ld_out = go.ld_out;
+  b.grad_loss = go.g;
+  b.grad_loss_dev = go.g_dev;
+  b.invT = 1.0f / c.p->temperature;
+  b.k = 1.4426950408889634f / c.p->temperature;
+  b.gamma = c.p->entropy_coef;
+  b.ws = ws;
+  const long long grid = std::min<long long>(b.n_tiles, static_cast<long long>(sms) * 8);
+  return launch(bwd_kernel(c.dt, go.dt), dim3(static_cast<unsigned>(grid)), dim3(kBwdThreads), 0,
+                1, s, &b);
+}
+
 rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return RL_ERR_CUDA;
@@ -330,21 +373,31 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s) {
   aa.cu = f.cu;
   aa.mask = c.mask;
   aa.rho = f.rho;
-  aa.teacher = (c.p->opd_coef != 0.0f) ? f.teacher : nullptr;
+  aa.teacher = (c.p->opd_coef != 0.0f && c.p->opd_topk == 0) ? f.teacher : nullptr;
   aa.opd_coef = c.p->opd_coef;
   aa.normalize_std = c.p->normalize_std;
   aa.unbiased_std = c.p->unbiased_std;
   aa.std_floor = c.p->std_floor;
   aa.advantages = f.out_adv;
   aa.group_sizes = f.out_gsize;
+  aa.estimator = c.p->estimator;
+  const size_t traj_bytes = (2 * static_cast<size_t>(f.n_traj) + 1) * sizeof(int);
+  aa.smem_traj = traj_bytes <= static_cast<size_t>(kAdvSmemBytes);
   aa.ws = ws;
-  rl_status st = launch(adv_kernel(), dim3(1), dim3(kAdvThreads), 0, 1, s, &aa);
+  rl_status st = launch(adv_kernel(), dim3(1), dim3(kAdvThreads),
+                        aa.smem_traj ? static_cast<int>(traj_bytes) : 0, 1, s, &aa);
   if (st != RL_OK) return st;
 
-  const bool grad = go != nullptr;
+  // GSPO: the gradient of a token depends on its whole trajectory, so the
+  // call runs as forward sweep -> per-trajectory pass -> gradient sweep.
+  const bool gspo = c.p->estimator == RL_EST_GSPO;
+  const GradOut* go_sweep = gspo ? nullptr : go;
+
+  const bool grad = go_sweep != nullptr;
   const size_t es = elem_size(c.dt);
   const bool in_bulk = aligned16(c.logits) && ((c.ld * es) % 16 == 0);
   const bool out_vec = grad && aligned16(go->dl) && ((go->ld_out * elem_size(go->dt)) % 16 == 0);
+  (void)go_sweep;
   if (c.R > 0 && use_stream(c.V * static_cast<long long>(es), in_bulk)) {
     StreamPlan sp;
     st = plan_stream(dev, &sp);
@@ -424,6 +477,20 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s) {
     if (st != RL_OK) return st;
   }
 
+  if (gspo && c.R > 0 && f.n_traj > 0) {
+    SeqArgs qa;
+    qa.cu = f.cu;
+    qa.rho = f.rho;
+    qa.old = f.old;
+    qa.q = f.q;
+    qa.mask = c.mask;
+    qa.s = scalars(c.p);
+    qa.ws = ws;
+    st = launch(seq_kernel(), dim3(static_cast<unsigned>(f.n_traj)), dim3(kSeqThreads), 0, 1, s,
+                &qa);
+    if (st != RL_OK) return st;
+  }
+
   if (f.stats) {
     StatArgs ta;
     ta.R = c.R;
@@ -437,6 +504,7 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s) {
                 &ta);
     if (st != RL_OK) return st;
   }
+  if (gspo && go && c.R > 0) return launch_bwd(c, *go, ws, s);
   return RL_OK;
 }
 
@@ -508,34 +576,9 @@ rl_status rl_loss_bwd(const void* logits, rl_dtype logits_dtype, int64_t n_rows,
   const WsLayout L = WsLayout::make(n_rows, 0, 0);
   if (workspace_bytes < L.total) return RL_ERR_WORKSPACE_TOO_SMALL;
   if (n_rows == 0) return RL_OK;
-  int dev = 0, sms = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return RL_ERR_CUDA;
-  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-    return RL_ERR_CUDA;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  BwdArgs b;
-  b.logits = logits;
-  b.ld = ld;
-  b.R = n_rows;
-  b.V = static_cast<int>(vocab);
-  b.tiles_per_row = static_cast<int>((vocab + kBwdTile - 1) / kBwdTile);
-  b.n_tiles = n_rows * b.tiles_per_row;
-  b.in_vec = aligned16(logits) && ((ld * elem_size(logits_dtype)) % 16 == 0);
-  b.out_vec = aligned16(dlogits) && ((ld_out * elem_size(dlogits_dtype)) % 16 == 0);
-  b.targets = targets;
-  b.mask = loss_mask;
-  b.dlogits = dlogits;
-  b.ld_out = ld_out;
-  b.grad_loss = grad_loss;
-  b.grad_loss_dev = grad_loss_device;
-  b.invT = 1.0f / params->temperature;
-  b.k = 1.4426950408889634f / params->temperature;
-  b.gamma = params->entropy_coef;
-  b.ws = WsPtrs::at(const_cast<void*>(workspace), L);
-  const long long grid = std::min<long long>(b.n_tiles, static_cast<long long>(sms) * 8);
   record(t_ev_begin, s);
-  st = launch(bwd_kernel(logits_dtype, dlogits_dtype), dim3(static_cast<unsigned>(grid)),
-              dim3(kBwdThreads), 0, 1, s, &b);
+  st = launch_bwd(c, go, WsPtrs::at(const_cast<void*>(workspace), L), s);
   record(t_ev_end, s);
   return st;
 }

@@ -32,7 +32,8 @@ struct WsHeader {
   uint32_t err_bits;   // OR of kErr* bits
   uint32_t ticket;     // last-block counter of the statistics reduction
   long long n_tokens;  // N = sum of the loss mask, written by the advantage kernel
-  uint32_t pad[60];
+  long long n_seq;     // trajectories with at least one training token
+  uint32_t pad[58];
 };
 static_assert(sizeof(WsHeader) == 256, "header is one 256-byte segment");
 
@@ -47,7 +48,7 @@ constexpr int kStatThreads = 256;
 constexpr int kMaxStatBlocks = 256;  // one partial per thread of the final block
 
 struct WsLayout {
-  size_t hdr, g_mu, g_den, g_flag, a_traj, a_row;
+  size_t hdr, g_mu, g_den, g_flag, a_traj, traj_n, a_row;
   size_t r_logp, r_H, r_lse, r_G, r_ell, r_pg, r_k3, r_r, r_rc, r_flags;
   size_t parts, total;
 
@@ -70,6 +71,7 @@ struct WsLayout {
     L.g_den = o; o += up(sizeof(double) * (size_t)n_groups);
     L.g_flag = o; o += up(sizeof(int) * (size_t)n_groups);
     L.a_traj = o; o += up(sizeof(float) * (size_t)n_traj);
+    L.traj_n = o; o += up(sizeof(int) * (size_t)n_traj);
     L.total = o;
     return L;
   }
@@ -82,6 +84,7 @@ struct WsPtrs {
   double* g_den;
   int* g_flag;
   float* a_traj;
+  int* traj_n;  // training tokens per trajectory
   float* a_row;
   float *logp, *H, *lse, *G, *ell, *pg, *k3, *r, *rc;
   uint8_t* flags;
@@ -95,6 +98,7 @@ struct WsPtrs {
     p.g_den = reinterpret_cast<double*>(b + L.g_den);
     p.g_flag = reinterpret_cast<int*>(b + L.g_flag);
     p.a_traj = reinterpret_cast<float*>(b + L.a_traj);
+    p.traj_n = reinterpret_cast<int*>(b + L.traj_n);
     p.a_row = reinterpret_cast<float*>(b + L.a_row);
     p.logp = reinterpret_cast<float*>(b + L.r_logp);
     p.H = reinterpret_cast<float*>(b + L.r_H);
@@ -117,7 +121,18 @@ struct LossScalars {
   float k;         // log2(e) / T: logits -> base-2 exponent units
   float eps_lo, eps_hi, dual_c, beta, gamma, corr_lo, corr_hi;
   int corr;        // rl_correction
+  int topk;        // K of the top-K OPD signal applied in the sweep epilogue (0 = none)
+  float opd_coef;
+  const int* topk_ids;       // [R, K]
+  const float* topk_teacher; // [R, K]
 };
+
+// Correction weight of a token (Sec. 3.4) from its ratio rc = exp(old - rollout).
+__host__ __device__ __forceinline__ float correction_weight(float rc, const LossScalars& s) {
+  if (s.corr == RL_CORR_NONE) return 1.0f;
+  if (s.corr == RL_CORR_TIS) return fminf(fmaxf(rc, s.corr_lo), s.corr_hi);
+  return (rc < s.corr_lo || rc > s.corr_hi) ? 0.0f : rc;
+}
 
 // ------------------------------------------------------------------ PTX
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -435,10 +450,8 @@ __device__ __forceinline__ TokenTerms token_terms(float logp, float H, float rho
   float rc = 1.0f;
   if (s.corr != RL_CORR_NONE) {
     rc = expf(old - rho);
-    const bool outside = (rc < s.corr_lo) || (rc > s.corr_hi);
-    const float wt = (s.corr == RL_CORR_TIS) ? fminf(fmaxf(rc, s.corr_lo), s.corr_hi)
-                                             : (outside ? 0.0f : rc);
-    if (outside) fl |= kFlagCorrClip;
+    if ((rc < s.corr_lo) || (rc > s.corr_hi)) fl |= kFlagCorrClip;
+    const float wt = correction_weight(rc, s);
     pg *= wt;
     gpg *= wt;
   }
@@ -458,6 +471,33 @@ __device__ __forceinline__ TokenTerms token_terms(float logp, float H, float rho
   t.rc = rc;
   t.flags = fl;
   return t;
+}
+
+// Top-K on-policy distillation signal of one row (Sec. 5.2): the sum over
+// the candidate set of w_k (log p_k - teacher_k), with p_k the trainer's
+// probabilities of the candidates (from the row's logits and its lse) and
+// w_k = p_k / sum_j p_j. Candidates outside [0, V) are skipped.
+template <class In>
+__device__ __forceinline__ float topk_signal(const void* row, int V, const int* ids,
+                                            const float* teacher, int K, float invT, float lse) {
+  // two passes over the K candidates (the largest log-prob, then the
+  // weighted sum); the second pass reloads the few logits from cache
+  float mx = -INFINITY;
+  for (int k = 0; k < K; ++k) {
+    const int id = ids[k];
+    if (id >= 0 && id < V) mx = fmaxf(mx, In::load1(row, id) * invT - lse);
+  }
+  if (mx == -INFINITY) return 0.0f;
+  float sw = 0.0f, acc = 0.0f;
+  for (int k = 0; k < K; ++k) {
+    const int id = ids[k];
+    if (id < 0 || id >= V) continue;
+    const float lp = In::load1(row, id) * invT - lse;
+    const float w = expf(lp - mx);
+    sw += w;
+    acc += w * (lp - teacher[k]);
+  }
+  return acc / sw;
 }
 
 }  // namespace milesloss

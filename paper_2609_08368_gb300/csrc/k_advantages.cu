@@ -1,18 +1,23 @@
-// Group-relative advantages (GRPO, Sec. 2 and Sec. 9.1), the per-row
-// advantage with optional on-policy-distillation shaping (Sec. 5.2), the
-// masked token count N, and validation of group ids and row offsets.
+// Advantages of the configured estimator (Sec. 3.4: GRPO, GSPO, REINFORCE++
+// plain and baseline-relative), the per-row advantage with the one-sample
+// on-policy-distillation shaping (Sec. 5.2), the masked token count N, the
+// training tokens of every trajectory, and validation of group ids and row
+// offsets.
 //
-// One CTA of 1024 threads does all of it; the inputs are a few KB of
-// per-trajectory data plus one byte and one float per row, so the kernel
-// is a small fraction of a call. Every sum runs in a fixed order (lane-
-// strided partial sums, xor-butterfly merges), so results are bit-for-bit
-// reproducible, and all statistics are accumulated in double precision.
+// One CTA of 1024 threads does all of it: the inputs are a few KB of
+// per-trajectory data plus one byte and one float per row. Row offsets and
+// per-trajectory counts are staged in shared memory when they fit, so the
+// per-row trajectory lookup (a binary search) stays on chip. Every sum runs
+// in a fixed order (lane-strided partial sums, xor-butterfly merges) in
+// double precision, so results are bit-for-bit reproducible.
 #include "common.cuh"
 #include "kernels.h"
 
 namespace milesloss {
 
 namespace {
+
+constexpr int kWarps = kAdvThreads / 32;
 
 __device__ __forceinline__ double warp_sum(double v) {
 #pragma unroll
@@ -35,28 +40,67 @@ __device__ __forceinline__ double warp_min(double v) {
   return v;
 }
 
+// Block-wide sums in a fixed order (valid in every thread).
+__device__ double block_sum(double v, double* sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  v = warp_sum(v);
+  __syncthreads();
+  if (lane == 0) sh[warp] = v;
+  __syncthreads();
+  double t = 0.0;
+  for (int w = 0; w < kWarps; ++w) t += sh[w];
+  return t;
+}
+__device__ double block_max(double v, double* sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  v = warp_max(v);
+  __syncthreads();
+  if (lane == 0) sh[warp] = v;
+  __syncthreads();
+  double t = -INFINITY;
+  for (int w = 0; w < kWarps; ++w) t = fmax(t, sh[w]);
+  return t;
+}
+
+// Trajectory of row t: the last i with cu[i] <= t (cu valid: cu[0] = 0 <= t < cu[n]).
+__device__ __forceinline__ int traj_of(const int* cu, int n_traj, long long t) {
+  int lo = 0, hi = n_traj;
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (static_cast<long long>(cu[mid]) <= t) lo = mid; else hi = mid;
+  }
+  return lo;
+}
+
 __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) {
+  extern __shared__ __align__(16) int dyn[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  constexpr int kWarps = kAdvThreads / 32;
   __shared__ unsigned int s_err;
-  __shared__ unsigned long long s_cnt[kWarps];
+  __shared__ double s_red[kWarps];
   WsPtrs ws = a.ws;
+  // shared copies of cu (n_traj + 1) and the per-trajectory token counts
+  const bool on_chip = a.smem_traj;
+  int* cu = on_chip ? dyn : const_cast<int*>(a.cu);
+  int* cnt_i = on_chip ? dyn + (a.n_traj + 1) : ws.traj_n;
   if (tid == 0) {
     s_err = 0;
     ws.hdr->err_bits = 0;
     ws.hdr->ticket = 0;
+  }
+  for (int i = tid; i <= a.n_traj; i += kAdvThreads) {
+    if (on_chip) cu[i] = a.cu[i];
+    if (i < a.n_traj) cnt_i[i] = 0;
   }
   __syncthreads();
 
   // ---- validation
   unsigned int err = 0;
   for (int i = tid; i < a.n_traj; i += kAdvThreads) {
-    if (a.cu[i] > a.cu[i + 1]) err |= kErrSeqlens;
+    if (cu[i] > cu[i + 1]) err |= kErrSeqlens;
     const int g = a.gid[i];
     if (g < 0 || g >= a.n_groups) err |= kErrGroup;
   }
-  if (tid == 0 && (a.cu[0] != 0 || static_cast<long long>(a.cu[a.n_traj]) != a.R))
-    err |= kErrSeqlens;
+  if (tid == 0 && (cu[0] != 0 || static_cast<long long>(cu[a.n_traj]) != a.R)) err |= kErrSeqlens;
   if (err) atomicOr(&s_err, err);
 
   // ---- group statistics: one warp per group, members found by scanning.
@@ -86,7 +130,7 @@ __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) 
     }
     ss = warp_sum(ss);
     // A group whose rewards are all equal (this includes one-member groups)
-    // carries no advantage signal: its advantages are exactly zero.
+    // carries no advantage signal: its GRPO advantages are exactly zero.
     const int flat = (n == 0) || (wmax == wmin);
     double den = 1.0;
     if (a.normalize_std && !flat) {
@@ -101,43 +145,86 @@ __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) 
     }
   }
   __syncthreads();
+  const bool cu_ok = (s_err & kErrSeqlens) == 0;
+  const bool rpp = a.estimator == RL_EST_REINFORCEPP || a.estimator == RL_EST_REINFORCEPP_BASELINE;
 
-  // ---- per-trajectory advantage
-  for (int i = tid; i < a.n_traj; i += kAdvThreads) {
+  // ---- per-trajectory base value (kept in double in a register-free way:
+  // recomputed from the group table where needed)
+  auto base_value = [&](int i) -> double {
     const int g = a.gid[i];
-    double A = 0.0;
-    if (g >= 0 && g < a.n_groups && !ws.g_flag[g])
-      A = (static_cast<double>(a.rewards[i]) - ws.g_mu[g]) / ws.g_den[g];
+    const bool gok = g >= 0 && g < a.n_groups;
+    const double w = a.rewards[i];
+    if (a.estimator == RL_EST_REINFORCEPP) return w;
+    if (a.estimator == RL_EST_REINFORCEPP_BASELINE) return gok ? w - ws.g_mu[g] : 0.0;
+    if (!gok || ws.g_flag[g]) return 0.0;  // GRPO, GSPO
+    return (w - ws.g_mu[g]) / ws.g_den[g];
+  };
+
+  // ---- per-row pass 1: N and the training tokens of each trajectory
+  unsigned long long n_tok = 0;
+  for (long long t = tid; t < a.R; t += kAdvThreads) {
+    if (a.mask[t] == 0) continue;
+    ++n_tok;
+    if (cu_ok && a.n_traj > 0) atomicAdd(&cnt_i[traj_of(cu, a.n_traj, t)], 1);
+  }
+  const double N = block_sum(static_cast<double>(n_tok), s_red);  // exact below 2^53
+
+  // ---- REINFORCE++: normalise the returns over the training tokens
+  double mu = 0.0, den = 1.0;
+  bool zero_all = false;
+  if (rpp) {
+    double sb = 0.0, bmax = -INFINITY, bmin = INFINITY;
+    for (int i = tid; i < a.n_traj; i += kAdvThreads) {
+      const int n_i = cnt_i[i];
+      if (n_i == 0) continue;
+      const double b = base_value(i);
+      sb += b * n_i;
+      bmax = fmax(bmax, b);
+      bmin = fmin(bmin, b);
+    }
+    sb = block_sum(sb, s_red);
+    bmax = block_max(bmax, s_red);
+    bmin = -block_max(-bmin, s_red);
+    zero_all = !(N > 0.0) || !(bmax != bmin);
+    mu = N > 0.0 ? sb / N : 0.0;
+    double ss = 0.0;
+    for (int i = tid; i < a.n_traj; i += kAdvThreads) {
+      const int n_i = cnt_i[i];
+      if (n_i == 0) continue;
+      const double d = base_value(i) - mu;
+      ss += d * d * n_i;
+    }
+    ss = block_sum(ss, s_red);
+    if (a.normalize_std) {
+      const double ddof = a.unbiased_std ? 1.0 : 0.0;
+      const double var = N > ddof ? ss / (N - ddof) : 0.0;
+      den = fmax(sqrt(var), static_cast<double>(a.std_floor));
+    }
+  }
+
+  // ---- per-trajectory advantage and the count of trajectories that train
+  int n_seq = 0;
+  for (int i = tid; i < a.n_traj; i += kAdvThreads) {
+    double A = base_value(i);
+    if (rpp) A = zero_all ? 0.0 : (A - mu) / den;
     ws.a_traj[i] = static_cast<float>(A);
     if (a.advantages) a.advantages[i] = static_cast<float>(A);
+    const int n_i = cnt_i[i];
+    if (on_chip) ws.traj_n[i] = n_i;
+    n_seq += (n_i > 0);
   }
-  __syncthreads();
-  const bool cu_ok = (s_err & kErrSeqlens) == 0;
+  const double n_seq_all = block_sum(static_cast<double>(n_seq), s_red);
 
-  // ---- per-row advantage (trajectory of row t: last i with cu[i] <= t) and N
-  unsigned long long cnt = 0;
+  // ---- per-row pass 2: the row's advantage, with the one-sample OPD shaping
   for (long long t = tid; t < a.R; t += kAdvThreads) {
     float A = 0.0f;
-    if (cu_ok && a.n_traj > 0) {
-      int lo = 0, hi = a.n_traj;  // invariant: cu[lo] <= t < cu[hi]
-      while (hi - lo > 1) {
-        const int mid = (lo + hi) >> 1;
-        if (static_cast<long long>(a.cu[mid]) <= t) lo = mid; else hi = mid;
-      }
-      A = ws.a_traj[lo];
-    }
+    if (cu_ok && a.n_traj > 0) A = ws.a_traj[traj_of(cu, a.n_traj, t)];
     if (a.teacher) A -= a.opd_coef * (a.rho[t] - a.teacher[t]);
     ws.a_row[t] = A;
-    cnt += (a.mask[t] != 0);
   }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
-  if (lane == 0) s_cnt[warp] = cnt;
-  __syncthreads();
   if (tid == 0) {
-    unsigned long long N = 0;
-    for (int w = 0; w < kWarps; ++w) N += s_cnt[w];
     ws.hdr->n_tokens = static_cast<long long>(N);
+    ws.hdr->n_seq = static_cast<long long>(n_seq_all);
     if (s_err) atomicOr(&ws.hdr->err_bits, s_err);
   }
 }

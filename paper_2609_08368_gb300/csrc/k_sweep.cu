@@ -303,6 +303,12 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
       float H = lnS - tot.u * kLn2 / tot.s;
       float logp = zy_all * a.s.invT - lse;
       if (bad) { logp = 0.0f; H = 0.0f; }
+      if (a.s.topk > 0 && !bad) {
+        // top-K on-policy distillation signal (Sec. 5.2), a fixed per-token reward
+        const long long o = row * a.s.topk;
+        A -= a.s.opd_coef * topk_signal<In>(lg + row * a.ld * static_cast<long long>(sizeof(St)), a.V, a.s.topk_ids + o,
+                                            a.s.topk_teacher + o, a.s.topk, a.s.invT, lse);
+      }
       TokenTerms tt = token_terms(logp, H, rho, q, a.q != nullptr, old, a.old != nullptr, A, a.s);
       if (bad) tt = TokenTerms{0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, kFlagBad};
       if (crank == 0) {

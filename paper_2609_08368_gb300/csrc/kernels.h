@@ -13,6 +13,9 @@ constexpr int kAdvThreads = 1024;
 constexpr int kBwdThreads = 256;
 constexpr int kStreamConsumers = 512;     // consumer threads of k_stream (+ one producer warp)
 constexpr int kMaxSlots = 16;             // ring slots of k_stream
+constexpr int kSeqThreads = 256;
+constexpr int kAdvSmemBytes = 48 * 1024;  // on-chip row offsets + counts when they fit
+constexpr int kMaxTopK = 64;
 
 struct SweepArgs {
   const void* logits;
@@ -72,8 +75,20 @@ struct AdvArgs {
   float opd_coef;
   int normalize_std, unbiased_std;
   float std_floor;
+  int estimator;   // rl_estimator
+  int smem_traj;   // cu_seqlens and per-trajectory counts staged in shared memory
   float* advantages;   // may be null
   int* group_sizes;    // may be null
+  WsPtrs ws;
+};
+
+struct SeqArgs {
+  const int* cu;
+  const float* rho;
+  const float* old;
+  const float* q;
+  const uint8_t* mask;
+  LossScalars s;
   WsPtrs ws;
 };
 
@@ -109,6 +124,7 @@ const void* sweep_kernel(rl_dtype in, rl_dtype out, bool grad, int threads);
 const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad);
 const void* bwd_kernel(rl_dtype in, rl_dtype out);
 const void* adv_kernel();
+const void* seq_kernel();
 const void* stats_kernel();
 
 }  // namespace milesloss

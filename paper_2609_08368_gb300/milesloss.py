@@ -17,6 +17,7 @@ from . import build as _build
 RL_OK = 0
 RL_BF16, RL_F32 = 0, 1
 CORRECTIONS = {"none": 0, "tis": 1, "clip_or_pop": 2}
+ESTIMATORS = {"grpo": 0, "reinforcepp": 1, "reinforcepp_baseline": 2, "gspo": 3}
 STATS_BYTES = 128
 
 
@@ -35,16 +36,27 @@ class RlLossParams(ctypes.Structure):
         ("corr_lo", ctypes.c_float),
         ("corr_hi", ctypes.c_float),
         ("opd_coef", ctypes.c_float),
+        ("estimator", ctypes.c_int32),
+        ("opd_topk", ctypes.c_int32),
+        ("opd_topk_ids", ctypes.c_void_p),
+        ("opd_topk_teacher", ctypes.c_void_p),
     ]
 
 
 def make_params(temperature=1.0, eps_lo=0.2, eps_hi=0.2, dual_clip_c=0.0, kl_coef=0.0,
                 entropy_coef=0.0, std_floor=1e-6, normalize_std=True, unbiased_std=True,
-                correction="none", corr_lo=0.0, corr_hi=2.0, opd_coef=0.0) -> RlLossParams:
+                correction="none", corr_lo=0.0, corr_hi=2.0, opd_coef=0.0, estimator="grpo",
+                opd_topk=0, opd_topk_ids=None, opd_topk_teacher=None) -> RlLossParams:
+    """One rl_loss_params. ``opd_topk_ids`` / ``opd_topk_teacher`` are device
+    tensors ([n_rows, K] int32 / fp32); the caller keeps them alive."""
     return RlLossParams(temperature, eps_lo, eps_hi, dual_clip_c, kl_coef, entropy_coef,
                         std_floor, int(bool(normalize_std)), int(bool(unbiased_std)),
                         CORRECTIONS[correction] if isinstance(correction, str) else int(correction),
-                        corr_lo, corr_hi, opd_coef)
+                        corr_lo, corr_hi, opd_coef,
+                        ESTIMATORS[estimator] if isinstance(estimator, str) else int(estimator),
+                        int(opd_topk),
+                        None if opd_topk_ids is None else opd_topk_ids.data_ptr(),
+                        None if opd_topk_teacher is None else opd_topk_teacher.data_ptr())
 
 
 class MilesLossError(RuntimeError):

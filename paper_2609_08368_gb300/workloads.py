@@ -50,6 +50,8 @@ class Recipe:
     seed: int = 1000
     old_noise: float | None = None  # optional old (pi_old) log-probs
     teacher_noise: float | None = None  # optional OPD teacher log-probs
+    topk: int = 0                   # OPD top-K candidates per row (the student's K most likely)
+    topk_noise: float = 0.3         # teacher log-prob of a candidate = student's + N(0, s^2)
 
     @property
     def n_traj(self) -> int:
@@ -107,6 +109,8 @@ class Workload:
     loss_mask: torch.Tensor     # [R] uint8
     n_groups: int
     params: dict
+    topk_ids: torch.Tensor | None = None      # [R, K] int32
+    topk_teacher: torch.Tensor | None = None  # [R, K] f32
 
     @property
     def n_rows(self) -> int:
@@ -123,7 +127,8 @@ class Workload:
                         mv(self.rollout_logprobs), mv(self.ref_logprobs),
                         mv(self.old_logprobs), mv(self.teacher_logprobs),
                         mv(self.rewards), mv(self.group_id), mv(self.cu_seqlens),
-                        mv(self.loss_mask), self.n_groups, dict(self.params))
+                        mv(self.loss_mask), self.n_groups, dict(self.params),
+                        mv(self.topk_ids), mv(self.topk_teacher))
 
 
 def _rewards(kind: str, n_traj: int, group_size: int, rng: np.random.Generator):
@@ -153,6 +158,10 @@ def _mask(kind: str, n_traj: int, traj_len: int, rng: np.random.Generator):
             m[i, :min(traj_len, int(rng.integers(32, 129)))] = 0
     elif kind == "prefix_frac0.25":
         m[:, :traj_len // 4] = 0
+    elif kind == "prefix_u0_half":
+        # prompt prefixes of U[0, traj_len/2] tokens: unequal training lengths
+        for i in range(n_traj):
+            m[i, :int(rng.integers(0, traj_len // 2 + 1))] = 0
     elif kind == "tool_spans":
         # Model-token spans U[64,512] alternate with masked tool-output spans
         # U[128,2048], starting with a model span.
@@ -224,6 +233,21 @@ def make(rec: Recipe, device="cpu", ld: int | None = None) -> Workload:
     old = noisy(rec.old_noise) if rec.old_noise is not None else None
     teacher = noisy(rec.teacher_noise) if rec.teacher_noise is not None else None
 
+    topk_ids = topk_teacher = None
+    if rec.topk > 0:
+        # the student's K most likely tokens and the teacher's log-probs of them
+        K = min(rec.topk, V)
+        topk_ids = torch.empty((R, K), dtype=torch.int32, device=device)
+        topk_teacher = torch.empty((R, K), dtype=torch.float32, device=device)
+        for lo in range(0, R, 512):
+            hi = min(R, lo + 512)
+            s = logits[lo:hi, :V].to(torch.float64) / T
+            vals, ids = torch.topk(s, K, dim=1)
+            lps = vals - torch.logsumexp(s, dim=1, keepdim=True)
+            e = torch.randn((hi - lo, K), generator=gen, device=device, dtype=torch.float64)
+            topk_ids[lo:hi] = ids.to(torch.int32)
+            topk_teacher[lo:hi] = (lps + rec.topk_noise * e).to(torch.float32)
+
     w = _rewards(rec.reward, n_traj, rec.group_size, rng)
     gid = (np.arange(n_traj) // rec.group_size).astype(np.int32)
     cu = (np.arange(n_traj + 1) * rec.traj_len).astype(np.int32)
@@ -233,4 +257,4 @@ def make(rec: Recipe, device="cpu", ld: int | None = None) -> Workload:
         return torch.from_numpy(a).to(device)
 
     return Workload(rec, logits, targets, rho, ref, old, teacher, dev(w), dev(gid),
-                    dev(cu), dev(mask), rec.n_prompts, dict(rec.params))
+                    dev(cu), dev(mask), rec.n_prompts, dict(rec.params), topk_ids, topk_teacher)

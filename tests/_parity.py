@@ -21,7 +21,16 @@ GUARD = 1e-5
 
 
 def oracle_params(params: dict) -> oracle.LossParams:
-    return oracle.LossParams(**params)
+    return oracle.LossParams(**{k: v for k, v in params.items()
+                                if k not in ("opd_topk_ids", "opd_topk_teacher")})
+
+
+def gpu_params(w, params=None) -> dict:
+    """The call's parameters with the top-K OPD inputs attached when used."""
+    p = dict(w.params if params is None else params)
+    if p.get("opd_topk", 0) > 0:
+        p.update(opd_topk_ids=w.topk_ids, opd_topk_teacher=w.topk_teacher)
+    return p
 
 
 def host_logits(w, rows=None) -> np.ndarray:
@@ -45,6 +54,7 @@ def run_gpu(w, mode="fused", dl_dtype=None, grad_loss=1.0, ld_out=None, params=N
     buf = api.alloc(R, n_traj, w.n_groups, w.logits.device, vocab=w.vocab,
                     dlogits_dtype=None if mode == "fwd" else dl_dtype, ld_out=ld_out,
                     fill_nan=True)
+    params = gpu_params(w, params)
     if mode == "fused":
         api.fwd_bwd(w, buf, params=params, grad_loss=grad_loss)
     else:
@@ -66,7 +76,8 @@ def run_oracle(w, grad_loss=1.0, want_dlogits=True, params=None):
                           np_(w.ref_logprobs), np_(w.rewards), np_(w.group_id),
                           np_(w.cu_seqlens), w.n_groups, np_(w.loss_mask), p,
                           grad_loss=grad_loss, old=np_(w.old_logprobs),
-                          teacher=np_(w.teacher_logprobs), want_dlogits=want_dlogits)
+                          teacher=np_(w.teacher_logprobs), want_dlogits=want_dlogits,
+                          topk_ids=np_(w.topk_ids), topk_teacher=np_(w.topk_teacher))
 
 
 def logp_tol(w) -> float:
@@ -148,13 +159,24 @@ def compare_forward(w, g, o, params=None):
     # GPU counts exactly (up to tokens in the guard band); against the
     # oracle's float64 log-probs they differ only inside the band.
     old = np_(w.old_logprobs)
-    c_gpu, band_g = clip_counts(p, g["logp"].astype(np.float64), np_(w.rollout_logprobs),
-                                np_(w.ref_logprobs), o["A_row"], g["H"], np_(w.loss_mask), old)
-    c_ora, band_o = clip_counts(p, o["logp"], np_(w.rollout_logprobs), np_(w.ref_logprobs),
-                                o["A_row"], o["H"], np_(w.loss_mask), old)
-    for k in c_gpu:
-        assert abs(st[k] - c_gpu[k]) <= band_g, (k, st[k], c_gpu[k], band_g)
-        assert abs(st[k] - c_ora[k]) <= band_g + band_o, (k, st[k], c_ora[k])
+    if p.estimator == "gspo":
+        # sequence-level decisions: every training token of a trajectory
+        # carries its sequence's flags; tokens of sequences whose ratio lies in
+        # the guard band of a threshold may fall either way
+        m = np_(w.loss_mask).astype(bool)
+        th = [1 - p.eps_lo, 1 + p.eps_hi] + ([p.dual_clip_c] if p.dual_clip_c else [])
+        band = int(sum(((np.abs(o["r"] - t) <= GUARD * t) & m).sum() for t in th))
+        for k in ("n_clip_hi", "n_clip_lo", "n_dual_clip", "n_corr_clip"):
+            assert abs(st[k] - o["stats"][k]) <= band, (k, st[k], o["stats"][k], band)
+    else:
+        c_gpu, band_g = clip_counts(p, g["logp"].astype(np.float64), np_(w.rollout_logprobs),
+                                    np_(w.ref_logprobs), o["A_row"], g["H"], np_(w.loss_mask),
+                                    old)
+        c_ora, band_o = clip_counts(p, o["logp"], np_(w.rollout_logprobs), np_(w.ref_logprobs),
+                                    o["A_row"], o["H"], np_(w.loss_mask), old)
+        for k in c_gpu:
+            assert abs(st[k] - c_gpu[k]) <= band_g, (k, st[k], c_gpu[k], band_g)
+            assert abs(st[k] - c_ora[k]) <= band_g + band_o, (k, st[k], c_ora[k])
     os_ = o["stats"]
     scale = max(abs(os_["loss"]), float(np.abs(o["ell"][np_(w.loss_mask).astype(bool)]).mean())
                 if o["N"] else 0.0)

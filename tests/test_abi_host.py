@@ -123,6 +123,11 @@ INVALID = [
     dict(params=dict(correction=5), old=FAKE),
     dict(params=dict(opd_coef=0.5)),                   # no teacher log-probs
     dict(params=dict(opd_coef=float("nan")), teacher=FAKE),
+    dict(params=dict(estimator=4)),
+    dict(params=dict(estimator=-1)),
+    dict(params=dict(opd_coef=0.5, opd_topk=4)),        # no candidate ids / teacher log-probs
+    dict(params=dict(opd_coef=0.5, opd_topk=65), teacher=FAKE),
+    dict(params=dict(opd_topk=-1)),
 ]
 
 
@@ -155,10 +160,12 @@ def test_bwd_and_fwd_validate_too(lib):
 
 
 def test_params_struct_layout_matches_header():
-    assert ctypes.sizeof(ml.RlLossParams) == 52
+    assert ctypes.sizeof(ml.RlLossParams) == 80
     text = open(HEADER).read()
-    body = text[text.index("typedef struct {", text.index("rl_correction;")):
+    body = text[text.index("typedef struct {", text.index("} rl_estimator;")):
                 text.index("} rl_loss_params;")]
-    fields = re.findall(r"\b(?:float|int32_t)\s+([a-z_0-9]+(?:\s*,\s*[a-z_0-9]+)*)\s*;", body)
+    body = re.sub(r"/\*.*?\*/", "", body, flags=re.S)
+    fields = re.findall(r"(?:float|int32_t|const int32_t\s*\*|const float\s*\*)\s*"
+                        r"([a-z_0-9]+(?:\s*,\s*[a-z_0-9]+)*)\s*;", body)
     names = [n.strip() for group in fields for n in group.split(",")]
     assert names == [f[0] for f in ml.RlLossParams._fields_]

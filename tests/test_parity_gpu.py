@@ -176,6 +176,41 @@ def test_temperature_entropy_kl_correction_opd():
 
 
 @pytest.mark.parametrize("kind", ["cluster", "stream"])
+@pytest.mark.parametrize("params", [
+    dict(estimator="reinforcepp"),
+    dict(estimator="reinforcepp_baseline", dual_clip_c=2.0, kl_coef=0.05),
+    dict(estimator="reinforcepp", normalize_std=False, unbiased_std=False),
+    dict(estimator="gspo", dual_clip_c=1.5, kl_coef=0.05, entropy_coef=0.01),
+    dict(estimator="gspo", correction="tis", corr_lo=0.0, corr_hi=1.1, eps_lo=0.1, eps_hi=0.1),
+    dict(estimator="gspo", correction="clip_or_pop", corr_lo=0.9, corr_hi=1.1, temperature=0.8),
+], ids=["rpp", "rpp_base", "rpp_center", "gspo", "gspo_tis", "gspo_pop"])
+def test_advantage_estimators(monkeypatch, kind, params):
+    """REINFORCE++ (plain, baseline-relative) and GSPO (Sec. 3.4), fused and
+    split, on both sweep kernels; trajectories of unequal training length."""
+    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=3, group_size=4, traj_len=20, vocab=9000,
+                    rho_noise=0.3, ref_noise=0.2, old_noise=0.1, mask="prefix_u0_half")
+    w = wl.make(rec, DEV)
+    _full_check(w, params=params)
+    _full_check(w, mode="split", params=params)
+
+
+@pytest.mark.parametrize("kind", ["cluster", "stream"])
+@pytest.mark.parametrize("K", [1, 4, 16])
+def test_opd_topk(monkeypatch, kind, K):
+    """The top-K on-policy distillation signal (Sec. 5.2) from candidate sets
+    and teacher log-probs, in the sweep epilogue."""
+    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=2, group_size=4, traj_len=24, vocab=12000,
+                    rho_noise=0.3, ref_noise=0.2, topk=K, topk_noise=0.4)
+    w = wl.make(rec, DEV)
+    for params in (dict(opd_coef=0.5, opd_topk=K, dual_clip_c=2.0),
+                   dict(opd_coef=-0.3, opd_topk=K, estimator="reinforcepp_baseline")):
+        _full_check(w, params=params)
+        _full_check(w, mode="split", params=params)
+
+
+@pytest.mark.parametrize("kind", ["cluster", "stream"])
 def test_no_training_tokens_and_empty_call(monkeypatch, kind):
     monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
     rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=1, group_size=2, traj_len=8, vocab=300)
