@@ -47,6 +47,7 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="glm")
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--e2e-chunk-rows", type=int, default=4096)
     ap.add_argument("--cpu-sample-rows", type=int, default=3072)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -301,6 +302,7 @@ def run_ours(args, rank, world, local):
     w = wl.make(rec, dev)
     R, V = w.n_rows, w.vocab
     dl_dtype = w.logits.dtype
+    dt_name = "bf16" if w.logits.dtype == torch.bfloat16 else "f32"
     buf = api.alloc(R, int(w.rewards.shape[0]), w.n_groups, dev, vocab=V, dlogits_dtype=dl_dtype)
     stream = torch.cuda.current_stream()
 
@@ -342,7 +344,7 @@ def run_ours(args, rank, world, local):
     rows_all = sum_over_ranks(float(R), world)
     value = rows_all * K / (ms_total / 1e3)
 
-    bpr = algorithmic_bytes_per_row(w, dl_dtype)
+    bpr = algorithmic_bytes_per_row(w, dl_dtype)  # before w is released for the e2e leg
     launch_bytes = bpr * R
     sweep_avg = statistics.fmean(sweep_ms)
     peaks, peak_kind = measured_peaks()
@@ -350,11 +352,20 @@ def run_ours(args, rank, world, local):
     achieved = launch_bytes / (sweep_avg / 1e3) / 1e9
     step_gbs = launch_bytes / (ms_step / 1e3) / 1e9
 
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rps, secs, n = oracle_sample(w, args.cpu_sample_rows)
+        cpu = {"value": rps, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+               "sample": f"{n} random rows of the {R} x {V} batch (every per-row output and "
+                         f"dLogits of those rows; call-wide advantages and N), {secs:.1f} s"}
+
     # end to end through host buffers (pinned), one call per step
     e2e = None
     if not args.no_e2e and args.e2e_steps > 0:
         host_w = _pinned_copy(w)
-        call = api.HostCall(host_w, dev, dev_w=w, buf=buf)
+        del w, buf  # the pipelined call keeps its own two chunk buffers
+        torch.cuda.empty_cache()
+        call = api.PipelinedHostCall(host_w, dev, chunk_rows=args.e2e_chunk_rows)
         call()
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -369,15 +380,10 @@ def run_ours(args, rank, world, local):
         ms_e2e = max_over_ranks(e0.elapsed_time(e1), world) / args.e2e_steps
         e2e = {"value": rows_all / (ms_e2e / 1e3), "unit": "tokens/s",
                "ms_per_step": ms_e2e, "steps": args.e2e_steps,
+               "how": f"pinned host buffers, rl_loss_fwd_bwd_rows over chunks of "
+                      f"{args.e2e_chunk_rows} rows, copies overlapped with the sweep",
                "h2d_bytes_per_step": call.bytes_in(), "d2h_bytes_per_step": call.bytes_out()}
         del call, host_w
-
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        rps, secs, n = oracle_sample(w, args.cpu_sample_rows)
-        cpu = {"value": rps, "unit": "tokens/s", "cores": 1, "kind": "oracle",
-               "sample": f"{n} random rows of the {R} x {V} batch (every per-row output and "
-                         f"dLogits of those rows; call-wide advantages and N), {secs:.1f} s"}
 
     traffic = profiled_traffic(R)
     line = {
@@ -386,7 +392,7 @@ def run_ours(args, rank, world, local):
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": f"{args.workload}: {R} rows ({rec.n_traj} traj x {rec.traj_len} "
                                f"tokens, groups of {rec.group_size}) x vocab {V}, "
-                               f"{'bf16' if w.logits.dtype == torch.bfloat16 else 'f32'} logits "
+                               f"{dt_name} logits "
                                f"-> dLogits",
                    "rows": R, "vocab": V, "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2 (20+ GB per step), no flush"},

@@ -234,6 +234,42 @@ rl_status rl_loss_fwd_bwd(const void* logits, rl_dtype logits_dtype, int64_t n_r
                           rl_dtype dlogits_dtype, int64_t ld_out, void* workspace,
                           size_t workspace_bytes, rl_stream stream);
 
+/* Phases of rl_loss_fwd_bwd_rows. */
+enum {
+  RL_PHASE_BEGIN = 1, /* advantages, N and validation over the whole call      */
+  RL_PHASE_ROWS = 2,  /* the vocabulary sweep over rows [row_begin, row_end)   */
+  RL_PHASE_END = 4,   /* the loss and its statistics over the whole call       */
+  RL_PHASE_ALL = 7
+};
+
+/* rl_loss_fwd_bwd for logits that exist a block of rows at a time (the usual
+ * way to bound the memory of the language-model head): one BEGIN, any number
+ * of ROWS calls that together cover the rows once, one END, all on the same
+ * workspace and stream (or ordered by the caller across streams). The
+ * arguments are those of rl_loss_fwd_bwd for the whole call (n_rows, the
+ * per-row inputs and outputs, rewards, groups, cu_seqlens), except:
+ *  logits    rows [row_begin, row_end): logits points at row row_begin with
+ *            row stride ld (the chunk buffer); NULL outside ROWS
+ *  dlogits   the same rows of dLogits, pointing at row row_begin; NULL runs
+ *            the chunk forward-only (log-probs, entropy, loss terms; the
+ *            per-row state stays in the workspace)
+ * rl_loss_fwd_bwd_rows(RL_PHASE_ALL, 0, n_rows, ...) is rl_loss_fwd_bwd.
+ * GSPO needs every log-prob before any gradient: with RL_EST_GSPO only that
+ * whole call is accepted (RL_ERR_UNSUPPORTED otherwise). */
+rl_status rl_loss_fwd_bwd_rows(int32_t phase, int64_t row_begin, int64_t row_end,
+                               const void* logits, rl_dtype logits_dtype, int64_t n_rows,
+                               int64_t vocab, int64_t ld, const int32_t* targets,
+                               const float* rollout_logprobs, const float* ref_logprobs,
+                               const float* old_logprobs, const float* teacher_logprobs,
+                               const float* rewards, const int32_t* group_id,
+                               const int32_t* cu_seqlens, int32_t n_traj, int32_t n_groups,
+                               const uint8_t* loss_mask, const rl_loss_params* params,
+                               float* token_logprobs, float* entropy, float* advantages,
+                               int32_t* group_sizes, rl_loss_stats* stats, float grad_loss,
+                               const float* grad_loss_device, void* dlogits,
+                               rl_dtype dlogits_dtype, int64_t ld_out, void* workspace,
+                               size_t workspace_bytes, rl_stream stream);
+
 /* rl_loss_fwd_bwd for callers that cannot allocate device memory at call
  * time (the paper has no counterpart; this is a deployment convenience).
  * Frameworks that reserve nearly all of HBM for their own pool, plain-C

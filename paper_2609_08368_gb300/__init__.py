@@ -17,6 +17,7 @@ from .milesloss import (  # noqa: F401
     rl_loss_check_device_error,
     rl_loss_fwd,
     rl_loss_fwd_bwd,
+    rl_loss_fwd_bwd_rows,
     rl_loss_workspace_size,
     rl_set_sweep_events,
     status_string,

@@ -117,3 +117,122 @@ class HostCall:
         self.out["entropy"].copy_(self.buf.entropy, non_blocking=True)
         self.out["stats"].copy_(self.buf.stats, non_blocking=True)
         return self.out
+
+
+def _rows_call(w, buf, phase, r0, r1, logits, dlogits, params=None, grad_loss=1.0, stream=None):
+    ml.rl_loss_fwd_bwd_rows(phase, r0, r1, w.n_rows, logits, w.targets, w.rollout_logprobs,
+                            w.ref_logprobs, w.old_logprobs, w.teacher_logprobs, w.rewards,
+                            w.group_id, w.cu_seqlens, w.n_groups, w.loss_mask,
+                            params if params is not None else w.params, buf.token_logprobs,
+                            buf.entropy, buf.advantages, buf.group_sizes, buf.stats, dlogits,
+                            buf.workspace, w.vocab,
+                            logits_dtype=(w.logits.dtype if w.logits is not None
+                                          else (logits.dtype if logits is not None
+                                                else torch.bfloat16)),
+                            grad_loss=grad_loss, stream=stream)
+
+
+def fwd_bwd_chunked(w, buf: Buffers, chunk_rows: int, params=None, grad_loss=1.0,
+                    forward_only=False):
+    """The fused call as BEGIN, one ROWS call per block of ``chunk_rows`` rows
+    (each reading a view of the logits and writing a view of dLogits), END."""
+    R = w.n_rows
+    _rows_call(w, buf, ml.RL_PHASE_BEGIN, 0, R, None, None, params, grad_loss)
+    for r0 in range(0, R, chunk_rows):
+        r1 = min(R, r0 + chunk_rows)
+        dl = None if forward_only else buf.dlogits[r0:r1]
+        _rows_call(w, buf, ml.RL_PHASE_ROWS, r0, r1, w.logits[r0:r1], dl, params, grad_loss)
+    _rows_call(w, buf, ml.RL_PHASE_END, 0, R, None, None, params, grad_loss)
+
+
+class PipelinedHostCall:
+    """The fused call with logits and dLogits in pinned HOST memory, streamed
+    through two device chunk buffers: per chunk of rows, the host-to-device
+    copy (one stream), the vocabulary sweep (the caller's stream) and the
+    device-to-host copy of dLogits (a third stream) overlap with the other
+    chunks'. The small per-row inputs go to the device whole before the sweep
+    (BEGIN needs all of them)."""
+
+    SMALL = ("targets", "rollout_logprobs", "ref_logprobs", "old_logprobs", "teacher_logprobs",
+             "rewards", "group_id", "cu_seqlens", "loss_mask", "topk_ids", "topk_teacher")
+
+    def __init__(self, host_w, device, chunk_rows=4096, dlogits_dtype=None):
+        from . import workloads as wl
+        self.host = host_w
+        self.chunk = chunk_rows
+        R, V = host_w.n_rows, host_w.vocab
+        self.dl_dtype = dlogits_dtype or host_w.logits.dtype
+
+        def dev(t):
+            return None if t is None else torch.empty_like(t, device=device)
+        self.dev = wl.Workload(host_w.recipe, None, dev(host_w.targets),
+                               dev(host_w.rollout_logprobs), dev(host_w.ref_logprobs),
+                               dev(host_w.old_logprobs), dev(host_w.teacher_logprobs),
+                               dev(host_w.rewards), dev(host_w.group_id), dev(host_w.cu_seqlens),
+                               dev(host_w.loss_mask), host_w.n_groups, dict(host_w.params),
+                               dev(host_w.topk_ids), dev(host_w.topk_teacher))
+        n = min(chunk_rows, R)
+        self.lg = [torch.empty((n, V), dtype=host_w.logits.dtype, device=device) for _ in range(2)]
+        self.dl = [torch.empty((n, V), dtype=self.dl_dtype, device=device) for _ in range(2)]
+        self.buf = alloc(R, int(host_w.rewards.shape[0]), host_w.n_groups, device, vocab=V)
+        pin = dict(pin_memory=True)
+        self.out = dict(
+            dlogits=torch.empty((R, V), dtype=self.dl_dtype, **pin),
+            token_logprobs=torch.empty(R, dtype=torch.float32, **pin),
+            entropy=torch.empty(R, dtype=torch.float32, **pin),
+            stats=torch.empty(ml.STATS_BYTES, dtype=torch.uint8, **pin))
+        self.s_in = torch.cuda.Stream(device=device)
+        self.s_out = torch.cuda.Stream(device=device)
+        self.params = dict(host_w.params)
+        if self.params.get("opd_topk", 0) > 0:
+            self.params.update(opd_topk_ids=self.dev.topk_ids,
+                               opd_topk_teacher=self.dev.topk_teacher)
+
+    def bytes_in(self) -> int:
+        h = self.host
+        return h.logits[:, :h.vocab].numel() * h.logits.element_size() + sum(
+            getattr(h, k).numel() * getattr(h, k).element_size()
+            for k in self.SMALL if getattr(h, k) is not None)
+
+    def bytes_out(self) -> int:
+        return sum(t.numel() * t.element_size() for t in self.out.values())
+
+    def __call__(self, grad_loss=1.0):
+        comp = torch.cuda.current_stream()
+        h, d = self.host, self.dev
+        R, V = h.n_rows, h.vocab
+        for k in self.SMALL:
+            if getattr(h, k) is not None:
+                getattr(d, k).copy_(getattr(h, k), non_blocking=True)
+        _rows_call(d, self.buf, ml.RL_PHASE_BEGIN, 0, R, None, None, self.params, grad_loss)
+        comp_done = [None, None]
+        out_done = [None, None]
+        for i, r0 in enumerate(range(0, R, self.chunk)):
+            r1 = min(R, r0 + self.chunk)
+            b, n = i % 2, r1 - r0
+            if comp_done[b] is not None:   # the sweep two chunks back read lg[b]
+                self.s_in.wait_event(comp_done[b])
+            with torch.cuda.stream(self.s_in):
+                self.lg[b][:n].copy_(h.logits[r0:r1, :V], non_blocking=True)
+                in_done = torch.cuda.Event()
+                in_done.record(self.s_in)
+            comp.wait_event(in_done)
+            if out_done[b] is not None:    # dl[b] was copied out
+                comp.wait_event(out_done[b])
+            _rows_call(d, self.buf, ml.RL_PHASE_ROWS, r0, r1, self.lg[b][:n], self.dl[b][:n],
+                       self.params, grad_loss)
+            comp_done[b] = torch.cuda.Event()
+            comp_done[b].record(comp)
+            self.s_out.wait_event(comp_done[b])
+            with torch.cuda.stream(self.s_out):
+                self.out["dlogits"][r0:r1].copy_(self.dl[b][:n], non_blocking=True)
+                out_done[b] = torch.cuda.Event()
+                out_done[b].record(self.s_out)
+        _rows_call(d, self.buf, ml.RL_PHASE_END, 0, R, None, None, self.params, grad_loss)
+        self.out["token_logprobs"].copy_(self.buf.token_logprobs, non_blocking=True)
+        self.out["entropy"].copy_(self.buf.entropy, non_blocking=True)
+        self.out["stats"].copy_(self.buf.stats, non_blocking=True)
+        for e in out_done:
+            if e is not None:
+                comp.wait_event(e)
+        return self.out

@@ -263,10 +263,10 @@ struct Common {
   const rl_loss_params* p;
 };
 
-rl_status check_common(const Common& c) {
+rl_status check_common(const Common& c, bool need_logits = true) {
   if (!dtype_ok(c.dt)) return RL_ERR_INVALID_ARG;
   if (c.R < 0 || c.V < 1 || c.V > INT_MAX / 8 || c.ld < c.V) return RL_ERR_INVALID_ARG;
-  if (c.R > 0 && (!c.logits || !c.targets || !c.mask)) return RL_ERR_INVALID_ARG;
+  if (c.R > 0 && ((need_logits && !c.logits) || !c.targets || !c.mask)) return RL_ERR_INVALID_ARG;
   return check_params(c.p);
 }
 
@@ -282,8 +282,8 @@ struct FwdIn {
   size_t ws_bytes;
 };
 
-rl_status check_fwd(const FwdIn& f) {
-  rl_status st = check_common(f.c);
+rl_status check_fwd(const FwdIn& f, bool need_logits = true) {
+  rl_status st = check_common(f.c, need_logits);
   if (st != RL_OK) return st;
   const rl_loss_params* p = f.c.p;
   if (f.n_traj < 0 || f.n_groups < 0) return RL_ERR_INVALID_ARG;
@@ -314,13 +314,32 @@ struct GradOut {
   long long ld_out;
 };
 
-rl_status check_grad(const Common& c, const GradOut& o) {
+rl_status check_grad(const Common& c, const GradOut& o, bool need_out = true) {
   if (!finite(o.g)) return RL_ERR_INVALID_ARG;
   if (!dtype_ok(o.dt)) return RL_ERR_INVALID_ARG;
   if (o.ld_out < c.V) return RL_ERR_INVALID_ARG;
-  if (c.R > 0 && !o.dl) return RL_ERR_INVALID_ARG;
+  if (c.R > 0 && need_out && !o.dl) return RL_ERR_INVALID_ARG;
   return RL_OK;
 }
+
+// The per-row arrays of a workspace view shifted to start at row r0.
+WsPtrs rows_from(WsPtrs w, long long r0) {
+  w.a_row += r0;
+  w.logp += r0;
+  w.H += r0;
+  w.lse += r0;
+  w.G += r0;
+  w.ell += r0;
+  w.pg += r0;
+  w.k3 += r0;
+  w.r += r0;
+  w.rc += r0;
+  w.flags += r0;
+  return w;
+}
+
+template <class T>
+T* shift(T* p, long long r0) { return p ? p + r0 : p; }
 
 void record(cudaEvent_t ev, cudaStream_t s) {
   if (ev && t_ev_begin && t_ev_end) cudaEventRecord(ev, s);
@@ -356,13 +375,22 @@ rl_status launch_bwd(const Common& c, const GradOut& go, const WsPtrs& ws, cudaS
                 1, s, &b);
 }
 
-rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s) {
+// phase: RL_PHASE_BEGIN (advantages, N), RL_PHASE_ROWS (the sweep over rows
+// [r0, r1), whose logits / dLogits pointers address row r0), RL_PHASE_END
+// (the statistics); rl_loss_fwd / rl_loss_fwd_bwd run all three on [0, R).
+rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase = RL_PHASE_ALL,
+                  long long r0 = 0, long long r1 = -1) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return RL_ERR_CUDA;
-  const Common& c = f.c;
-  const WsLayout L = WsLayout::make(c.R, f.n_traj, f.n_groups);
-  const WsPtrs ws = WsPtrs::at(f.ws, L);
+  const Common& call = f.c;
+  if (r1 < 0) r1 = call.R;
+  const WsLayout L = WsLayout::make(call.R, f.n_traj, f.n_groups);
+  const WsPtrs ws_all = WsPtrs::at(f.ws, L);
+  rl_status st = RL_OK;
 
+  if (phase & RL_PHASE_BEGIN) {
+  const Common& c = call;
+  const WsPtrs& ws = ws_all;
   // advantages, N, validation
   AdvArgs aa;
   aa.R = c.R;
@@ -384,14 +412,35 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s) {
   const size_t traj_bytes = (2 * static_cast<size_t>(f.n_traj) + 1) * sizeof(int);
   aa.smem_traj = traj_bytes <= static_cast<size_t>(kAdvSmemBytes);
   aa.ws = ws;
-  rl_status st = launch(adv_kernel(), dim3(1), dim3(kAdvThreads),
-                        aa.smem_traj ? static_cast<int>(traj_bytes) : 0, 1, s, &aa);
+  st = launch(adv_kernel(), dim3(1), dim3(kAdvThreads),
+              aa.smem_traj ? static_cast<int>(traj_bytes) : 0, 1, s, &aa);
   if (st != RL_OK) return st;
+  }
 
   // GSPO: the gradient of a token depends on its whole trajectory, so the
   // call runs as forward sweep -> per-trajectory pass -> gradient sweep.
-  const bool gspo = c.p->estimator == RL_EST_GSPO;
+  const bool gspo = call.p->estimator == RL_EST_GSPO;
   const GradOut* go_sweep = gspo ? nullptr : go;
+
+  // the sweep sees rows [r0, r1) as a call of its own: per-row pointers and
+  // the workspace's per-row arrays start at row r0
+  Common c = call;
+  c.R = (phase & RL_PHASE_ROWS) ? r1 - r0 : 0;
+  c.targets = shift(call.targets, r0);
+  c.mask = shift(call.mask, r0);
+  FwdIn fr = f;
+  fr.c = c;
+  fr.rho = shift(f.rho, r0);
+  fr.q = shift(f.q, r0);
+  fr.old = shift(f.old, r0);
+  fr.out_logp = shift(f.out_logp, r0);
+  fr.out_H = shift(f.out_H, r0);
+  const WsPtrs ws = rows_from(ws_all, r0);
+  LossScalars sc = scalars(call.p);
+  if (sc.topk) {
+    sc.topk_ids = shift(sc.topk_ids, r0 * sc.topk);
+    sc.topk_teacher = shift(sc.topk_teacher, r0 * sc.topk);
+  }
 
   const bool grad = go_sweep != nullptr;
   const size_t es = elem_size(c.dt);
@@ -417,17 +466,17 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s) {
     ta.n_slots = sp.slots;
     ta.out_vec = out_vec;
     ta.targets = c.targets;
-    ta.rho = f.rho;
-    ta.q = f.q;
-    ta.old = f.old;
+    ta.rho = fr.rho;
+    ta.q = fr.q;
+    ta.old = fr.old;
     ta.mask = c.mask;
-    ta.out_logp = f.out_logp;
-    ta.out_H = f.out_H;
+    ta.out_logp = fr.out_logp;
+    ta.out_H = fr.out_H;
     ta.dlogits = grad ? go->dl : nullptr;
     ta.ld_out = grad ? go->ld_out : 0;
     ta.grad_loss = grad ? go->g : 0.0f;
     ta.grad_loss_dev = grad ? go->g_dev : nullptr;
-    ta.s = scalars(c.p);
+    ta.s = sc;
     ta.ws = ws;
     const long long grid = std::min<long long>(ctas, c.R);
     record(t_ev_begin, s);
@@ -458,17 +507,17 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s) {
     sa.in_bulk = in_bulk;
     sa.out_vec = out_vec;
     sa.targets = c.targets;
-    sa.rho = f.rho;
-    sa.q = f.q;
-    sa.old = f.old;
+    sa.rho = fr.rho;
+    sa.q = fr.q;
+    sa.old = fr.old;
     sa.mask = c.mask;
-    sa.out_logp = f.out_logp;
-    sa.out_H = f.out_H;
+    sa.out_logp = fr.out_logp;
+    sa.out_H = fr.out_H;
     sa.dlogits = grad ? go->dl : nullptr;
     sa.ld_out = grad ? go->ld_out : 0;
     sa.grad_loss = grad ? go->g : 0.0f;
     sa.grad_loss_dev = grad ? go->g_dev : nullptr;
-    sa.s = scalars(c.p);
+    sa.s = sc;
     sa.ws = ws;
     record(t_ev_begin, s);
     st = launch(fn, dim3(static_cast<unsigned>(n_cl * pl.C)), dim3(pl.threads), pl.smem, pl.C,
@@ -477,34 +526,34 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s) {
     if (st != RL_OK) return st;
   }
 
-  if (gspo && c.R > 0 && f.n_traj > 0) {
+  if (gspo && (phase & RL_PHASE_ROWS) && call.R > 0 && f.n_traj > 0) {
     SeqArgs qa;
     qa.cu = f.cu;
     qa.rho = f.rho;
     qa.old = f.old;
     qa.q = f.q;
-    qa.mask = c.mask;
-    qa.s = scalars(c.p);
-    qa.ws = ws;
+    qa.mask = call.mask;
+    qa.s = scalars(call.p);
+    qa.ws = ws_all;
     st = launch(seq_kernel(), dim3(static_cast<unsigned>(f.n_traj)), dim3(kSeqThreads), 0, 1, s,
                 &qa);
     if (st != RL_OK) return st;
   }
 
-  if (f.stats) {
+  if ((phase & RL_PHASE_END) && f.stats) {
     StatArgs ta;
-    ta.R = c.R;
-    ta.mask = c.mask;
+    ta.R = call.R;
+    ta.mask = call.mask;
     ta.rho = f.rho;
     ta.out = f.stats;
-    ta.ws = ws;
-    long long blocks = (c.R + kStatThreads * 4 - 1) / (kStatThreads * 4);
+    ta.ws = ws_all;
+    long long blocks = (call.R + kStatThreads * 4 - 1) / (kStatThreads * 4);
     blocks = std::max<long long>(1, std::min<long long>(blocks, kMaxStatBlocks));
     st = launch(stats_kernel(), dim3(static_cast<unsigned>(blocks)), dim3(kStatThreads), 0, 1, s,
                 &ta);
     if (st != RL_OK) return st;
   }
-  if (gspo && go && c.R > 0) return launch_bwd(c, *go, ws, s);
+  if (gspo && go && (phase & RL_PHASE_ROWS) && call.R > 0) return launch_bwd(call, *go, ws_all, s);
   return RL_OK;
 }
 
@@ -558,6 +607,42 @@ rl_status rl_loss_fwd_bwd(const void* logits, rl_dtype logits_dtype, int64_t n_r
   st = check_grad(f.c, go);
   if (st != RL_OK) return st;
   return run_fwd(f, &go, reinterpret_cast<cudaStream_t>(stream));
+}
+
+rl_status rl_loss_fwd_bwd_rows(int32_t phase, int64_t row_begin, int64_t row_end,
+                               const void* logits, rl_dtype logits_dtype, int64_t n_rows,
+                               int64_t vocab, int64_t ld, const int32_t* targets,
+                               const float* rollout_logprobs, const float* ref_logprobs,
+                               const float* old_logprobs, const float* teacher_logprobs,
+                               const float* rewards, const int32_t* group_id,
+                               const int32_t* cu_seqlens, int32_t n_traj, int32_t n_groups,
+                               const uint8_t* loss_mask, const rl_loss_params* params,
+                               float* token_logprobs, float* entropy, float* advantages,
+                               int32_t* group_sizes, rl_loss_stats* stats, float grad_loss,
+                               const float* grad_loss_device, void* dlogits,
+                               rl_dtype dlogits_dtype, int64_t ld_out, void* workspace,
+                               size_t workspace_bytes, rl_stream stream) {
+  if (phase < 1 || phase > RL_PHASE_ALL) return RL_ERR_INVALID_ARG;
+  if (row_begin < 0 || row_end < row_begin || row_end > n_rows) return RL_ERR_INVALID_ARG;
+  const bool sweep = (phase & RL_PHASE_ROWS) && row_end > row_begin;
+  FwdIn f{{logits, logits_dtype, n_rows, vocab, ld, targets, loss_mask, params},
+          rollout_logprobs, ref_logprobs, old_logprobs, teacher_logprobs, rewards,
+          group_id, cu_seqlens, n_traj, n_groups, token_logprobs, entropy, advantages,
+          group_sizes, stats, workspace, workspace_bytes};
+  rl_status st = check_fwd(f, sweep);
+  if (st != RL_OK) return st;
+  GradOut go{grad_loss, grad_loss_device, dlogits, dlogits_dtype, ld_out};
+  const bool grad = dlogits != nullptr;  // NULL: the chunk runs forward-only
+  if (grad) {
+    st = check_grad(f.c, go, sweep);
+    if (st != RL_OK) return st;
+  }
+  // GSPO needs every row's log-prob before any gradient: whole calls only
+  if (params->estimator == RL_EST_GSPO && (phase != RL_PHASE_ALL || row_begin != 0 ||
+                                           row_end != n_rows))
+    return RL_ERR_UNSUPPORTED;
+  return run_fwd(f, grad ? &go : nullptr, reinterpret_cast<cudaStream_t>(stream), phase,
+                 row_begin, row_end);
 }
 
 rl_status rl_loss_bwd(const void* logits, rl_dtype logits_dtype, int64_t n_rows, int64_t vocab,

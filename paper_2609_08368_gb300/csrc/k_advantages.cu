@@ -160,12 +160,20 @@ __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) 
     return (w - ws.g_mu[g]) / ws.g_den[g];
   };
 
-  // ---- per-row pass 1: N and the training tokens of each trajectory
+  // ---- per-row pass 1: N, and (for the estimators that use them) the
+  // training tokens of each trajectory. Consecutive rows mostly share a
+  // trajectory, so the lanes of a warp that do add once per trajectory.
+  const bool need_counts = rpp || a.estimator == RL_EST_GSPO;
   unsigned long long n_tok = 0;
-  for (long long t = tid; t < a.R; t += kAdvThreads) {
-    if (a.mask[t] == 0) continue;
-    ++n_tok;
-    if (cu_ok && a.n_traj > 0) atomicAdd(&cnt_i[traj_of(cu, a.n_traj, t)], 1);
+  for (long long t0 = 0; t0 < a.R; t0 += kAdvThreads) {
+    const long long t = t0 + tid;
+    const bool trains = t < a.R && a.mask[t] != 0;
+    n_tok += trains;
+    if (need_counts && cu_ok && a.n_traj > 0) {
+      const int i = trains ? traj_of(cu, a.n_traj, t) : -1;
+      const unsigned grp = __match_any_sync(0xffffffffu, i);
+      if (trains && (__ffs(grp) - 1) == lane) atomicAdd(&cnt_i[i], __popc(grp));
+    }
   }
   const double N = block_sum(static_cast<double>(n_tok), s_red);  // exact below 2^53
 

@@ -16,6 +16,7 @@ from . import build as _build
 
 RL_OK = 0
 RL_BF16, RL_F32 = 0, 1
+RL_PHASE_BEGIN, RL_PHASE_ROWS, RL_PHASE_END, RL_PHASE_ALL = 1, 2, 4, 7
 CORRECTIONS = {"none": 0, "tis": 1, "clip_or_pop": 2}
 ESTIMATORS = {"grpo": 0, "reinforcepp": 1, "reinforcepp_baseline": 2, "gspo": 3}
 STATS_BYTES = 128
@@ -90,12 +91,15 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
     fwd_common = [P, I32, I64, I64, I64, P, P, P, P, P, P, P, P, I32, I32, P, PP, P, P, P, P, P]
     lib.rl_loss_fwd.argtypes = fwd_common + [P, SZ, P]
     lib.rl_loss_fwd_bwd.argtypes = fwd_common + [F32, P, P, I32, I64, P, SZ, P]
+    lib.rl_loss_fwd_bwd_rows.argtypes = [I32, I64, I64] + fwd_common + [F32, P, P, I32, I64, P,
+                                                                        SZ, P]
     lib.rl_loss_bwd.argtypes = [P, I32, I64, I64, I64, P, P, PP, F32, P, P, SZ, P, I32, I64, P]
     lib.rl_loss_check_device_error.argtypes = [P]
     lib.rl_status_string.argtypes = [I32]
     lib.rl_status_string.restype = ctypes.c_char_p
     lib.rl_set_sweep_events.argtypes = [P, P]
-    for name in ("rl_loss_workspace_size", "rl_loss_fwd", "rl_loss_fwd_bwd", "rl_loss_bwd",
+    for name in ("rl_loss_workspace_size", "rl_loss_fwd", "rl_loss_fwd_bwd", "rl_loss_fwd_bwd_rows",
+                 "rl_loss_bwd",
                  "rl_loss_check_device_error", "rl_set_sweep_events", "rl_loss_abi_version"):
         getattr(lib, name).restype = ctypes.c_int32
     _lib = lib
@@ -177,6 +181,36 @@ def rl_loss_fwd_bwd(logits, targets, rollout_logprobs, ref_logprobs, old_logprob
                                   _dtype_code(dlogits), int(dlogits.stride(0)), _ptr(workspace),
                                   workspace.numel() * workspace.element_size(), _stream(stream)),
            "rl_loss_fwd_bwd")
+
+
+def rl_loss_fwd_bwd_rows(phase, row_begin, row_end, n_rows, logits, targets, rollout_logprobs,
+                         ref_logprobs, old_logprobs, teacher_logprobs, rewards, group_id,
+                         cu_seqlens, n_groups, loss_mask, params, token_logprobs, entropy,
+                         advantages, group_sizes, stats, dlogits, workspace, vocab,
+                         logits_dtype=None, grad_loss=1.0, grad_loss_device=None, stream=None):
+    """One phase (or several) of the chunked call. ``logits`` / ``dlogits``
+    hold rows [row_begin, row_end) (their row 0 is row row_begin) or are None
+    outside the ROWS phase (``dlogits`` None: forward only); every other
+    per-row tensor covers all n_rows."""
+    import torch
+    n_traj = int(rewards.shape[0]) if rewards is not None else 0
+    if logits is not None:
+        ldt, ld = _dtype_code(logits), int(logits.stride(0))
+    else:
+        ldt = _dtype_code(torch.empty(0, dtype=logits_dtype or torch.bfloat16))
+        ld = int(vocab)
+    if dlogits is not None:
+        ddt, ld_out = _dtype_code(dlogits), int(dlogits.stride(0))
+    else:
+        ddt, ld_out = ldt, int(vocab)
+    _check(load().rl_loss_fwd_bwd_rows(
+        int(phase), int(row_begin), int(row_end), _ptr(logits), ldt, int(n_rows), int(vocab), ld,
+        _ptr(targets), _ptr(rollout_logprobs), _ptr(ref_logprobs), _ptr(old_logprobs),
+        _ptr(teacher_logprobs), _ptr(rewards), _ptr(group_id), _ptr(cu_seqlens), n_traj,
+        int(n_groups), _ptr(loss_mask), ctypes.byref(_params(params)), _ptr(token_logprobs),
+        _ptr(entropy), _ptr(advantages), _ptr(group_sizes), _ptr(stats), float(grad_loss),
+        _ptr(grad_loss_device), _ptr(dlogits), ddt, ld_out, _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)), "rl_loss_fwd_bwd_rows")
 
 
 def rl_loss_bwd(logits, targets, loss_mask, params, workspace, dlogits, grad_loss=1.0,

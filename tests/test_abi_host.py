@@ -169,3 +169,23 @@ def test_params_struct_layout_matches_header():
                         r"([a-z_0-9]+(?:\s*,\s*[a-z_0-9]+)*)\s*;", body)
     names = [n.strip() for group in fields for n in group.split(",")]
     assert names == [f[0] for f in ml.RlLossParams._fields_]
+
+
+def test_chunked_entry_validates(lib):
+    v = ctypes.c_void_p
+    p = ml.make_params()
+    gspo = ml.make_params(estimator="gspo")
+
+    def call(phase, r0, r1, params=p, logits=FAKE, dl=FAKE):
+        return lib.rl_loss_fwd_bwd_rows(
+            phase, r0, r1, v(logits), 0, 16, 64, 64, v(FAKE), v(FAKE), None, None, None,
+            v(FAKE), v(FAKE), v(FAKE), 2, 1, v(FAKE), ctypes.byref(params), v(FAKE), v(FAKE),
+            v(FAKE), v(FAKE), v(FAKE), 1.0, None, v(dl), 0, 64, v(FAKE * 2), 1 << 30, None)
+    assert call(0, 0, 16) == RL_ERR_INVALID_ARG            # no phase
+    assert call(8, 0, 16) == RL_ERR_INVALID_ARG            # unknown phase bit
+    assert call(ml.RL_PHASE_ROWS, 4, 2) == RL_ERR_INVALID_ARG
+    assert call(ml.RL_PHASE_ROWS, 0, 17) == RL_ERR_INVALID_ARG
+    assert call(ml.RL_PHASE_ROWS, -1, 3) == RL_ERR_INVALID_ARG
+    assert call(ml.RL_PHASE_ROWS, 0, 8, logits=None) == RL_ERR_INVALID_ARG
+    assert call(ml.RL_PHASE_ALL, 0, 8, params=gspo) == 2     # GSPO: whole calls only
+    assert call(ml.RL_PHASE_ROWS, 0, 16, params=gspo) == 2

@@ -356,3 +356,50 @@ def test_full_size_sampled_rows(name):
         assert abs(g["stats"][k] - v) <= band, (k, g["stats"][k], v, band)
     del g, w
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("kind", ["cluster", "stream"])
+def test_chunked_call_equals_whole_call(monkeypatch, kind):
+    """BEGIN, ROWS over blocks of rows (ragged last block), END give the same
+    bits as one rl_loss_fwd_bwd; a forward-only chunk leaves dLogits alone."""
+    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=2, group_size=4, traj_len=40, vocab=20480,
+                    rho_noise=0.3, ref_noise=0.2, topk=4)
+    w = wl.make(rec, DEV)
+    params = P.gpu_params(w, dict(w.params, opd_coef=0.3, opd_topk=4))
+    whole = P.run_gpu(w, params=params)
+    for chunk in (7, 100, w.n_rows):
+        buf = api.alloc(w.n_rows, int(w.rewards.shape[0]), w.n_groups, DEV, vocab=w.vocab,
+                        dlogits_dtype=w.logits.dtype, fill_nan=True)
+        api.fwd_bwd_chunked(w, buf, chunk, params=params)
+        torch.cuda.synchronize()
+        assert ml.rl_loss_check_device_error(buf.workspace) == 0
+        assert torch.equal(buf.dlogits, whole["dlogits_t"])
+        np.testing.assert_array_equal(buf.token_logprobs.cpu().numpy(), whole["logp"])
+        np.testing.assert_array_equal(buf.entropy.cpu().numpy(), whole["H"])
+        assert buf.read_stats() == whole["stats"]
+    buf = api.alloc(w.n_rows, int(w.rewards.shape[0]), w.n_groups, DEV, vocab=w.vocab,
+                    dlogits_dtype=w.logits.dtype, fill_nan=True)
+    api.fwd_bwd_chunked(w, buf, 64, params=params, forward_only=True)
+    torch.cuda.synchronize()
+    assert torch.isnan(buf.dlogits.float()).all()
+    np.testing.assert_array_equal(buf.token_logprobs.cpu().numpy(), whole["logp"])
+    assert buf.read_stats() == whole["stats"]
+
+
+def test_pipelined_host_call_matches_device_call():
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=2, group_size=4, traj_len=64, vocab=40000,
+                    rho_noise=0.2, ref_noise=0.1)
+    w = wl.make(rec, DEV)
+    whole = P.run_gpu(w)
+    host = w.to("cpu")
+    for k in ("logits", "targets", "rollout_logprobs", "ref_logprobs", "rewards", "group_id",
+              "cu_seqlens", "loss_mask"):
+        setattr(host, k, getattr(host, k).pin_memory())
+    call = api.PipelinedHostCall(host, DEV, chunk_rows=100)
+    for _ in range(2):
+        out = call()
+        torch.cuda.synchronize()
+        assert torch.equal(out["dlogits"], whole["dlogits_t"].cpu())
+        np.testing.assert_array_equal(out["token_logprobs"].numpy(), whole["logp"])
+        assert ml.parse_stats(out["stats"].numpy().tobytes()) == whole["stats"]
