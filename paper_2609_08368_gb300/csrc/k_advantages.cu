@@ -18,6 +18,7 @@ namespace milesloss {
 namespace {
 
 constexpr int kWarps = kAdvThreads / 32;
+constexpr int kRowBlock = 16;  // consecutive rows per thread in the row passes
 
 __device__ __forceinline__ double warp_sum(double v) {
 #pragma unroll
@@ -163,17 +164,39 @@ __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) 
   // ---- per-row pass 1: N, and (for the estimators that use them) the
   // training tokens of each trajectory. Consecutive rows mostly share a
   // trajectory, so the lanes of a warp that do add once per trajectory.
+  // Each thread takes blocks of kRowBlock consecutive rows (one 16-byte load
+  // of the mask when the block is whole and aligned), so that the loads of a
+  // pass are few and independent.
   const bool need_counts = rpp || a.estimator == RL_EST_GSPO;
+  const bool lookup = cu_ok && a.n_traj > 0;
+  const bool mask_vec = (reinterpret_cast<uintptr_t>(a.mask) & 15u) == 0;
   unsigned long long n_tok = 0;
-  for (long long t0 = 0; t0 < a.R; t0 += kAdvThreads) {
-    const long long t = t0 + tid;
-    const bool trains = t < a.R && a.mask[t] != 0;
-    n_tok += trains;
-    if (need_counts && cu_ok && a.n_traj > 0) {
-      const int i = trains ? traj_of(cu, a.n_traj, t) : -1;
-      const unsigned grp = __match_any_sync(0xffffffffu, i);
-      if (trains && (__ffs(grp) - 1) == lane) atomicAdd(&cnt_i[i], __popc(grp));
+  for (long long b0 = static_cast<long long>(tid) * kRowBlock; b0 < a.R;
+       b0 += static_cast<long long>(kAdvThreads) * kRowBlock) {
+    const int nb = static_cast<int>(min(static_cast<long long>(kRowBlock), a.R - b0));
+    uint8_t m[kRowBlock];
+    if (nb == kRowBlock && mask_vec) {
+      *reinterpret_cast<uint4*>(m) = *reinterpret_cast<const uint4*>(a.mask + b0);
+    } else {
+      for (int j = 0; j < nb; ++j) m[j] = a.mask[b0 + j];
     }
+    int i = (need_counts && lookup) ? traj_of(cu, a.n_traj, b0) : 0;
+    int run = 0;
+#pragma unroll
+    for (int j = 0; j < kRowBlock; ++j) {
+      if (j >= nb) break;
+      const bool tr = m[j] != 0;
+      n_tok += tr;
+      if (need_counts && lookup) {
+        while (i + 1 < a.n_traj && cu[i + 1] <= b0 + j) {  // next trajectory
+          if (run) atomicAdd(&cnt_i[i], run);
+          run = 0;
+          ++i;
+        }
+        run += tr;
+      }
+    }
+    if (need_counts && lookup && run) atomicAdd(&cnt_i[i], run);
   }
   const double N = block_sum(static_cast<double>(n_tok), s_red);  // exact below 2^53
 
@@ -224,11 +247,22 @@ __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) 
   const double n_seq_all = block_sum(static_cast<double>(n_seq), s_red);
 
   // ---- per-row pass 2: the row's advantage, with the one-sample OPD shaping
-  for (long long t = tid; t < a.R; t += kAdvThreads) {
-    float A = 0.0f;
-    if (cu_ok && a.n_traj > 0) A = ws.a_traj[traj_of(cu, a.n_traj, t)];
-    if (a.teacher) A -= a.opd_coef * (a.rho[t] - a.teacher[t]);
-    ws.a_row[t] = A;
+  for (long long b0 = static_cast<long long>(tid) * kRowBlock; b0 < a.R;
+       b0 += static_cast<long long>(kAdvThreads) * kRowBlock) {
+    const int nb = static_cast<int>(min(static_cast<long long>(kRowBlock), a.R - b0));
+    int i = lookup ? traj_of(cu, a.n_traj, b0) : 0;
+#pragma unroll
+    for (int j = 0; j < kRowBlock; ++j) {
+      if (j >= nb) break;
+      const long long t = b0 + j;
+      float A = 0.0f;
+      if (lookup) {
+        while (i + 1 < a.n_traj && cu[i + 1] <= t) ++i;
+        A = ws.a_traj[i];
+      }
+      if (a.teacher) A -= a.opd_coef * (a.rho[t] - a.teacher[t]);
+      ws.a_row[t] = A;
+    }
   }
   if (tid == 0) {
     ws.hdr->n_tokens = static_cast<long long>(N);
