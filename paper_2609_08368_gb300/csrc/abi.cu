@@ -547,7 +547,7 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     ta.rho = f.rho;
     ta.out = f.stats;
     ta.ws = ws_all;
-    long long blocks = (call.R + kStatThreads * 4 - 1) / (kStatThreads * 4);
+    long long blocks = (call.R + kStatThreads - 1) / kStatThreads;  // one row per thread
     blocks = std::max<long long>(1, std::min<long long>(blocks, kMaxStatBlocks));
     st = launch(stats_kernel(), dim3(static_cast<unsigned>(blocks)), dim3(kStatThreads), 0, 1, s,
                 &ta);

@@ -52,6 +52,18 @@ __device__ double block_sum(double v, double* sh) {
   for (int w = 0; w < kWarps; ++w) t += sh[w];
   return t;
 }
+// Exact integer block sum (valid in every thread).
+__device__ unsigned long long block_sum_u(unsigned long long v, unsigned long long* sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  __syncthreads();
+  if (lane == 0) sh[warp] = v;
+  __syncthreads();
+  unsigned long long t = 0;
+  for (int w = 0; w < kWarps; ++w) t += sh[w];
+  return t;
+}
 __device__ double block_max(double v, double* sh) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   v = warp_max(v);
@@ -78,6 +90,7 @@ __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   __shared__ unsigned int s_err;
   __shared__ double s_red[kWarps];
+  __shared__ unsigned long long s_cnt[kWarps];
   WsPtrs ws = a.ws;
   // shared copies of cu (n_traj + 1) and the per-trajectory token counts
   const bool on_chip = a.smem_traj;
@@ -174,18 +187,23 @@ __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) 
   for (long long b0 = static_cast<long long>(tid) * kRowBlock; b0 < a.R;
        b0 += static_cast<long long>(kAdvThreads) * kRowBlock) {
     const int nb = static_cast<int>(min(static_cast<long long>(kRowBlock), a.R - b0));
-    uint8_t m[kRowBlock];
+    // the block's mask bytes, packed four to a register (byte j in word j / 4)
+    uint32_t m[kRowBlock / 4];
     if (nb == kRowBlock && mask_vec) {
-      *reinterpret_cast<uint4*>(m) = *reinterpret_cast<const uint4*>(a.mask + b0);
+      const uint4 v = *reinterpret_cast<const uint4*>(a.mask + b0);
+      m[0] = v.x; m[1] = v.y; m[2] = v.z; m[3] = v.w;
     } else {
-      for (int j = 0; j < nb; ++j) m[j] = a.mask[b0 + j];
+#pragma unroll
+      for (int q = 0; q < kRowBlock / 4; ++q) m[q] = 0u;
+      for (int j = 0; j < nb; ++j)
+        m[j >> 2] |= (a.mask[b0 + j] != 0 ? 1u : 0u) << (8 * (j & 3));
     }
     int i = (need_counts && lookup) ? traj_of(cu, a.n_traj, b0) : 0;
     int run = 0;
 #pragma unroll
     for (int j = 0; j < kRowBlock; ++j) {
       if (j >= nb) break;
-      const bool tr = m[j] != 0;
+      const bool tr = ((m[j >> 2] >> (8 * (j & 3))) & 0xffu) != 0;
       n_tok += tr;
       if (need_counts && lookup) {
         while (i + 1 < a.n_traj && cu[i + 1] <= b0 + j) {  // next trajectory
@@ -198,7 +216,7 @@ __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) 
     }
     if (need_counts && lookup && run) atomicAdd(&cnt_i[i], run);
   }
-  const double N = block_sum(static_cast<double>(n_tok), s_red);  // exact below 2^53
+  const double N = static_cast<double>(block_sum_u(n_tok, s_cnt));
 
   // ---- REINFORCE++: normalise the returns over the training tokens
   double mu = 0.0, den = 1.0;
@@ -244,29 +262,45 @@ __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) 
     if (on_chip) ws.traj_n[i] = n_i;
     n_seq += (n_i > 0);
   }
-  const double n_seq_all = block_sum(static_cast<double>(n_seq), s_red);
+  const unsigned long long n_seq_all = block_sum_u(static_cast<unsigned long long>(n_seq), s_cnt);
 
-  // ---- per-row pass 2: the row's advantage, with the one-sample OPD shaping
+  // ---- per-row pass 2: the row's advantage, with the one-sample OPD shaping.
+  // The trajectory's advantage is reloaded only when a block crosses into the
+  // next trajectory, and a whole aligned block leaves in four 16-byte stores.
+  const bool row_vec = (reinterpret_cast<uintptr_t>(ws.a_row) & 15u) == 0;
   for (long long b0 = static_cast<long long>(tid) * kRowBlock; b0 < a.R;
        b0 += static_cast<long long>(kAdvThreads) * kRowBlock) {
     const int nb = static_cast<int>(min(static_cast<long long>(kRowBlock), a.R - b0));
     int i = lookup ? traj_of(cu, a.n_traj, b0) : 0;
+    float A_i = lookup ? ws.a_traj[i] : 0.0f;
+    float out[kRowBlock];
 #pragma unroll
     for (int j = 0; j < kRowBlock; ++j) {
-      if (j >= nb) break;
-      const long long t = b0 + j;
-      float A = 0.0f;
-      if (lookup) {
-        while (i + 1 < a.n_traj && cu[i + 1] <= t) ++i;
-        A = ws.a_traj[i];
+      if (lookup && j < nb && i + 1 < a.n_traj && cu[i + 1] <= b0 + j) {
+        do { ++i; } while (i + 1 < a.n_traj && cu[i + 1] <= b0 + j);  // next trajectory
+        A_i = ws.a_traj[i];
       }
-      if (a.teacher) A -= a.opd_coef * (a.rho[t] - a.teacher[t]);
-      ws.a_row[t] = A;
+      out[j] = A_i;
+    }
+    if (a.teacher) {
+#pragma unroll
+      for (int j = 0; j < kRowBlock; ++j)
+        if (j < nb) out[j] -= a.opd_coef * (a.rho[b0 + j] - a.teacher[b0 + j]);
+    }
+    if (nb == kRowBlock && row_vec) {
+      float4* dst = reinterpret_cast<float4*>(ws.a_row + b0);
+#pragma unroll
+      for (int q = 0; q < kRowBlock / 4; ++q)
+        dst[q] = make_float4(out[4 * q], out[4 * q + 1], out[4 * q + 2], out[4 * q + 3]);
+    } else {
+#pragma unroll
+      for (int j = 0; j < kRowBlock; ++j)
+        if (j < nb) ws.a_row[b0 + j] = out[j];
     }
   }
   if (tid == 0) {
     ws.hdr->n_tokens = static_cast<long long>(N);
-    ws.hdr->n_seq = static_cast<long long>(n_seq_all);
+    ws.hdr->n_seq = static_cast<long long>(n_seq_all);  // exact integer counts
     if (s_err) atomicOr(&ws.hdr->err_bits, s_err);
   }
 }

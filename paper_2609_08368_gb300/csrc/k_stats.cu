@@ -3,10 +3,10 @@
 // rollout logp| (the train/rollout divergence of Sec. 9.2) and the
 // correction ratio (Sec. 3.4), min / max ratio, and exact clip counts.
 //
-// Each block reduces a fixed strided set of rows into double-precision
-// partial sums (butterfly merges in a fixed order), stores them in the
-// workspace, and the last block to finish (an atomic ticket, no waiting)
-// merges the partials in block order. The grid size depends only on the row
+// Each block reduces a fixed strided set of rows into partial sums
+// (butterfly merges in a fixed order), stores them in the workspace, and the
+// last block to finish (an atomic ticket, no waiting) merges the partials in
+// double precision in block order. The grid size depends only on the row
 // count, so the scalar loss is bit-for-bit reproducible.
 #include "common.cuh"
 #include "kernels.h"
@@ -15,19 +15,23 @@ namespace milesloss {
 
 namespace {
 
+// Per-block partial sums: fp32 within a block (a fixed-order tree over at
+// most kStatThreads rows; its rounding is far below the statistics'
+// tolerance), exact integer counts; the last block merges the partials in
+// double precision.
 struct Part {
-  double v[9];  // ell, pg, k3, H, r, |r-1|, |logp-rho|, rc, |rc-1|
+  float v[9];  // ell, pg, k3, H, r, |r-1|, |logp-rho|, rc, |rc-1|
   float rmin, rmax;
-  unsigned long long c[5];  // n, clip_hi, clip_lo, dual, corr_clip
+  unsigned int c[5];  // n, clip_hi, clip_lo, dual, corr_clip
 };
 
 __device__ __forceinline__ void part_zero(Part& p) {
 #pragma unroll
-  for (int i = 0; i < 9; ++i) p.v[i] = 0.0;
+  for (int i = 0; i < 9; ++i) p.v[i] = 0.0f;
   p.rmin = INFINITY;
   p.rmax = -INFINITY;
 #pragma unroll
-  for (int i = 0; i < 5; ++i) p.c[i] = 0ull;
+  for (int i = 0; i < 5; ++i) p.c[i] = 0u;
 }
 
 __device__ __forceinline__ void part_merge_shfl(Part& p, int o) {
@@ -43,13 +47,13 @@ __device__ __forceinline__ void part_merge_shfl(Part& p, int o) {
 __device__ void block_reduce(Part& p, Part* sh) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   constexpr int kWarps = kStatThreads / 32;
-#pragma unroll 1
+#pragma unroll
   for (int o = 16; o > 0; o >>= 1) part_merge_shfl(p, o);
   if (lane == 0) sh[warp] = p;
   __syncthreads();
   if (warp == 0) {
     if (lane < kWarps) p = sh[lane]; else part_zero(p);
-#pragma unroll 1
+#pragma unroll
     for (int o = 16; o > 0; o >>= 1) part_merge_shfl(p, o);
   }
 }
@@ -61,19 +65,46 @@ __device__ __forceinline__ void to_stat(const Part& p, StatPart& s) {
   s.n = p.c[0]; s.n_hi = p.c[1]; s.n_lo = p.c[2]; s.n_dual = p.c[3]; s.n_corr = p.c[4];
 }
 
-__device__ __forceinline__ void from_stat(const StatPart* sp, Part& p) {
+// The final merge, in double precision: one partial per thread, then a
+// fixed-order tree.
+struct Final {
+  double v[9];
+  float rmin, rmax;
+  unsigned long long c[5];
+};
+
+__device__ __forceinline__ void final_load(const StatPart* sp, Final& f) {
   const double* d = reinterpret_cast<const double*>(sp);
 #pragma unroll
-  for (int i = 0; i < 9; ++i) p.v[i] = __ldcg(d + i);
-  p.rmin = __ldcg(&sp->rmin);
-  p.rmax = __ldcg(&sp->rmax);
+  for (int i = 0; i < 9; ++i) f.v[i] = __ldcg(d + i);
+  f.rmin = __ldcg(&sp->rmin);
+  f.rmax = __ldcg(&sp->rmax);
   const unsigned long long* c = &sp->n;
 #pragma unroll
-  for (int i = 0; i < 5; ++i) p.c[i] = __ldcg(c + i);
+  for (int i = 0; i < 5; ++i) f.c[i] = __ldcg(c + i);
+}
+
+__device__ __forceinline__ void final_zero(Final& f) {
+#pragma unroll
+  for (int i = 0; i < 9; ++i) f.v[i] = 0.0;
+  f.rmin = INFINITY;
+  f.rmax = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < 5; ++i) f.c[i] = 0ull;
+}
+
+__device__ __forceinline__ void final_merge_shfl(Final& f, int o) {
+#pragma unroll
+  for (int i = 0; i < 9; ++i) f.v[i] += __shfl_xor_sync(0xffffffffu, f.v[i], o);
+  f.rmin = fminf(f.rmin, __shfl_xor_sync(0xffffffffu, f.rmin, o));
+  f.rmax = fmaxf(f.rmax, __shfl_xor_sync(0xffffffffu, f.rmax, o));
+#pragma unroll
+  for (int i = 0; i < 5; ++i) f.c[i] += __shfl_xor_sync(0xffffffffu, f.c[i], o);
 }
 
 __global__ void __launch_bounds__(kStatThreads) k_stats(const StatArgs a) {
   __shared__ Part sh[kStatThreads / 32];
+  __shared__ Final shf[kStatThreads / 32];
   __shared__ int s_last;
   WsPtrs ws = a.ws;
   Part p;
@@ -89,10 +120,10 @@ __global__ void __launch_bounds__(kStatThreads) k_stats(const StatArgs a) {
     p.v[2] += ws.k3[t];
     p.v[3] += ws.H[t];
     p.v[4] += r;
-    p.v[5] += fabs(static_cast<double>(r) - 1.0);
-    p.v[6] += fabs(static_cast<double>(ws.logp[t]) - static_cast<double>(a.rho[t]));
+    p.v[5] += fabsf(r - 1.0f);
+    p.v[6] += fabsf(ws.logp[t] - a.rho[t]);
     p.v[7] += rc;
-    p.v[8] += fabs(static_cast<double>(rc) - 1.0);
+    p.v[8] += fabsf(rc - 1.0f);
     p.rmin = fminf(p.rmin, r);
     p.rmax = fmaxf(p.rmax, r);
     p.c[0] += 1;
@@ -112,30 +143,40 @@ __global__ void __launch_bounds__(kStatThreads) k_stats(const StatArgs a) {
   if (!s_last) return;
   __threadfence();
 
-  // Last block: merge the partials in block order.
-  if (static_cast<int>(threadIdx.x) < static_cast<int>(gridDim.x)) from_stat(&ws.parts[threadIdx.x], p);
-  else part_zero(p);
-  block_reduce(p, sh);
+  // Last block: merge the partials in block order (one per thread, then a tree).
+  Final fin;
+  if (static_cast<int>(threadIdx.x) < static_cast<int>(gridDim.x)) final_load(&ws.parts[threadIdx.x], fin);
+  else final_zero(fin);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) final_merge_shfl(fin, o);
+  if (lane == 0) shf[warp] = fin;
+  __syncthreads();
+  if (warp == 0) {
+    if (lane < kStatThreads / 32) fin = shf[lane]; else final_zero(fin);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) final_merge_shfl(fin, o);
+  }
   if (threadIdx.x == 0) {
     rl_loss_stats o;
-    const unsigned long long n = p.c[0];
+    const unsigned long long n = fin.c[0];
     const double inv = n ? 1.0 / static_cast<double>(n) : 0.0;
-    o.loss = p.v[0] * inv;
-    o.pg_loss_mean = p.v[1] * inv;
-    o.kl_mean = p.v[2] * inv;
-    o.entropy_mean = p.v[3] * inv;
-    o.ratio_mean = p.v[4] * inv;
-    o.ratio_absdev_mean = p.v[5] * inv;
-    o.logprob_absdiff_mean = p.v[6] * inv;
-    o.corr_ratio_mean = p.v[7] * inv;
-    o.corr_absdev_mean = p.v[8] * inv;
-    o.ratio_min = n ? p.rmin : 0.0f;
-    o.ratio_max = n ? p.rmax : 0.0f;
+    o.loss = fin.v[0] * inv;
+    o.pg_loss_mean = fin.v[1] * inv;
+    o.kl_mean = fin.v[2] * inv;
+    o.entropy_mean = fin.v[3] * inv;
+    o.ratio_mean = fin.v[4] * inv;
+    o.ratio_absdev_mean = fin.v[5] * inv;
+    o.logprob_absdiff_mean = fin.v[6] * inv;
+    o.corr_ratio_mean = fin.v[7] * inv;
+    o.corr_absdev_mean = fin.v[8] * inv;
+    o.ratio_min = n ? fin.rmin : 0.0f;
+    o.ratio_max = n ? fin.rmax : 0.0f;
     o.n_tokens = static_cast<int64_t>(n);
-    o.n_clip_hi = static_cast<int64_t>(p.c[1]);
-    o.n_clip_lo = static_cast<int64_t>(p.c[2]);
-    o.n_dual_clip = static_cast<int64_t>(p.c[3]);
-    o.n_corr_clip = static_cast<int64_t>(p.c[4]);
+    o.n_clip_hi = static_cast<int64_t>(fin.c[1]);
+    o.n_clip_lo = static_cast<int64_t>(fin.c[2]);
+    o.n_dual_clip = static_cast<int64_t>(fin.c[3]);
+    o.n_corr_clip = static_cast<int64_t>(fin.c[4]);
     *a.out = o;
     ws.hdr->ticket = 0;
   }
