@@ -109,8 +109,16 @@ def row_log_softmax(z: np.ndarray, y: np.ndarray, temperature: float):
     p = np.exp(logp_all)
     rows = np.arange(s.shape[0])
     logp = logp_all[rows, np.asarray(y, dtype=np.int64)]
-    H = -(p * logp_all).sum(axis=1)
+    H = -_p_log_p(p, logp_all).sum(axis=1)
     return logp, H, lse
+
+
+def _p_log_p(p, logp_all):
+    """p log p with the limit 0 log 0 = 0 for a category of probability zero
+    (a logit of -inf): such a category contributes nothing, as if it were
+    absent from the vocabulary."""
+    zero = np.isneginf(logp_all)
+    return np.where(zero, 0.0, p * np.where(zero, 0.0, logp_all))
 
 
 # --------------------------------------------------------------------------
@@ -470,7 +478,9 @@ def dlogits_rows(z, y, temperature, lse, H, G, mask, N, grad_loss, entropy_coef)
     scale = (grad_loss * m / N / float(temperature)) if N > 0 else np.zeros_like(m)
     Gc = np.asarray(G, np.float64)[:, None]
     Hc = np.asarray(H, np.float64)[:, None]
-    return scale[:, None] * (Gc * (onehot - pj) + entropy_coef * pj * (logp_all + Hc))
+    # the entropy term p_j (log p_j + H) vanishes with p_j (a logit of -inf)
+    ent = np.where(np.isneginf(logp_all), 0.0, pj * (np.where(np.isneginf(logp_all), 0.0, logp_all) + Hc))
+    return scale[:, None] * (Gc * (onehot - pj) + entropy_coef * ent)
 
 
 # --------------------------------------------------------------------------

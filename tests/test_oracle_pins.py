@@ -80,6 +80,41 @@ def test_entropy_extremes():
     assert H[0] < 1e-80 and abs(logp[0]) < 1e-80
 
 
+def test_minus_inf_logits_are_absent_categories():
+    """A logit of -inf is a category of probability zero: the log-prob,
+    entropy and lse equal those of the row with that category removed, its
+    own dLogit is 0 (the limit 0 log 0 = 0), and the other dLogits equal the
+    reduced row's. A row with one live category has H = 0 and log p = 0."""
+    rng = np.random.default_rng(11)
+    V = 37
+    z = rng.normal(0.0, 2.0, size=(3, V))
+    dead = np.zeros((3, V), dtype=bool)
+    dead[0, [1, 5, 30]] = True
+    dead[1, 10:36] = True
+    dead[2, 0] = True
+    y = np.array([0, 3, 7])
+    zi = np.where(dead, -np.inf, z)
+    G = rng.normal(size=3)
+    mask = np.ones(3, dtype=np.uint8)
+    for T, gamma in ((1.0, 0.0), (0.7, 0.05)):
+        lp, H, lse = oracle.row_log_softmax(zi, y, T)
+        d = oracle.dlogits_rows(zi, y, T, lse, H, G, mask, 3, 1.0, gamma)
+        assert np.all(np.isfinite(d)) and np.all(d[dead] == 0.0)
+        for r in range(3):
+            keep = ~dead[r]
+            yr = np.array([int(keep[:y[r]].sum())])
+            lp_r, H_r, lse_r = oracle.row_log_softmax(z[r:r + 1, keep], yr, T)
+            assert abs(lp[r] - lp_r[0]) < 1e-13 and abs(H[r] - H_r[0]) < 1e-13
+            assert abs(lse[r] - lse_r[0]) < 1e-13
+            d_r = oracle.dlogits_rows(z[r:r + 1, keep], yr, T, lse_r, H_r, G[r:r + 1],
+                                      mask[r:r + 1], 3, 1.0, gamma)
+            assert np.allclose(d[r, keep], d_r[0], rtol=1e-13, atol=1e-16)
+    one = np.full((1, 9), -np.inf)
+    one[0, 4] = 1.5
+    lp, H, _ = oracle.row_log_softmax(one, np.array([4]), 1.0)
+    assert lp[0] == 0.0 and H[0] == 0.0
+
+
 def test_log_softmax_mpmath_brute_force():
     mpmath = pytest.importorskip("mpmath")
     mpmath.mp.dps = 50
