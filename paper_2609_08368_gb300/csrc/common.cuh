@@ -280,6 +280,18 @@ __device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
 }
 __device__ __forceinline__ float2 ex2x2(float2 t) { return make_float2(ex2(t.x), ex2(t.y)); }
 
+// The entropy term's factor (ca + cb z) of a logit z. A logit of -inf has
+// probability zero and its p (ca + cb z) must be 0, not 0 * inf: the factor
+// takes z no lower than kZFloor, far below any logit whose probability is
+// not zero, where the vanishing p makes the product 0 whatever the floor.
+constexpr float kZFloor = -1.0e20f;
+__device__ __forceinline__ float ent_factor(float z, float ca, float cb) {
+  return fmaf(cb, fmaxf(z, kZFloor), ca);
+}
+__device__ __forceinline__ float2 ent_factor2(float2 z, float2 ca2, float2 cb2) {
+  return ffma2(cb2, make_float2(fmaxf(z.x, kZFloor), fmaxf(z.y, kZFloor)), ca2);
+}
+
 // Streaming 16-byte global load that does not allocate in L1.
 __device__ __forceinline__ uint4 ld_stream_u4(const void* p) {
   uint4 v;

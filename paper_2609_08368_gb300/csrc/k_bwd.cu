@@ -41,7 +41,7 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
     const float dzy = cc * (G * -expm1f(logp) + a.gamma * expf(logp) * (logp + H));
     auto value = [&](float z, int j) {
       if (j == y) return dzy;
-      return (cc == 0.0f) ? 0.0f : ex2(fmaf(z, a.k, -L2)) * fmaf(cb, z, ca);
+      return (cc == 0.0f) ? 0.0f : ex2(fmaf(z, a.k, -L2)) * ent_factor(z, ca, cb);
     };
     if (a.in_vec && a.out_vec) {
       // j0 is a multiple of V8 (kBwdTile is), so every vector is aligned.
@@ -55,7 +55,7 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
           for (int e = 0; e < V8; ++e) f[e] = 0.0f;
         } else {
 #pragma unroll
-          for (int e = 0; e < V8; ++e) f[e] = ex2(fmaf(f[e], a.k, -L2)) * fmaf(cb, f[e], ca);
+          for (int e = 0; e < V8; ++e) f[e] = ex2(fmaf(f[e], a.k, -L2)) * ent_factor(f[e], ca, cb);
           if (static_cast<unsigned>(y - jb) < static_cast<unsigned>(V8)) {
 #pragma unroll
             for (int e = 0; e < V8; ++e)

@@ -121,7 +121,7 @@ __device__ __forceinline__ void pass_b_chunk(const uint4* sv, int nv, char* dchu
 #pragma unroll
     for (int e = 0; e < P; ++e) {
       if (kMode == 2) {
-        f[e] = fmul2(ex2x2(ffma2(f[e], k2, off2)), ffma2(cb2, f[e], ca2));
+        f[e] = fmul2(ex2x2(ffma2(f[e], k2, off2)), ent_factor2(f[e], ca2, cb2));
       } else {
         f[e] = ex2x2(ffma2(f[e], k2, off2));
         if (kMode == 1) f[e] = make_float2(-f[e].x, -f[e].y);
@@ -261,47 +261,44 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
     const int yv = yok ? y / V8 : -1;  // thread 0 only
 
     // ---------------- pass A
+    // One sweep of each chunk in shared memory: the exponentials take as
+    // reference the thread's running maximum from before the chunk (for the
+    // first chunk, the maximum of the thread's first vector), while the
+    // chunk's maximum is tracked on the side and raises the reference after
+    // the chunk. Sums taken against a reference below the maximum are the
+    // same sums scaled by a power of two; they stay finite unless a logit
+    // exceeds the reference by more than 127 / k, and that case (an
+    // overflow, detected as inf) or a -inf logit (NaN) redoes the chunk
+    // against its own maximum, skipping -inf logits exactly.
     Run run;
     for (int c = 0; c < n_chunks; ++c) {
       const uint4* sv = wait_slot(q0 + c);
       const int nv = min(CV, row_vec - c * CV);
-      uint4 w[2];
-      int nw = 0;
-      typename In::MaxAcc macc = In::kMaxInit;
-#pragma unroll
-      for (int r = 0; r < 2; ++r) {
-        const int v = tid + r * kCons;
-        if (v < nv) {
-          w[r] = sv[v];
-          macc = In::max_acc(macc, w[r]);
-          nw = r + 1;
-        }
-      }
-      for (int v = tid + 2 * kCons; v < nv; v += kCons) macc = In::max_acc(macc, sv[v]);
       if (tid == 0 && yv >= c * CV && yv < c * CV + nv) zy = In::load1(sv, y - c * CV * V8);
-      run.raise(In::max_val(macc), k);
-      if (run.m != -INFINITY) {
-        const Run keep = run;
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-          if (r < nw) {
-            float2 f[P];
-            In::unpack2(w[r], f);
-#pragma unroll
-            for (int e = 0; e < P; ++e) run.add_pair<false>(f[e], k2, (e & 1) ? run.s1 : run.s0,
-                                                            (e & 1) ? run.u1 : run.u0);
-          }
-        }
-        for (int v = tid + 2 * kCons; v < nv; v += kCons) {
+      if (run.m == -INFINITY && tid < nv) run.raise(In::vmax(sv[tid]), k);
+      typename In::MaxAcc macc = In::kMaxInit;
+      const Run keep = run;
+      bool redo = run.m == -INFINITY;  // no finite reference yet: two sweeps
+      if (!redo) {
+#pragma unroll 2
+        for (int v = tid; v < nv; v += kCons) {
+          const uint4 w = sv[v];
+          macc = In::max_acc(macc, w);
           float2 f[P];
-          In::unpack2(sv[v], f);
+          In::unpack2(w, f);
 #pragma unroll
-          for (int e = 0; e < P; ++e) run.add_pair<false>(f[e], k2, run.s0, run.u0);
+          for (int e = 0; e < P; ++e) run.add_pair<false>(f[e], k2, (e & 1) ? run.s1 : run.s0,
+                                                          (e & 1) ? run.u1 : run.u0);
         }
         const Tri cur = run.tri();
-        if (__isnanf(cur.u) || __isnanf(cur.s)) {
-          // -inf logits in this chunk: redo it, skipping them exactly
-          run = keep;
+        redo = !(fabsf(cur.s) < INFINITY) || !(fabsf(cur.u) < INFINITY);  // inf or NaN
+      } else {
+        for (int v = tid; v < nv; v += kCons) macc = In::max_acc(macc, sv[v]);
+      }
+      if (redo) {
+        run = keep;
+        run.raise(In::max_val(macc), k);
+        if (run.m != -INFINITY) {
           for (int v = tid; v < nv; v += kCons) {
             float2 f[P];
             In::unpack2(sv[v], f);
@@ -309,6 +306,8 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
             for (int e = 0; e < P; ++e) run.add_pair<true>(f[e], k2, run.s0, run.u0);
           }
         }
+      } else {
+        run.raise(In::max_val(macc), k);
       }
       release_slot(q0 + c);
     }
@@ -433,7 +432,7 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
 #pragma unroll
             for (int e = 0; e < P; ++e) {
               f[e] = ci.y ? ex2x2(ffma2(f[e], k2, off2))
-                          : fmul2(ex2x2(ffma2(f[e], k2, off2)), ffma2(cb2, f[e], ca2));
+                          : fmul2(ex2x2(ffma2(f[e], k2, off2)), ent_factor2(f[e], ca2, cb2));
               if (ci.y && ci.z) f[e] = make_float2(-f[e].x, -f[e].y);
             }
             const float* fv = reinterpret_cast<const float*>(f);
@@ -446,7 +445,7 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
         const float z = In::load1(grow, j);
         float x = 0.0f;
         if (!ci.x) {
-          x = ci.y ? ex2(fmaf(z, k, cf.x)) : ex2(fmaf(z, k, cf.x)) * fmaf(cf.z, z, cf.y);
+          x = ci.y ? ex2(fmaf(z, k, cf.x)) : ex2(fmaf(z, k, cf.x)) * ent_factor(z, cf.y, cf.z);
           if (ci.y && ci.z) x = -x;
         }
         Out::store1(drow, j, x);

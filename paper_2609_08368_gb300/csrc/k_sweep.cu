@@ -392,13 +392,13 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
           In::unpack2(sv[v], f);
 #pragma unroll
           for (int e = 0; e < P; ++e)
-            f[e] = fmul2(ex2x2(ffma2(f[e], k2, off2)), ffma2(cb2, f[e], ca2));
+            f[e] = fmul2(ex2x2(ffma2(f[e], k2, off2)), ent_factor2(f[e], ca2, cb2));
           Out::template storev<V8>(drow + static_cast<size_t>(v) * V8 * Out::kSize,
                                    reinterpret_cast<const float*>(f), 0u);
         }
         for (int j = vo_elems + tid; j < cnt; j += kThreads) {
           const float z = (j < vec_elems) ? In::load1(sb, j) : In::load1(grow, j);
-          Out::store1(drow, j, ex2(fmaf(z, k, c.x)) * fmaf(c.z, z, c.y));
+          Out::store1(drow, j, ex2(fmaf(z, k, c.x)) * ent_factor(z, c.y, c.z));
         }
       }
       __syncthreads();

@@ -10,6 +10,7 @@ import pytest
 import torch
 
 import _parity as P
+import oracle
 from paper_2609_08368_gb300 import api, workloads as wl
 from paper_2609_08368_gb300 import milesloss as ml
 
@@ -152,6 +153,64 @@ def test_padded_and_misaligned_rows():
     assert torch.isnan(g["dlogits_t"][:, 1000:]).all()
     o = P.run_oracle(w)
     P.assert_dlogits_close(g["dlogits_t"][:, :1000].float().cpu().numpy(), o["dlogits"])
+
+
+def _extreme_rows(w):
+    """Rows that stress the running-maximum and -inf handling of the sweeps:
+    -inf logits (scattered, nearly all, a whole leading block, all but the
+    target), a spike far above the rest (at the row's end, in its first
+    chunk, on the target), a constant row, a ramp whose maximum is last,
+    and a row shifted to -1000."""
+    V = w.vocab
+    z = w.logits[:, :V]
+    y = w.targets.long()
+    g = torch.Generator(device="cpu").manual_seed(5)
+    ninf = float("-inf")
+    keep_y = lambda r, row: row.index_fill_(0, y[r:r + 1], float(z[r, y[r]]))  # noqa: E731
+    sc = torch.rand(V, generator=g) < 0.1
+    row = z[0].clone(); row[sc.to(z.device)] = ninf; z[0] = keep_y(0, row)
+    row = torch.full((V,), ninf, dtype=z.dtype, device=z.device)
+    live = torch.randperm(V, generator=g)[:100].to(z.device)
+    row[live] = z[1, live]; z[1] = keep_y(1, row)
+    z[2, V - 1] = 150.0
+    if int(y[2]) == V - 1:
+        w.targets[2] = 0
+    z[3, V - 1] = 150.0
+    w.targets[3] = V - 1
+    z[4] = 5.0
+    z[5] = torch.linspace(-60.0, 60.0, V, device=z.device).to(z.dtype)
+    z[6] = (z[6].float() - 1000.0).to(z.dtype)
+    row = z[7].clone(); row[:min(V, 8192)] = ninf; z[7] = keep_y(7, row)
+    z[8, V // 4] = 100.0
+    row = torch.full((V,), ninf, dtype=z.dtype, device=z.device); z[9] = keep_y(9, row)
+
+
+@pytest.mark.parametrize("kind", ["cluster", "stream"])
+@pytest.mark.parametrize("extra", [dict(), dict(entropy_coef=0.01, temperature=0.7)])
+def test_extreme_logits(monkeypatch, kind, extra):
+    """Extreme rows (see _extreme_rows) on both sweep kernels, fused and
+    split, with and without the entropy term and temperature; a row of 200 KB
+    runs in the streaming kernel in two ring chunks."""
+    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=4, vocab=100000)
+    w = wl.make(rec, DEV)
+    _extreme_rows(w)
+    params = dict(w.params, **extra)
+    # rollout and reference log-probs near the new rows' own (a log-ratio
+    # past ~88 would overflow the fp32 exponentials of the ratio and of k3)
+    lp, _, _ = oracle.row_log_softmax(P.host_logits(w), P.np_(w.targets),
+                                      params.get("temperature", 1.0))
+    lp = torch.from_numpy(lp).float().to(DEV)
+    w.rollout_logprobs.copy_(lp + 0.05 * torch.sin(torch.arange(w.n_rows, device=DEV)))
+    if w.ref_logprobs is not None:
+        w.ref_logprobs.copy_(lp - 0.03)
+    if w.old_logprobs is not None:
+        w.old_logprobs.copy_(lp + 0.01)
+    g, o = _full_check(w, params=params)
+    for k in ("logp", "H"):
+        assert np.all(np.isfinite(g[k])), k
+    assert abs(float(g["H"][9])) < 1e-6 and abs(float(g["logp"][9])) < 1e-6
+    _full_check(w, mode="split", params=params)
 
 
 @pytest.mark.parametrize("logit_dtype,dl_dtype", [("bf16", torch.float32), ("f32", torch.bfloat16)])
