@@ -50,17 +50,22 @@ __device__ __forceinline__ uint64_t l2_policy_evict_last() {
   return p;
 }
 
+// A thread's (or a group's) partial sums over a row, against a reference r
+// in log2 units (a multiple of k = log2(e) / T of a logit):
+//   s = sum_j 2^(z_j k - r),  u = sum_j 2^(z_j k - r) (z_j k - r).
+// Any finite r gives the same row statistics: lse = r ln 2 + ln s and
+// H = ln s - u ln 2 / s.
 struct Tri {
-  float m, s, u;
+  float m, s, u;  // m = r
 };
 
-__device__ __forceinline__ Tri warp_merge(Tri t, float k) {
+__device__ __forceinline__ Tri warp_merge(Tri t) {
   float M = t.m;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
   float s = 0.0f, u = 0.0f;
   if (t.s > 0.0f) {
-    const float d = (t.m - M) * k, f = ex2(d);
+    const float d = t.m - M, f = ex2(d);
     s = f * t.s;
     u = f * fmaf(d, t.s, t.u);
   }
@@ -72,27 +77,44 @@ __device__ __forceinline__ Tri warp_merge(Tri t, float k) {
   return Tri{M, s, u};
 }
 
-// Running (max, sums) of one thread over the chunks of a row.
+// Running sums of one thread over the chunks of a row. The reference starts
+// at the maximum of the thread's first vector and is moved only by whole
+// powers of two of the sums (rebase), so no per-element maximum is needed.
 struct Run {
-  float m = -INFINITY, mt = -INFINITY;
+  float r = -INFINITY;
   float2 s0 = {0.0f, 0.0f}, s1 = {0.0f, 0.0f}, u0 = {0.0f, 0.0f}, u1 = {0.0f, 0.0f};
 
-  __device__ __forceinline__ void raise(float cm, float k) {
-    if (!(cm > m)) return;
-    if (m != -INFINITY) {
-      const float d = (m - cm) * k, f = ex2(d);
+  // move the reference up to nr (sums rescaled by 2^(r - nr))
+  __device__ __forceinline__ void raise(float nr) {
+    if (!(nr > r)) return;
+    if (r != -INFINITY) {
+      const float d = r - nr, f = ex2(d);
       const float2 f2 = make_float2(f, f), d2 = make_float2(d, d);
       u0 = fmul2(f2, ffma2(d2, s0, u0));
       u1 = fmul2(f2, ffma2(d2, s1, u1));
       s0 = fmul2(f2, s0);
       s1 = fmul2(f2, s1);
     }
-    m = cm;
-    mt = cm * k;
+    r = nr;
+  }
+  // After a chunk whose sums are finite: when they exceed 2^16, move the
+  // reference up by their binary exponent e (s scales by 2^-e exactly).
+  __device__ __forceinline__ void rebase() {
+    const float2 s = fadd2(s0, s1);
+    const int e = ((__float_as_int(s.x + s.y) >> 23) & 0xff) - 127;
+    if (e > 16) {
+      const float f = __int_as_float((127 - e) << 23), d = -static_cast<float>(e);
+      const float2 f2 = make_float2(f, f), d2 = make_float2(d, d);
+      u0 = fmul2(f2, ffma2(d2, s0, u0));
+      u1 = fmul2(f2, ffma2(d2, s1, u1));
+      s0 = fmul2(f2, s0);
+      s1 = fmul2(f2, s1);
+      r -= d;
+    }
   }
   template <bool kSafe>
   __device__ __forceinline__ void add_pair(float2 z, float2 k2, float2& s, float2& u) {
-    float2 t = ffma2(z, k2, make_float2(-mt, -mt));
+    float2 t = ffma2(z, k2, make_float2(-r, -r));
     if (kSafe) {
       if (z.x == -INFINITY) t.x = -127.0f;
       if (z.y == -INFINITY) t.y = -127.0f;
@@ -103,7 +125,7 @@ struct Run {
   }
   __device__ __forceinline__ Tri tri() const {
     const float2 s = fadd2(s0, s1), u = fadd2(u0, u1);
-    return Tri{m, s.x + s.y, u.x + u.y};
+    return Tri{r, s.x + s.y, u.x + u.y};
   }
 };
 
@@ -261,44 +283,39 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
     const int yv = yok ? y / V8 : -1;  // thread 0 only
 
     // ---------------- pass A
-    // One sweep of each chunk in shared memory: the exponentials take as
-    // reference the thread's running maximum from before the chunk (for the
-    // first chunk, the maximum of the thread's first vector), while the
-    // chunk's maximum is tracked on the side and raises the reference after
-    // the chunk. Sums taken against a reference below the maximum are the
-    // same sums scaled by a power of two; they stay finite unless a logit
-    // exceeds the reference by more than 127 / k, and that case (an
-    // overflow, detected as inf) or a -inf logit (NaN) redoes the chunk
-    // against its own maximum, skipping -inf logits exactly.
+    // One sweep of each chunk in shared memory against the thread's running
+    // reference (for the first chunk, the maximum of the thread's first
+    // vector): the sums are finite unless a logit lies more than 127 / k
+    // above the reference, and that case (an overflow, seen as inf) or a
+    // -inf logit (NaN) redoes the chunk against the chunk's own maximum,
+    // skipping -inf logits exactly.
     Run run;
     for (int c = 0; c < n_chunks; ++c) {
       const uint4* sv = wait_slot(q0 + c);
       const int nv = min(CV, row_vec - c * CV);
       if (tid == 0 && yv >= c * CV && yv < c * CV + nv) zy = In::load1(sv, y - c * CV * V8);
-      if (run.m == -INFINITY && tid < nv) run.raise(In::vmax(sv[tid]), k);
-      typename In::MaxAcc macc = In::kMaxInit;
+      if (run.r == -INFINITY && tid < nv) run.raise(In::vmax(sv[tid]) * k);
       const Run keep = run;
-      bool redo = run.m == -INFINITY;  // no finite reference yet: two sweeps
+      bool redo = run.r == -INFINITY;  // no finite reference yet
       if (!redo) {
-#pragma unroll 2
+#pragma unroll 4
         for (int v = tid; v < nv; v += kCons) {
-          const uint4 w = sv[v];
-          macc = In::max_acc(macc, w);
           float2 f[P];
-          In::unpack2(w, f);
+          In::unpack2(sv[v], f);
 #pragma unroll
           for (int e = 0; e < P; ++e) run.add_pair<false>(f[e], k2, (e & 1) ? run.s1 : run.s0,
                                                           (e & 1) ? run.u1 : run.u0);
         }
         const Tri cur = run.tri();
         redo = !(fabsf(cur.s) < INFINITY) || !(fabsf(cur.u) < INFINITY);  // inf or NaN
-      } else {
-        for (int v = tid; v < nv; v += kCons) macc = In::max_acc(macc, sv[v]);
+        if (!redo) run.rebase();
       }
       if (redo) {
+        typename In::MaxAcc macc = In::kMaxInit;
+        for (int v = tid; v < nv; v += kCons) macc = In::max_acc(macc, sv[v]);
         run = keep;
-        run.raise(In::max_val(macc), k);
-        if (run.m != -INFINITY) {
+        run.raise(In::max_val(macc) * k);
+        if (run.r != -INFINITY) {
           for (int v = tid; v < nv; v += kCons) {
             float2 f[P];
             In::unpack2(sv[v], f);
@@ -306,8 +323,6 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
             for (int e = 0; e < P; ++e) run.add_pair<true>(f[e], k2, run.s0, run.u0);
           }
         }
-      } else {
-        run.raise(In::max_val(macc), k);
       }
       release_slot(q0 + c);
     }
@@ -315,21 +330,22 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
     for (int j = tail0 + tid; j < a.V; j += kCons) {
       const float z = In::load1(grow, j);
       if (z == -INFINITY) continue;
-      if (z > t.m) {
+      const float zk = z * k;
+      if (zk > t.m) {
         if (t.s > 0.0f) {
-          const float d = (t.m - z) * k, f = ex2(d);
+          const float d = t.m - zk, f = ex2(d);
           t.u = f * fmaf(d, t.s, t.u);
           t.s *= f;
         }
-        t.m = z;
+        t.m = zk;
       }
-      const float tt = fmaf(z, k, -t.m * k), x = ex2(tt);
+      const float tt = fmaf(z, k, -t.m), x = ex2(tt);
       t.s += x;
       t.u = fmaf(x, tt, t.u);
     }
 
     // ---------------- merge
-    t = warp_merge(t, k);
+    t = warp_merge(t);
     if (lane == 0) red[warp] = make_float4(t.m, t.s, t.u, 0.0f);
     cons_sync();
     if (tid == 0 && fix_ptr) Out::store1(fix_ptr, 0, fix_val);  // previous row's y entry
@@ -340,7 +356,7 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
         const float4 v = red[lane];
         x = Tri{v.x, v.y, v.z};
       }
-      t = warp_merge(x, k);
+      t = warp_merge(x);
     }
 
     // ---------------- epilogue (thread 0)
@@ -351,7 +367,7 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
       const bool bad = !yok;
       if (bad) atomicOr(&ws.hdr->err_bits, kErrTarget);
       const float lnS = logf(t.s);
-      const float lse = t.m * a.s.invT + lnS;
+      const float lse = fmaf(t.m, kLn2f, lnS);  // the reference is in log2 units
       float H = lnS - t.u * kLn2f / t.s;
       float logp = zy * a.s.invT - lse;
       if (bad) { logp = 0.0f; H = 0.0f; }
@@ -379,7 +395,7 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
         const float cc = (msk && !bad) ? cscale : 0.0f;
         const float ca = cc * (-tt.G + a.s.gamma * (H - lse));
         const float cb = cc * a.s.gamma * a.s.invT;
-        const float L2 = t.m * k + __log2f(t.s);
+        const float L2 = t.m + __log2f(t.s);
         const bool zero = (cc == 0.0f) || (ca == 0.0f && cb == 0.0f);
         const bool fold = !zero && (cb == 0.0f);
         const float off = fold ? (__log2f(fabsf(ca)) - L2) : -L2;
