@@ -344,6 +344,30 @@ def run_ours(args, rank, world, local):
     rows_all = sum_over_ranks(float(R), world)
     value = rows_all * K / (ms_total / 1e3)
 
+    # the other two ways to call the loss, timed beside the fused call (median
+    # of 20 after 3 warm-ups, whole call, CUDA events): the forward alone
+    # (reads the logits once) and the split pair rl_loss_fwd + rl_loss_bwd
+    # (reads them twice)
+    also = {}
+    for name, fn in (("fwd_only", lambda: api.fwd(w, buf)),
+                     ("split_fwd_bwd", lambda: (api.fwd(w, buf), api.bwd(w, buf)))):
+        for _ in range(3):
+            fn()
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(20)]
+        for b, e in evs:
+            b.record(stream)
+            fn()
+            e.record(stream)
+        torch.cuda.synchronize()
+        also[name + "_ms"] = statistics.median(b.elapsed_time(e) for b, e in evs)
+    err = ml.rl_loss_check_device_error(buf.workspace)
+    if err:
+        raise RuntimeError(f"device error: {ml.status_string(err)}")
+    logit_bytes = R * V * w.logits.element_size()
+    also["fwd_only_read_gbs"] = logit_bytes / (also["fwd_only_ms"] / 1e3) / 1e9
+    also["split_fwd_bwd_tokens_per_s"] = R / (also["split_fwd_bwd_ms"] / 1e3)
+
     bpr = algorithmic_bytes_per_row(w, dl_dtype)  # before w is released for the e2e leg
     launch_bytes = bpr * R
     sweep_avg = statistics.fmean(sweep_ms)
@@ -389,7 +413,7 @@ def run_ours(args, rank, world, local):
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "scaling": "weak", "vs_baseline": None, "dtype": dt_name, "data": "synthetic",
         "config": {"workload": f"{args.workload}: {R} rows ({rec.n_traj} traj x {rec.traj_len} "
                                f"tokens, groups of {rec.group_size}) x vocab {V}, "
                                f"{dt_name} logits "
@@ -402,8 +426,10 @@ def run_ours(args, rank, world, local):
                      "bytes_per_launch": launch_bytes, "sweep_ms": sweep_avg,
                      "peak_kind": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"
                      if peak_kind == "measured" else "fallback 6.8 TB/s",
-                     "frac_of_8tbs": achieved / NOMINAL_HBM_GBS},
+                     "frac_of_8tbs": achieved / NOMINAL_HBM_GBS,
+                     "traffic_gbs": None if traffic is None else traffic / (sweep_avg / 1e3) / 1e9},
         "step_hbm_gbs": step_gbs,
+        "also": also,
         "cpu_baseline": cpu,
         "e2e": e2e,
         "gpu_launches": 3 * K,

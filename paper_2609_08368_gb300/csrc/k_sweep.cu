@@ -9,11 +9,11 @@
 // bulk async copies (cp.async.bulk, completion counted on an mbarrier per
 // stage). Several CTAs share an SM, so one CTA's per-row synchronisation
 // overlaps the others' arithmetic. Per row:
-//   pass M  every thread takes the maximum m of its own elements;
-//   pass A  it sums S = sum 2^(t - m k) and U = sum 2^(t - m k) (t - m k),
-//           t = z log2(e)/T, two lanes per instruction (f32x2);
-//           warp shuffles, then one warp, merge the threads' (m, S, U) in a
-//           fixed order;
+//   pass A  every thread sums S = sum 2^(t - r) and U = sum 2^(t - r) (t - r),
+//           t = z log2(e)/T, two lanes per instruction (f32x2), against a
+//           reference r taken from its first vector (a second sweep for the
+//           maximum runs only on overflow or -inf logits); warp shuffles,
+//           then one warp, merge the threads' (r, S, U) in a fixed order;
 //   exchange thread 0 pushes the CTA's (m, S, U, z_y) into every peer's
 //           shared memory with st.async, counted on the peer's mbarrier,
 //           and merges the C triples in rank order once they have all
@@ -37,20 +37,23 @@ namespace {
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s per bounded wait
 constexpr float kLn2 = 0.69314718055994531f;
 
+// Partial sums against a reference r in log2 units (t = z k, k = log2(e)/T):
+// s = sum 2^(t - r), u = sum 2^(t - r) (t - r). Any finite r gives the same
+// row statistics: lse = r ln 2 + ln s, H = ln s - u ln 2 / s.
 struct Tri {
-  float m, s, u;  // max of z; sum of 2^(t - m k); sum of 2^(t - m k) (t - m k)
+  float m, s, u;  // m = r
 };
 
-// Warp-wide merge in a fixed order: the maximum first, then every lane
-// rescales its sums once to that maximum, then plain butterfly sums.
-// Every lane ends with the same triple.
-__device__ __forceinline__ Tri warp_merge(Tri t, float k) {
+// Warp-wide merge in a fixed order: the largest reference first, then every
+// lane rescales its sums once to it, then plain butterfly sums. Every lane
+// ends with the same triple.
+__device__ __forceinline__ Tri warp_merge(Tri t) {
   float M = t.m;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
   float s = 0.0f, u = 0.0f;
   if (t.s > 0.0f) {
-    const float d = (t.m - M) * k, f = ex2(d);
+    const float d = t.m - M, f = ex2(d);
     s = f * t.s;
     u = f * fmaf(d, t.s, t.u);
   }
@@ -64,9 +67,9 @@ __device__ __forceinline__ Tri warp_merge(Tri t, float k) {
 
 // Block-wide merge; the result is valid in warp 0. Contains a __syncthreads.
 template <int kWarps>
-__device__ __forceinline__ Tri block_merge(Tri t, float k, float4* red) {
+__device__ __forceinline__ Tri block_merge(Tri t, float4* red) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  t = warp_merge(t, k);
+  t = warp_merge(t);
   if (lane == 0) red[warp] = make_float4(t.m, t.s, t.u, 0.0f);
   __syncthreads();
   if (warp == 0) {
@@ -75,13 +78,13 @@ __device__ __forceinline__ Tri block_merge(Tri t, float k, float4* red) {
       const float4 v = red[lane];
       x = Tri{v.x, v.y, v.z};
     }
-    t = warp_merge(x, k);
+    t = warp_merge(x);
   }
   return t;
 }
 
 // Sum of 2^(t - mt) and of 2^(t - mt) (t - mt) over the thread's vectors,
-// t = z k, for a fixed mt (the thread's own maximum times k). kSafe skips
+// t = z k, for a fixed reference mt in log2 units. kSafe skips
 // -inf logits exactly (0 * -inf would otherwise give NaN); it runs only
 // when the fast pass produced a NaN.
 template <class In, int kThreads, bool kSafe>
@@ -130,6 +133,23 @@ __device__ __forceinline__ void sum_pass(const uint4* sv, int n_vec, float k, fl
   const float2 s = fadd2(s0, s1), u = fadd2(u0, u1);
   s_out = s.x + s.y;
   u_out = u.x + u.y;
+}
+
+// The thread's sums against its own maximum over the slice, skipping -inf
+// logits exactly: the rare path (no finite first vector, an overflow, or a
+// -inf logit), kept out of line so that it costs the fast path no registers.
+template <class In, int kThreads>
+__device__ __noinline__ Tri slow_sums(const uint4* sv, int n_vec, float k) {
+  typename In::MaxAcc macc = In::kMaxInit;
+  for (int v = threadIdx.x; v < n_vec; v += kThreads) macc = In::max_acc(macc, sv[v]);
+  const float r = In::max_val(macc) * k;
+  Tri t{-INFINITY, 0.0f, 0.0f};
+  if (r != -INFINITY) {
+    float su, uu;
+    sum_pass<In, kThreads, true>(sv, n_vec, k, r, su, uu);
+    t = Tri{r, su, uu};
+  }
+  return t;
 }
 
 template <class In, class Out, bool kGrad, int kThreads, int kMinBlocks>
@@ -233,30 +253,46 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
       }
     }
 
-    // ---------------- pass M: the thread's own maximum
-    typename In::MaxAcc macc = In::kMaxInit;
-    for (int v = tid; v < n_vec; v += kThreads) macc = In::max_acc(macc, sv[v]);
-    float mz = In::max_val(macc);
-    for (int j = vec_elems + tid; j < cnt; j += kThreads) mz = fmaxf(mz, In::load1(grow, j));
-
-    // ---------------- pass A: sums at the fixed maximum
-    Tri t{mz, 0.0f, 0.0f};
-    if (mz != -INFINITY) {
-      const float mt = mz * k;
-      float su, uu;
-      sum_pass<In, kThreads, false>(sv, n_vec, k, mt, su, uu);
-      if (__isnanf(uu) || __isnanf(su)) sum_pass<In, kThreads, true>(sv, n_vec, k, mt, su, uu);
-      for (int j = vec_elems + tid; j < cnt; j += kThreads) {
-        const float z = In::load1(grow, j);
-        if (z == -INFINITY) continue;
-        const float tt = fmaf(z, k, -mt), x = ex2(tt);
-        su += x;
-        uu = fmaf(x, tt, uu);
+    // ---------------- pass A: one sweep against the maximum of the thread's
+    // first vector. The sums stay finite unless a logit lies more than
+    // 127 / k above that reference; that case (inf) or a -inf logit (NaN)
+    // takes the thread's maximum over the slice and sums again, skipping
+    // -inf logits exactly. Sums past 2^16 move the reference up by their
+    // binary exponent (an exact rescale) before the merge.
+    Tri t{-INFINITY, 0.0f, 0.0f};
+    if (tid < n_vec) {
+      const float r = In::vmax(sv[tid]) * k;
+      if (r != -INFINITY) {
+        float su, uu;
+        sum_pass<In, kThreads, false>(sv, n_vec, k, r, su, uu);
+        if (fabsf(su) < INFINITY && fabsf(uu) < INFINITY) t = Tri{r, su, uu};
       }
-      t.s = su;
-      t.u = uu;
+      if (t.m == -INFINITY) t = slow_sums<In, kThreads>(sv, n_vec, k);
+      const int e = ((__float_as_int(t.s) >> 23) & 0xff) - 127;
+      if (e > 16) {
+        const float f = __int_as_float((127 - e) << 23), d = static_cast<float>(e);
+        t.u = f * fmaf(-d, t.s, t.u);
+        t.s *= f;
+        t.m += d;
+      }
     }
-    t = block_merge<kWarps>(t, k, red);
+    for (int j = vec_elems + tid; j < cnt; j += kThreads) {  // elements past the vectors
+      const float z = In::load1(grow, j);
+      if (z == -INFINITY) continue;
+      const float zk = z * k;
+      if (zk > t.m) {
+        if (t.s > 0.0f) {
+          const float d = t.m - zk, f = ex2(d);
+          t.u = f * fmaf(d, t.s, t.u);
+          t.s *= f;
+        }
+        t.m = zk;
+      }
+      const float tt = fmaf(z, k, -t.m), x = ex2(tt);
+      t.s += x;
+      t.u = fmaf(x, tt, t.u);
+    }
+    t = block_merge<kWarps>(t, red);
 
     // ---------------- exchange and epilogue (thread 0)
     const bool yok = (tid == 0) && (y >= 0) && (y < a.V);
@@ -289,7 +325,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
         for (int r = 0; r < C; ++r) {
           const float4 e = xs[r];
           if (e.y > 0.0f) {
-            const float d = (e.x - M) * k, f = ex2(d);
+            const float d = e.x - M, f = ex2(d);
             tot.s += f * e.y;
             tot.u += f * fmaf(d, e.y, e.z);
           }
@@ -299,7 +335,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
       const bool bad = !yok;
       if (bad) atomicOr(&ws.hdr->err_bits, kErrTarget);
       const float lnS = logf(tot.s);
-      const float lse = tot.m * a.s.invT + lnS;
+      const float lse = fmaf(tot.m, kLn2, lnS);  // the reference is in log2 units
       float H = lnS - tot.u * kLn2 / tot.s;
       float logp = zy_all * a.s.invT - lse;
       if (bad) { logp = 0.0f; H = 0.0f; }
@@ -330,7 +366,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
         const float cc = (msk && !bad) ? cscale : 0.0f;
         const float ca = cc * (-tt.G + a.s.gamma * (H - lse));
         const float cb = cc * a.s.gamma * a.s.invT;
-        const float L2 = tot.m * k + __log2f(tot.s);
+        const float L2 = tot.m + __log2f(tot.s);
         const bool zero = (cc == 0.0f) || (ca == 0.0f && cb == 0.0f);
         const bool fold = !zero && (cb == 0.0f);
         // fold: p_j ca = sign(ca) 2^(z_j k - L2 + log2|ca|)
