@@ -178,19 +178,32 @@ def sweep_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(rows_now: int):
+def profiled_traffic(rows_now: int, workload: str, vocab: int):
     """DRAM bytes of one sweep launch from the committed ncu summary, if it
-    was taken on the current kernel source; scaled by rows if captured on a
-    smaller case of the same vocabulary."""
+    was taken on the current kernel source and on this workload's recipe and
+    vocabulary; scaled by rows if captured on a smaller case."""
     if not os.path.exists(PROFILE_SUMMARY):
         return None
     text = open(PROFILE_SUMMARY).read()
     src = re.search(r"source_sha256:\s*([0-9a-f]+)", text)
     tb = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
     rows = re.search(r"rows_per_launch:\s*([0-9]+)", text)
-    if not (src and tb and rows) or src.group(1) != sweep_source_hash():
+    wk = re.search(r"workload:\s*(\S+)", text)
+    voc = re.search(r"vocab:\s*([0-9]+)", text)
+    if not (src and tb and rows and wk and voc) or src.group(1) != sweep_source_hash():
+        return None
+    if wk.group(1) != workload or int(voc.group(1)) != vocab:
         return None
     return float(tb.group(1)) * rows_now / int(rows.group(1))
+
+
+def sweep_kernel_name(vocab: int, elem_size: int) -> str:
+    """The sweep kernel the library picks for these rows (rows of 160 KB and
+    more, 16-byte aligned, stream through one CTA each; shorter rows go to the
+    cluster kernel)."""
+    if vocab * elem_size >= 160 * 1024:
+        return "k_stream (fused fwd+bwd vocabulary sweep, one CTA per row)"
+    return "k_sweep (fused fwd+bwd vocabulary sweep, clusters sharing a row)"
 
 
 def algorithmic_bytes_per_row(w, dl_dtype) -> int:
@@ -369,6 +382,7 @@ def run_ours(args, rank, world, local):
     also["split_fwd_bwd_tokens_per_s"] = R / (also["split_fwd_bwd_ms"] / 1e3)
 
     bpr = algorithmic_bytes_per_row(w, dl_dtype)  # before w is released for the e2e leg
+    kernel_name = sweep_kernel_name(V, w.logits.element_size())
     launch_bytes = bpr * R
     sweep_avg = statistics.fmean(sweep_ms)
     peaks, peak_kind = measured_peaks()
@@ -409,7 +423,7 @@ def run_ours(args, rank, world, local):
                "h2d_bytes_per_step": call.bytes_in(), "d2h_bytes_per_step": call.bytes_out()}
         del call, host_w
 
-    traffic = profiled_traffic(R)
+    traffic = profiled_traffic(R, args.workload, V)
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True,
@@ -422,7 +436,7 @@ def run_ours(args, rank, world, local):
                    "l2": "inputs larger than L2 (20+ GB per step), no flush"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
-                     "kernel": "k_stream (fused fwd+bwd vocabulary sweep, one CTA per row)",
+                     "kernel": kernel_name,
                      "bytes_per_launch": launch_bytes, "sweep_ms": sweep_avg,
                      "peak_kind": f"{peak_kind} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)"
                      if peak_kind == "measured" else "fallback 6.8 TB/s",
