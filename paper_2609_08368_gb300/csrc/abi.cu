@@ -370,9 +370,15 @@ rl_status launch_bwd(const Common& c, const GradOut& go, const WsPtrs& ws, cudaS
   b.k = 1.4426950408889634f / c.p->temperature;
   b.gamma = c.p->entropy_coef;
   b.ws = ws;
-  const long long grid = std::min<long long>(b.n_tiles, static_cast<long long>(sms) * 8);
-  return launch(bwd_kernel(c.dt, go.dt), dim3(static_cast<unsigned>(grid)), dim3(kBwdThreads), 0,
-                1, s, &b);
+  // one wave of resident blocks (grid-stride over the tiles): a second,
+  // partial wave would run with fewer loads in flight
+  const void* fn = bwd_kernel(c.dt, go.dt);
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kBwdThreads, 0) != cudaSuccess)
+    return RL_ERR_CUDA;
+  const long long grid =
+      std::min<long long>(b.n_tiles, static_cast<long long>(sms) * std::max(per_sm, 1));
+  return launch(fn, dim3(static_cast<unsigned>(grid)), dim3(kBwdThreads), 0, 1, s, &b);
 }
 
 // phase: RL_PHASE_BEGIN (advantages, N), RL_PHASE_ROWS (the sweep over rows

@@ -2,9 +2,10 @@
 // backward path): the logits are read once more, row statistics come from
 // the workspace.
 //   dZ_tj = g (m_t / N) (1/T) [G_t (1[j = y_t] - p_j) + gamma p_j (log p_j + H_t)]
-// A tile is a contiguous run of kBwdTile columns of one row; blocks stride
-// over tiles. Loads are 16-byte streaming loads that skip L1, stores are
-// 16-byte streaming stores when the rows are aligned.
+// A tile is a contiguous run of kTile columns of one row; blocks stride
+// over tiles. Each thread issues all of its 16-byte streaming loads of a tile
+// (L1 skipped) before using any, then writes 16-byte streaming stores; rows
+// that are not 16-byte aligned take the scalar path.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -22,18 +23,45 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
   if (a.grad_loss_dev) g *= *a.grad_loss_dev;
   const float cscale = (N > 0) ? g / static_cast<float>(N) * a.invT : 0.0f;
 
-  for (long long tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x) {
+  constexpr int kTile = kBwdTile;
+  constexpr int kPer = kTile / V8 / kBwdThreads;  // vectors per thread per tile
+  const bool vec = a.in_vec && a.out_vec;
+  // vectors of a tile (the last tile of a row may be partial; unaligned rows
+  // take the scalar path)
+  auto tile_nv = [&](long long tile) {
+    const int j0 = static_cast<int>(tile % a.tiles_per_row) * kTile;
+    return vec ? (min(a.V, j0 + kTile) - j0) / V8 : 0;
+  };
+  // All of a thread's 16-byte streaming loads of a tile are issued before
+  // any is used, and the next tile's loads are issued before this tile's
+  // arithmetic, so each thread keeps up to 2 kPer loads in flight.
+  auto load_tile = [&](long long tile, uint4* raw) {
     const long long row = tile / a.tiles_per_row;
-    const int j0 = static_cast<int>(tile % a.tiles_per_row) * kBwdTile;
-    const int j1 = min(a.V, j0 + kBwdTile);
+    const int j0 = static_cast<int>(tile % a.tiles_per_row) * kTile;
+    const int nv = tile_nv(tile);
+    const char* zrow = static_cast<const char*>(a.logits) + row * a.ld * static_cast<long long>(sizeof(St));
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+      const int v = threadIdx.x + i * kBwdThreads;
+      if (v < nv) raw[i] = ld_stream_u4(zrow + static_cast<size_t>(j0 + v * V8) * sizeof(St));
+    }
+  };
+  uint4 raw[kPer], nxt[kPer];
+  if (blockIdx.x < a.n_tiles) load_tile(blockIdx.x, raw);
+  for (long long tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x) {
+    if (tile + gridDim.x < a.n_tiles) load_tile(tile + gridDim.x, nxt);
+    const long long row = tile / a.tiles_per_row;
+    const int j0 = static_cast<int>(tile % a.tiles_per_row) * kTile;
+    const int j1 = min(a.V, j0 + kTile);
+    const char* zrow = static_cast<const char*>(a.logits) + row * a.ld * static_cast<long long>(sizeof(St));
+    char* drow = static_cast<char*>(a.dlogits) + row * a.ld_out * static_cast<long long>(Out::kSize);
+    const int nv = tile_nv(tile);
     const bool bad = (ws.flags[row] & kFlagBad) != 0;
     const float cc = (a.mask[row] && !bad) ? cscale : 0.0f;
     const float G = ws.G[row], H = ws.H[row], lse = ws.lse[row];
     const float ca = cc * (-G + a.gamma * (H - lse));
     const float cb = cc * a.gamma * a.invT;
     const float L2 = lse * 1.4426950408889634f;
-    const char* zrow = static_cast<const char*>(a.logits) + row * a.ld * static_cast<long long>(sizeof(St));
-    char* drow = static_cast<char*>(a.dlogits) + row * a.ld_out * static_cast<long long>(Out::kSize);
     const int y = a.targets[row];
     // The sampled token's entry: cc [G (1 - p_y) + gamma p_y (log p_y + H)]
     // with 1 - p_y = -expm1(logp), accurate when p_y is close to 1.
@@ -43,33 +71,31 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
       if (j == y) return dzy;
       return (cc == 0.0f) ? 0.0f : ex2(fmaf(z, a.k, -L2)) * ent_factor(z, ca, cb);
     };
-    if (a.in_vec && a.out_vec) {
-      // j0 is a multiple of V8 (kBwdTile is), so every vector is aligned.
-      const int nv = (j1 - j0) / V8;
-      for (int v = threadIdx.x; v < nv; v += kBwdThreads) {
-        const int jb = j0 + v * V8;
-        float f[V8];
-        In::unpack(ld_stream_u4(zrow + static_cast<size_t>(jb) * sizeof(St)), f);
-        if (cc == 0.0f) {
 #pragma unroll
-          for (int e = 0; e < V8; ++e) f[e] = 0.0f;
-        } else {
+    for (int i = 0; i < kPer; ++i) {
+      const int v = threadIdx.x + i * kBwdThreads;
+      if (v >= nv) continue;
+      const int jb = j0 + v * V8;
+      float f[V8];
+      In::unpack(raw[i], f);
+      if (cc == 0.0f) {
 #pragma unroll
-          for (int e = 0; e < V8; ++e) f[e] = ex2(fmaf(f[e], a.k, -L2)) * ent_factor(f[e], ca, cb);
-          if (static_cast<unsigned>(y - jb) < static_cast<unsigned>(V8)) {
+        for (int e = 0; e < V8; ++e) f[e] = 0.0f;
+      } else {
 #pragma unroll
-            for (int e = 0; e < V8; ++e)
-              if (jb + e == y) f[e] = dzy;
-          }
+        for (int e = 0; e < V8; ++e) f[e] = ex2(fmaf(f[e], a.k, -L2)) * ent_factor(f[e], ca, cb);
+        if (static_cast<unsigned>(y - jb) < static_cast<unsigned>(V8)) {
+#pragma unroll
+          for (int e = 0; e < V8; ++e)
+            if (jb + e == y) f[e] = dzy;
         }
-        Out::template storev<V8>(drow + static_cast<size_t>(jb) * Out::kSize, f, 0u);
       }
-      for (int j = j0 + nv * V8 + threadIdx.x; j < j1; j += kBwdThreads)
-        Out::store1(drow, j, value(In::load1(zrow, j), j));
-    } else {
-      for (int j = j0 + threadIdx.x; j < j1; j += kBwdThreads)
-        Out::store1(drow, j, value(In::load1(zrow, j), j));
+      Out::template storev<V8>(drow + static_cast<size_t>(jb) * Out::kSize, f, 0u);
     }
+    for (int j = j0 + nv * V8 + threadIdx.x; j < j1; j += kBwdThreads)
+      Out::store1(drow, j, value(In::load1(zrow, j), j));
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) raw[i] = nxt[i];
   }
 }
 

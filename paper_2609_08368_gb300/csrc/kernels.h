@@ -117,7 +117,7 @@ struct BwdArgs {
   WsPtrs ws;
 };
 
-constexpr int kBwdTile = kBwdThreads * 8 * 4;  // elements of one row per tile
+constexpr int kBwdTile = kBwdThreads * 8 * 4;  // elements of one row per backward tile
 
 // Kernel entry points (device function pointers usable with cudaLaunchKernelEx).
 const void* sweep_kernel(rl_dtype in, rl_dtype out, bool grad, int threads);
