@@ -15,6 +15,7 @@ replicas). ``--impl reference`` times the float64 CPU oracle instead.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import os
@@ -55,6 +56,10 @@ def parse_args():
                     help="fewer groups (a smaller case of the same workload, for profiling)")
     ap.add_argument("--traj-len", type=int, default=None,
                     help="shorter trajectories (a smaller case, for profiling)")
+    ap.add_argument("--estimator", default=None,
+                    choices=["grpo", "reinforcepp", "reinforcepp_baseline", "gspo"],
+                    help="another advantage estimator than the workload's (for profiling "
+                         "the kernels of that path)")
     return ap.parse_args()
 
 
@@ -312,6 +317,8 @@ def run_ours(args, rank, world, local):
     rec = wl.RECIPES[args.workload]
     rec = wl.shrink(rec, n_prompts=args.n_prompts, traj_len=args.traj_len,
                     seed=rec.seed + 1000 * rank)  # each replica has its own batch
+    if args.estimator:
+        rec = dataclasses.replace(rec, params=dict(rec.params, estimator=args.estimator))
     w = wl.make(rec, dev)
     R, V = w.n_rows, w.vocab
     dl_dtype = w.logits.dtype
@@ -391,7 +398,9 @@ def run_ours(args, rank, world, local):
     step_gbs = launch_bytes / (ms_step / 1e3) / 1e9
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    # (the sampled-row oracle timing covers the token-level estimators only)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and \
+            w.params.get("estimator", "grpo") != "gspo":
         rps, secs, n = oracle_sample(w, args.cpu_sample_rows)
         cpu = {"value": rps, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                "sample": f"{n} random rows of the {R} x {V} batch (every per-row output and "

@@ -26,36 +26,49 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
   constexpr int kTile = kBwdTile;
   constexpr int kPer = kTile / V8 / kBwdThreads;  // vectors per thread per tile
   const bool vec = a.in_vec && a.out_vec;
+  // Tile (row, t) of this block, advanced by gridDim.x tiles per step
+  // without a division in the loop.
+  const int tpr = a.tiles_per_row;
+  const long long dq = gridDim.x / tpr;
+  const int dr = static_cast<int>(gridDim.x % tpr);
+  auto advance = [&](long long& row, int& t) {
+    row += dq;
+    t += dr;
+    if (t >= tpr) { t -= tpr; ++row; }
+  };
   // vectors of a tile (the last tile of a row may be partial; unaligned rows
   // take the scalar path)
-  auto tile_nv = [&](long long tile) {
-    const int j0 = static_cast<int>(tile % a.tiles_per_row) * kTile;
+  auto tile_nv = [&](int t) {
+    const int j0 = t * kTile;
     return vec ? (min(a.V, j0 + kTile) - j0) / V8 : 0;
   };
   // All of a thread's 16-byte streaming loads of a tile are issued before
   // any is used, and the next tile's loads are issued before this tile's
   // arithmetic, so each thread keeps up to 2 kPer loads in flight.
-  auto load_tile = [&](long long tile, uint4* raw) {
-    const long long row = tile / a.tiles_per_row;
-    const int j0 = static_cast<int>(tile % a.tiles_per_row) * kTile;
-    const int nv = tile_nv(tile);
-    const char* zrow = static_cast<const char*>(a.logits) + row * a.ld * static_cast<long long>(sizeof(St));
+  auto load_tile = [&](long long row, int t, uint4* raw) {
+    const int nv = tile_nv(t);
+    const char* zrow = static_cast<const char*>(a.logits) + row * a.ld * static_cast<long long>(sizeof(St)) +
+                       static_cast<size_t>(t) * kTile * sizeof(St);
 #pragma unroll
     for (int i = 0; i < kPer; ++i) {
       const int v = threadIdx.x + i * kBwdThreads;
-      if (v < nv) raw[i] = ld_stream_u4(zrow + static_cast<size_t>(j0 + v * V8) * sizeof(St));
+      if (v < nv) raw[i] = ld_stream_u4(zrow + static_cast<size_t>(v) * 16);
     }
   };
+  long long row = blockIdx.x / tpr;
+  int t = static_cast<int>(blockIdx.x % tpr);
   uint4 raw[kPer], nxt[kPer];
-  if (blockIdx.x < a.n_tiles) load_tile(blockIdx.x, raw);
-  for (long long tile = blockIdx.x; tile < a.n_tiles; tile += gridDim.x) {
-    if (tile + gridDim.x < a.n_tiles) load_tile(tile + gridDim.x, nxt);
-    const long long row = tile / a.tiles_per_row;
-    const int j0 = static_cast<int>(tile % a.tiles_per_row) * kTile;
+  if (row < a.R) load_tile(row, t, raw);
+  while (row < a.R) {
+    long long nrow = row;
+    int nt = t;
+    advance(nrow, nt);
+    if (nrow < a.R) load_tile(nrow, nt, nxt);
+    const int j0 = t * kTile;
     const int j1 = min(a.V, j0 + kTile);
     const char* zrow = static_cast<const char*>(a.logits) + row * a.ld * static_cast<long long>(sizeof(St));
     char* drow = static_cast<char*>(a.dlogits) + row * a.ld_out * static_cast<long long>(Out::kSize);
-    const int nv = tile_nv(tile);
+    const int nv = tile_nv(t);
     const bool bad = (ws.flags[row] & kFlagBad) != 0;
     const float cc = (a.mask[row] && !bad) ? cscale : 0.0f;
     const float G = ws.G[row], H = ws.H[row], lse = ws.lse[row];
@@ -63,10 +76,15 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
     const float cb = cc * a.gamma * a.invT;
     const float L2 = lse * 1.4426950408889634f;
     const int y = a.targets[row];
-    // The sampled token's entry: cc [G (1 - p_y) + gamma p_y (log p_y + H)]
-    // with 1 - p_y = -expm1(logp), accurate when p_y is close to 1.
-    const float logp = ws.logp[row];
-    const float dzy = cc * (G * -expm1f(logp) + a.gamma * expf(logp) * (logp + H));
+    const bool has_y = y >= j0 && y < j1;
+    // The sampled token's entry (only in the tile that holds it):
+    // cc [G (1 - p_y) + gamma p_y (log p_y + H)] with 1 - p_y = -expm1(logp),
+    // accurate when p_y is close to 1.
+    float dzy = 0.0f;
+    if (has_y) {
+      const float logp = ws.logp[row];
+      dzy = cc * (G * -expm1f(logp) + a.gamma * expf(logp) * (logp + H));
+    }
     auto value = [&](float z, int j) {
       if (j == y) return dzy;
       return (cc == 0.0f) ? 0.0f : ex2(fmaf(z, a.k, -L2)) * ent_factor(z, ca, cb);
@@ -84,7 +102,7 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
       } else {
 #pragma unroll
         for (int e = 0; e < V8; ++e) f[e] = ex2(fmaf(f[e], a.k, -L2)) * ent_factor(f[e], ca, cb);
-        if (static_cast<unsigned>(y - jb) < static_cast<unsigned>(V8)) {
+        if (has_y && static_cast<unsigned>(y - jb) < static_cast<unsigned>(V8)) {
 #pragma unroll
           for (int e = 0; e < V8; ++e)
             if (jb + e == y) f[e] = dzy;
@@ -96,6 +114,8 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
       Out::store1(drow, j, value(In::load1(zrow, j), j));
 #pragma unroll
     for (int i = 0; i < kPer; ++i) raw[i] = nxt[i];
+    row = nrow;
+    t = nt;
   }
 }
 
