@@ -30,12 +30,6 @@ bool finite(float x) { return std::isfinite(x); }
 
 rl_status cuda_fail(cudaError_t e) { return e == cudaSuccess ? RL_OK : RL_ERR_CUDA; }
 
-int env_int(const char* name, int dflt) {
-  const char* v = std::getenv(name);
-  if (!v || !*v) return dflt;
-  return std::atoi(v);
-}
-
 rl_status set_smem(const void* fn, int dev, int bytes) {
   std::lock_guard<std::mutex> lk(g_mu);
   auto key = std::make_pair(dev, fn);
@@ -210,48 +204,6 @@ rl_status plan_sweep(rl_dtype dt, long long V, int dev, SweepPlan* out) {
     }
   }
   return RL_ERR_UNSUPPORTED;  // vocabulary too large for an 8-CTA cluster
-}
-
-// Rows of 160 KB and more with 16-byte aligned starts go to the streaming
-// kernel (one CTA per row, second read served by L2); shorter or unaligned
-// rows to the cluster kernel, which keeps them on chip. Measured on GB300:
-// bf16 rows of 151,936-154,880 columns run 5-8 % faster streamed, fp32 rows
-// of 32,768 columns 10 % faster in clusters. MILESLOSS_SWEEP_KIND=stream|cluster
-// overrides the choice.
-constexpr long long kStreamMinRowBytes = 160 * 1024;
-
-bool use_stream(long long row_bytes, bool in_bulk) {
-  const char* k = std::getenv("MILESLOSS_SWEEP_KIND");
-  if (k && std::string(k) == "cluster") return false;
-  if (k && std::string(k) == "stream") return in_bulk;
-  return in_bulk && row_bytes >= kStreamMinRowBytes;
-}
-
-struct StreamPlan {
-  int chunk, slots, smem;
-};
-
-// Two 112 KB slots (one CTA per SM): few, large chunks keep the per-chunk
-// handshakes rare (measured best among 16-112 KB chunks with 2-14 slots).
-// Overridable through MILESLOSS_STREAM_CHUNK / MILESLOSS_STREAM_SLOTS.
-rl_status plan_stream(int dev, StreamPlan* out) {
-  int optin = 0;
-  if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
-    return RL_ERR_CUDA;
-  const int chunk = env_int("MILESLOSS_STREAM_CHUNK", 114688);
-  if (chunk < 1024 || chunk > 131072 || chunk % 128) return RL_ERR_UNSUPPORTED;
-  int slots = (optin - kSweepSmemExtra) / chunk;
-  if (slots > kMaxSlots) slots = kMaxSlots;
-  const int forced = env_int("MILESLOSS_STREAM_SLOTS", 0);
-  if (forced) {
-    if (forced < 1 || forced > slots) return RL_ERR_UNSUPPORTED;
-    slots = forced;
-  }
-  if (slots < 1) return RL_ERR_UNSUPPORTED;
-  out->chunk = chunk;
-  out->slots = slots;
-  out->smem = slots * chunk + kSweepSmemExtra;
-  return RL_OK;
 }
 
 struct Common {

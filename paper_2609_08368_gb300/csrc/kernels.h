@@ -1,6 +1,8 @@
 // Internal interface between the C-ABI layer (abi.cu) and the kernels.
 #pragma once
 
+#include <cstdlib>
+
 #include "common.cuh"
 
 namespace milesloss {
@@ -122,6 +124,21 @@ constexpr int kBwdTile = kBwdThreads * 8 * 4;  // elements of one row per backwa
 // Kernel entry points (device function pointers usable with cudaLaunchKernelEx).
 const void* sweep_kernel(rl_dtype in, rl_dtype out, bool grad, int threads);
 const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad);
+
+// An integer from the environment (tuning overrides), or dflt.
+inline int env_int(const char* name, int dflt) {
+  const char* v = std::getenv(name);
+  if (!v || !*v) return dflt;
+  return std::atoi(v);
+}
+
+// The streaming kernel's launch plan (defined beside the kernel, k_stream.cu):
+// whether rows of row_bytes go to it, and its ring of shared-memory slots.
+struct StreamPlan {
+  int chunk, slots, smem;
+};
+bool use_stream(long long row_bytes, bool in_bulk);
+rl_status plan_stream(int dev, StreamPlan* out);
 const void* bwd_kernel(rl_dtype in, rl_dtype out);
 const void* adv_kernel();
 const void* seq_kernel();

@@ -213,6 +213,24 @@ def test_extreme_logits(monkeypatch, kind, extra):
     _full_check(w, mode="split", params=params)
 
 
+@pytest.mark.parametrize("ld,ld_out", [(100008, 100000), (100003, 100003), (100000, 100011)])
+def test_long_rows_padded_and_misaligned(ld, ld_out):
+    """Rows of 200 KB (the streaming kernel's size) with a padded row stride,
+    rows whose starts are not 16-byte aligned (the cluster kernel's element-wise
+    path takes them), and a dLogits stride that is not 16-byte aligned (scalar
+    stores); fused and split."""
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=6, vocab=100000)
+    w = wl.make(rec, DEV, ld=ld)
+    for mode in ("fused", "split"):
+        g = P.run_gpu(w, mode=mode, ld_out=ld_out)
+        assert g["err"] == 0, ml.status_string(g["err"])
+        o = P.run_oracle(w)
+        P.compare_forward(w, g, o)
+        P.assert_dlogits_close(g["dlogits_t"][:, :w.vocab].float().cpu().numpy(), o["dlogits"])
+        if ld_out > w.vocab:
+            assert torch.isnan(g["dlogits_t"][:, w.vocab:]).all()
+
+
 @pytest.mark.parametrize("logit_dtype,dl_dtype", [("bf16", torch.float32), ("f32", torch.bfloat16)])
 def test_mixed_dtypes(logit_dtype, dl_dtype):
     rec = wl.shrink(wl.RECIPES["fp32" if logit_dtype == "f32" else "tiny"], n_prompts=2,
