@@ -48,11 +48,20 @@ def alloc(n_rows: int, n_traj: int, n_groups: int, device, vocab: int | None = N
     return Buffers(f32(n_rows), f32(n_rows), f32(n_traj), gs, st, ws, dl)
 
 
+def _params(w, params):
+    """The call's parameters; with top-K OPD on, the workload's candidate ids
+    and teacher log-probs are attached unless the caller gave them."""
+    p = dict(w.params if params is None else params)
+    if p.get("opd_topk", 0) > 0 and "opd_topk_ids" not in p and w.topk_ids is not None:
+        p.update(opd_topk_ids=w.topk_ids, opd_topk_teacher=w.topk_teacher)
+    return p
+
+
 def fwd_bwd(w, buf: Buffers, params=None, grad_loss=1.0, grad_loss_device=None, stream=None):
     """One fused forward+backward call on a ``workloads.Workload``."""
     ml.rl_loss_fwd_bwd(w.logits, w.targets, w.rollout_logprobs, w.ref_logprobs, w.old_logprobs,
                        w.teacher_logprobs, w.rewards, w.group_id, w.cu_seqlens, w.n_groups,
-                       w.loss_mask, params if params is not None else w.params,
+                       w.loss_mask, _params(w, params),
                        buf.token_logprobs, buf.entropy, buf.advantages, buf.group_sizes,
                        buf.stats, buf.dlogits, buf.workspace, grad_loss=grad_loss,
                        grad_loss_device=grad_loss_device, vocab=w.vocab, stream=stream)
@@ -61,14 +70,14 @@ def fwd_bwd(w, buf: Buffers, params=None, grad_loss=1.0, grad_loss_device=None, 
 def fwd(w, buf: Buffers, params=None, stream=None):
     ml.rl_loss_fwd(w.logits, w.targets, w.rollout_logprobs, w.ref_logprobs, w.old_logprobs,
                    w.teacher_logprobs, w.rewards, w.group_id, w.cu_seqlens, w.n_groups,
-                   w.loss_mask, params if params is not None else w.params, buf.token_logprobs,
+                   w.loss_mask, _params(w, params), buf.token_logprobs,
                    buf.entropy, buf.advantages, buf.group_sizes, buf.stats, buf.workspace,
                    vocab=w.vocab, stream=stream)
 
 
 def bwd(w, buf: Buffers, params=None, grad_loss=1.0, grad_loss_device=None, stream=None):
     ml.rl_loss_bwd(w.logits, w.targets, w.loss_mask,
-                   params if params is not None else w.params, buf.workspace, buf.dlogits,
+                   _params(w, params), buf.workspace, buf.dlogits,
                    grad_loss=grad_loss, grad_loss_device=grad_loss_device, vocab=w.vocab,
                    stream=stream)
 
@@ -123,7 +132,7 @@ def _rows_call(w, buf, phase, r0, r1, logits, dlogits, params=None, grad_loss=1.
     ml.rl_loss_fwd_bwd_rows(phase, r0, r1, w.n_rows, logits, w.targets, w.rollout_logprobs,
                             w.ref_logprobs, w.old_logprobs, w.teacher_logprobs, w.rewards,
                             w.group_id, w.cu_seqlens, w.n_groups, w.loss_mask,
-                            params if params is not None else w.params, buf.token_logprobs,
+                            _params(w, params), buf.token_logprobs,
                             buf.entropy, buf.advantages, buf.group_sizes, buf.stats, dlogits,
                             buf.workspace, w.vocab,
                             logits_dtype=(w.logits.dtype if w.logits is not None

@@ -156,7 +156,7 @@ struct SweepPlan {
 // stages as still fit; if no cluster size fits, one CTA per SM.
 // Overridable for tuning through MILESLOSS_SWEEP_CLUSTER / _STAGES /
 // _THREADS / _CTAS_PER_SM.
-rl_status plan_sweep(rl_dtype dt, long long V, int dev, SweepPlan* out) {
+rl_status plan_sweep(rl_dtype dt, long long V, int dev, int extra, SweepPlan* out) {
   int optin = 0, per_sm = 0, reserved = 0;
   if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) !=
@@ -175,8 +175,9 @@ rl_status plan_sweep(rl_dtype dt, long long V, int dev, SweepPlan* out) {
   const int vec = 16 / es;
   const int forced_c = env_int("MILESLOSS_SWEEP_CLUSTER", 0);
   const int forced_s = env_int("MILESLOSS_SWEEP_STAGES", 0);
-  const int hard = optin - kSweepSmemExtra;                            // one CTA per SM
-  const int share = per_sm / target - reserved - kSweepSmemExtra;      // `target` per SM
+  const int fixed = kSweepSmemExtra + extra;                           // scratch (+ top-K)
+  const int hard = optin - fixed;                                      // one CTA per SM
+  const int share = per_sm / target - reserved - fixed;                // `target` per SM
   for (int pass = 0; pass < 2; ++pass) {
     const int budget = pass == 0 ? share : hard;
     for (int C = 1; C <= kMaxCluster; C *= 2) {
@@ -197,7 +198,7 @@ rl_status plan_sweep(rl_dtype dt, long long V, int dev, SweepPlan* out) {
       out->S = S;
       out->slice = static_cast<int>(slice);
       out->stage_bytes = static_cast<int>(stage);
-      out->smem = static_cast<int>(S * stage) + kSweepSmemExtra;
+      out->smem = static_cast<int>(S * stage) + fixed;
       out->threads = threads;
       out->variant = variant;
       return RL_OK;
@@ -247,7 +248,9 @@ rl_status check_fwd(const FwdIn& f, bool need_logits = true) {
   if (f.c.R > 0 && p->opd_coef != 0.0f && p->opd_topk == 0 && !f.teacher)
     return RL_ERR_INVALID_ARG;
   if (f.c.R > 0 && p->opd_coef != 0.0f && p->opd_topk > 0 &&
-      (!p->opd_topk_ids || !p->opd_topk_teacher))
+      (!p->opd_topk_ids || !p->opd_topk_teacher ||
+       (reinterpret_cast<uintptr_t>(p->opd_topk_ids) & 3u) ||
+       (reinterpret_cast<uintptr_t>(p->opd_topk_teacher) & 3u)))
     return RL_ERR_INVALID_ARG;
   // GSPO scores whole trajectories with one advantage: no per-token shaping
   if (p->estimator == RL_EST_GSPO && p->opd_coef != 0.0f) return RL_ERR_UNSUPPORTED;
@@ -404,12 +407,11 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
   const size_t es = elem_size(c.dt);
   const bool in_bulk = aligned16(c.logits) && ((c.ld * es) % 16 == 0);
   const bool out_vec = grad && aligned16(go->dl) && ((go->ld_out * elem_size(go->dt)) % 16 == 0);
-  (void)go_sweep;
   if (c.R > 0 && use_stream(c.V * static_cast<long long>(es), in_bulk)) {
     StreamPlan sp;
-    st = plan_stream(dev, &sp);
+    st = plan_stream(dev, sc.topk ? kTopKSmem : 0, &sp);
     if (st != RL_OK) return st;
-    const void* fn = stream_kernel(c.dt, grad ? go->dt : c.dt, grad);
+    const void* fn = stream_kernel(c.dt, grad ? go->dt : c.dt, grad, sc.topk > 0);
     st = set_smem(fn, dev, sp.smem);
     if (st != RL_OK) return st;
     int ctas = 0;
@@ -444,9 +446,9 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     if (st != RL_OK) return st;
   } else if (c.R > 0) {
     SweepPlan pl;
-    st = plan_sweep(c.dt, c.V, dev, &pl);
+    st = plan_sweep(c.dt, c.V, dev, sc.topk ? kTopKSmem : 0, &pl);
     if (st != RL_OK) return st;
-    const void* fn = sweep_kernel(c.dt, grad ? go->dt : c.dt, grad, pl.variant);
+    const void* fn = sweep_kernel(c.dt, grad ? go->dt : c.dt, grad, pl.variant, sc.topk > 0);
     st = set_smem(fn, dev, pl.smem);
     if (st != RL_OK) return st;
     int clusters = 0;

@@ -44,6 +44,7 @@ struct StatPart {
   unsigned long long n, n_hi, n_lo, n_dual, n_corr;
 };
 
+constexpr int kMaxTopK = 64;
 constexpr int kStatThreads = 256;
 constexpr int kMaxStatBlocks = 256;  // one partial per thread of the final block
 
@@ -489,27 +490,112 @@ __device__ __forceinline__ TokenTerms token_terms(float logp, float H, float rho
 // the candidate set of w_k (log p_k - teacher_k), with p_k the trainer's
 // probabilities of the candidates (from the row's logits and its lse) and
 // w_k = p_k / sum_j p_j. Candidates outside [0, V) are skipped.
+//
+// Since w_k is proportional to exp(z_k / T), the signal is
+//   sum_k w_k (z_k / T - teacher_k) / sum_k w_k  -  lse,
+// so partial sums over any subset of the candidates can be formed before lse
+// is known and merged like the row statistics (a largest term, then sums
+// rescaled to it): TopKPart below, with zmax the largest z_k / T of the part,
+// sw = sum exp(z_k / T - zmax) and acc = sum exp(z_k / T - zmax)(z_k / T - teacher_k).
+//
+// One warp holds a row's candidates (K <= 64: lane l has candidates l and
+// l + 32). Their ids and teacher log-probs are copied into shared memory one
+// row ahead (cp.async: no registers held; each lane copies, and later reads,
+// only its own entries). The candidates' logits are then taken from the copy
+// of the row already in shared memory, which costs no DRAM access.
+struct TopKBuf {
+  int ids[kMaxTopK];
+  float teacher[kMaxTopK];
+};
+
+struct TopKLane {
+  int id0, id1;  // -1: no candidate (past K or outside [0, V))
+  float z0, z1;
+};
+
+struct TopKPart {
+  float zmax, sw, acc;
+};
+
+__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.wait_all;" ::: "memory");
+}
+
+__device__ __forceinline__ void topk_prefetch(TopKBuf* buf, const int* ids, const float* teacher,
+                                              int K, int lane) {
+  if (lane < K) {
+    cp_async4(&buf->ids[lane], ids + lane);
+    cp_async4(&buf->teacher[lane], teacher + lane);
+  }
+  if (lane + 32 < K) {
+    cp_async4(&buf->ids[lane + 32], ids + lane + 32);
+    cp_async4(&buf->teacher[lane + 32], teacher + lane + 32);
+  }
+  cp_async_commit();
+}
+
+// The lane's candidate ids of the row (after cp_async_wait_all for its buffer).
+__device__ __forceinline__ TopKLane topk_ids(const TopKBuf* buf, int V, int K, int lane) {
+  TopKLane c{-1, -1, 0.0f, 0.0f};
+  if (lane < K) {
+    const int id = buf->ids[lane];
+    if (id >= 0 && id < V) c.id0 = id;
+  }
+  if (lane + 32 < K) {
+    const int id = buf->ids[lane + 32];
+    if (id >= 0 && id < V) c.id1 = id;
+  }
+  return c;
+}
+
+// Take the lane's candidates that lie in columns [c0, c1) from a copy of
+// those columns (element j at src[j - c0]).
 template <class In>
-__device__ __forceinline__ float topk_signal(const void* row, int V, const int* ids,
-                                            const float* teacher, int K, float invT, float lse) {
-  // two passes over the K candidates (the largest log-prob, then the
-  // weighted sum); the second pass reloads the few logits from cache
-  float mx = -INFINITY;
-  for (int k = 0; k < K; ++k) {
-    const int id = ids[k];
-    if (id >= 0 && id < V) mx = fmaxf(mx, In::load1(row, id) * invT - lse);
+__device__ __forceinline__ void topk_gather(TopKLane& c, const void* src, int c0, int c1) {
+  if (c.id0 >= c0 && c.id0 < c1) c.z0 = In::load1(src, c.id0 - c0);
+  if (c.id1 >= c0 && c.id1 < c1) c.z1 = In::load1(src, c.id1 - c0);
+}
+
+__device__ __forceinline__ TopKPart topk_merge(TopKPart a, TopKPart b) {
+  const float M = fmaxf(a.zmax, b.zmax);
+  if (M == -INFINITY) return TopKPart{-INFINITY, 0.0f, 0.0f};
+  const float fa = a.sw > 0.0f ? expf(a.zmax - M) : 0.0f;
+  const float fb = b.sw > 0.0f ? expf(b.zmax - M) : 0.0f;
+  return TopKPart{M, fa * a.sw + fb * b.sw, fa * a.acc + fb * b.acc};
+}
+
+// The warp's part over its lanes' candidates whose ids satisfy `mine`
+// (fixed-order butterfly; every lane ends with it).
+template <class Mine>
+__device__ __forceinline__ TopKPart topk_part(const TopKLane& c, const TopKBuf* buf, int lane,
+                                              float invT, Mine mine) {
+  const bool u0 = c.id0 >= 0 && mine(c.id0), u1 = c.id1 >= 0 && mine(c.id1);
+  const float s0 = c.z0 * invT, s1 = c.z1 * invT;
+  float M = fmaxf(u0 ? s0 : -INFINITY, u1 ? s1 : -INFINITY);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  if (M == -INFINITY) return TopKPart{-INFINITY, 0.0f, 0.0f};
+  const float w0 = u0 ? expf(s0 - M) : 0.0f, w1 = u1 ? expf(s1 - M) : 0.0f;
+  float sw = w0 + w1;
+  float acc = (u0 ? w0 * (s0 - buf->teacher[lane]) : 0.0f) +
+              (u1 ? w1 * (s1 - buf->teacher[lane + 32]) : 0.0f);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    sw += __shfl_xor_sync(0xffffffffu, sw, o);
+    acc += __shfl_xor_sync(0xffffffffu, acc, o);
   }
-  if (mx == -INFINITY) return 0.0f;
-  float sw = 0.0f, acc = 0.0f;
-  for (int k = 0; k < K; ++k) {
-    const int id = ids[k];
-    if (id < 0 || id >= V) continue;
-    const float lp = In::load1(row, id) * invT - lse;
-    const float w = expf(lp - mx);
-    sw += w;
-    acc += w * (lp - teacher[k]);
-  }
-  return acc / sw;
+  return TopKPart{M, sw, acc};
+}
+
+__device__ __forceinline__ float topk_value(const TopKPart& p, float lse) {
+  return p.sw > 0.0f ? p.acc / p.sw - lse : 0.0f;
 }
 
 }  // namespace milesloss

@@ -156,7 +156,7 @@ __device__ __forceinline__ void pass_b_chunk(const uint4* sv, int nv, char* dchu
   }
 }
 
-template <class In, class Out, bool kGrad>
+template <class In, class Out, bool kGrad, bool kTopK>
 __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const StreamArgs a) {
   using St = typename In::storage;
   constexpr int V8 = In::kVec;
@@ -178,6 +178,8 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
   float4* red = reinterpret_cast<float4*>(empty + kMaxSlots);  // [kConsWarps]
   float4* bc = red + kConsWarps;                                // [2]
   int4* bci = reinterpret_cast<int4*>(bc + 2);                  // [1]
+  // [2] top-K candidates of this row and the next (launched with kTopKSmem more)
+  TopKBuf* tkb = reinterpret_cast<TopKBuf*>(smem + static_cast<size_t>(NS) * CB + kSweepSmemExtra);
 
   if (tid == 0) {
     for (int s = 0; s < NS; ++s) {
@@ -262,6 +264,11 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
     if (lane == 0) mbar_arrive(smem_u32(&empty[q % NS]));
   };
 
+  constexpr bool topk = kTopK;  // top-K OPD on (a.s.topk > 0): its own instantiation
+  if (topk && warp == 0 && rows_mine > 0)
+    topk_prefetch(&tkb[0], a.s.topk_ids + static_cast<long long>(blockIdx.x) * a.s.topk,
+                  a.s.topk_teacher + static_cast<long long>(blockIdx.x) * a.s.topk, a.s.topk, lane);
+
   long long q0 = 0;  // task number of the row's first chunk (same count as the producer's)
   for (long long i = 0; i < rows_mine; ++i) {
     const long long row = blockIdx.x + i * gridDim.x;
@@ -283,6 +290,19 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
       if (yok && y >= tail0) zy = In::load1(grow, y);
     }
     const int yv = yok ? y / V8 : -1;  // thread 0 only
+    // top-K OPD candidates (warp 0): this row's ids arrived during the last
+    // row; their logits are taken from the chunks as pass A sweeps them; the
+    // next row's ids and teacher values are copied meanwhile
+    TopKLane tk{-1, -1, 0.0f, 0.0f};
+    const TopKBuf* tk_row = &tkb[i & 1];
+    if (topk && warp == 0) {
+      cp_async_wait_all();
+      tk = topk_ids(tk_row, a.V, a.s.topk, lane);
+      if (i + 1 < rows_mine) {
+        const long long o = (row + gridDim.x) * a.s.topk;
+        topk_prefetch(&tkb[(i + 1) & 1], a.s.topk_ids + o, a.s.topk_teacher + o, a.s.topk, lane);
+      }
+    }
 
     // ---------------- pass A
     // One sweep of each chunk in shared memory against the thread's running
@@ -296,6 +316,7 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
       const uint4* sv = wait_slot(q0 + c);
       const int nv = min(CV, row_vec - c * CV);
       if (tid == 0 && yv >= c * CV && yv < c * CV + nv) zy = In::load1(sv, y - c * CV * V8);
+      if (topk && warp == 0) topk_gather<In>(tk, sv, c * CV * V8, (c * CV + nv) * V8);
       if (run.r == -INFINITY && tid < nv) run.raise(In::vmax(sv[tid]) * k);
       const Run keep = run;
       bool redo = run.r == -INFINITY;  // no finite reference yet
@@ -329,6 +350,8 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
       release_slot(q0 + c);
     }
     Tri t = run.tri();
+    if (topk && warp == 0 && tail0 < a.V)  // candidates past the last whole vector
+      topk_gather<In>(tk, reinterpret_cast<const St*>(grow) + tail0, tail0, a.V);
     for (int j = tail0 + tid; j < a.V; j += kCons) {
       const float z = In::load1(grow, j);
       if (z == -INFINITY) continue;
@@ -360,6 +383,12 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
       }
       t = warp_merge(x);
     }
+    // top-K OPD signal (Sec. 5.2), a fixed per-token reward; warp 0 holds the
+    // row's statistics and candidates
+    float opd = 0.0f;
+    if (topk && warp == 0)
+      opd = topk_value(topk_part(tk, tk_row, lane, a.s.invT, [](int) { return true; }),
+                       fmaf(t.m, kLn2f, logf(t.s)));
 
     // ---------------- epilogue (thread 0)
     char* drow = kGrad ? static_cast<char*>(a.dlogits) +
@@ -373,12 +402,7 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
       float H = lnS - t.u * kLn2f / t.s;
       float logp = zy * a.s.invT - lse;
       if (bad) { logp = 0.0f; H = 0.0f; }
-      if (a.s.topk > 0 && !bad) {
-        // top-K on-policy distillation signal (Sec. 5.2), a fixed per-token reward
-        const long long o = row * a.s.topk;
-        A -= a.s.opd_coef * topk_signal<In>(grow, a.V, a.s.topk_ids + o,
-                                            a.s.topk_teacher + o, a.s.topk, a.s.invT, lse);
-      }
+      if (a.s.topk > 0 && !bad) A -= a.s.opd_coef * opd;
       TokenTerms tt = token_terms(logp, H, rho, q, a.q != nullptr, old, a.old != nullptr, A, a.s);
       if (bad) tt = TokenTerms{0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, kFlagBad};
       if (a.out_logp) a.out_logp[row] = logp;
@@ -476,8 +500,9 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
 }
 
 template <class In, class Out, bool kGrad>
-const void* fn() {
-  return reinterpret_cast<const void*>(&k_stream<In, Out, kGrad>);
+const void* fn(bool topk) {
+  return topk ? reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, true>)
+              : reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, false>);
 }
 
 }  // namespace
@@ -500,13 +525,13 @@ bool use_stream(long long row_bytes, bool in_bulk) {
 // Two 112 KB slots (one CTA per SM): few, large chunks keep the per-chunk
 // handshakes rare (measured best among 16-112 KB chunks with 2-14 slots).
 // Overridable through MILESLOSS_STREAM_CHUNK / MILESLOSS_STREAM_SLOTS.
-rl_status plan_stream(int dev, StreamPlan* out) {
+rl_status plan_stream(int dev, int extra, StreamPlan* out) {
   int optin = 0;
   if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
     return RL_ERR_CUDA;
   const int chunk = env_int("MILESLOSS_STREAM_CHUNK", 114688);
   if (chunk < 1024 || chunk > 131072 || chunk % 128) return RL_ERR_UNSUPPORTED;
-  int slots = (optin - kSweepSmemExtra) / chunk;
+  int slots = (optin - kSweepSmemExtra - extra) / chunk;
   if (slots > kMaxSlots) slots = kMaxSlots;
   const int forced = env_int("MILESLOSS_STREAM_SLOTS", 0);
   if (forced) {
@@ -516,14 +541,16 @@ rl_status plan_stream(int dev, StreamPlan* out) {
   if (slots < 1) return RL_ERR_UNSUPPORTED;
   out->chunk = chunk;
   out->slots = slots;
-  out->smem = slots * chunk + kSweepSmemExtra;
+  out->smem = slots * chunk + kSweepSmemExtra + extra;
   return RL_OK;
 }
 
-const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad) {
-  if (!grad) return in == RL_BF16 ? fn<InBf16, OutBf16, false>() : fn<InF32, OutF32, false>();
-  if (in == RL_BF16) return out == RL_BF16 ? fn<InBf16, OutBf16, true>() : fn<InBf16, OutF32, true>();
-  return out == RL_BF16 ? fn<InF32, OutBf16, true>() : fn<InF32, OutF32, true>();
+const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad, bool topk) {
+  if (!grad)
+    return in == RL_BF16 ? fn<InBf16, OutBf16, false>(topk) : fn<InF32, OutF32, false>(topk);
+  if (in == RL_BF16)
+    return out == RL_BF16 ? fn<InBf16, OutBf16, true>(topk) : fn<InBf16, OutF32, true>(topk);
+  return out == RL_BF16 ? fn<InF32, OutBf16, true>(topk) : fn<InF32, OutF32, true>(topk);
 }
 
 }  // namespace milesloss

@@ -17,7 +17,7 @@ constexpr int kStreamConsumers = 512;     // consumer threads of k_stream (+ one
 constexpr int kMaxSlots = 16;             // ring slots of k_stream
 constexpr int kSeqThreads = 256;
 constexpr int kAdvSmemBytes = 48 * 1024;  // on-chip row offsets + counts when they fit
-constexpr int kMaxTopK = 64;
+constexpr int kTopKSmem = 2 * (2 * kMaxTopK * 4);  // two rows of top-K ids + teacher values
 
 struct SweepArgs {
   const void* logits;
@@ -122,8 +122,11 @@ struct BwdArgs {
 constexpr int kBwdTile = kBwdThreads * 8 * 4;  // elements of one row per backward tile
 
 // Kernel entry points (device function pointers usable with cudaLaunchKernelEx).
-const void* sweep_kernel(rl_dtype in, rl_dtype out, bool grad, int threads);
-const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad);
+// topk: top-K OPD on (a separate instantiation, so that calls without it
+// carry none of its code)
+const void* sweep_kernel(rl_dtype in, rl_dtype out, bool grad, int threads, bool topk);
+const void* sweep_kernel_topk(rl_dtype in, rl_dtype out, bool grad, int threads);
+const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad, bool topk);
 
 // An integer from the environment (tuning overrides), or dflt.
 inline int env_int(const char* name, int dflt) {
@@ -138,7 +141,9 @@ struct StreamPlan {
   int chunk, slots, smem;
 };
 bool use_stream(long long row_bytes, bool in_bulk);
-rl_status plan_stream(int dev, StreamPlan* out);
+// extra: shared memory beyond the ring and the fixed scratch (kTopKSmem with
+// top-K OPD on, else 0)
+rl_status plan_stream(int dev, int extra, StreamPlan* out);
 const void* bwd_kernel(rl_dtype in, rl_dtype out);
 const void* adv_kernel();
 const void* seq_kernel();
