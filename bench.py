@@ -226,10 +226,62 @@ def algorithmic_bytes_per_row(w, dl_dtype) -> int:
 
 # ---------------------------------------------------------------- CPU oracle
 
-def oracle_sample(w, n_rows: int, seed: int = 7):
+def _oracle_rows_task(task):
+    """One block of sampled rows through the float64 oracle, in a worker
+    process (spawned; it attaches to the parent's shared logits)."""
+    from multiprocessing import shared_memory
+
+    import oracle
+
+    (shm_name, shape, dtype, lo, hi, y, rho, q, A_row, mask, N, params) = task
+    shm = shared_memory.SharedMemory(name=shm_name)
+    try:
+        z = np.ndarray(shape, dtype=dtype, buffer=shm.buf)[lo:hi]
+        oracle.rl_loss_rows(z, y, rho, q, A_row, mask, N, oracle.LossParams(**params))
+    finally:
+        shm.close()
+    return hi - lo
+
+
+def _oracle_worker_init():
+    """Worker start-up: import the oracle and run it once on a tiny row so
+    that first-call costs stay out of the timed samples."""
+    import oracle
+
+    oracle.rl_loss_rows(np.zeros((1, 8)), np.zeros(1, np.int64), np.zeros(1), None, np.zeros(1),
+                        np.ones(1, bool), 1, oracle.LossParams())
+
+
+class OraclePool:
+    """A pool of spawned worker processes, one per host core this process
+    may run on, that time the oracle on blocks of sampled rows. Started
+    before any sampling, so that no fork follows CUDA initialisation."""
+
+    def __init__(self, workers: int | None = None):
+        import multiprocessing as mp
+
+        self.workers = workers or max(1, len(os.sched_getaffinity(0)))
+        self.pool = (mp.get_context("spawn").Pool(self.workers, initializer=_oracle_worker_init)
+                     if self.workers > 1 else None)
+        if self.pool is not None:
+            try:  # workers up and importing done; if they cannot start, time in this process
+                self.pool.map_async(int, range(self.workers)).get(timeout=300)
+            except Exception:  # noqa: BLE001
+                self.pool.terminate()
+                self.pool.join()
+                self.pool, self.workers = None, 1
+
+    def close(self):
+        if self.pool is not None:
+            self.pool.close()
+            self.pool.join()
+
+
+def oracle_sample(w, n_rows: int, seed: int = 7, pool: "OraclePool | None" = None):
     """Times the float64 CPU oracle on ``n_rows`` rows of the workload (every
     per-row output and dLogits of those rows, with the call-wide advantages
-    and token count of the whole batch). Returns (rows/s, seconds, rows)."""
+    and token count of the whole batch), on the pool's worker processes (one
+    per core) or in this process. Returns (rows/s, seconds, rows, cores)."""
     import oracle
 
     p = oracle.LossParams(**w.params)
@@ -245,16 +297,41 @@ def oracle_sample(w, n_rows: int, seed: int = 7):
     mask = host(w.loss_mask)
     y, rho = host(w.targets)[rows], host(w.rollout_logprobs)[rows]
     q = None if w.ref_logprobs is None else host(w.ref_logprobs)[rows]
-    t0 = time.perf_counter()
-    A, _ = oracle.group_advantages(host(w.rewards), host(w.group_id), w.n_groups, p)
-    A_row = oracle.row_advantages(A, host(w.cu_seqlens), w.n_rows)
-    N = int(mask.astype(bool).sum())
-    for lo in range(0, len(rows), 128):
-        hi = min(len(rows), lo + 128)
-        oracle.rl_loss_rows(z[lo:hi], y[lo:hi], rho[lo:hi], None if q is None else q[lo:hi],
-                            A_row[rows[lo:hi]], mask[rows[lo:hi]].astype(bool), N, p)
-    dt = time.perf_counter() - t0
-    return len(rows) / dt, dt, len(rows)
+    block = 32
+    if pool is None or pool.pool is None:
+        t0 = time.perf_counter()
+        A, _ = oracle.group_advantages(host(w.rewards), host(w.group_id), w.n_groups, p)
+        A_row = oracle.row_advantages(A, host(w.cu_seqlens), w.n_rows)
+        N = int(mask.astype(bool).sum())
+        for lo in range(0, len(rows), block):
+            hi = min(len(rows), lo + block)
+            oracle.rl_loss_rows(z[lo:hi], y[lo:hi], rho[lo:hi], None if q is None else q[lo:hi],
+                                A_row[rows[lo:hi]], mask[rows[lo:hi]].astype(bool), N, p)
+        dt = time.perf_counter() - t0
+        return len(rows) / dt, dt, len(rows), 1
+    from multiprocessing import shared_memory
+
+    shm = shared_memory.SharedMemory(create=True, size=max(1, z.nbytes))
+    try:
+        zs = np.ndarray(z.shape, dtype=z.dtype, buffer=shm.buf)
+        zs[:] = z
+        t0 = time.perf_counter()
+        A, _ = oracle.group_advantages(host(w.rewards), host(w.group_id), w.n_groups, p)
+        A_row = oracle.row_advantages(A, host(w.cu_seqlens), w.n_rows)
+        N = int(mask.astype(bool).sum())
+        tasks = [(shm.name, z.shape, z.dtype, lo, min(len(rows), lo + block),
+                  y[lo:lo + block], rho[lo:lo + block], None if q is None else q[lo:lo + block],
+                  A_row[rows[lo:lo + block]], mask[rows[lo:lo + block]].astype(bool), N,
+                  dict(w.params))
+                 for lo in range(0, len(rows), block)]
+        done = sum(pool.pool.map(_oracle_rows_task, tasks, chunksize=1))
+        dt = time.perf_counter() - t0
+        del zs
+    finally:
+        shm.close()
+        shm.unlink()
+    assert done == len(rows)
+    return len(rows) / dt, dt, len(rows), pool.workers
 
 
 def run_reference(args, rank, world):
@@ -264,19 +341,24 @@ def run_reference(args, rank, world):
         return
     from paper_2609_08368_gb300 import workloads as wl
 
+    pool = OraclePool()  # spawned before any CUDA work
     rec = wl.RECIPES[args.workload]
     w = wl.make(rec, "cuda" if torch.cuda.is_available() else "cpu")
-    rows_per_step = 128
-    for _ in range(args.warmup):
-        oracle_sample(w, rows_per_step, seed=1)
-    times = []
-    for k in range(args.steps):
-        _, dt, n = oracle_sample(w, rows_per_step, seed=100 + k)
-        times.append(dt)
+    rows_per_step = min(512, 32 * pool.workers)  # one 32-row block per worker
+    try:
+        for _ in range(args.warmup):
+            oracle_sample(w, rows_per_step, seed=1, pool=pool)
+        times = []
+        for k in range(args.steps):
+            _, dt, n, cores = oracle_sample(w, rows_per_step, seed=100 + k, pool=pool)
+            times.append(dt)
+    finally:
+        pool.close()
     total = sum(times)
     value = rows_per_step * args.steps / total
     sample = (f"{rows_per_step} random rows of the {rec.n_rows} x {rec.vocab} batch per step "
-              f"(all per-row outputs and dLogits; call-wide advantages and N)")
+              f"(all per-row outputs and dLogits; call-wide advantages and N), "
+              f"{cores} worker processes")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * total / args.steps,
@@ -284,7 +366,7 @@ def run_reference(args, rank, world):
             "data": "synthetic",
             "config": {"workload": f"{args.workload}: {rec.n_rows} rows x vocab {rec.vocab}",
                        "rows": rec.n_rows, "vocab": rec.vocab},
-            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
@@ -401,10 +483,15 @@ def run_ours(args, rank, world, local):
     # (the sampled-row oracle timing covers the token-level estimators only)
     if rank == 0 and world == 1 and not args.no_cpu_baseline and \
             w.params.get("estimator", "grpo") != "gspo":
-        rps, secs, n = oracle_sample(w, args.cpu_sample_rows)
-        cpu = {"value": rps, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+        pool = OraclePool()
+        try:
+            rps, secs, n, cores = oracle_sample(w, args.cpu_sample_rows, pool=pool)
+        finally:
+            pool.close()
+        cpu = {"value": rps, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                "sample": f"{n} random rows of the {R} x {V} batch (every per-row output and "
-                         f"dLogits of those rows; call-wide advantages and N), {secs:.1f} s"}
+                         f"dLogits of those rows; call-wide advantages and N), {secs:.1f} s "
+                         f"wall on {cores} worker processes"}
 
     # end to end through host buffers (pinned), one call per step
     e2e = None
