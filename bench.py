@@ -211,6 +211,14 @@ def sweep_kernel_name(vocab: int, elem_size: int) -> str:
     return "k_sweep (fused fwd+bwd vocabulary sweep, clusters sharing a row)"
 
 
+def launches_per_call(params: dict, n_groups: int) -> int:
+    """Kernels one fused call launches: group statistics (when there are
+    groups), advantages, the sweep and the statistics; GSPO adds the
+    per-trajectory pass and the gradient sweep."""
+    n = 3 + (1 if n_groups > 8 else 0)  # up to 8 groups, k_advantages computes them itself
+    return n + (2 if params.get("estimator", "grpo") == "gspo" else 0)
+
+
 def algorithmic_bytes_per_row(w, dl_dtype) -> int:
     """Logits read once + dLogits written once + the per-row inputs and
     outputs (target, rollout log-prob, optional ref / old / teacher
@@ -472,6 +480,7 @@ def run_ours(args, rank, world, local):
 
     bpr = algorithmic_bytes_per_row(w, dl_dtype)  # before w is released for the e2e leg
     kernel_name = sweep_kernel_name(V, w.logits.element_size())
+    w_params, n_groups = dict(w.params), w.n_groups
     launch_bytes = bpr * R
     sweep_avg = statistics.fmean(sweep_ms)
     peaks, peak_kind = measured_peaks()
@@ -542,7 +551,7 @@ def run_ours(args, rank, world, local):
         "also": also,
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": 3 * K,
+        "gpu_launches": launches_per_call(w_params, n_groups) * K,
         "clocks": clk,
         "loss": stats["loss"],
     }

@@ -370,9 +370,15 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
   aa.advantages = f.out_adv;
   aa.group_sizes = f.out_gsize;
   aa.estimator = c.p->estimator;
-  const size_t traj_bytes = (2 * static_cast<size_t>(f.n_traj) + 1) * sizeof(int);
+  // cu_seqlens, per-trajectory counts and advantages, group ids, rewards
+  const size_t traj_bytes = (5 * static_cast<size_t>(f.n_traj) + 1) * sizeof(int);
   aa.smem_traj = traj_bytes <= static_cast<size_t>(kAdvSmemBytes);
   aa.ws = ws;
+  if (f.n_groups > kInlineGroups) {
+    const int gb = std::min(f.n_groups, kMaxGroupBlocks);
+    st = launch(groups_kernel(), dim3(static_cast<unsigned>(gb)), dim3(32), 0, 1, s, &aa);
+    if (st != RL_OK) return st;
+  }
   st = launch(adv_kernel(), dim3(1), dim3(kAdvThreads),
               aa.smem_traj ? static_cast<int>(traj_bytes) : 0, 1, s, &aa);
   if (st != RL_OK) return st;

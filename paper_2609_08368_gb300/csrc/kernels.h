@@ -146,6 +146,11 @@ bool use_stream(long long row_bytes, bool in_bulk);
 rl_status plan_stream(int dev, int extra, StreamPlan* out);
 const void* bwd_kernel(rl_dtype in, rl_dtype out);
 const void* adv_kernel();
+const void* groups_kernel();  // one 32-thread block per group (grid-stride)
+constexpr int kMaxGroupBlocks = 65535;
+// Up to this many groups, k_advantages computes the group statistics itself
+// (a launch costs more than their double arithmetic on one SM).
+constexpr int kInlineGroups = 8;
 const void* seq_kernel();
 const void* stats_kernel();
 

@@ -231,6 +231,25 @@ def test_long_rows_padded_and_misaligned(ld, ld_out):
             assert torch.isnan(g["dlogits_t"][:, w.vocab:]).all()
 
 
+@pytest.mark.parametrize("estimator", ["grpo", "reinforcepp", "gspo"])
+@pytest.mark.parametrize("n_prompts", [8, 1200])
+def test_ragged_and_empty_trajectories(estimator, n_prompts):
+    """Trajectories of random lengths, some empty, with their row offsets in
+    shared memory (32 trajectories) or, past what fits there, in global memory
+    (4,800 trajectories)."""
+    rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=n_prompts, group_size=4, traj_len=3,
+                    vocab=512)
+    w = wl.make(rec, DEV)
+    rng = np.random.default_rng(n_prompts)
+    n_traj = int(w.rewards.shape[0])
+    cuts = np.sort(rng.integers(0, w.n_rows + 1, size=n_traj - 1))
+    cu = np.concatenate([[0], cuts, [w.n_rows]]).astype(np.int32)
+    assert (np.diff(cu) == 0).any()
+    w.cu_seqlens.copy_(torch.from_numpy(cu))
+    w.loss_mask.copy_(torch.from_numpy((rng.random(w.n_rows) < 0.7).astype(np.uint8)))
+    _full_check(w, params=dict(w.params, estimator=estimator))
+
+
 @pytest.mark.parametrize("logit_dtype,dl_dtype", [("bf16", torch.float32), ("f32", torch.bfloat16)])
 def test_mixed_dtypes(logit_dtype, dl_dtype):
     rec = wl.shrink(wl.RECIPES["fp32" if logit_dtype == "f32" else "tiny"], n_prompts=2,
