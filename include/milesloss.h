@@ -128,7 +128,8 @@ typedef struct {
    * opd_topk_teacher[t*K + k]. The signal is sum_k w_k (log p_k - teacher_k)
    * with the trainer's probabilities p_k of the candidates renormalised over
    * the set as weights w_k; it is subtracted, times opd_coef, from the token's
-   * advantage and is not differentiated. */
+   * advantage and is not differentiated. Both arrays are device memory,
+   * 4-byte aligned (else RL_ERR_INVALID_ARG); K <= 64. */
   const int32_t* opd_topk_ids;
   const float* opd_topk_teacher;
 } rl_loss_params;

@@ -12,10 +12,11 @@
 // the headline workload, against a 126 MB L2), so the second read of a row
 // is served by L2 and HBM sees each logit once (checked with the DRAM byte
 // counters). The sixteen consumer warps:
-//   pass A  per chunk, each thread folds its vectors into an online
-//           (max, S, U) in packed f32x2 (rescaling when its maximum grows),
-//           then releases the slot;
-//   merge   butterfly merges, maximum first, in a fixed order;
+//   pass A  per chunk, each thread sums its vectors into (S, U) in packed
+//           f32x2 against a running reference that moves by whole powers of
+//           two (no per-element maximum), then releases the slot; warp 0
+//           also takes the row's top-K OPD candidates from the chunk;
+//   merge   butterfly merges, largest reference first, in a fixed order;
 //   epilogue one thread evaluates the per-token objective and the gradient
 //           coefficients;
 //   pass B  per chunk, dLogits from the re-read chunk, 16-byte streaming

@@ -16,7 +16,7 @@ constexpr int kBwdThreads = 256;
 constexpr int kStreamConsumers = 512;     // consumer threads of k_stream (+ one producer warp)
 constexpr int kMaxSlots = 16;             // ring slots of k_stream
 constexpr int kSeqThreads = 256;
-constexpr int kAdvSmemBytes = 48 * 1024;  // on-chip row offsets + counts when they fit
+constexpr int kAdvSmemBytes = 48 * 1024;  // on-chip trajectory tables when they fit
 constexpr int kTopKSmem = 2 * (2 * kMaxTopK * 4);  // two rows of top-K ids + teacher values
 
 struct SweepArgs {
@@ -78,7 +78,8 @@ struct AdvArgs {
   int normalize_std, unbiased_std;
   float std_floor;
   int estimator;   // rl_estimator
-  int smem_traj;   // cu_seqlens and per-trajectory counts staged in shared memory
+  int smem_traj;   // trajectory tables (cu_seqlens, group ids, rewards, counts,
+                   // advantages) staged in shared memory
   float* advantages;   // may be null
   int* group_sizes;    // may be null
   WsPtrs ws;

@@ -68,6 +68,16 @@ def test_workspace_size(lib):
 FAKE = 1 << 20  # never dereferenced: every case below fails validation first
 
 
+class _Ptr:
+    """A fake device pointer with the tensor method make_params reads."""
+
+    def __init__(self, addr):
+        self.addr = addr
+
+    def data_ptr(self):
+        return self.addr
+
+
 def _fwd_bwd_args(**over):
     p = ml.make_params(**over.pop("params", {}))
     a = dict(logits=FAKE, dt=ml.RL_BF16, R=16, V=64, ld=64, targets=FAKE, rho=FAKE, q=None,
@@ -128,6 +138,10 @@ INVALID = [
     dict(params=dict(opd_coef=0.5, opd_topk=4)),        # no candidate ids / teacher log-probs
     dict(params=dict(opd_coef=0.5, opd_topk=65), teacher=FAKE),
     dict(params=dict(opd_topk=-1)),
+    dict(params=dict(opd_coef=0.5, opd_topk=4, opd_topk_ids=_Ptr(FAKE + 2),  # not 4-byte aligned
+                     opd_topk_teacher=_Ptr(FAKE))),
+    dict(params=dict(opd_coef=0.5, opd_topk=4, opd_topk_ids=_Ptr(FAKE),
+                     opd_topk_teacher=_Ptr(FAKE + 1))),
 ]
 
 
