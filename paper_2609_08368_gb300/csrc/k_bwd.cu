@@ -45,8 +45,10 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
   // All of a thread's 16-byte streaming loads of a tile are issued before
   // any is used, and the next tile's loads are issued before this tile's
   // arithmetic, so each thread keeps up to 2 kPer loads in flight.
+  // rows that do not train (or have a bad target) get zeros: no read
+  auto reads = [&](long long row) { return a.mask[row] != 0 && !(ws.flags[row] & kFlagBad); };
   auto load_tile = [&](long long row, int t, uint4* raw) {
-    const int nv = tile_nv(t);
+    const int nv = reads(row) ? tile_nv(t) : 0;
     const char* zrow = static_cast<const char*>(a.logits) + row * a.ld * static_cast<long long>(sizeof(St)) +
                        static_cast<size_t>(t) * kTile * sizeof(St);
 #pragma unroll
@@ -69,8 +71,8 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
     const char* zrow = static_cast<const char*>(a.logits) + row * a.ld * static_cast<long long>(sizeof(St));
     char* drow = static_cast<char*>(a.dlogits) + row * a.ld_out * static_cast<long long>(Out::kSize);
     const int nv = tile_nv(t);
-    const bool bad = (ws.flags[row] & kFlagBad) != 0;
-    const float cc = (a.mask[row] && !bad) ? cscale : 0.0f;
+    const bool rd = reads(row);
+    const float cc = rd ? cscale : 0.0f;
     const float G = ws.G[row], H = ws.H[row], lse = ws.lse[row];
     const float ca = cc * (-G + a.gamma * (H - lse));
     const float cb = cc * a.gamma * a.invT;
@@ -95,11 +97,11 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
       if (v >= nv) continue;
       const int jb = j0 + v * V8;
       float f[V8];
-      In::unpack(raw[i], f);
-      if (cc == 0.0f) {
+      if (cc == 0.0f) {  // (a row that does not train was not read)
 #pragma unroll
         for (int e = 0; e < V8; ++e) f[e] = 0.0f;
       } else {
+        In::unpack(raw[i], f);
 #pragma unroll
         for (int e = 0; e < V8; ++e) f[e] = ex2(fmaf(f[e], a.k, -L2)) * ent_factor(f[e], ca, cb);
         if (has_y && static_cast<unsigned>(y - jb) < static_cast<unsigned>(V8)) {
@@ -111,7 +113,7 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
       Out::template storev<V8>(drow + static_cast<size_t>(jb) * Out::kSize, f, 0u);
     }
     for (int j = j0 + nv * V8 + threadIdx.x; j < j1; j += kBwdThreads)
-      Out::store1(drow, j, value(In::load1(zrow, j), j));
+      Out::store1(drow, j, cc == 0.0f ? 0.0f : value(In::load1(zrow, j), j));
 #pragma unroll
     for (int i = 0; i < kPer; ++i) raw[i] = nxt[i];
     row = nrow;
