@@ -156,6 +156,8 @@ struct SweepPlan {
 // stages as still fit; if no cluster size fits, one CTA per SM.
 // Overridable for tuning through MILESLOSS_SWEEP_CLUSTER / _STAGES /
 // _THREADS / _CTAS_PER_SM.
+constexpr long long kMinSliceBytes = 32 * 1024;  // smallest cluster slice a fused plan takes
+
 rl_status plan_sweep(rl_dtype dt, long long V, int dev, int extra, bool grad, SweepPlan* out) {
   int optin = 0, per_sm = 0, reserved = 0;
   if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
@@ -211,6 +213,25 @@ rl_status plan_sweep(rl_dtype dt, long long V, int dev, int extra, bool grad, Sw
         fill(C, S);
         return RL_OK;
       }
+    }
+  }
+  // Fused calls: the largest cluster whose slices are still at least
+  // kMinSliceBytes (slices of 32-48 KB measured best on GB300; 20-24 KB
+  // slices ran 10-25 % slower: bf16 rows of 40,960 / 49,152 columns), with
+  // as many stages as fit a fifth of the SM's shared memory, else one.
+  if (grad && !forced_c && !forced_s && threads == 256 && target == 5) {
+    int C = 1;
+    for (int c = 2; c <= kMaxCluster; c *= 2) {
+      const long long slice = slice_of(c);
+      if (slice * (c - 1) >= V || slice * es < kMinSliceBytes) break;
+      C = c;
+    }
+    const long long stage = (slice_of(C) * es + 127) / 128 * 128;
+    if (stage <= hard) {
+      int S = stage <= share ? static_cast<int>(share / stage) : 1;
+      if (S > kMaxStages) S = kMaxStages;
+      fill(C, S);
+      return RL_OK;
     }
   }
   for (int pass = 0; pass < 2; ++pass) {
