@@ -215,16 +215,28 @@ rl_status plan_sweep(rl_dtype dt, long long V, int dev, int extra, bool grad, Sw
       }
     }
   }
-  // Fused calls: the largest cluster whose slices are still at least
-  // kMinSliceBytes (slices of 32-48 KB measured best on GB300; 20-24 KB
-  // slices ran 10-25 % slower: bf16 rows of 40,960 / 49,152 columns), with
-  // as many stages as fit a fifth of the SM's shared memory, else one.
+  // Fused calls: for bf16 rows, the cluster of 2 or more CTAs whose slices
+  // are 48-64 KB when there is one; otherwise (and for fp32) the largest cluster whose slices
+  // are still at least kMinSliceBytes; as many stages as fit a fifth of the
+  // SM's shared memory, else one. Measured on GB300 (bf16 rows): 20-24 KB
+  // slices ran 10-25 % slower than 32-64 KB ones (40,960 / 49,152 columns),
+  // 64 KB slices beat 32 KB ones by 2-7 % (65,536 / 131,072 columns); for
+  // fp32 rows of 32,768 columns 32 KB slices beat 64 KB ones by 3 %.
   if (grad && !forced_c && !forced_s && threads == 256 && target == 5) {
     int C = 1;
     for (int c = 2; c <= kMaxCluster; c *= 2) {
       const long long slice = slice_of(c);
       if (slice * (c - 1) >= V || slice * es < kMinSliceBytes) break;
       C = c;
+    }
+    if (dt == RL_BF16) {
+      for (int c = 2; c <= kMaxCluster; c *= 2) {  // (a whole 64 KB row in one CTA was slower)
+        const long long b = slice_of(c) * es;
+        if (b >= 48 * 1024 && b <= 64 * 1024 && slice_of(c) * (c - 1) < V) {
+          C = c;
+          break;
+        }
+      }
     }
     const long long stage = (slice_of(C) * es + 127) / 128 * 128;
     if (stage <= hard) {

@@ -508,13 +508,14 @@ const void* fn(bool topk) {
 
 }  // namespace
 
-// Rows of 160 KB and more with 16-byte aligned starts go to the streaming
+// Rows of 280 KB and more with 16-byte aligned starts go to the streaming
 // kernel (one CTA per row, second read served by L2); shorter or unaligned
-// rows to the cluster kernel, which keeps them on chip. Measured on GB300:
-// bf16 rows of 151,936-154,880 columns run faster streamed, fp32 rows of
-// 32,768 columns faster in clusters. MILESLOSS_SWEEP_KIND=stream|cluster
-// overrides the choice.
-constexpr long long kStreamMinRowBytes = 160 * 1024;
+// rows to the cluster kernel, which keeps them on chip. Measured on GB300
+// (bf16, fused): rows of 151,936-154,880 columns (297-310 KB) run faster
+// streamed (0.955 against 0.941 of the copy peak), rows of 81,920-131,072
+// columns (160-256 KB) faster in clusters (0.94-0.96 against 0.89-0.94).
+// MILESLOSS_SWEEP_KIND=stream|cluster overrides the choice.
+constexpr long long kStreamMinRowBytes = 280 * 1024;
 
 bool use_stream(long long row_bytes, bool in_bulk) {
   const char* k = std::getenv("MILESLOSS_SWEEP_KIND");

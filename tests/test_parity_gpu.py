@@ -213,12 +213,14 @@ def test_extreme_logits(monkeypatch, kind, extra):
     _full_check(w, mode="split", params=params)
 
 
+@pytest.mark.parametrize("kind", ["cluster", "stream"])
 @pytest.mark.parametrize("ld,ld_out", [(100008, 100000), (100003, 100003), (100000, 100011)])
-def test_long_rows_padded_and_misaligned(ld, ld_out):
-    """Rows of 200 KB (the streaming kernel's size) with a padded row stride,
-    rows whose starts are not 16-byte aligned (the cluster kernel's element-wise
-    path takes them), and a dLogits stride that is not 16-byte aligned (scalar
-    stores); fused and split."""
+def test_long_rows_padded_and_misaligned(monkeypatch, kind, ld, ld_out):
+    """Rows of 200 KB on both sweep kernels with a padded row stride, rows
+    whose starts are not 16-byte aligned (the cluster kernel's element-wise
+    path takes them whatever the kind), and a dLogits stride that is not
+    16-byte aligned (scalar stores); fused and split."""
+    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=6, vocab=100000)
     w = wl.make(rec, DEV, ld=ld)
     for mode in ("fused", "split"):
