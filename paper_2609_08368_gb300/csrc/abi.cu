@@ -481,7 +481,7 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
   const size_t es = elem_size(c.dt);
   const bool in_bulk = aligned16(c.logits) && ((c.ld * es) % 16 == 0);
   const bool out_vec = grad && aligned16(go->dl) && ((go->ld_out * elem_size(go->dt)) % 16 == 0);
-  if (c.R > 0 && use_stream(c.V * static_cast<long long>(es), in_bulk)) {
+  if (c.R > 0 && use_stream(c.V * static_cast<long long>(es), in_bulk, grad)) {
     StreamPlan sp;
     st = plan_stream(dev, sc.topk ? kTopKSmem : 0, &sp);
     if (st != RL_OK) return st;

@@ -508,20 +508,24 @@ const void* fn(bool topk) {
 
 }  // namespace
 
-// Rows of 280 KB and more with 16-byte aligned starts go to the streaming
-// kernel (one CTA per row, second read served by L2); shorter or unaligned
-// rows to the cluster kernel, which keeps them on chip. Measured on GB300
-// (bf16, fused): rows of 151,936-154,880 columns (297-310 KB) run faster
-// streamed (0.955 against 0.941 of the copy peak), rows of 81,920-131,072
-// columns (160-256 KB) faster in clusters (0.94-0.96 against 0.89-0.94).
-// MILESLOSS_SWEEP_KIND=stream|cluster overrides the choice.
-constexpr long long kStreamMinRowBytes = 280 * 1024;
+// Rows with 16-byte aligned starts go to the streaming kernel (one CTA per
+// row, second read served by L2) from 280 KB in a fused call and from 160 KB
+// in a forward-only one; shorter or unaligned rows to the cluster kernel,
+// which keeps them on chip. Measured on GB300 (bf16, fractions of the copy
+// peak): fused, rows of 151,936-154,880 columns (297-310 KB) streamed 0.955
+// against 0.941 in clusters, rows of 81,920-131,072 columns (160-256 KB) in
+// clusters 0.94-0.96 against 0.89-0.94 streamed; forward only, rows of
+// 160-310 KB streamed 0.92-1.09 against 0.78-0.88, rows of 96-128 KB in
+// clusters 0.87-0.92 against 0.79. MILESLOSS_SWEEP_KIND=stream|cluster
+// overrides the choice.
+constexpr long long kStreamMinRowBytes = 280 * 1024;     // fused calls
+constexpr long long kStreamMinRowBytesFwd = 160 * 1024;  // forward-only calls
 
-bool use_stream(long long row_bytes, bool in_bulk) {
+bool use_stream(long long row_bytes, bool in_bulk, bool grad) {
   const char* k = std::getenv("MILESLOSS_SWEEP_KIND");
   if (k && std::string(k) == "cluster") return false;
   if (k && std::string(k) == "stream") return in_bulk;
-  return in_bulk && row_bytes >= kStreamMinRowBytes;
+  return in_bulk && row_bytes >= (grad ? kStreamMinRowBytes : kStreamMinRowBytesFwd);
 }
 
 // Two 112 KB slots (one CTA per SM): few, large chunks keep the per-chunk

@@ -141,7 +141,7 @@ inline int env_int(const char* name, int dflt) {
 struct StreamPlan {
   int chunk, slots, smem;
 };
-bool use_stream(long long row_bytes, bool in_bulk);
+bool use_stream(long long row_bytes, bool in_bulk, bool grad);
 // extra: shared memory beyond the ring and the fixed scratch (kTopKSmem with
 // top-K OPD on, else 0)
 rl_status plan_stream(int dev, int extra, StreamPlan* out);

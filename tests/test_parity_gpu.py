@@ -404,7 +404,7 @@ def test_bitwise_reproducible_and_fwd_matches_fused():
     assert a["stats"] == c["stats"]
 
 
-@pytest.mark.parametrize("vocab", [30000, 40000])  # cluster kernel, streaming kernel
+@pytest.mark.parametrize("vocab", [30000, 100000])  # forward: cluster kernel, streaming kernel
 def test_batch_invariance_of_row_outputs(vocab):
     """A row's log-prob and entropy do not depend on where it sits or on how
     many other rows share the call."""
