@@ -82,6 +82,28 @@ def bwd(w, buf: Buffers, params=None, grad_loss=1.0, grad_loss_device=None, stre
                    stream=stream)
 
 
+class GraphedCall:
+    """The fused call on fixed tensors, captured once in a CUDA graph; each
+    call replays it on the current stream. The library only enqueues kernels
+    (no allocation, no synchronisation), so the capture holds the whole call;
+    the inputs may change in place between replays. For small calls the host
+    launch cost of the three to four kernels is then paid once."""
+
+    def __init__(self, w, buf: Buffers, params=None, grad_loss=1.0):
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            fwd_bwd(w, buf, params=params, grad_loss=grad_loss)  # kernel attributes set outside capture
+        torch.cuda.current_stream().wait_stream(s)
+        torch.cuda.synchronize()
+        self.graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.graph):
+            fwd_bwd(w, buf, params=params, grad_loss=grad_loss)
+
+    def __call__(self):
+        self.graph.replay()
+
+
 class HostCall:
     """Fused forward+backward with the inputs and results in pinned HOST
     memory: every call copies the inputs host -> device, runs the loss, and

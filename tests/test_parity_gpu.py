@@ -263,19 +263,11 @@ def test_fused_call_replays_from_a_cuda_graph(monkeypatch, kind):
     w = wl.make(rec, DEV)
     buf = api.alloc(w.n_rows, int(w.rewards.shape[0]), w.n_groups, DEV, vocab=w.vocab,
                     dlogits_dtype=w.logits.dtype)
-    s = torch.cuda.Stream()
-    s.wait_stream(torch.cuda.current_stream())
-    with torch.cuda.stream(s):
-        api.fwd_bwd(w, buf)  # warm-up: per-device kernel attributes set outside capture
-    torch.cuda.current_stream().wait_stream(s)
-    torch.cuda.synchronize()
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph):
-        api.fwd_bwd(w, buf)
+    call = api.GraphedCall(w, buf)
     for step in range(2):
         if step:
             w.logits.mul_(0.5)  # new inputs, same buffers
-        graph.replay()
+        call()
         torch.cuda.synchronize()
         got = (buf.dlogits.clone(), buf.token_logprobs.clone(), buf.read_stats()["loss"])
         api.fwd_bwd(w, buf)
