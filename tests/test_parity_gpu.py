@@ -333,6 +333,23 @@ def test_opd_topk(monkeypatch, kind, K):
         _full_check(w, mode="split", params=params)
 
 
+@pytest.mark.parametrize("kind,cluster", [("cluster", 0), ("cluster", 8), ("stream", 0)])
+@pytest.mark.parametrize("K", [4, 64])
+def test_opd_topk_long_rows(monkeypatch, kind, cluster, K):
+    """Top-K OPD on rows of 200 KB: candidates spread over the CTAs of a
+    cluster (4 by the plan, 8 forced; their partial sums merge in the row
+    exchange) or over the streaming kernel's two ring chunks."""
+    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+    if cluster:
+        monkeypatch.setenv("MILESLOSS_SWEEP_CLUSTER", str(cluster))
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=12, vocab=100000,
+                    rho_noise=0.3, ref_noise=0.2, topk=K, topk_noise=0.4)
+    w = wl.make(rec, DEV)
+    params = dict(w.params, opd_coef=0.5, opd_topk=K)
+    _full_check(w, params=params)
+    _full_check(w, mode="split", params=params)
+
+
 @pytest.mark.parametrize("kind", ["cluster", "stream"])
 def test_no_training_tokens_and_empty_call(monkeypatch, kind):
     monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
