@@ -186,7 +186,8 @@ def _extreme_rows(w):
 
 
 @pytest.mark.parametrize("kind", ["cluster", "stream"])
-@pytest.mark.parametrize("extra", [dict(), dict(entropy_coef=0.01, temperature=0.7)])
+@pytest.mark.parametrize("extra", [dict(), dict(entropy_coef=0.01, temperature=0.7),
+                                   dict(temperature=0.05)])
 def test_extreme_logits(monkeypatch, kind, extra):
     """Extreme rows (see _extreme_rows) on both sweep kernels, fused and
     split, with and without the entropy term and temperature; a row of 200 KB
