@@ -8,7 +8,7 @@
 // mbarrier (one arrival per consumer warp). The producer walks the task list
 // row by row: the chunks of the row for pass A, then the same chunks again
 // for pass B. Pass A's copies are marked evict-last in L2 and pass B's
-// evict-first: with one CTA per SM only ~one row per SM is live (~46 MB on
+// evict-first (a forward-only call reads each chunk once: evict-first too): with one CTA per SM only ~one row per SM is live (~46 MB on
 // the headline workload, against a 126 MB L2), so the second read of a row
 // is served by L2 and HBM sees each logit once (checked with the DRAM byte
 // counters). The sixteen consumer warps:
@@ -221,7 +221,7 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
           const uint32_t bar = smem_u32(&full[s]);
           mbar_arrive_expect_tx(bar, bytes);
           bulk_g2s(smem_u32(ring + static_cast<size_t>(s) * CB), src_row + static_cast<size_t>(v0) * 16,
-                   bytes, bar, t < n_chunks ? pol_a : pol_b);
+                   bytes, bar, (kGrad && t < n_chunks) ? pol_a : pol_b);
         }
       }
       // A timeout leaves copies in flight: wait (bounded) for the last one
