@@ -1,0 +1,52 @@
+"""Host-side helpers of bench.py and the tensor API, on CPU: the launch count
+per call, the sweep-kernel naming rule, the profiled traffic's validity checks,
+the algorithmic bytes per row, and the top-K parameter attachment."""
+
+import os
+import sys
+
+import torch
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import bench  # noqa: E402
+from paper_2609_08368_gb300 import api, workloads as wl  # noqa: E402
+
+
+def test_launches_per_call():
+    assert bench.launches_per_call({}, 4) == 3                     # glm: groups inline
+    assert bench.launches_per_call({}, 64) == 4                    # fp32: k_groups too
+    assert bench.launches_per_call({"estimator": "gspo"}, 4) == 5  # + k_seq, k_bwd
+    assert bench.launches_per_call({"estimator": "reinforcepp"}, 1) == 3
+
+
+def test_sweep_kernel_name_follows_the_fused_threshold():
+    assert bench.sweep_kernel_name(154880, 2).startswith("k_stream")
+    assert bench.sweep_kernel_name(131072, 2).startswith("k_sweep")
+    assert bench.sweep_kernel_name(32768, 4).startswith("k_sweep")
+    assert bench.sweep_kernel_name(80000, 4).startswith("k_stream")
+
+
+def test_profiled_traffic_only_for_its_workload_and_sources():
+    t = bench.profiled_traffic(65536, "glm", 154880)
+    assert t is None or t > 4e10  # valid only while the sources hash to the capture's
+    assert bench.profiled_traffic(65536, "glm", 100000) is None
+    assert bench.profiled_traffic(131072, "fp32", 32768) is None
+
+
+def test_algorithmic_bytes_per_row():
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=2, traj_len=2, vocab=1000)
+    w = wl.make(rec, "cpu")
+    # bf16 in and out, plus target, rollout, ref log-prob, mask, logp and H out
+    assert bench.algorithmic_bytes_per_row(w, torch.bfloat16) == 1000 * 4 + 4 + 4 + 4 + 1 + 4 + 4
+    assert bench.algorithmic_bytes_per_row(w, torch.float32) == 1000 * 6 + 21
+
+
+def test_api_attaches_top_k_inputs():
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=2, traj_len=2, vocab=64, topk=4)
+    w = wl.make(rec, "cpu")
+    p = api._params(w, dict(w.params, opd_topk=4, opd_coef=0.5))
+    assert p["opd_topk_ids"] is w.topk_ids and p["opd_topk_teacher"] is w.topk_teacher
+    assert "opd_topk_ids" not in api._params(w, None)
