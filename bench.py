@@ -203,10 +203,10 @@ def profiled_traffic(rows_now: int, workload: str, vocab: int):
 
 
 def sweep_kernel_name(vocab: int, elem_size: int) -> str:
-    """The sweep kernel the library picks for these rows (rows of 280 KB and
-    more, 16-byte aligned, stream through one CTA each; shorter rows go to the
-    cluster kernel)."""
-    if vocab * elem_size >= 280 * 1024:
+    """The sweep kernel the library picks for these rows in a fused call
+    (rows of 192 KB and more, 16-byte aligned, stream through one CTA each;
+    shorter rows go to the cluster kernel)."""
+    if vocab * elem_size >= 192 * 1024:
         return "k_stream (fused fwd+bwd vocabulary sweep, one CTA per row)"
     return "k_sweep (fused fwd+bwd vocabulary sweep, clusters sharing a row)"
 

@@ -483,7 +483,7 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
   const bool out_vec = grad && aligned16(go->dl) && ((go->ld_out * elem_size(go->dt)) % 16 == 0);
   if (c.R > 0 && use_stream(c.V * static_cast<long long>(es), in_bulk, grad)) {
     StreamPlan sp;
-    st = plan_stream(dev, sc.topk ? kTopKSmem : 0, &sp);
+    st = plan_stream(dev, sc.topk ? kTopKSmem : 0, c.V * static_cast<long long>(es), grad, &sp);
     if (st != RL_OK) return st;
     const void* fn = stream_kernel(c.dt, grad ? go->dt : c.dt, grad, sc.topk > 0);
     st = set_smem(fn, dev, sp.smem);
@@ -498,6 +498,8 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     ta.V = static_cast<int>(c.V);
     ta.chunk_bytes = sp.chunk;
     ta.n_slots = sp.slots;
+    ta.n_hold = sp.hold;
+    ta.split_first = sp.split_first;
     ta.out_vec = out_vec;
     ta.targets = c.targets;
     ta.rho = fr.rho;

@@ -6,12 +6,15 @@
 // (bulk async copies, non-multicast) into a ring of shared-memory slots,
 // each slot with a "full" mbarrier (transaction bytes) and an "empty"
 // mbarrier (one arrival per consumer warp). The producer walks the task list
-// row by row: the chunks of the row for pass A, then the same chunks again
-// for pass B. Pass A's copies are marked evict-last in L2 and pass B's
-// evict-first (a forward-only call reads each chunk once: evict-first too): with one CTA per SM only ~one row per SM is live (~46 MB on
-// the headline workload, against a 126 MB L2), so the second read of a row
-// is served by L2 and HBM sees each logit once (checked with the DRAM byte
-// counters). The sixteen consumer warps:
+// row by row: the chunks of the row for pass A, then, for pass B, the same
+// chunks in reverse order except the last, which pass B takes from the slot
+// pass A left it in (the consumers release that slot only after pass B has
+// used it). Pass A's copies of chunks that are read again are marked
+// evict-last in L2, every other copy evict-first: with one CTA per SM only
+// ~one row per SM is live (~46 MB on the headline workload, against a
+// 126 MB L2), so the second read of a row is served by L2 and HBM sees each
+// logit about once (checked with the DRAM byte counters); the reverse order
+// re-reads the most recently copied chunk first. The sixteen consumer warps:
 //   pass A  per chunk, each thread sums its vectors into (S, U) in packed
 //           f32x2 against a running reference that moves by whole powers of
 //           two (no per-element maximum), then releases the slot; warp 0
@@ -19,7 +22,7 @@
 //   merge   butterfly merges, largest reference first, in a fixed order;
 //   epilogue one thread evaluates the per-token objective and the gradient
 //           coefficients;
-//   pass B  per chunk, dLogits from the re-read chunk, 16-byte streaming
+//   pass B  per chunk, last to first, dLogits from the chunk, 16-byte streaming
 //           stores; the sampled token's entry is rewritten during the next
 //           row's epilogue (after a barrier that orders every store before it).
 // Definitions: Sec. 3.4 (ratio), Sec. 2 / 9.1 (advantage), Sec. 2.4 (mask).
@@ -171,6 +174,15 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
   const int row_vec = a.V / V8;                  // whole 16-byte vectors per row
   const int tail0 = row_vec * V8;                // first element not in a vector
   const int n_chunks = (row_vec + CV - 1) / CV;
+  // Chunk c starts at vector cs(c) and holds cn(c) vectors. With
+  // split_first the first chunk takes the remainder, rounded up to a multiple
+  // of 8 vectors (128 bytes) so that every later chunk starts 128-byte aligned
+  // and the last chunks, which pass B takes from shared memory, are (nearly)
+  // full; otherwise the last chunk is the ragged one.
+  const int rem = row_vec - (n_chunks - 1) * CV;
+  const int f0 = a.split_first ? min(CV, (rem + 7) & ~7) : CV;
+  auto cs = [&](int c) { return c == 0 ? 0 : min(row_vec, f0 + (c - 1) * CV); };
+  auto cn = [&](int c) { return cs(c + 1) - cs(c); };
   const float k = a.s.k;
 
   unsigned char* ring = smem;
@@ -205,9 +217,13 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
         const long long row = blockIdx.x + i * gridDim.x;
         const char* src_row = lg + row * a.ld * static_cast<long long>(sizeof(St));
         // a row that does not train has an all-zero gradient: no second read
-        const int tasks = (kGrad && a.mask[row]) ? 2 * n_chunks : n_chunks;
+        const bool again = kGrad && a.mask[row] && n_chunks > 0;
+        const int h = again ? min(a.n_hold, n_chunks) : 0;
+        const int tasks = again ? 2 * n_chunks - h : n_chunks;
         for (int t = 0; t < tasks; ++t, ++q) {
-          const int c = t % n_chunks;
+          // pass A: chunks 0 .. n-1; pass B: chunks n-h-1 .. 0 (the last h
+          // stay in their slots)
+          const int c = (t < n_chunks) ? t : 2 * n_chunks - h - 1 - t;
           const int s = static_cast<int>(q % NS);
           if (q >= NS &&
               !mbar_wait_bounded(smem_u32(&empty[s]), static_cast<uint32_t>(((q / NS) - 1) & 1),
@@ -216,12 +232,12 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
             atomicOr(&ws.hdr->err_bits, kErrTimeout);
             break;
           }
-          const int v0 = c * CV;
-          const uint32_t bytes = static_cast<uint32_t>(min(CV, row_vec - v0)) * 16u;
+          const int v0 = cs(c);
+          const uint32_t bytes = static_cast<uint32_t>(cn(c)) * 16u;
           const uint32_t bar = smem_u32(&full[s]);
           mbar_arrive_expect_tx(bar, bytes);
           bulk_g2s(smem_u32(ring + static_cast<size_t>(s) * CB), src_row + static_cast<size_t>(v0) * 16,
-                   bytes, bar, (kGrad && t < n_chunks) ? pol_a : pol_b);
+                   bytes, bar, (again && t < n_chunks - h) ? pol_a : pol_b);
         }
       }
       // A timeout leaves copies in flight: wait (bounded) for the last one
@@ -275,6 +291,8 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
     const long long row = blockIdx.x + i * gridDim.x;
     const char* grow = lg + row * a.ld * static_cast<long long>(sizeof(St));
     const bool trains = a.mask[row] != 0;
+    // pass B takes the last h chunks from the slots pass A left them in
+    const int h = (kGrad && trains && n_chunks > 0) ? min(a.n_hold, n_chunks) : 0;
 
     int y = 0;
     float rho = 0.0f, q = 0.0f, old = 0.0f, A = 0.0f, zy = 0.0f;
@@ -315,9 +333,9 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
     Run run;
     for (int c = 0; c < n_chunks; ++c) {
       const uint4* sv = wait_slot(q0 + c);
-      const int nv = min(CV, row_vec - c * CV);
-      if (tid == 0 && yv >= c * CV && yv < c * CV + nv) zy = In::load1(sv, y - c * CV * V8);
-      if (topk && warp == 0) topk_gather<In>(tk, sv, c * CV * V8, (c * CV + nv) * V8);
+      const int v0 = cs(c), nv = cn(c);
+      if (tid == 0 && yv >= v0 && yv < v0 + nv) zy = In::load1(sv, y - v0 * V8);
+      if (topk && warp == 0) topk_gather<In>(tk, sv, v0 * V8, (v0 + nv) * V8);
       if (run.r == -INFINITY && tid < nv) run.raise(In::vmax(sv[tid]) * k);
       const Run keep = run;
       bool redo = run.r == -INFINITY;  // no finite reference yet
@@ -348,7 +366,7 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
           }
         }
       }
-      release_slot(q0 + c);
+      if (c < n_chunks - h) release_slot(q0 + c);
     }
     Tri t = run.tri();
     if (topk && warp == 0 && tail0 < a.V)  // candidates past the last whole vector
@@ -444,10 +462,14 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
       const float2 off2 = make_float2(cf.x, cf.x);
       const float2 ca2 = make_float2(cf.y, cf.y), cb2 = make_float2(cf.z, cf.z);
       const bool vec_out = a.out_vec != 0;
-      for (int c = 0; c < n_chunks; ++c) {
-        const long long qq = q0 + n_chunks + c;
-        const int nv = min(CV, row_vec - c * CV);
-        char* dchunk = drow + static_cast<long long>(c) * CV * V8 * Out::kSize;
+      for (int j = 0; j < n_chunks; ++j) {
+        // chunks n-h .. n-1 are still in the slots of tasks q0 + n - h ..
+        // q0 + n - 1 (a wait on a completed phase returns at once); then
+        // tasks q0 + n .. q0 + 2n - h - 1 bring chunks n-h-1 .. 0
+        const int c = (j < h) ? n_chunks - h + j : n_chunks - 1 - j;
+        const long long qq = (j < h) ? q0 + n_chunks - h + j : q0 + n_chunks + (j - h);
+        const int nv = cn(c);
+        char* dchunk = drow + static_cast<long long>(cs(c)) * V8 * Out::kSize;
         if (ci.x) {
           // zero gradient: the chunk's data is not needed; a training row's
           // chunk was still copied, so its slot is waited on and released to
@@ -494,7 +516,7 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
         Out::store1(drow, j, x);
       }
     }
-    q0 += (kGrad && trains) ? 2 * n_chunks : n_chunks;
+    q0 += (kGrad && trains) ? 2 * n_chunks - h : n_chunks;
   }
   cons_sync();
   if (tid == 0 && fix_ptr) Out::store1(fix_ptr, 0, fix_val);
@@ -509,16 +531,16 @@ const void* fn(bool topk) {
 }  // namespace
 
 // Rows with 16-byte aligned starts go to the streaming kernel (one CTA per
-// row, second read served by L2) from 280 KB in a fused call and from 160 KB
-// in a forward-only one; shorter or unaligned rows to the cluster kernel,
-// which keeps them on chip. Measured on GB300 (bf16, fractions of the copy
-// peak): fused, rows of 151,936-154,880 columns (297-310 KB) streamed 0.955
-// against 0.941 in clusters, rows of 81,920-131,072 columns (160-256 KB) in
-// clusters 0.94-0.96 against 0.89-0.94 streamed; forward only, rows of
+// row, second read served by L2 or shared memory) from 192 KB in a fused
+// call and from 160 KB in a forward-only one; shorter or unaligned rows to
+// the cluster kernel, which keeps them on chip. Measured on GB300 (bf16,
+// fractions of the copy peak): fused, rows of 200-310 KB streamed
+// 0.966-0.984 against 0.939-0.959 in clusters, rows of 128-160 KB in
+// clusters 0.94-0.96 against 0.88-0.91 streamed; forward only, rows of
 // 160-310 KB streamed 0.92-1.09 against 0.78-0.88, rows of 96-128 KB in
 // clusters 0.87-0.92 against 0.79. MILESLOSS_SWEEP_KIND=stream|cluster
 // overrides the choice.
-constexpr long long kStreamMinRowBytes = 280 * 1024;     // fused calls
+constexpr long long kStreamMinRowBytes = 192 * 1024;     // fused calls
 constexpr long long kStreamMinRowBytesFwd = 160 * 1024;  // forward-only calls
 
 bool use_stream(long long row_bytes, bool in_bulk, bool grad) {
@@ -528,14 +550,22 @@ bool use_stream(long long row_bytes, bool in_bulk, bool grad) {
   return in_bulk && row_bytes >= (grad ? kStreamMinRowBytes : kStreamMinRowBytesFwd);
 }
 
-// Two 112 KB slots (one CTA per SM): few, large chunks keep the per-chunk
-// handshakes rare (measured best among 16-112 KB chunks with 2-14 slots).
-// Overridable through MILESLOSS_STREAM_CHUNK / MILESLOSS_STREAM_SLOTS.
-rl_status plan_stream(int dev, int extra, StreamPlan* out) {
+// The ring (one CTA per SM), measured on GB300 among 44-112 KB chunks and
+// 0-3 kept chunks (bf16, fused): rows of 240 KB and more run best with three
+// 74 KB slots, the ragged remainder as the first chunk and the last two
+// chunks kept for pass B (0.966-0.984 of the copy peak, against 0.959-0.973
+// with two 112 KB slots); shorter rows with two 112 KB slots and the last
+// chunk kept (200 KB rows: 0.972-0.979, against 0.944 with 74 KB slots). A
+// forward-only call has no pass B: two 112 KB slots. Overridable through
+// MILESLOSS_STREAM_CHUNK / _SLOTS / _HOLD / _SPLIT.
+constexpr long long kLongRowBytes = 240 * 1024;
+
+rl_status plan_stream(int dev, int extra, long long row_bytes, bool grad, StreamPlan* out) {
   int optin = 0;
   if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
     return RL_ERR_CUDA;
-  const int chunk = env_int("MILESLOSS_STREAM_CHUNK", 114688);
+  const bool lng = grad && row_bytes >= kLongRowBytes;
+  const int chunk = env_int("MILESLOSS_STREAM_CHUNK", lng ? 75776 : 114688);
   if (chunk < 1024 || chunk > 131072 || chunk % 128) return RL_ERR_UNSUPPORTED;
   int slots = (optin - kSweepSmemExtra - extra) / chunk;
   if (slots > kMaxSlots) slots = kMaxSlots;
@@ -545,8 +575,12 @@ rl_status plan_stream(int dev, int extra, StreamPlan* out) {
     slots = forced;
   }
   if (slots < 1) return RL_ERR_UNSUPPORTED;
+  const int hold = env_int("MILESLOSS_STREAM_HOLD", lng ? 2 : 1);
+  if (hold < 0 || hold > slots) return RL_ERR_UNSUPPORTED;
   out->chunk = chunk;
   out->slots = slots;
+  out->hold = hold;
+  out->split_first = env_int("MILESLOSS_STREAM_SPLIT", lng ? 1 : 0) != 0;
   out->smem = slots * chunk + kSweepSmemExtra + extra;
   return RL_OK;
 }

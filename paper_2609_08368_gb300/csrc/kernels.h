@@ -49,6 +49,8 @@ struct StreamArgs {
   int V;
   int chunk_bytes;  // bytes per ring slot (multiple of 128)
   int n_slots;      // ring depth
+  int n_hold;       // last chunks of a row that pass B reads from shared memory (<= n_slots)
+  int split_first;  // 1: the first chunk takes the ragged remainder (rounded up to 128 bytes)
   int out_vec;      // dLogits rows are 16-byte aligned: vector stores
   const int* targets;
   const float* rho;
@@ -139,12 +141,13 @@ inline int env_int(const char* name, int dflt) {
 // The streaming kernel's launch plan (defined beside the kernel, k_stream.cu):
 // whether rows of row_bytes go to it, and its ring of shared-memory slots.
 struct StreamPlan {
-  int chunk, slots, smem;
+  int chunk, slots, hold, split_first, smem;
 };
 bool use_stream(long long row_bytes, bool in_bulk, bool grad);
 // extra: shared memory beyond the ring and the fixed scratch (kTopKSmem with
-// top-K OPD on, else 0)
-rl_status plan_stream(int dev, int extra, StreamPlan* out);
+// top-K OPD on, else 0); the ring's shape depends on the row length and on
+// whether the call writes dLogits
+rl_status plan_stream(int dev, int extra, long long row_bytes, bool grad, StreamPlan* out);
 const void* bwd_kernel(rl_dtype in, rl_dtype out);
 const void* adv_kernel();
 const void* groups_kernel();  // one 32-thread block per group (grid-stride)

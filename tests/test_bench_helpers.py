@@ -24,9 +24,11 @@ def test_launches_per_call():
 
 def test_sweep_kernel_name_follows_the_fused_threshold():
     assert bench.sweep_kernel_name(154880, 2).startswith("k_stream")
-    assert bench.sweep_kernel_name(131072, 2).startswith("k_sweep")
+    assert bench.sweep_kernel_name(131072, 2).startswith("k_stream")
+    assert bench.sweep_kernel_name(98304, 2).startswith("k_stream")
+    assert bench.sweep_kernel_name(98303, 2).startswith("k_sweep")
     assert bench.sweep_kernel_name(32768, 4).startswith("k_sweep")
-    assert bench.sweep_kernel_name(80000, 4).startswith("k_stream")
+    assert bench.sweep_kernel_name(49152, 4).startswith("k_stream")
 
 
 def test_profiled_traffic_only_for_its_workload_and_sources():

@@ -41,6 +41,8 @@ def _no_overrides(monkeypatch):
     monkeypatch.delenv("MILESLOSS_SWEEP_KIND", raising=False)
     monkeypatch.delenv("MILESLOSS_STREAM_CHUNK", raising=False)
     monkeypatch.delenv("MILESLOSS_STREAM_SLOTS", raising=False)
+    monkeypatch.delenv("MILESLOSS_STREAM_HOLD", raising=False)
+    monkeypatch.delenv("MILESLOSS_STREAM_SPLIT", raising=False)
 
 
 def _full_check(w, mode="fused", dl_dtype=None, params=None):
@@ -68,12 +70,19 @@ def test_parity_each_sweep_kernel(monkeypatch, kind, name):
     _full_check(wl.make(SHRUNK[name], DEV), mode="split")
 
 
-@pytest.mark.parametrize("chunk,slots", [(16384, 14), (4096, 2), (12288, 3), (1024, 1),
-                                         (65536, 3)])
-def test_stream_ring_shapes(monkeypatch, chunk, slots):
+@pytest.mark.parametrize("chunk,slots,hold,split", [
+    (16384, 14, 1, 0), (16384, 14, 5, 1), (4096, 2, 0, 0), (4096, 2, 2, 1), (12288, 3, 2, 1),
+    (12288, 3, 3, 0), (1024, 1, 1, 1), (1024, 1, 0, 0), (65536, 3, 2, 1), (75776, 3, 2, 1),
+    (8192, 4, 4, 1)])
+def test_stream_ring_shapes(monkeypatch, chunk, slots, hold, split):
+    """The streaming kernel's ring: chunk sizes, slot counts, chunks kept in
+    shared memory for pass B (0 to every slot) and the ragged chunk first or
+    last, on rows of 2 to 88 chunks."""
     monkeypatch.setenv("MILESLOSS_SWEEP_KIND", "stream")
     monkeypatch.setenv("MILESLOSS_STREAM_CHUNK", str(chunk))
     monkeypatch.setenv("MILESLOSS_STREAM_SLOTS", str(slots))
+    monkeypatch.setenv("MILESLOSS_STREAM_HOLD", str(hold))
+    monkeypatch.setenv("MILESLOSS_STREAM_SPLIT", str(split))
     # ragged rows: 45,003 bf16 columns = 5,625 vectors and a 3-element tail
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=24, vocab=45003,
                     rho_noise=0.3)
