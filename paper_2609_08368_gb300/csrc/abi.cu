@@ -489,7 +489,8 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     st = set_smem(fn, dev, sp.smem);
     if (st != RL_OK) return st;
     int ctas = 0;
-    st = resident_clusters(fn, dev, 1, sp.smem, kStreamConsumers + 32, &ctas);
+    const int threads = stream_threads(sc.topk > 0);
+    st = resident_clusters(fn, dev, 1, sp.smem, threads, &ctas);
     if (st != RL_OK) return st;
     StreamArgs ta;
     ta.logits = c.logits;
@@ -516,7 +517,7 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     ta.ws = ws;
     const long long grid = std::min<long long>(ctas, c.R);
     record(t_ev_begin, s);
-    st = launch(fn, dim3(static_cast<unsigned>(grid)), dim3(kStreamConsumers + 32), sp.smem, 1, s,
+    st = launch(fn, dim3(static_cast<unsigned>(grid)), dim3(threads), sp.smem, 1, s,
                 &ta);
     record(t_ev_end, s);
     if (st != RL_OK) return st;

@@ -17,9 +17,11 @@
 // re-reads the most recently copied chunk first. The sixteen consumer warps:
 //   pass A  per chunk, each thread sums its vectors into (S, U) in packed
 //           f32x2 against a running reference that moves by whole powers of
-//           two (no per-element maximum), then releases the slot; warp 0
-//           also takes the row's top-K OPD candidates from the chunk;
+//           two (no per-element maximum), then releases the slot;
 //   merge   butterfly merges, largest reference first, in a fixed order;
+//           with top-K OPD on, warp 0 also takes the row's top-K part from
+//           the top-K warp (one more warp, which gathers the candidates from
+//           the ring slots as pass A's chunks arrive);
 //   epilogue one thread evaluates the per-token objective and the gradient
 //           coefficients;
 //   pass B  per chunk, last to first, dLogits from the chunk, 16-byte streaming
@@ -161,7 +163,7 @@ __device__ __forceinline__ void pass_b_chunk(const uint4* sv, int nv, char* dchu
 }
 
 template <class In, class Out, bool kGrad, bool kTopK>
-__global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const StreamArgs a) {
+__global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_stream(const StreamArgs a) {
   using St = typename In::storage;
   constexpr int V8 = In::kVec;
   constexpr int P = V8 / 2;
@@ -191,13 +193,23 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
   float4* red = reinterpret_cast<float4*>(empty + kMaxSlots);  // [kConsWarps]
   float4* bc = red + kConsWarps;                                // [2]
   int4* bci = reinterpret_cast<int4*>(bc + 2);                  // [1]
+  TopKPart* tkp = reinterpret_cast<TopKPart*>(bci + 1);         // [2] top-K parts by row parity
+  uint64_t* tk_full = reinterpret_cast<uint64_t*>(tkp + 2);     // [2] part written
+  uint64_t* tk_empty = tk_full + 2;                             // [2] part read
+  static_assert(2 * kMaxSlots * 8 + (kConsWarps + 3) * 16 + 2 * sizeof(TopKPart) + 4 * 8 <=
+                    kSweepSmemExtra,
+                "k_stream scratch");
   // [2] top-K candidates of this row and the next (launched with kTopKSmem more)
   TopKBuf* tkb = reinterpret_cast<TopKBuf*>(smem + static_cast<size_t>(NS) * CB + kSweepSmemExtra);
 
   if (tid == 0) {
     for (int s = 0; s < NS; ++s) {
       mbar_init(smem_u32(&full[s]), 1);
-      mbar_init(smem_u32(&empty[s]), kConsWarps);
+      mbar_init(smem_u32(&empty[s]), kConsWarps + (kTopK ? 1 : 0));
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(smem_u32(&tk_full[b]), 1);
+      mbar_init(smem_u32(&tk_empty[b]), 1);
     }
     fence_mbar_init();
   }
@@ -255,6 +267,82 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
     return;
   }
 
+  if (kTopK && warp == kConsWarps + 1) {
+    // ------------------------------------------------------------- top-K OPD
+    // One more warp takes each row's top-K candidate logits from the ring
+    // slots as pass A's chunks arrive (it waits on every task's "full"
+    // barrier and is one more arrival on its "empty" barrier) and computes the
+    // candidates' part of the signal, which needs no row statistics, while the
+    // consumers finish pass A; warp 0 takes the part after the merge. The
+    // parts are double-buffered by row parity, each buffer with a "written"
+    // and a "read" mbarrier (one arrival each), so this warp may run up to a
+    // row ahead. (A named barrier synced by both warps once per row cost
+    // ~1 us per row on GB300: 6.72 against 6.26 ms on 65,536 x 154,880.) The
+    // row's ids and teacher values were copied during the previous row.
+    bool tdead = false;
+    auto twait = [&](long long q) {
+      const int s = static_cast<int>(q % NS);
+      if (!tdead &&
+          !mbar_wait_bounded(smem_u32(&full[s]), static_cast<uint32_t>((q / NS) & 1), kWaitLimitNs)) {
+        tdead = true;
+        atomicOr(&ws.hdr->err_bits, kErrTimeout);
+      }
+      return reinterpret_cast<const uint4*>(ring + static_cast<size_t>(s) * CB);
+    };
+    auto tarrive = [&](long long q) {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&empty[q % NS]));
+    };
+    const int K = a.s.topk;
+    if (rows_mine > 0)
+      topk_prefetch(&tkb[0], a.s.topk_ids + static_cast<long long>(blockIdx.x) * K,
+                    a.s.topk_teacher + static_cast<long long>(blockIdx.x) * K, K, lane);
+    long long q0 = 0;
+    for (long long i = 0; i < rows_mine; ++i) {
+      const long long row = blockIdx.x + i * gridDim.x;
+      const bool trains = a.mask[row] != 0;
+      const int h = (kGrad && trains && n_chunks > 0) ? min(a.n_hold, n_chunks) : 0;
+      const TopKBuf* tk_row = &tkb[i & 1];
+      cp_async_wait_all();
+      TopKLane tk = topk_ids(tk_row, a.V, K, lane);
+      if (i + 1 < rows_mine) {
+        const long long o = (row + gridDim.x) * K;
+        topk_prefetch(&tkb[(i + 1) & 1], a.s.topk_ids + o, a.s.topk_teacher + o, K, lane);
+      }
+      for (int c = 0; c < n_chunks; ++c) {
+        const uint4* sv = twait(q0 + c);
+        const int v0 = cs(c);
+        topk_gather<In>(tk, sv, v0 * V8, (v0 + cn(c)) * V8);
+        tarrive(q0 + c);
+      }
+      if (tail0 < a.V)  // candidates past the last whole vector
+        topk_gather<In>(tk, reinterpret_cast<const St*>(lg + row * a.ld * static_cast<long long>(sizeof(St))) + tail0,
+                        tail0, a.V);
+      const TopKPart p = topk_part(tk, tk_row, lane, a.s.invT, [](int) { return true; });
+      // the part of row i - 2 (same buffer) has been read
+      if (i >= 2 && !tdead &&
+          !mbar_wait_bounded(smem_u32(&tk_empty[i & 1]), static_cast<uint32_t>(((i >> 1) - 1) & 1),
+                             kWaitLimitNs)) {
+        tdead = true;
+        atomicOr(&ws.hdr->err_bits, kErrTimeout);
+      }
+      if (lane == 0) {
+        tkp[i & 1] = p;
+        mbar_arrive(smem_u32(&tk_full[i & 1]));
+      }
+      // pass B's copies: this warp's arrivals keep the slots' counts
+      if (kGrad && trains) {
+        for (int j = h; j < n_chunks; ++j) {
+          const long long qq = q0 + n_chunks + (j - h);
+          twait(qq);
+          tarrive(qq);
+        }
+      }
+      q0 += (kGrad && trains) ? 2 * n_chunks - h : n_chunks;
+    }
+    return;
+  }
+
   // -------------------------------------------------------------- consumers
   const long long N = ws.hdr->n_tokens;
   float g = a.grad_loss;
@@ -281,11 +369,6 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
     if (lane == 0) mbar_arrive(smem_u32(&empty[q % NS]));
   };
 
-  constexpr bool topk = kTopK;  // top-K OPD on (a.s.topk > 0): its own instantiation
-  if (topk && warp == 0 && rows_mine > 0)
-    topk_prefetch(&tkb[0], a.s.topk_ids + static_cast<long long>(blockIdx.x) * a.s.topk,
-                  a.s.topk_teacher + static_cast<long long>(blockIdx.x) * a.s.topk, a.s.topk, lane);
-
   long long q0 = 0;  // task number of the row's first chunk (same count as the producer's)
   for (long long i = 0; i < rows_mine; ++i) {
     const long long row = blockIdx.x + i * gridDim.x;
@@ -309,19 +392,6 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
       if (yok && y >= tail0) zy = In::load1(grow, y);
     }
     const int yv = yok ? y / V8 : -1;  // thread 0 only
-    // top-K OPD candidates (warp 0): this row's ids arrived during the last
-    // row; their logits are taken from the chunks as pass A sweeps them; the
-    // next row's ids and teacher values are copied meanwhile
-    TopKLane tk{-1, -1, 0.0f, 0.0f};
-    const TopKBuf* tk_row = &tkb[i & 1];
-    if (topk && warp == 0) {
-      cp_async_wait_all();
-      tk = topk_ids(tk_row, a.V, a.s.topk, lane);
-      if (i + 1 < rows_mine) {
-        const long long o = (row + gridDim.x) * a.s.topk;
-        topk_prefetch(&tkb[(i + 1) & 1], a.s.topk_ids + o, a.s.topk_teacher + o, a.s.topk, lane);
-      }
-    }
 
     // ---------------- pass A
     // One sweep of each chunk in shared memory against the thread's running
@@ -335,7 +405,6 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
       const uint4* sv = wait_slot(q0 + c);
       const int v0 = cs(c), nv = cn(c);
       if (tid == 0 && yv >= v0 && yv < v0 + nv) zy = In::load1(sv, y - v0 * V8);
-      if (topk && warp == 0) topk_gather<In>(tk, sv, v0 * V8, (v0 + nv) * V8);
       if (run.r == -INFINITY && tid < nv) run.raise(In::vmax(sv[tid]) * k);
       const Run keep = run;
       bool redo = run.r == -INFINITY;  // no finite reference yet
@@ -369,8 +438,6 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
       if (c < n_chunks - h) release_slot(q0 + c);
     }
     Tri t = run.tri();
-    if (topk && warp == 0 && tail0 < a.V)  // candidates past the last whole vector
-      topk_gather<In>(tk, reinterpret_cast<const St*>(grow) + tail0, tail0, a.V);
     for (int j = tail0 + tid; j < a.V; j += kCons) {
       const float z = In::load1(grow, j);
       if (z == -INFINITY) continue;
@@ -402,12 +469,20 @@ __global__ void __launch_bounds__(kStreamConsumers + 32, 1) k_stream(const Strea
       }
       t = warp_merge(x);
     }
-    // top-K OPD signal (Sec. 5.2), a fixed per-token reward; warp 0 holds the
-    // row's statistics and candidates
+    // top-K OPD signal (Sec. 5.2), a fixed per-token reward: the top-K warp's
+    // part of this row and the row's lse (warp 0)
     float opd = 0.0f;
-    if (topk && warp == 0)
-      opd = topk_value(topk_part(tk, tk_row, lane, a.s.invT, [](int) { return true; }),
-                       fmaf(t.m, kLn2f, logf(t.s)));
+    if (kTopK && warp == 0) {
+      if (!dead &&
+          !mbar_wait_bounded(smem_u32(&tk_full[i & 1]), static_cast<uint32_t>((i >> 1) & 1),
+                             kWaitLimitNs)) {
+        dead = true;
+        atomicOr(&ws.hdr->err_bits, kErrTimeout);
+      }
+      opd = topk_value(tkp[i & 1], fmaf(t.m, kLn2f, logf(t.s)));
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&tk_empty[i & 1]));
+    }
 
     // ---------------- epilogue (thread 0)
     char* drow = kGrad ? static_cast<char*>(a.dlogits) +

@@ -14,6 +14,9 @@ constexpr int kSweepSmemExtra = 1024;     // mbarriers + exchange + reduction sc
 constexpr int kAdvThreads = 1024;
 constexpr int kBwdThreads = 256;
 constexpr int kStreamConsumers = 512;     // consumer threads of k_stream (+ one producer warp)
+// k_stream's block: the consumers, the producer warp and, with top-K OPD, the
+// top-K warp
+constexpr int stream_threads(bool topk) { return kStreamConsumers + (topk ? 64 : 32); }
 constexpr int kMaxSlots = 16;             // ring slots of k_stream
 constexpr int kSeqThreads = 256;
 constexpr int kAdvSmemBytes = 48 * 1024;  // on-chip trajectory tables when they fit

@@ -360,6 +360,27 @@ def test_opd_topk_long_rows(monkeypatch, kind, cluster, K):
     _full_check(w, mode="split", params=params)
 
 
+@pytest.mark.parametrize("vocab,ring", [
+    (45003, (4096, 2, 1, 0)), (45003, (4096, 3, 2, 1)), (45003, (1024, 1, 0, 0)),
+    (45003, (16384, 4, 4, 1)), (45003, (75776, 3, 2, 1)), (131072, None)])
+def test_opd_topk_stream_ring_shapes(monkeypatch, vocab, ring):
+    """Top-K OPD in the streaming kernel, whose top-K warp waits on and
+    releases every ring slot and hands each row's part to warp 0: chunk
+    sizes, slot counts, kept chunks and both splits (rows of 1 to 88 chunks,
+    a ragged tail past the last whole vector), and the default plan of
+    256 KB rows (three 74 KB slots, two kept)."""
+    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", "stream")
+    if ring:
+        for name, v in zip(("CHUNK", "SLOTS", "HOLD", "SPLIT"), ring):
+            monkeypatch.setenv("MILESLOSS_STREAM_" + name, str(v))
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=16, vocab=vocab,
+                    rho_noise=0.3, ref_noise=0.2, topk=16, topk_noise=0.4)
+    w = wl.make(rec, DEV)
+    params = dict(w.params, opd_coef=0.5, opd_topk=16)
+    _full_check(w, params=params)
+    _full_check(w, mode="split", params=params)
+
+
 @pytest.mark.parametrize("kind", ["cluster", "stream"])
 def test_no_training_tokens_and_empty_call(monkeypatch, kind):
     monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
