@@ -495,8 +495,9 @@ __device__ __forceinline__ TokenTerms token_terms(float logp, float H, float rho
 //   sum_k w_k (z_k / T - teacher_k) / sum_k w_k  -  lse,
 // so partial sums over any subset of the candidates can be formed before lse
 // is known and merged like the row statistics (a largest term, then sums
-// rescaled to it): TopKPart below, with zmax the largest z_k / T of the part,
-// sw = sum exp(z_k / T - zmax) and acc = sum exp(z_k / T - zmax)(z_k / T - teacher_k).
+// rescaled to it): TopKPart below, with m the largest z_k k of the part (log2
+// units, k = log2(e) / T, as the row statistics), sw = sum 2^(z_k k - m) and
+// acc = sum 2^(z_k k - m)(z_k / T - teacher_k).
 //
 // One warp holds a row's candidates (K <= 64: lane l has candidates l and
 // l + 32). Their ids and teacher log-probs are copied into shared memory one
@@ -514,7 +515,7 @@ struct TopKLane {
 };
 
 struct TopKPart {
-  float zmax, sw, acc;
+  float m, sw, acc;
 };
 
 __device__ __forceinline__ void cp_async4(void* dst, const void* src) {
@@ -563,29 +564,40 @@ __device__ __forceinline__ void topk_gather(TopKLane& c, const void* src, int c0
   if (c.id1 >= c0 && c.id1 < c1) c.z1 = In::load1(src, c.id1 - c0);
 }
 
-__device__ __forceinline__ TopKPart topk_merge(TopKPart a, TopKPart b) {
-  const float M = fmaxf(a.zmax, b.zmax);
-  if (M == -INFINITY) return TopKPart{-INFINITY, 0.0f, 0.0f};
-  const float fa = a.sw > 0.0f ? expf(a.zmax - M) : 0.0f;
-  const float fb = b.sw > 0.0f ? expf(b.zmax - M) : 0.0f;
-  return TopKPart{M, fa * a.sw + fb * b.sw, fa * a.acc + fb * b.acc};
+// The parts of a row's CTAs (x = m, y = sw, z = acc), merged in rank order:
+// the largest reference first, then every part rescaled to it (independent
+// exponentials, no chain through the parts).
+__device__ __forceinline__ TopKPart topk_merge_all(const float4* parts, int n) {
+  float M = -INFINITY;
+  for (int r = 0; r < n; ++r) M = fmaxf(M, parts[r].x);
+  TopKPart p{M, 0.0f, 0.0f};
+  if (M == -INFINITY) return p;
+  for (int r = 0; r < n; ++r) {
+    const float4 e = parts[r];
+    if (e.y > 0.0f) {
+      const float f = ex2(e.x - M);
+      p.sw = fmaf(f, e.y, p.sw);
+      p.acc = fmaf(f, e.z, p.acc);
+    }
+  }
+  return p;
 }
 
 // The warp's part over its lanes' candidates whose ids satisfy `mine`
-// (fixed-order butterfly; every lane ends with it).
+// (fixed-order butterfly; every lane ends with it); k = log2(e) / T.
 template <class Mine>
 __device__ __forceinline__ TopKPart topk_part(const TopKLane& c, const TopKBuf* buf, int lane,
-                                              float invT, Mine mine) {
+                                              float invT, float k, Mine mine) {
   const bool u0 = c.id0 >= 0 && mine(c.id0), u1 = c.id1 >= 0 && mine(c.id1);
-  const float s0 = c.z0 * invT, s1 = c.z1 * invT;
-  float M = fmaxf(u0 ? s0 : -INFINITY, u1 ? s1 : -INFINITY);
+  const float t0 = c.z0 * k, t1 = c.z1 * k;
+  float M = fmaxf(u0 ? t0 : -INFINITY, u1 ? t1 : -INFINITY);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
   if (M == -INFINITY) return TopKPart{-INFINITY, 0.0f, 0.0f};
-  const float w0 = u0 ? expf(s0 - M) : 0.0f, w1 = u1 ? expf(s1 - M) : 0.0f;
+  const float w0 = u0 ? ex2(t0 - M) : 0.0f, w1 = u1 ? ex2(t1 - M) : 0.0f;
   float sw = w0 + w1;
-  float acc = (u0 ? w0 * (s0 - buf->teacher[lane]) : 0.0f) +
-              (u1 ? w1 * (s1 - buf->teacher[lane + 32]) : 0.0f);
+  float acc = (u0 ? w0 * fmaf(c.z0, invT, -buf->teacher[lane]) : 0.0f) +
+              (u1 ? w1 * fmaf(c.z1, invT, -buf->teacher[lane + 32]) : 0.0f);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     sw += __shfl_xor_sync(0xffffffffu, sw, o);
@@ -594,8 +606,10 @@ __device__ __forceinline__ TopKPart topk_part(const TopKLane& c, const TopKBuf* 
   return TopKPart{M, sw, acc};
 }
 
+// sw >= 1 (the largest candidate contributes 1), so a fast division is exact
+// enough
 __device__ __forceinline__ float topk_value(const TopKPart& p, float lse) {
-  return p.sw > 0.0f ? p.acc / p.sw - lse : 0.0f;
+  return p.sw > 0.0f ? __fdividef(p.acc, p.sw) - lse : 0.0f;
 }
 
 }  // namespace milesloss

@@ -318,7 +318,7 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
       if (tail0 < a.V)  // candidates past the last whole vector
         topk_gather<In>(tk, reinterpret_cast<const St*>(lg + row * a.ld * static_cast<long long>(sizeof(St))) + tail0,
                         tail0, a.V);
-      const TopKPart p = topk_part(tk, tk_row, lane, a.s.invT, [](int) { return true; });
+      const TopKPart p = topk_part(tk, tk_row, lane, a.s.invT, k, [](int) { return true; });
       // the part of row i - 2 (same buffer) has been read
       if (i >= 2 && !tdead &&
           !mbar_wait_bounded(smem_u32(&tk_empty[i & 1]), static_cast<uint32_t>(((i >> 1) - 1) & 1),

@@ -321,7 +321,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
       topk_gather<In>(tk, sb, lo, lo + vec_elems);
       topk_gather<In>(tk, grow + static_cast<size_t>(vec_elems) * sizeof(St), lo + vec_elems, lo + cnt);
       const int c0 = lo, c1 = lo + cnt;
-      tkp = topk_part(tk, tk_row, tid, a.s.invT, [c0, c1](int id) { return id >= c0 && id < c1; });
+      tkp = topk_part(tk, tk_row, tid, a.s.invT, k, [c0, c1](int id) { return id >= c0 && id < c1; });
     }
     t = block_merge<kWarps>(t, red);
 
@@ -338,7 +338,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
       }
       const int slot = static_cast<int>(it & 1);
       const float4 mine = make_float4(t.m, t.s, t.u, zy);
-      const float4 mine_tk = make_float4(tkp.zmax, tkp.sw, tkp.acc, 0.0f);
+      const float4 mine_tk = make_float4(tkp.m, tkp.sw, tkp.acc, 0.0f);
       zy_all = zy;
       if (C > 1) {
         float4* xs = xch + slot * 2 * kMaxCluster;
@@ -369,10 +369,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
           }
           if (r == owner) zy_all = e.w;
         }
-        if (topk) {  // the CTAs' top-K parts, merged in rank order
-          tkp = TopKPart{-INFINITY, 0.0f, 0.0f};
-          for (int r = 0; r < C; ++r) tkp = topk_merge(tkp, TopKPart{xt[r].x, xt[r].y, xt[r].z});
-        }
+        if (topk) tkp = topk_merge_all(xt, C);  // the CTAs' top-K parts
       }
     }
     if (tid == 0) {
