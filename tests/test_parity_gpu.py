@@ -243,6 +243,33 @@ def test_long_rows_padded_and_misaligned(monkeypatch, kind, ld, ld_out):
             assert torch.isnan(g["dlogits_t"][:, w.vocab:]).all()
 
 
+@pytest.mark.parametrize("logits,vocab,ld,dl_dtype,ld_out", [
+    ("bf16", 140003, 140008, torch.bfloat16, 140008),
+    ("bf16", 140003, 140008, torch.float32, 140011),
+    ("bf16", 131075, 131080, torch.float32, 131076),
+    ("f32", 65541, 65544, torch.bfloat16, 65544),
+    ("f32", 65541, 65544, torch.float32, 65547)])
+def test_long_row_plan_shapes(logits, vocab, ld, dl_dtype, ld_out):
+    """The streaming kernel's plan for rows of 240 KB and more (three 74 KB
+    slots, the ragged remainder first, two chunks kept for pass B), chosen by
+    the library for 16-byte aligned rows: vector counts that are not a
+    multiple of 8 (the last chunk a few vectors short of a slot), elements
+    past the last whole vector, bf16 and fp32 logits and dLogits, and
+    dLogits strides that are 16-byte aligned (vector stores) or not (scalar
+    stores); fused and split."""
+    base = wl.RECIPES["glm" if logits == "bf16" else "fp32"]
+    rec = wl.shrink(base, n_prompts=1, group_size=4, traj_len=6, vocab=vocab, rho_noise=0.3)
+    w = wl.make(rec, DEV, ld=ld)
+    for mode in ("fused", "split"):
+        g = P.run_gpu(w, mode=mode, dl_dtype=dl_dtype, ld_out=ld_out)
+        assert g["err"] == 0, ml.status_string(g["err"])
+        o = P.run_oracle(w)
+        P.compare_forward(w, g, o)
+        P.assert_dlogits_close(g["dlogits_t"][:, :vocab].float().cpu().numpy(), o["dlogits"])
+        if ld_out > vocab:
+            assert torch.isnan(g["dlogits_t"][:, vocab:]).all()
+
+
 @pytest.mark.parametrize("estimator", ["grpo", "reinforcepp", "gspo"])
 @pytest.mark.parametrize("n_prompts", [8, 1200])
 def test_ragged_and_empty_trajectories(estimator, n_prompts):
