@@ -60,6 +60,9 @@ def parse_args():
                     choices=["grpo", "reinforcepp", "reinforcepp_baseline", "gspo"],
                     help="another advantage estimator than the workload's (for profiling "
                          "the kernels of that path)")
+    ap.add_argument("--opd-topk", type=int, default=0,
+                    help="top-K on-policy distillation with K candidates per row, coefficient "
+                         "0.5 (for profiling the sweeps' top-K instantiations)")
     return ap.parse_args()
 
 
@@ -222,13 +225,15 @@ def launches_per_call(params: dict, n_groups: int) -> int:
 def algorithmic_bytes_per_row(w, dl_dtype) -> int:
     """Logits read once + dLogits written once + the per-row inputs and
     outputs (target, rollout log-prob, optional ref / old / teacher
-    log-probs, mask byte, log-prob and entropy out)."""
+    log-probs, mask byte, log-prob and entropy out, top-K OPD candidates)."""
     es_in = w.logits.element_size()
     es_out = torch.tensor([], dtype=dl_dtype).element_size()
     small = 4 + 4 + 1 + 4 + 4
     for t in (w.ref_logprobs, w.old_logprobs, w.teacher_logprobs):
         if t is not None:
             small += 4
+    if w.topk_ids is not None:  # top-K OPD: candidate ids and teacher log-probs
+        small += 8 * int(w.topk_ids.shape[1])
     return w.vocab * (es_in + es_out) + small
 
 
@@ -409,6 +414,9 @@ def run_ours(args, rank, world, local):
                     seed=rec.seed + 1000 * rank)  # each replica has its own batch
     if args.estimator:
         rec = dataclasses.replace(rec, params=dict(rec.params, estimator=args.estimator))
+    if args.opd_topk:
+        rec = dataclasses.replace(rec, topk=args.opd_topk,
+                                  params=dict(rec.params, opd_topk=args.opd_topk, opd_coef=0.5))
     w = wl.make(rec, dev)
     R, V = w.n_rows, w.vocab
     dl_dtype = w.logits.dtype
@@ -489,9 +497,10 @@ def run_ours(args, rank, world, local):
     step_gbs = launch_bytes / (ms_step / 1e3) / 1e9
 
     cpu = None
-    # (the sampled-row oracle timing covers the token-level estimators only)
+    # (the sampled-row oracle timing covers the token-level estimators
+    # without top-K OPD only)
     if rank == 0 and world == 1 and not args.no_cpu_baseline and \
-            w.params.get("estimator", "grpo") != "gspo":
+            w.params.get("estimator", "grpo") != "gspo" and not args.opd_topk:
         pool = OraclePool()
         try:
             rps, secs, n, cores = oracle_sample(w, args.cpu_sample_rows, pool=pool)
@@ -528,7 +537,9 @@ def run_ours(args, rank, world, local):
                "h2d_bytes_per_step": call.bytes_in(), "d2h_bytes_per_step": call.bytes_out()}
         del call, host_w
 
-    traffic = profiled_traffic(R, args.workload, V)
+    # the committed capture is of the default path (GRPO-style fused sweep,
+    # no top-K): it does not describe the others
+    traffic = None if (args.estimator or args.opd_topk) else profiled_traffic(R, args.workload, V)
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True,
@@ -538,6 +549,8 @@ def run_ours(args, rank, world, local):
                                f"{dt_name} logits "
                                f"-> dLogits",
                    "rows": R, "vocab": V, "parallelism": f"replicas x{world}",
+                   **({"estimator": args.estimator} if args.estimator else {}),
+                   **({"opd_topk": args.opd_topk} if args.opd_topk else {}),
                    "l2": "inputs larger than L2 (20+ GB per step), no flush"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,

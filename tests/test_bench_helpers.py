@@ -2,6 +2,7 @@
 per call, the sweep-kernel naming rule, the profiled traffic's validity checks,
 the algorithmic bytes per row, and the top-K parameter attachment."""
 
+import dataclasses
 import os
 import sys
 
@@ -46,6 +47,10 @@ def test_algorithmic_bytes_per_row():
     # bf16 in and out, plus target, rollout, ref log-prob, mask, logp and H out
     assert bench.algorithmic_bytes_per_row(w, torch.bfloat16) == 1000 * 4 + 4 + 4 + 4 + 1 + 4 + 4
     assert bench.algorithmic_bytes_per_row(w, torch.float32) == 1000 * 6 + 21
+    # top-K OPD adds each row's K candidate ids and teacher log-probs
+    rec = dataclasses.replace(rec, topk=4, params=dict(rec.params, opd_topk=4, opd_coef=0.5))
+    w = wl.make(rec, "cpu")
+    assert bench.algorithmic_bytes_per_row(w, torch.bfloat16) == 1000 * 4 + 21 + 4 * 8
 
 
 def test_api_attaches_top_k_inputs():
