@@ -46,6 +46,48 @@ MUTANTS = [
     ("entropy bonus sign", "ell = pg + p.kl_coef * k3 - p.entropy_coef * H",
      "ell = pg + p.kl_coef * k3 + p.entropy_coef * H"),
     ("ratio inverted", "r = np.exp(logp - base)", "r = np.exp(base - logp)"),
+    ("lse drops its max", "lse = m[:, 0] + np.log(np.exp(s - m).sum(axis=1))",
+     "lse = np.log(np.exp(s - m).sum(axis=1))"),
+    ("temperature ignored in the log-softmax", "s = _widen(z) / float(temperature)\n    m = s.max",
+     "s = _widen(z)\n    m = s.max"),
+    ("first row of each trajectory without advantage", "A_row[cu[i]:cu[i + 1]] = A_traj[i]",
+     "A_row[cu[i] + 1:cu[i + 1]] = A_traj[i]"),
+    ("token mean over all rows", "return float(np.asarray(ell, np.float64)[m].sum() / N), N",
+     "return float(np.asarray(ell, np.float64)[m].sum() / m.size), N"),
+    ("ratio deviation metric without the absolute value",
+     "ratio_absdev_mean=float(np.abs(r - 1.0).sum() / N)", "ratio_absdev_mean=float((r - 1.0).sum() / N)"),
+    ("TIS lower clamp dropped", "wt = np.minimum(np.maximum(rc, p.corr_lo), p.corr_hi)",
+     "wt = np.minimum(rc, p.corr_hi)"),
+    ("clip_hi tests eps_lo", "clip_hi = clipped & (r > 1.0 + p.eps_hi)",
+     "clip_hi = clipped & (r > 1.0 + p.eps_lo)"),
+    ("clip_lo tests eps_hi", "clip_lo = clipped & (r < 1.0 - p.eps_lo)",
+     "clip_lo = clipped & (r < 1.0 - p.eps_hi)"),
+    ("clip interval with the eps swapped", "np.clip(r, 1.0 - p.eps_lo, 1.0 + p.eps_hi)",
+     "np.clip(r, 1.0 - p.eps_hi, 1.0 + p.eps_lo)"),
+    ("KL gradient subtracted", "G = g_pg + p.kl_coef * g_kl", "G = g_pg - p.kl_coef * g_kl"),
+    ("top-K log-probs miss the lse", "lps = s[rows, ids] - np.asarray(lse, np.float64)[:, None]",
+     "lps = s[rows, ids]"),
+    ("GSPO ratio over masked tokens too",
+     "s_i = float(np.exp((logp[rows][mm] - base[rows][mm]).sum() / n_i[i]))",
+     "s_i = float(np.exp((logp[rows] - base[rows]).sum() / n_i[i]))"),
+    ("GSPO share without 1/n_i", "scale = N / (n_seq * n_i[i])", "scale = N / n_seq"),
+    ("GSPO clip_hi tests eps_lo", "clip_hi[rows] = clipped and s_i > 1.0 + p.eps_hi",
+     "clip_hi[rows] = clipped and s_i > 1.0 + p.eps_lo"),
+    ("GSPO dual clip for A > 0",
+     "        if p.dual_clip_c > 0.0 and A < 0.0:\n            d = -A * p.dual_clip_c\n            if d < pgi:",
+     "        if p.dual_clip_c > 0.0 and A > 0.0:\n            d = -A * p.dual_clip_c\n            if d < pgi:"),
+    ("dLogits entropy term subtracted", "+ entropy_coef * ent)", "- entropy_coef * ent)"),
+    ("dual clip for A > 0", "dual = (A < 0.0) & (d < pg)", "dual = (A > 0.0) & (d < pg)"),
+    ("REINFORCE++ std over all rows",
+     "sigma = float(np.sqrt(((b_row[m] - mu) ** 2).sum() / (N - ddof))) if N > ddof else 0.0",
+     "sigma = float(np.sqrt(((b_row - mu) ** 2).sum() / (N - ddof))) if N > ddof else 0.0"),
+    ("clip-or-pop lower bound exclusive", "outside = (rc < p.corr_lo) | (rc > p.corr_hi)",
+     "outside = (rc <= p.corr_lo) | (rc > p.corr_hi)"),
+    ("entropy from unnormalised probabilities", "    p = np.exp(logp_all)\n", "    p = np.exp(s - m)\n"),
+    ("ratio minimum over masked rows too", "ratio_min=float(r.min()),", "ratio_min=float(obj['r'].min()),"),
+    ("divergence metric signed",
+     "logprob_absdiff_mean=float(np.abs(np.asarray(logp, np.float64)[m]",
+     "logprob_absdiff_mean=float((np.asarray(logp, np.float64)[m]"),
 ]
 
 
@@ -76,7 +118,7 @@ def test_every_planted_mistake_fails_the_pins(tmp_path):
     for name, a, _ in MUTANTS:  # (a site found more than once is mutated at its first)
         assert a in orig, f"mutation site not found: {name}"
     jobs = [("unmutated", orig)] + [(name, orig.replace(a, b, 1)) for name, a, b in MUTANTS]
-    with ThreadPoolExecutor(max_workers=min(8, os.cpu_count() or 1)) as ex:
+    with ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1)) as ex:
         passed = list(ex.map(lambda j: _pins_pass(str(tmp_path / f"m{j[0]}"), j[1]),
                              enumerate(s for _, s in jobs)))
     assert passed[0], "the unmutated copy must pass its pins"

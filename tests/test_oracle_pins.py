@@ -198,8 +198,11 @@ def test_row_advantages_and_opd_shaping():
 
 # ---------------------------------------------------------------- objective
 
-def test_ppo_tokens_golden():
-    c = _golden()["ppo_tokens"]
+@pytest.mark.parametrize("name", ["ppo_tokens", "ppo_tokens_asymmetric_lo", "ppo_tokens_asymmetric_hi"])
+def test_ppo_tokens_golden(name):
+    """Hand-derived PPO tokens: symmetric clip with dual clip, and both
+    asymmetric intervals (each bound and each flag tied to its own eps)."""
+    c = _golden()[name]
     A = np.array([_ev(v) for v in c["A"]])
     logp = np.array([_ev(v) for v in c["log_r"]])
     o = oracle.token_objective(logp, np.zeros_like(logp), None, A, np.zeros_like(A),
@@ -293,6 +296,49 @@ def test_corrections_tis_and_clip_or_pop():
     np.testing.assert_allclose(pop["G"], pop["wt"] * base["G"], rtol=1e-15)
     with pytest.raises(ValueError):
         oracle.token_objective(logp, rho, None, A, np.zeros(5), LossParams(correction="tis"))
+
+
+def test_tis_lower_clamp_golden():
+    c = _golden()["tis_lower_clamp"]
+    old = np.array([math.log(_ev(c["rc"]))])
+    o = oracle.token_objective(old.copy(), np.zeros(1), None, np.ones(1), np.zeros(1),
+                               LossParams(**c["params"]), old=old)
+    for k in ("wt", "pg", "G"):
+        assert abs(o[k][0] - _ev(c["expect"][k])) < 1e-15, k
+    assert int(o["corr_clip"][0]) == c["expect"]["corr_clip"]
+
+
+def test_clip_or_pop_bounds_are_inclusive():
+    """A correction ratio exactly at either bound keeps its weight; the next
+    double outside pops the token (weight 0)."""
+    for lo, hi in ((0.5, 2.0), (0.8, 1.25)):
+        for bound in (lo, hi):
+            d, t, up, dn = _threshold_probe(bound)
+            assert float(np.exp(np.float64(d))) == t  # the double the oracle forms from d
+            outer = dn if bound == lo else up
+            p = LossParams(correction="clip_or_pop", corr_lo=t if bound == lo else lo,
+                           corr_hi=t if bound == hi else hi)
+            old = np.array([d, outer])
+            o = oracle.token_objective(old.copy(), np.zeros(2), None, np.ones(2), np.zeros(2), p,
+                                       old=old)
+            assert o["wt"][0] == t and o["corr_clip"][0] == 0
+            assert o["wt"][1] == 0.0 and o["corr_clip"][1] == 1
+
+
+def test_metrics_golden():
+    """The reported metrics are means, minima and maxima over the tokens that
+    train, of absolute deviations where the definition says so."""
+    c = _golden()["metrics_over_training_tokens"]
+    lr = np.array([_ev(v) for v in c["log_r"]])
+    logp = np.array([-0.5, -1.0, -2.0])
+    rho = logp - lr
+    H = np.array([_ev(v) for v in c["H"]])
+    mask = np.array(c["mask"])
+    p = LossParams(entropy_coef=c["entropy_coef"])
+    obj = oracle.token_objective(logp, rho, None, np.zeros(3), H, p)
+    st = oracle.loss_stats(obj, logp, rho, H, mask)
+    for k, v in c["expect"].items():
+        assert abs(st[k] - _ev(v)) < 1e-14, (k, st[k])
 
 
 def test_masked_mean_edge_cases():
@@ -495,6 +541,21 @@ def test_gspo_golden():
     assert abs(L - _ev(c["expect"]["loss"])) < 1e-14
     np.testing.assert_allclose(o["G"], [_ev(v) for v in c["expect"]["G"]], atol=1e-14)
     np.testing.assert_allclose(o["r"], _ev(c["expect"]["r"]), atol=1e-15)
+
+
+def test_gspo_asymmetric_clip_golden():
+    c = _golden()["gspo_asymmetric_clip"]
+    lr = np.array([_ev(v) for v in c["log_ratio"]])
+    logp = np.array([-1.0, -2.0])
+    rho = logp - lr
+    o = oracle.sequence_objective(logp, rho, None, np.array([_ev(c["A"])]), np.zeros(2),
+                                  np.array([0, 2]), np.array([1, 1]), LossParams(**c["params"]))
+    L, _ = oracle.masked_token_mean(o["ell"], np.array([1, 1]))
+    assert abs(L - _ev(c["expect"]["loss"])) < 1e-14
+    np.testing.assert_allclose(o["G"], [_ev(v) for v in c["expect"]["G"]], atol=1e-14)
+    np.testing.assert_allclose(o["r"], _ev(c["expect"]["r"]), atol=1e-14)
+    for k in ("clip_hi", "clip_lo"):
+        assert o[k].astype(int).tolist() == c["expect"][k]
 
 
 def test_gspo_on_one_token_trajectories_is_token_ppo():
