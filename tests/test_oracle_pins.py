@@ -341,6 +341,23 @@ def test_metrics_golden():
         assert abs(st[k] - _ev(v)) < 1e-14, (k, st[k])
 
 
+def test_metrics_with_correction_kl_clip_golden():
+    """Counts and means over the training tokens, with a masked row that would
+    be clipped, corrected and carry KL."""
+    c = _golden()["metrics_with_correction_kl_clip"]
+    logp = np.full(3, -1.0)
+    old = logp - np.array([_ev(v) for v in c["log_r"]])
+    rho = old - np.array([_ev(v) for v in c["log_rc"]])
+    q = logp + np.array([_ev(v) for v in c["delta"]])
+    A = np.array([_ev(v) for v in c["A"]])
+    mask = np.array(c["mask"])
+    H = np.zeros(3)
+    obj = oracle.token_objective(logp, rho, q, A, H, LossParams(**c["params"]), old=old)
+    st = oracle.loss_stats(obj, logp, rho, H, mask)
+    for k, v in c["expect"].items():
+        assert abs(st[k] - _ev(v)) < 1e-14, (k, st[k])
+
+
 def test_masked_mean_edge_cases():
     assert oracle.masked_token_mean(np.array([1.0, 2.0]), np.array([0, 0])) == (0.0, 0)
     L, N = oracle.masked_token_mean(np.array([1.0, 2.0, 4.0]), np.array([1, 0, 1]))
@@ -556,6 +573,20 @@ def test_gspo_asymmetric_clip_golden():
     np.testing.assert_allclose(o["r"], _ev(c["expect"]["r"]), atol=1e-14)
     for k in ("clip_hi", "clip_lo"):
         assert o[k].astype(int).tolist() == c["expect"][k]
+
+
+def test_gspo_with_an_untrained_trajectory_golden():
+    c = _golden()["gspo_with_an_untrained_trajectory"]
+    lr = np.array([_ev(v) for v in c["log_ratio"]])
+    logp = np.array([-1.0, -2.0, -0.5])
+    rho = logp - lr
+    mask = np.array(c["mask"])
+    o = oracle.sequence_objective(logp, rho, None, np.array([_ev(v) for v in c["A"]]), np.zeros(3),
+                                  np.array(c["cu"]), mask, LossParams(estimator="gspo"))
+    L, _ = oracle.masked_token_mean(o["ell"], mask)
+    assert abs(L - _ev(c["expect"]["loss"])) < 1e-14
+    np.testing.assert_allclose(o["G"], [_ev(v) for v in c["expect"]["G"]], atol=1e-14)
+    np.testing.assert_allclose(o["r"], [_ev(v) for v in c["expect"]["r"]], atol=1e-14)
 
 
 def test_gspo_on_one_token_trajectories_is_token_ppo():
