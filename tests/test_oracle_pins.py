@@ -378,6 +378,52 @@ def test_full_pipeline_golden(name):
     np.testing.assert_allclose(out["dlogits"], want, atol=1e-14, rtol=0)
 
 
+def _call_inputs(c):
+    z = np.array([[_ev(v) for v in row] for row in c["z"]])
+    return (z, np.array(c["y"]), np.array([_ev(v) for v in c["rho"]]),
+            np.array([_ev(v) for v in c["w"]]), np.array(c["gid"]), np.array(c["cu"]),
+            c["n_groups"], np.array(c["mask"]))
+
+
+def test_full_call_kl_opd_golden():
+    """The whole call wires the KL reference and the one-sample OPD teacher
+    into the advantages, the objective and dLogits."""
+    c = _golden()["full_call_kl_opd"]
+    z, y, rho, w, gid, cu, n_groups, mask = _call_inputs(c)
+    q = rho + np.array([_ev(v) for v in c["delta"]])  # rho = logp here
+    out = oracle.rl_loss(z, y, rho, q, w, gid, cu, n_groups, mask, LossParams(**c["params"]),
+                         teacher=np.array([_ev(v) for v in c["teacher"]]))
+    e = c["expect"]
+    np.testing.assert_allclose(out["A_row"], [_ev(v) for v in e["A_row"]], atol=1e-14, rtol=0)
+    np.testing.assert_allclose(out["G"], [_ev(v) for v in e["G"]], atol=1e-14, rtol=0)
+    assert abs(out["loss"] - _ev(e["loss"])) < 1e-14
+    want = np.array([[_ev(v) for v in row] for row in e["dlogits"]])
+    np.testing.assert_allclose(out["dlogits"], want, atol=1e-14, rtol=0)
+
+
+def test_full_call_topk_opd_golden():
+    """The whole call shapes the advantages with the top-K signal of each
+    row's own statistics (one row per chunk)."""
+    c = _golden()["full_call_topk_opd"]
+    z, y, rho, w, gid, cu, n_groups, mask = _call_inputs(c)
+    ids = np.array(c["topk_ids"])
+    tt = np.array([[_ev(v) for v in row] for row in c["topk_teacher"]])
+    out = oracle.rl_loss(z, y, rho, None, w, gid, cu, n_groups, mask, LossParams(**c["params"]),
+                         chunk=1, topk_ids=ids, topk_teacher=tt)
+    np.testing.assert_allclose(out["A_row"], [_ev(v) for v in c["expect"]["A_row"]], atol=1e-14,
+                               rtol=0)
+    assert abs(out["loss"] - _ev(c["expect"]["loss"])) < 1e-14
+
+
+def test_full_call_gspo_golden():
+    """The whole call gives GSPO each trajectory's advantage."""
+    c = _golden()["full_call_gspo_two_row_trajectories"]
+    z, y, rho, w, gid, cu, n_groups, mask = _call_inputs(c)
+    out = oracle.rl_loss(z, y, rho, None, w, gid, cu, n_groups, mask, LossParams(**c["params"]))
+    np.testing.assert_allclose(out["G"], [_ev(v) for v in c["expect"]["G"]], atol=1e-14, rtol=0)
+    assert abs(out["loss"] - _ev(c["expect"]["loss"])) < 1e-14
+
+
 def test_cross_entropy_special_case():
     """A = 1, rho = logp, beta = gamma = 0, T = 1, all tokens train: r = 1,
     L = -1 and dZ = (p - onehot)/N, the gradient of the mean cross-entropy."""
