@@ -238,9 +238,13 @@ def opd_topk_estimate(z_rows, temperature, lse, cand_ids, teacher_lp):
     set, of log pi_student - log pi_teacher, weighted by the student's
     probabilities renormalised over the set (the reverse KL restricted to
     the set). The student's log-probs are the trainer's, from the logits;
-    the estimate is a fixed per-token signal (no gradient flows through it)."""
+    the estimate is a fixed per-token signal (no gradient flows through it).
+    A candidate id outside [0, V) is an input error (raised, never wrapped
+    around to another column)."""
     s = _widen(z_rows) / float(temperature)
     ids = np.asarray(cand_ids, np.int64)
+    if ids.size and (ids.min() < 0 or ids.max() >= s.shape[1]):
+        raise ValueError("top-K candidate id outside [0, vocab)")
     rows = np.arange(s.shape[0])[:, None]
     lps = s[rows, ids] - np.asarray(lse, np.float64)[:, None]
     ps = np.exp(lps)

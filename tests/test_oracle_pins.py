@@ -593,6 +593,12 @@ def test_opd_topk_estimate_pins():
     c = rng.integers(0, V, size=(R, 1))
     est1 = oracle.opd_topk_estimate(z, T, lse, c, log_t[np.arange(R)[:, None], c])
     np.testing.assert_allclose(est1, (log_s.numpy() - log_t)[np.arange(R), c[:, 0]], atol=1e-12)
+    # a candidate outside [0, V) is rejected, not wrapped to another column
+    for bad in (-1, V):
+        ids_bad = ids.copy()
+        ids_bad[2, 4] = bad
+        with pytest.raises(ValueError):
+            oracle.opd_topk_estimate(z, T, lse, ids_bad, log_t)
 
 
 def test_gspo_golden():
