@@ -18,6 +18,7 @@ from .rl_loss_ref import (  # noqa: F401
     training_tokens_per_trajectory,
     opd_topk_estimate,
     sequence_objective,
+    correction_ratio,
     token_objective,
     masked_token_mean,
     loss_stats,

@@ -14,8 +14,10 @@ What the paper fixes (Miles v0.1, arxiv 2609.08368):
     prompt, i.e. rewards are centred within their group                (Sec. 2, Sec. 9.1)
   * a group whose attempts all got the same reward carries no signal  (Sec. 2.2, Table 2)
   * tokens the model did not generate are loss-masked                 (Sec. 2.4)
-  * truncated importance sampling (TIS): clamp the ratio to an interval,
-    default [0, 2], and use it as a per-token weight on the PG loss;
+  * truncated importance sampling (TIS): clamp the ratio
+    exp(log pi_train - log pi_rollout) to an interval, default [0, 2], and
+    use it as a per-token weight on the PG loss (log pi_train: given old
+    log-probs, or the trainer's own log-prob of this pass, held constant);
     clip-or-pop: weight 0 outside the interval, the unclipped ratio inside;
     reported metrics: pre-clamp ratio, clipped fraction, mean |r - 1|  (Sec. 3.4)
   * OPD shaping: subtract coef * (log pi_student - log pi_teacher) of the
@@ -256,6 +258,16 @@ def opd_topk_estimate(z_rows, temperature, lse, cand_ids, teacher_lp):
 # (a3) per-token objective
 # --------------------------------------------------------------------------
 
+def correction_ratio(logp, rho, old=None):
+    """The train/rollout ratio the corrections act on (Sec. 3.4):
+    rc = exp(log pi_train - log pi_rollout). log pi_train is ``old`` when the
+    caller gives the trainer's log-probs from a separate pass, else the
+    trainer's own log-prob of the token in this pass. Either way the ratio
+    is a constant per-token weight: no gradient flows through it."""
+    train = np.asarray(logp if old is None else old, np.float64)
+    return np.exp(train - np.asarray(rho, np.float64))
+
+
 def token_objective(logp, rho, q, A_row, H, p: LossParams, old=None):
     """Per-token loss terms and the derivative of the token loss w.r.t. logp.
 
@@ -266,8 +278,9 @@ def token_objective(logp, rho, q, A_row, H, p: LossParams, old=None):
                        clipped and r < 1-eps_lo.
     dual clip:         if c_dual > 0 and A < 0: d = -A c_dual; if d < pg
                        (strict) then pg = d and the token is dual-clipped.
-    correction (Sec. 3.4), needs ``old``: rc = exp(old - rho) is the
-                       train/rollout ratio, a constant weight:
+    correction (Sec. 3.4): rc = correction_ratio(logp, rho, old), the
+                       train/rollout ratio (exp(old - rho), or without old
+                       exp(logp - rho) of this pass), a constant weight:
                        TIS wt = min(max(rc, lo), hi);
                        clip-or-pop wt = rc if lo <= rc <= hi else 0;
                        pg <- wt * pg.
@@ -301,9 +314,7 @@ def token_objective(logp, rho, q, A_row, H, p: LossParams, old=None):
     if p.correction != "none":
         if p.correction not in CORRECTIONS:
             raise ValueError(p.correction)
-        if old is None:
-            raise ValueError("a ratio correction needs old log-probs")
-        rc = np.exp(np.asarray(old, np.float64) - rho)
+        rc = correction_ratio(logp, rho, old)
         outside = (rc < p.corr_lo) | (rc > p.corr_hi)
         corr_clip = outside
         if p.correction == "tis":
@@ -359,9 +370,7 @@ def sequence_objective(logp, rho, q, A_traj, H, cu_seqlens, mask, p: LossParams,
     rc = np.ones(R)
     corr_clip = np.zeros(R, bool)
     if p.correction != "none":
-        if old is None:
-            raise ValueError("a ratio correction needs old log-probs")
-        rc = np.exp(np.asarray(old, np.float64) - rho)
+        rc = correction_ratio(logp, rho, old)
         outside = (rc < p.corr_lo) | (rc > p.corr_hi)
         corr_clip = outside
         wt = (np.minimum(np.maximum(rc, p.corr_lo), p.corr_hi) if p.correction == "tis"

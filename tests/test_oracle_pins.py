@@ -294,8 +294,24 @@ def test_corrections_tis_and_clip_or_pop():
     assert pop["corr_clip"].tolist() == [True, False, False, False, True]
     np.testing.assert_allclose(tis["pg"], tis["wt"] * base["pg"], rtol=1e-15)
     np.testing.assert_allclose(pop["G"], pop["wt"] * base["G"], rtol=1e-15)
-    with pytest.raises(ValueError):
-        oracle.token_objective(logp, rho, None, A, np.zeros(5), LossParams(correction="tis"))
+
+
+@pytest.mark.parametrize("correction", ["tis", "clip_or_pop"])
+def test_correction_without_old_logprobs_golden(correction):
+    """Without old log-probs the correction ratio is the trainer's own
+    log-prob of this pass against the rollout's (a constant weight), and the
+    PPO ratio is taken against the rollout log-prob (hand-derived)."""
+    c = _golden()["tis_own_ratio"]
+    logp = np.array([_ev(v) for v in c["log_r"]])
+    A = np.array([float(v) for v in c["A"]])
+    o = oracle.token_objective(logp, np.zeros(4), None, A, np.zeros(4),
+                               LossParams(correction=correction, **c["params"]))
+    e = c["expect"][correction]
+    for k in ("wt", "pg", "G"):
+        np.testing.assert_allclose(o[k], [_ev(v) for v in e[k]], atol=1e-14, err_msg=k)
+    assert o["corr_clip"].astype(int).tolist() == e["corr_clip"]
+    assert o["clip_hi"].astype(int).tolist() == e["clip_hi"]
+    np.testing.assert_allclose(o["rc"], o["r"], rtol=0, atol=0)
 
 
 def test_tis_lower_clamp_golden():
@@ -449,16 +465,19 @@ def _near_kink(out, p, guard=1e-4):
 
 
 @pytest.mark.parametrize("V", [2, 3, 5, 8])
-@pytest.mark.parametrize("variant", ["ppo_dual_kl_ent_T", "tis", "clip_or_pop", "opd"])
-def test_dlogits_central_finite_differences(V, variant):
+@pytest.mark.parametrize("variant", ["ppo_dual_kl_ent_T", "tis", "clip_or_pop", "opd",
+                                     "tis_own", "clip_or_pop_own"])
+def test_dlogits_central_finite_differences(V, variant, monkeypatch):
     rng = np.random.default_rng(100 + V)
     n_traj, L_ = 4, 2
     R = n_traj * L_
     p = LossParams(temperature=0.8, eps_lo=0.15, eps_hi=0.25, dual_clip_c=2.5,
                    kl_coef=0.3, entropy_coef=0.07)
-    if variant in ("tis", "clip_or_pop"):
+    own = variant.endswith("_own")  # the correction ratio from this pass's own log-prob
+    if variant in ("tis", "clip_or_pop", "tis_own", "clip_or_pop_own"):
         p = LossParams(temperature=1.3, eps_lo=0.2, eps_hi=0.2, kl_coef=0.1,
-                       entropy_coef=0.02, correction=variant, corr_lo=0.5, corr_hi=1.5)
+                       entropy_coef=0.02, correction=variant.replace("_own", ""), corr_lo=0.5,
+                       corr_hi=1.5)
     if variant == "opd":
         p = LossParams(temperature=1.0, eps_lo=0.2, eps_hi=0.2, opd_coef=0.7)
     for attempt in range(50):
@@ -467,7 +486,9 @@ def test_dlogits_central_finite_differences(V, variant):
         logp, _, _ = oracle.row_log_softmax(z, y, p.temperature)
         rho = logp + rng.normal(0, 0.6, size=R)
         q = logp + rng.normal(0, 0.5, size=R)
-        old = logp + rng.normal(0, 0.3, size=R) if p.correction != "none" else None
+        old = logp + rng.normal(0, 0.3, size=R) if (p.correction != "none" and not own) else None
+        if own:
+            rho = logp + rng.normal(0, 0.25, size=R)
         teacher = logp + rng.normal(0, 0.5, size=R)
         w = rng.random(n_traj)
         gid = np.array([0, 0, 1, 1])
@@ -481,6 +502,10 @@ def test_dlogits_central_finite_differences(V, variant):
         pytest.fail("no draw away from the kinks")
     if variant == "ppo_dual_kl_ent_T":
         assert out["clip_hi"].any() or out["clip_lo"].any() or out["dual"].any()
+    if own:
+        # the weight is a constant: hold the correction ratio at its value
+        frozen = out["rc"].copy()
+        monkeypatch.setattr(oracle.rl_loss_ref, "correction_ratio", lambda *a, **k: frozen)
     h = 1e-6
     num = np.zeros_like(z)
     for i in range(R):
@@ -662,7 +687,8 @@ def test_gspo_on_one_token_trajectories_is_token_ppo():
         np.testing.assert_allclose(seq[k], tok[k], atol=1e-13)
 
 
-@pytest.mark.parametrize("variant", ["gspo", "gspo_tis", "topk", "reinforcepp_baseline"])
+@pytest.mark.parametrize("variant", ["gspo", "gspo_tis", "topk", "reinforcepp_baseline",
+                                     "gspo_tis_own"])
 def test_dlogits_fd_estimators(variant, monkeypatch):
     rng = np.random.default_rng(200 + len(variant))
     V, n_traj, L_ = 6, 4, 3
@@ -671,7 +697,9 @@ def test_dlogits_fd_estimators(variant, monkeypatch):
     extra = dict(gspo=dict(estimator="gspo", dual_clip_c=2.0),
                  gspo_tis=dict(estimator="gspo", correction="tis", corr_lo=0.5, corr_hi=1.5),
                  topk=dict(opd_coef=0.6, opd_topk=3),
-                 reinforcepp_baseline=dict(estimator="reinforcepp_baseline"))[variant]
+                 reinforcepp_baseline=dict(estimator="reinforcepp_baseline"),
+                 gspo_tis_own=dict(estimator="gspo", correction="tis", corr_lo=0.5,
+                                   corr_hi=1.1))[variant]
     p = LossParams(**base, **extra)
     gid = np.array([0, 0, 1, 1])
     cu = np.arange(n_traj + 1) * L_
@@ -682,7 +710,8 @@ def test_dlogits_fd_estimators(variant, monkeypatch):
         logp, _, _ = oracle.row_log_softmax(z, y, p.temperature)
         rho = logp + rng.normal(0, 0.5, size=R)
         q = logp + rng.normal(0, 0.4, size=R)
-        old = logp + rng.normal(0, 0.3, size=R) if p.correction != "none" else None
+        own = variant.endswith("_own")
+        old = logp + rng.normal(0, 0.3, size=R) if (p.correction != "none" and not own) else None
         w = rng.random(n_traj)
         ids = np.stack([rng.choice(V, 3, replace=False) for _ in range(R)])
         tlp = np.log(rng.dirichlet(np.ones(V), size=R))[np.arange(R)[:, None], ids]
@@ -692,6 +721,11 @@ def test_dlogits_fd_estimators(variant, monkeypatch):
             break
     else:
         pytest.fail("no draw away from the kinks")
+    if own:
+        # the correction weight is a constant: hold the ratio at its value
+        frozen_rc = oracle.correction_ratio(out["logp"], rho)
+        assert (np.minimum(np.maximum(frozen_rc, 0.5), 1.1) != frozen_rc).any()
+        monkeypatch.setattr(oracle.rl_loss_ref, "correction_ratio", lambda *a, **k: frozen_rc)
     if variant == "topk":
         # the top-K signal is a fixed per-token reward: hold it at its value
         frozen = oracle.opd_topk_estimate(z, p.temperature, out["lse"], ids, tlp)
