@@ -36,12 +36,15 @@
  *    outputs. A workspace written by rl_loss_fwd must not be reused before
  *    the matching rl_loss_bwd has run.
  *  - Host-side argument errors return a status before anything is enqueued.
- *  - Data-dependent errors (a target outside [0, vocab), a group id outside
- *    [0, n_groups), cu_seqlens not non-decreasing from 0 to n_rows, a wait
- *    inside a kernel that ran out of time) never trap: the kernels finish,
- *    write zeros for the affected rows, and record the error in the
- *    workspace; read it with rl_loss_check_device_error after the stream is
- *    synchronised.
+ *  - Data-dependent errors (a target or a top-K candidate id outside
+ *    [0, vocab), a group id outside [0, n_groups), cu_seqlens not
+ *    non-decreasing from 0 to n_rows, a wait inside a kernel that ran out of
+ *    time) never trap: the kernels finish, write zeros for the affected rows,
+ *    and record the error in the workspace; read it with
+ *    rl_loss_check_device_error after the stream is synchronised. Every wait
+ *    inside a kernel is bounded (2 s); a CTA whose wait runs out stops
+ *    issuing copies, waits (bounded) for the copies it has in flight, writes
+ *    zeros for its remaining rows and returns.
  *  - Outputs are defined for every row, trained or not; rows with mask 0 get
  *    their log-prob and entropy and a zero dLogits row.
  *  - n_rows == 0 is a valid no-op apart from zeroed statistics.
@@ -69,14 +72,20 @@ typedef enum {
   RL_ERR_GROUP_OUT_OF_RANGE = 6,  /* device: a group id not in [0, n_groups)   */
   RL_ERR_BAD_SEQLENS = 7,         /* device: cu_seqlens not 0 <= ... <= n_rows,
                                      non-decreasing, ending at n_rows          */
-  RL_ERR_DEVICE_TIMEOUT = 8       /* device: a bounded wait gave up            */
+  RL_ERR_DEVICE_TIMEOUT = 8,      /* device: a bounded wait gave up            */
+  RL_ERR_TOPK_ID_OUT_OF_RANGE = 9 /* device: a top-K OPD candidate id not in
+                                     [0, vocab)                                */
 } rl_status;
 
 typedef enum { RL_BF16 = 0, RL_F32 = 1 } rl_dtype;
 
-/* Ratio corrections of Sec. 3.4. Both need old_logprobs: the PPO ratio is
- * then exp(logp - old) and the correction ratio rc = exp(old - rollout) is a
- * constant per-token weight on the policy-gradient term:
+/* Ratio corrections of Sec. 3.4: a constant per-token weight on the
+ * policy-gradient term from the train/rollout ratio
+ * rc = exp(log pi_train - log pi_rollout), where log pi_train is
+ * old_logprobs when given (the PPO ratio is then exp(logp - old)) and else
+ * the trainer's own log-prob of the token in this pass (the single-pass
+ * step: rc = exp(logp - rollout), held constant, and the PPO ratio is taken
+ * against the rollout log-probs too):
  *   RL_CORR_TIS          weight = min(max(rc, corr_lo), corr_hi)
  *   RL_CORR_CLIP_OR_POP  weight = rc if corr_lo <= rc <= corr_hi, else 0 */
 typedef enum { RL_CORR_NONE = 0, RL_CORR_TIS = 1, RL_CORR_CLIP_OR_POP = 2 } rl_correction;
@@ -129,7 +138,9 @@ typedef struct {
    * with the trainer's probabilities p_k of the candidates renormalised over
    * the set as weights w_k; it is subtracted, times opd_coef, from the token's
    * advantage and is not differentiated. Both arrays are device memory,
-   * 4-byte aligned (else RL_ERR_INVALID_ARG); K <= 64. */
+   * 4-byte aligned (else RL_ERR_INVALID_ARG); K <= 64. A row with a
+   * candidate id outside [0, vocab) gets zeros like a row with a bad target,
+   * and the call records RL_ERR_TOPK_ID_OUT_OF_RANGE. */
   const int32_t* opd_topk_ids;
   const float* opd_topk_teacher;
 } rl_loss_params;
@@ -156,6 +167,18 @@ typedef struct {
   int64_t n_corr_clip;         /* correction weight differs from rc (Sec. 3.4 clipped fraction) */
 } rl_loss_stats;
 
+/* A shard's partial statistics (row-sharded calls, below), in DEVICE memory.
+ * Combine the shards' copies element by element: `sum` and `count` by
+ * addition, `max` by maximum. */
+typedef struct {
+  double sum[9];   /* over the shard's training tokens: l, pg, k3, H, r, |r - 1|,
+                      |logp - rollout logp|, rc, |rc - 1|                        */
+  double count[5]; /* training tokens, clip_hi, clip_lo, dual clip, correction
+                      clip (exact integers)                                      */
+  double max[2];   /* -(minimum r) and maximum r over the shard's training
+                      tokens (-inf when it has none)                             */
+} rl_loss_partials;
+
 /* Bytes of device workspace that one call with these sizes needs (the same
  * value serves rl_loss_fwd, rl_loss_bwd and rl_loss_fwd_bwd). The workspace
  * is caller-owned, 256-byte aligned, needs no initialisation, and carries the
@@ -177,7 +200,8 @@ rl_status rl_loss_workspace_size(int64_t n_rows, int32_t n_traj, int32_t n_group
  *                    (required when kl_coef > 0)
  *  old_logprobs      [n_rows] fp32 log-probs of the policy before this update,
  *                    or NULL (then the PPO ratio is taken against the rollout
- *                    log-probs); required when a correction is set
+ *                    log-probs, and a correction uses this pass's own
+ *                    log-prob as log pi_train)
  *  teacher_logprobs  [n_rows] fp32 teacher log-probs for OPD, or NULL
  *                    (required when opd_coef != 0 and opd_topk == 0)
  *  rewards           [n_traj] fp32, one outcome reward per trajectory
@@ -271,6 +295,54 @@ rl_status rl_loss_fwd_bwd_rows(int32_t phase, int64_t row_begin, int64_t row_end
                                rl_dtype dlogits_dtype, int64_t ld_out, void* workspace,
                                size_t workspace_bytes, rl_stream stream);
 
+/* Phases of rl_loss_shard_fwd_bwd. */
+enum {
+  RL_SHARD_COUNT = 1,  /* this shard's training tokens per trajectory        */
+  RL_SHARD_SWEEP = 2,  /* advantages, the sweep over the shard's rows, dLogits
+                          and the shard's partial statistics                 */
+  RL_SHARD_FINISH = 4  /* the call's statistics from the combined partials   */
+};
+
+/* rl_loss_fwd_bwd with the rows of one call spread over several shards (one
+ * per GPU or rank: data parallelism, or context parallelism, which splits
+ * each long session over ranks, Sec. 9.1). Shard k holds the contiguous rows
+ * [row_offset, row_offset + n_rows) of a call of n_rows_total rows; the
+ * per-row arrays (logits, targets, log-probs, mask, token_logprobs, entropy,
+ * dlogits) cover those rows only, while rewards, group_id and cu_seqlens
+ * (row offsets in the whole call's numbering) describe the whole call on
+ * every shard. The loss needs two exchanges between the shards, which the
+ * caller performs (the library has no collective):
+ *   1. RL_SHARD_COUNT writes traj_counts[n_traj] (int32, device): the
+ *      training tokens of each trajectory within this shard. The caller sums
+ *      the array over the shards (an all-reduce) in place.
+ *   2. RL_SHARD_SWEEP, given the summed traj_counts, computes the advantages
+ *      (every shard the same), the sweep over its rows with the whole call's
+ *      N, dLogits (dlogits NULL: forward only) and writes `partials`. The
+ *      caller combines the shards' partials as rl_loss_partials says.
+ *   3. RL_SHARD_FINISH writes `stats` from the combined partials.
+ * Each shard's outputs for its rows (log-probs, entropies, dLogits) are those
+ * of the unsharded call; the statistics differ from it only in the order of
+ * their floating-point sums. Every phase of a shard uses the same
+ * workspace (rl_loss_workspace_size(n_rows, n_traj, n_groups)), in order, on
+ * one stream. GSPO, whose gradient needs whole trajectories, returns
+ * RL_ERR_UNSUPPORTED. Arguments a phase does not read may be NULL (COUNT:
+ * logits, outputs, dlogits, partials, stats; FINISH: everything but
+ * partials, stats and the stream). */
+rl_status rl_loss_shard_fwd_bwd(int32_t phase, int64_t row_offset, int64_t n_rows_total,
+                                const void* logits, rl_dtype logits_dtype, int64_t n_rows,
+                                int64_t vocab, int64_t ld, const int32_t* targets,
+                                const float* rollout_logprobs, const float* ref_logprobs,
+                                const float* old_logprobs, const float* teacher_logprobs,
+                                const float* rewards, const int32_t* group_id,
+                                const int32_t* cu_seqlens, int32_t n_traj, int32_t n_groups,
+                                const uint8_t* loss_mask, const rl_loss_params* params,
+                                float* token_logprobs, float* entropy, float* advantages,
+                                int32_t* group_sizes, int32_t* traj_counts,
+                                rl_loss_partials* partials, rl_loss_stats* stats,
+                                float grad_loss, const float* grad_loss_device, void* dlogits,
+                                rl_dtype dlogits_dtype, int64_t ld_out, void* workspace,
+                                size_t workspace_bytes, rl_stream stream);
+
 /* rl_loss_fwd_bwd for callers that cannot allocate device memory at call
  * time (the paper has no counterpart; this is a deployment convenience).
  * Frameworks that reserve nearly all of HBM for their own pool, plain-C
@@ -281,13 +353,16 @@ rl_status rl_loss_fwd_bwd_rows(int32_t phase, int64_t row_begin, int64_t row_end
  * at small trajectory and group counts). Larger calls return
  * RL_ERR_WORKSPACE_TOO_SMALL before anything is enqueued. Each device on
  * which the library's code is loaded keeps the array until the process
- * exits. The first call on a device looks up the array's device address
- * (cudaGetSymbolAddress, with that device current): make it before any
- * stream capture. No call allocates or frees memory. All calls on a device
- * share the array: calls that overlap on the GPU race and must be
+ * exits. Every call looks up the array's device address on the current
+ * device (cudaGetSymbolAddress, which allocates nothing); the first call on
+ * a device also loads the library's device code there, so make it before
+ * any stream capture. No call allocates or frees memory. All calls on a
+ * device share the array: calls that overlap on the GPU race and must be
  * serialised by the caller; what must start at zero is reset by every
- * call. The device-side error word is kept in the array and cannot be read
- * back; rows with a bad target still get zeros. */
+ * call. The data-dependent errors of a call (bad target, group id,
+ * cu_seqlens or top-K candidate, a wait that ran out) are recorded in the
+ * array as for rl_loss_fwd_bwd and read with
+ * rl_loss_noalloc_check_device_error; the affected rows get zeros. */
 rl_status rl_loss_fwd_bwd_noalloc(const void* logits, rl_dtype logits_dtype, int64_t n_rows,
                                   int64_t vocab, int64_t ld, const int32_t* targets,
                                   const float* rollout_logprobs, const float* ref_logprobs,
@@ -300,6 +375,13 @@ rl_status rl_loss_fwd_bwd_noalloc(const void* logits, rl_dtype logits_dtype, int
                                   const float* grad_loss_device, void* dlogits,
                                   rl_dtype dlogits_dtype, int64_t ld_out, rl_stream stream);
 
+/* The device-side error of the last rl_loss_fwd_bwd_noalloc call on the
+ * current device, read after its stream has been synchronised: RL_OK or the
+ * lowest recorded code, as rl_loss_check_device_error. Reads four bytes of
+ * the array with one blocking copy (cudaMemcpyFromSymbol, no allocation).
+ * A later no-alloc call on the device overwrites the value. */
+rl_status rl_loss_noalloc_check_device_error(void);
+
 /* After the stream that ran a call on `workspace` has been synchronised:
  * RL_OK, or the data-dependent error the kernels recorded (when several
  * kinds occurred, the lowest code). Performs one small blocking
@@ -308,6 +390,58 @@ rl_status rl_loss_check_device_error(const void* workspace);
 
 /* Static text for a status code; never NULL. */
 const char* rl_status_string(rl_status status);
+
+/* Launch-plan overrides: measurement aids and a test hook, not needed for
+ * normal use. The library picks every launch shape itself (the sweep kernel
+ * by row length, the cluster kernel's cluster size, ring depth and block
+ * shape, the streaming kernel's ring); these fields force one instead. -1
+ * in a field keeps the library's choice; rl_launch_overrides_init sets
+ * every field to -1. A forced value outside the compiled shapes makes later
+ * calls return RL_ERR_UNSUPPORTED before anything is enqueued.
+ *  sweep_kernel         0 = the cluster kernel, 1 = the streaming kernel
+ *                       (16-byte aligned rows only)
+ *  cluster_size         1, 2, 4 or 8 CTAs per row (cluster kernel)
+ *  cluster_stages       1..4 ring stages (cluster kernel)
+ *  cluster_threads      256 or 512 threads per CTA (cluster kernel)
+ *  cluster_ctas_per_sm  4 or 5 with 256 threads, 2 with 512
+ *  stream_chunk_bytes   ring slot size, a multiple of 128 in [1 KB, 128 KB]
+ *  stream_slots         ring slots (as many as fit by default)
+ *  stream_hold          last chunks of a row pass B reads from shared memory
+ *  stream_split_first   1: the ragged chunk first, 0: last
+ *  stream_prefetch_bytes bytes of the next row the streaming kernel asks L2
+ *                       to fetch once a row's first-pass copies are issued
+ *                       (0 = none; a multiple of 16)
+ *  stall_first_wait_ns  TEST HOOK, > 0: in each CTA of the vocabulary sweep,
+ *                       the first wait for logits waits instead on a barrier
+ *                       that nothing completes, bounded by this many
+ *                       nanoseconds. It runs out, the CTA gives up as it
+ *                       would on a copy that never arrives (stops issuing
+ *                       copies, waits for the ones in flight, writes zeros
+ *                       for its rows) and the call records
+ *                       RL_ERR_DEVICE_TIMEOUT. Nothing hangs and no fault is
+ *                       raised; it exists to test that path.
+ * The overrides are process-wide and apply to calls made after the setter
+ * returns. */
+typedef struct {
+  int32_t sweep_kernel;
+  int32_t cluster_size;
+  int32_t cluster_stages;
+  int32_t cluster_threads;
+  int32_t cluster_ctas_per_sm;
+  int32_t stream_chunk_bytes;
+  int32_t stream_slots;
+  int32_t stream_hold;
+  int32_t stream_split_first;
+  int32_t stream_prefetch_bytes;
+  int64_t stall_first_wait_ns;
+} rl_launch_overrides;
+
+/* Sets every field of *o to -1 (no override). */
+rl_status rl_launch_overrides_init(rl_launch_overrides* o);
+
+/* Installs *o as the process-wide overrides; NULL removes them. Returns
+ * RL_ERR_INVALID_ARG for a value outside a field's documented range. */
+rl_status rl_set_launch_overrides(const rl_launch_overrides* o);
 
 /* Optional timing hook for the calling host thread: when both are non-NULL,
  * later calls on this thread record `begin` / `end` (cudaEvent_t) on their

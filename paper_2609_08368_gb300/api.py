@@ -104,52 +104,6 @@ class GraphedCall:
         self.graph.replay()
 
 
-class HostCall:
-    """Fused forward+backward with the inputs and results in pinned HOST
-    memory: every call copies the inputs host -> device, runs the loss, and
-    copies dLogits, the per-row outputs and the statistics back. Device
-    buffers are allocated once at construction."""
-
-    INPUTS = ("logits", "targets", "rollout_logprobs", "ref_logprobs", "old_logprobs",
-              "teacher_logprobs", "rewards", "group_id", "cu_seqlens", "loss_mask")
-
-    def __init__(self, host_w, device, dlogits_dtype=None, dev_w=None, buf=None):
-        """``dev_w`` / ``buf``: existing device buffers of the same shapes to
-        reuse (their contents are overwritten by every call)."""
-        self.host = host_w
-        self.dev = host_w.to(device) if dev_w is None else dev_w
-        n_traj = int(host_w.rewards.shape[0])
-        dl_dtype = dlogits_dtype or host_w.logits.dtype
-        self.buf = buf if buf is not None else alloc(
-            host_w.n_rows, n_traj, host_w.n_groups, device, vocab=host_w.vocab,
-            dlogits_dtype=dl_dtype)
-        pin = dict(pin_memory=True)
-        self.out = dict(
-            dlogits=torch.empty(self.buf.dlogits.shape, dtype=dl_dtype, **pin),
-            token_logprobs=torch.empty(host_w.n_rows, dtype=torch.float32, **pin),
-            entropy=torch.empty(host_w.n_rows, dtype=torch.float32, **pin),
-            stats=torch.empty(ml.STATS_BYTES, dtype=torch.uint8, **pin))
-
-    def bytes_in(self) -> int:
-        return sum(getattr(self.host, k).numel() * getattr(self.host, k).element_size()
-                   for k in self.INPUTS if getattr(self.host, k) is not None)
-
-    def bytes_out(self) -> int:
-        return sum(t.numel() * t.element_size() for t in self.out.values())
-
-    def __call__(self, grad_loss=1.0):
-        for k in self.INPUTS:
-            h = getattr(self.host, k)
-            if h is not None:
-                getattr(self.dev, k).copy_(h, non_blocking=True)
-        fwd_bwd(self.dev, self.buf, grad_loss=grad_loss)
-        self.out["dlogits"].copy_(self.buf.dlogits, non_blocking=True)
-        self.out["token_logprobs"].copy_(self.buf.token_logprobs, non_blocking=True)
-        self.out["entropy"].copy_(self.buf.entropy, non_blocking=True)
-        self.out["stats"].copy_(self.buf.stats, non_blocking=True)
-        return self.out
-
-
 def _rows_call(w, buf, phase, r0, r1, logits, dlogits, params=None, grad_loss=1.0, stream=None):
     ml.rl_loss_fwd_bwd_rows(phase, r0, r1, w.n_rows, logits, w.targets, w.rollout_logprobs,
                             w.ref_logprobs, w.old_logprobs, w.teacher_logprobs, w.rewards,
@@ -267,3 +221,84 @@ class PipelinedHostCall:
             if e is not None:
                 comp.wait_event(e)
         return self.out
+
+
+# ------------------------------------------------------------ row-sharded calls
+
+class Shard:
+    """One shard of a row-sharded fused call (rl_loss_shard_fwd_bwd): the
+    workload ``w`` holds this shard's rows [row_offset, row_offset + rows) of
+    a call of ``n_rows_total`` rows, with the whole call's rewards, group ids
+    and cu_seqlens; ``buf`` its output buffers. ``count``, ``sweep`` and
+    ``finish`` run the three phases; between them the shards' ``counts`` are
+    summed and their ``partials`` combined (exchange_counts /
+    exchange_partials, or any equivalent)."""
+
+    def __init__(self, w, row_offset: int, n_rows_total: int, buf: Buffers, params=None,
+                 grad_loss=1.0):
+        self.w, self.row_offset, self.n_rows_total, self.buf = w, row_offset, n_rows_total, buf
+        self.params = _params(w, params)
+        self.grad_loss = grad_loss
+        dev = w.targets.device
+        self.counts = torch.zeros(int(w.rewards.shape[0]), dtype=torch.int32, device=dev)
+        self.partials = torch.zeros(ml.PARTIALS_DOUBLES, dtype=torch.float64, device=dev)
+
+    def _call(self, phase, forward_only=False):
+        w, b = self.w, self.buf
+        ml.rl_loss_shard_fwd_bwd(phase, self.row_offset, self.n_rows_total, w.logits, w.targets,
+                                 w.rollout_logprobs, w.ref_logprobs, w.old_logprobs,
+                                 w.teacher_logprobs, w.rewards, w.group_id, w.cu_seqlens,
+                                 w.n_groups, w.loss_mask, self.params, b.token_logprobs,
+                                 b.entropy, b.advantages, b.group_sizes, self.counts,
+                                 self.partials, b.stats, None if forward_only else b.dlogits,
+                                 b.workspace, w.vocab, grad_loss=self.grad_loss)
+
+    def count(self):
+        self._call(ml.RL_SHARD_COUNT)
+
+    def sweep(self, forward_only=False):
+        self._call(ml.RL_SHARD_SWEEP, forward_only)
+
+    def finish(self):
+        self._call(ml.RL_SHARD_FINISH)
+
+
+def exchange_counts(counts: torch.Tensor, group=None):
+    """Sum the shards' per-trajectory training-token counts over the ranks of
+    ``group`` (in place)."""
+    import torch.distributed as dist
+    dist.all_reduce(counts, op=dist.ReduceOp.SUM, group=group)
+
+
+def exchange_partials(partials: torch.Tensor, group=None):
+    """Combine the shards' rl_loss_partials over the ranks of ``group`` (in
+    place): sums and counts by addition, the two maxima by maximum."""
+    import torch.distributed as dist
+    dist.all_reduce(partials[:ml.PARTIALS_SUMS], op=dist.ReduceOp.SUM, group=group)
+    dist.all_reduce(partials[ml.PARTIALS_SUMS:], op=dist.ReduceOp.MAX, group=group)
+
+
+def sharded_fwd_bwd(shard: Shard, group=None):
+    """This rank's shard of a row-sharded fused call, one shard per rank,
+    with the two exchanges over torch.distributed."""
+    shard.count()
+    exchange_counts(shard.counts, group)
+    shard.sweep()
+    exchange_partials(shard.partials, group)
+    shard.finish()
+
+
+def sharded_fwd_bwd_local(shards):
+    """Several shards of one call driven from one process (for instance on
+    one GPU): the exchanges are sums and maxima over the shards' tensors."""
+    for s in shards:
+        s.count()
+    total = torch.stack([s.counts for s in shards]).sum(0)
+    for s in shards:
+        s.counts.copy_(total)
+        s.sweep()
+    p = torch.stack([s.partials for s in shards])
+    comb = torch.cat([p[:, :ml.PARTIALS_SUMS].sum(0), p[:, ml.PARTIALS_SUMS:].max(0).values])
+    for s in shards:
+        s.partials.copy_(comb)
+        s.finish()

@@ -18,6 +18,24 @@
 using namespace milesloss;
 
 namespace {
+std::mutex g_ov_mu;
+rl_launch_overrides g_ov = {-1, -1, -1, -1, -1, -1, -1, -1, -1, -1, -1};
+}  // namespace
+
+namespace milesloss {
+rl_launch_overrides current_overrides() {
+  std::lock_guard<std::mutex> lk(g_ov_mu);
+  return g_ov;
+}
+
+rl_status status_of_bits(uint32_t bits) {
+  for (int code = RL_ERR_TARGET_OUT_OF_RANGE; code <= RL_ERR_TOPK_ID_OUT_OF_RANGE; ++code)
+    if (bits & (1u << code)) return static_cast<rl_status>(code);
+  return RL_OK;
+}
+}  // namespace milesloss
+
+namespace {
 
 thread_local cudaEvent_t t_ev_begin = nullptr;
 thread_local cudaEvent_t t_ev_end = nullptr;
@@ -154,11 +172,11 @@ struct SweepPlan {
 // plan aims at five CTAs of 256 threads per SM: the smallest cluster whose
 // per-CTA slice fits a fifth of the SM's shared memory, then as many ring
 // stages as still fit; if no cluster size fits, one CTA per SM.
-// Overridable for tuning through MILESLOSS_SWEEP_CLUSTER / _STAGES /
-// _THREADS / _CTAS_PER_SM.
+// rl_set_launch_overrides can force the cluster size, stages and block shape.
 constexpr long long kMinSliceBytes = 32 * 1024;  // smallest cluster slice a fused plan takes
 
-rl_status plan_sweep(rl_dtype dt, long long V, int dev, int extra, bool grad, SweepPlan* out) {
+rl_status plan_sweep(rl_dtype dt, long long V, int dev, int extra, bool grad,
+                     const rl_launch_overrides& ov, SweepPlan* out) {
   int optin = 0, per_sm = 0, reserved = 0;
   if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) !=
@@ -168,15 +186,15 @@ rl_status plan_sweep(rl_dtype dt, long long V, int dev, int extra, bool grad, Sw
     return RL_ERR_CUDA;
   // Block shapes compiled: 256 threads for 5 or 4 CTAs per SM (48 or 64
   // registers), 512 threads for 2 CTAs per SM.
-  const int threads = env_int("MILESLOSS_SWEEP_THREADS", 256);
-  const int target = env_int("MILESLOSS_SWEEP_CTAS_PER_SM", threads == 256 ? 5 : 2);
+  const int threads = ov.cluster_threads > 0 ? ov.cluster_threads : 256;
+  const int target = ov.cluster_ctas_per_sm > 0 ? ov.cluster_ctas_per_sm : (threads == 256 ? 5 : 2);
   if (!((threads == 256 && (target == 4 || target == 5)) || (threads == 512 && target == 2)))
     return RL_ERR_UNSUPPORTED;
   const int variant = threads == 512 ? 512 : (target == 5 ? 255 : 256);
   const int es = static_cast<int>(elem_size(dt));
   const int vec = 16 / es;
-  const int forced_c = env_int("MILESLOSS_SWEEP_CLUSTER", 0);
-  const int forced_s = env_int("MILESLOSS_SWEEP_STAGES", 0);
+  const int forced_c = ov.cluster_size > 0 ? ov.cluster_size : 0;
+  const int forced_s = ov.cluster_stages > 0 ? ov.cluster_stages : 0;
   const int fixed = kSweepSmemExtra + extra;                           // scratch (+ top-K)
   const int hard = optin - fixed;                                      // one CTA per SM
   const int share = per_sm / target - reserved - fixed;                // `target` per SM
@@ -301,6 +319,12 @@ struct FwdIn {
   rl_loss_stats* stats;
   void* ws;
   size_t ws_bytes;
+  // a shard of a row-sharded call (rl_loss_shard_fwd_bwd)
+  long long row0 = 0;           // global index of the shard's first row
+  long long R_total = -1;       // rows of the whole call (-1: c.R)
+  const int* counts_in = nullptr;
+  int* counts_out = nullptr;
+  rl_loss_partials* part_out = nullptr;
 };
 
 rl_status check_fwd(const FwdIn& f, bool need_logits = true) {
@@ -312,7 +336,6 @@ rl_status check_fwd(const FwdIn& f, bool need_logits = true) {
   if (!f.cu) return RL_ERR_INVALID_ARG;
   if (f.c.R > 0 && !f.rho) return RL_ERR_INVALID_ARG;
   if (f.c.R > 0 && p->kl_coef > 0.0f && !f.q) return RL_ERR_INVALID_ARG;
-  if (f.c.R > 0 && p->correction != RL_CORR_NONE && !f.old) return RL_ERR_INVALID_ARG;
   if (f.c.R > 0 && p->opd_coef != 0.0f && p->opd_topk == 0 && !f.teacher)
     return RL_ERR_INVALID_ARG;
   if (f.c.R > 0 && p->opd_coef != 0.0f && p->opd_topk > 0 &&
@@ -423,6 +446,10 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
   // advantages, N, validation
   AdvArgs aa;
   aa.R = c.R;
+  aa.row0 = f.row0;
+  aa.R_total = f.R_total >= 0 ? f.R_total : c.R;
+  aa.counts_in = f.counts_in;
+  aa.counts_out = f.counts_out;
   aa.n_traj = f.n_traj;
   aa.n_groups = f.n_groups;
   aa.rewards = f.rewards;
@@ -481,9 +508,13 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
   const size_t es = elem_size(c.dt);
   const bool in_bulk = aligned16(c.logits) && ((c.ld * es) % 16 == 0);
   const bool out_vec = grad && aligned16(go->dl) && ((go->ld_out * elem_size(go->dt)) % 16 == 0);
-  if (c.R > 0 && use_stream(c.V * static_cast<long long>(es), in_bulk, grad)) {
+  const rl_launch_overrides ov = current_overrides();
+  const unsigned long long stall =
+      ov.stall_first_wait_ns > 0 ? static_cast<unsigned long long>(ov.stall_first_wait_ns) : 0ull;
+  if (c.R > 0 && use_stream(c.V * static_cast<long long>(es), in_bulk, grad, ov)) {
     StreamPlan sp;
-    st = plan_stream(dev, sc.topk ? kTopKSmem : 0, c.V * static_cast<long long>(es), grad, &sp);
+    st = plan_stream(dev, sc.topk ? kTopKSmem : 0, c.V * static_cast<long long>(es), grad, ov,
+                     &sp);
     if (st != RL_OK) return st;
     const void* fn = stream_kernel(c.dt, grad ? go->dt : c.dt, grad, sc.topk > 0);
     st = set_smem(fn, dev, sp.smem);
@@ -501,6 +532,7 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     ta.n_slots = sp.slots;
     ta.n_hold = sp.hold;
     ta.split_first = sp.split_first;
+    ta.prefetch = sp.prefetch;
     ta.out_vec = out_vec;
     ta.targets = c.targets;
     ta.rho = fr.rho;
@@ -515,6 +547,7 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     ta.grad_loss_dev = grad ? go->g_dev : nullptr;
     ta.s = sc;
     ta.ws = ws;
+    ta.stall_ns = stall;
     const long long grid = std::min<long long>(ctas, c.R);
     record(t_ev_begin, s);
     st = launch(fn, dim3(static_cast<unsigned>(grid)), dim3(threads), sp.smem, 1, s,
@@ -523,7 +556,7 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     if (st != RL_OK) return st;
   } else if (c.R > 0) {
     SweepPlan pl;
-    st = plan_sweep(c.dt, c.V, dev, sc.topk ? kTopKSmem : 0, grad, &pl);
+    st = plan_sweep(c.dt, c.V, dev, sc.topk ? kTopKSmem : 0, grad, ov, &pl);
     if (st != RL_OK) return st;
     const void* fn = sweep_kernel(c.dt, grad ? go->dt : c.dt, grad, pl.variant, sc.topk > 0);
     st = set_smem(fn, dev, pl.smem);
@@ -556,6 +589,7 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     sa.grad_loss_dev = grad ? go->g_dev : nullptr;
     sa.s = sc;
     sa.ws = ws;
+    sa.stall_ns = stall;
     record(t_ev_begin, s);
     st = launch(fn, dim3(static_cast<unsigned>(n_cl * pl.C)), dim3(pl.threads), pl.smem, pl.C,
                 s, &sa);
@@ -577,12 +611,13 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     if (st != RL_OK) return st;
   }
 
-  if ((phase & RL_PHASE_END) && f.stats) {
+  if ((phase & RL_PHASE_END) && (f.stats || f.part_out)) {
     StatArgs ta;
     ta.R = call.R;
     ta.mask = call.mask;
     ta.rho = f.rho;
     ta.out = f.stats;
+    ta.part_out = f.part_out;
     ta.ws = ws_all;
     long long blocks = (call.R + kStatThreads - 1) / kStatThreads;  // one row per thread
     blocks = std::max<long long>(1, std::min<long long>(blocks, kMaxStatBlocks));
@@ -682,6 +717,59 @@ rl_status rl_loss_fwd_bwd_rows(int32_t phase, int64_t row_begin, int64_t row_end
                  row_begin, row_end);
 }
 
+rl_status rl_loss_shard_fwd_bwd(int32_t phase, int64_t row_offset, int64_t n_rows_total,
+                                const void* logits, rl_dtype logits_dtype, int64_t n_rows,
+                                int64_t vocab, int64_t ld, const int32_t* targets,
+                                const float* rollout_logprobs, const float* ref_logprobs,
+                                const float* old_logprobs, const float* teacher_logprobs,
+                                const float* rewards, const int32_t* group_id,
+                                const int32_t* cu_seqlens, int32_t n_traj, int32_t n_groups,
+                                const uint8_t* loss_mask, const rl_loss_params* params,
+                                float* token_logprobs, float* entropy, float* advantages,
+                                int32_t* group_sizes, int32_t* traj_counts,
+                                rl_loss_partials* partials, rl_loss_stats* stats,
+                                float grad_loss, const float* grad_loss_device, void* dlogits,
+                                rl_dtype dlogits_dtype, int64_t ld_out, void* workspace,
+                                size_t workspace_bytes, rl_stream stream) {
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (phase == RL_SHARD_FINISH) {
+    if (!partials || !stats) return RL_ERR_INVALID_ARG;
+    FinishArgs fa{partials, stats};
+    return launch(finish_kernel(), dim3(1), dim3(32), 0, 1, s, &fa);
+  }
+  if (phase != RL_SHARD_COUNT && phase != RL_SHARD_SWEEP) return RL_ERR_INVALID_ARG;
+  if (row_offset < 0 || n_rows < 0 || n_rows_total < 0 || row_offset > n_rows_total - n_rows)
+    return RL_ERR_INVALID_ARG;
+  if (n_traj > 0 && !traj_counts) return RL_ERR_INVALID_ARG;
+  if (params && params->estimator == RL_EST_GSPO) return RL_ERR_UNSUPPORTED;
+  const bool count = phase == RL_SHARD_COUNT;
+  FwdIn f{{logits, logits_dtype, n_rows, vocab, ld, targets, loss_mask, params},
+          rollout_logprobs, ref_logprobs, old_logprobs, teacher_logprobs, rewards,
+          group_id, cu_seqlens, n_traj, n_groups, count ? nullptr : token_logprobs,
+          count ? nullptr : entropy, count ? nullptr : advantages,
+          count ? nullptr : group_sizes, nullptr, workspace, workspace_bytes};
+  f.row0 = row_offset;
+  f.R_total = n_rows_total;
+  if (count) {
+    f.counts_out = traj_counts;
+    rl_status st = check_fwd(f, false);
+    if (st != RL_OK) return st;
+    return run_fwd(f, nullptr, s, RL_PHASE_BEGIN);
+  }
+  if (!partials) return RL_ERR_INVALID_ARG;
+  f.counts_in = traj_counts;
+  f.part_out = partials;
+  rl_status st = check_fwd(f, n_rows > 0);
+  if (st != RL_OK) return st;
+  GradOut go{grad_loss, grad_loss_device, dlogits, dlogits_dtype, ld_out};
+  const bool grad = dlogits != nullptr;
+  if (grad) {
+    st = check_grad(f.c, go);
+    if (st != RL_OK) return st;
+  }
+  return run_fwd(f, grad ? &go : nullptr, s, RL_PHASE_ALL);
+}
+
 rl_status rl_loss_bwd(const void* logits, rl_dtype logits_dtype, int64_t n_rows, int64_t vocab,
                       int64_t ld, const int32_t* targets, const uint8_t* loss_mask,
                       const rl_loss_params* params, float grad_loss,
@@ -710,9 +798,7 @@ rl_status rl_loss_check_device_error(const void* workspace) {
   uint32_t bits = 0;
   if (cudaMemcpy(&bits, workspace, sizeof(bits), cudaMemcpyDeviceToHost) != cudaSuccess)
     return RL_ERR_CUDA;
-  for (int code = RL_ERR_TARGET_OUT_OF_RANGE; code <= RL_ERR_DEVICE_TIMEOUT; ++code)
-    if (bits & (1u << code)) return static_cast<rl_status>(code);
-  return RL_OK;
+  return status_of_bits(bits);
 }
 
 const char* rl_status_string(rl_status status) {
@@ -726,6 +812,7 @@ const char* rl_status_string(rl_status status) {
     case RL_ERR_GROUP_OUT_OF_RANGE: return "group id outside [0, n_groups)";
     case RL_ERR_BAD_SEQLENS: return "cu_seqlens not non-decreasing from 0 to n_rows";
     case RL_ERR_DEVICE_TIMEOUT: return "a bounded wait inside a kernel timed out";
+    case RL_ERR_TOPK_ID_OUT_OF_RANGE: return "top-K OPD candidate id outside [0, vocab)";
   }
   return "unknown status";
 }
@@ -736,6 +823,36 @@ rl_status rl_set_sweep_events(void* begin_event, void* end_event) {
   return RL_OK;
 }
 
-int32_t rl_loss_abi_version(void) { return 100; }
+rl_status rl_launch_overrides_init(rl_launch_overrides* o) {
+  if (!o) return RL_ERR_INVALID_ARG;
+  o->sweep_kernel = o->cluster_size = o->cluster_stages = o->cluster_threads = -1;
+  o->cluster_ctas_per_sm = o->stream_chunk_bytes = o->stream_slots = o->stream_hold = -1;
+  o->stream_split_first = o->stream_prefetch_bytes = -1;
+  o->stall_first_wait_ns = -1;
+  return RL_OK;
+}
+
+rl_status rl_set_launch_overrides(const rl_launch_overrides* o) {
+  rl_launch_overrides v;
+  rl_launch_overrides_init(&v);
+  if (o) {
+    auto in = [](int32_t x, int32_t lo, int32_t hi) { return x == -1 || (x >= lo && x <= hi); };
+    if (!in(o->sweep_kernel, 0, 1) || !in(o->cluster_size, 1, kMaxCluster) ||
+        !in(o->cluster_stages, 1, kMaxStages) || !in(o->cluster_threads, 256, 512) ||
+        !in(o->cluster_ctas_per_sm, 1, 8) || !in(o->stream_chunk_bytes, 1024, 131072) ||
+        !in(o->stream_slots, 1, kMaxSlots) || !in(o->stream_hold, 0, kMaxSlots) ||
+        !in(o->stream_split_first, 0, 1) || !in(o->stream_prefetch_bytes, 0, 1 << 20) ||
+        (o->stream_prefetch_bytes > 0 && o->stream_prefetch_bytes % 16) ||
+        o->stall_first_wait_ns < -1 ||
+        o->stall_first_wait_ns > 10000000000LL)
+      return RL_ERR_INVALID_ARG;
+    v = *o;
+  }
+  std::lock_guard<std::mutex> lk(g_ov_mu);
+  g_ov = v;
+  return RL_OK;
+}
+
+int32_t rl_loss_abi_version(void) { return 110; }
 
 }  // extern "C"

@@ -16,47 +16,38 @@
 // workspace would exceed it are rejected with RL_ERR_WORKSPACE_TOO_SMALL
 // before anything is enqueued.
 //
-// The first call on a device looks up the device address of the array
-// (cudaGetSymbolAddress, with that device current) and caches it; make that
-// first call before any stream capture. Nothing here calls cudaMalloc,
-// cudaFree or any allocating routine.
+// Every call looks up the device address of the array on the current
+// device (cudaGetSymbolAddress, with that device current). The address is
+// not cached: after cudaDeviceReset, or in a new primary context, the
+// library's device code is loaded again and the array may sit elsewhere.
+// The first call on a device also loads that code, so make it before any
+// stream capture. Nothing here calls cudaMalloc, cudaFree or any allocating
+// routine.
 //
 // All calls on a device share the one array and it keeps the previous
 // call's contents; the kernels reset what must start at zero (the error
 // word and the reduction ticket) at the start of every call. Calls that
 // overlap on the GPU (on different streams, or from different host
 // threads) race on the array and must be serialised by the caller. The
-// data-dependent error word lives in the array and is not reachable from
-// outside; rows with a bad target get zeros as in rl_loss_fwd_bwd.
+// data-dependent error word stays in the array after a call:
+// rl_loss_noalloc_check_device_error reads it back (cudaMemcpyFromSymbol,
+// no allocation); rows with a bad target get zeros as in rl_loss_fwd_bwd.
 #include <cuda_runtime.h>
 
-#include <mutex>
-
+#include "kernels.h"
 #include "milesloss.h"
 
 namespace {
 
 constexpr size_t kNoallocScratchBytes = size_t(8) << 20;
-constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
 
-std::mutex g_noalloc_mu;
-void* g_noalloc_addr[kMaxDevices] = {};
-
-// Device address of the scratch array on the current device (set-up once
-// per device).
+// Device address of the scratch array on the current device.
 rl_status scratch_address(void** out) {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return RL_ERR_CUDA;
-  if (dev < 0 || dev >= kMaxDevices) return RL_ERR_UNSUPPORTED;
-  std::lock_guard<std::mutex> lk(g_noalloc_mu);
-  if (!g_noalloc_addr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return RL_ERR_CUDA;
-    g_noalloc_addr[dev] = p;
-  }
-  *out = g_noalloc_addr[dev];
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return RL_ERR_CUDA;
+  *out = p;
   return RL_OK;
 }
 
@@ -83,4 +74,14 @@ extern "C" rl_status rl_loss_fwd_bwd_noalloc(
                          cu_seqlens, n_traj, n_groups, loss_mask, params, token_logprobs,
                          entropy, advantages, group_sizes, stats, grad_loss, grad_loss_device,
                          dlogits, dlogits_dtype, ld_out, scratch, kNoallocScratchBytes, stream);
+}
+
+extern "C" rl_status rl_loss_noalloc_check_device_error(void) {
+  // The error word is the first field of the workspace header, which starts
+  // the array (milesloss::WsLayout puts the header at offset 0).
+  uint32_t bits = 0;
+  if (cudaMemcpyFromSymbol(&bits, g_noalloc_scratch, sizeof(bits), 0, cudaMemcpyDeviceToHost) !=
+      cudaSuccess)
+    return RL_ERR_CUDA;
+  return milesloss::status_of_bits(bits);
 }

@@ -20,6 +20,7 @@ enum : uint32_t {
   kErrGroup = 1u << RL_ERR_GROUP_OUT_OF_RANGE,
   kErrSeqlens = 1u << RL_ERR_BAD_SEQLENS,
   kErrTimeout = 1u << RL_ERR_DEVICE_TIMEOUT,
+  kErrTopK = 1u << RL_ERR_TOPK_ID_OUT_OF_RANGE,
 };
 
 // Per-row flag bits kept in the workspace.
@@ -128,7 +129,7 @@ struct LossScalars {
   const float* topk_teacher; // [R, K]
 };
 
-// Correction weight of a token (Sec. 3.4) from its ratio rc = exp(old - rollout).
+// Correction weight of a token (Sec. 3.4) from its train/rollout ratio rc.
 __host__ __device__ __forceinline__ float correction_weight(float rc, const LossScalars& s) {
   if (s.corr == RL_CORR_NONE) return 1.0f;
   if (s.corr == RL_CORR_TIS) return fminf(fmaxf(rc, s.corr_lo), s.corr_hi);
@@ -188,6 +189,47 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
   }
 }
 
+// A CTA's shared "give up" flag: once one party of the CTA has given up on a
+// wait, the others stop waiting too (their next wait returns at once), so a
+// CTA that meets one timeout finishes in about one wait limit instead of one
+// limit per remaining wait.
+//
+// Waits for the phase with the given parity. Returns false without waiting
+// when *abort is already set, and gives up when *abort becomes set or after
+// ~limit_ns; a party that gives up on its own time limit records the timeout
+// in *err. On false the caller must not read what the phase guards. Every
+// party that returns false (re)sets *abort itself, so that whoever it later
+// synchronises with (a barrier, an mbarrier arrival) sees the flag.
+__device__ __forceinline__ bool mbar_wait_or_abort(uint32_t bar, uint32_t parity,
+                                                   uint64_t limit_ns, volatile int* abort,
+                                                   uint32_t* err) {
+  // the flag is read first: a party that runs on after giving up must not
+  // trust a parity test, which a barrier two phases behind would pass (the
+  // flag load and the first test are independent, so their latencies overlap)
+  const int gave_up = *abort;
+  const bool done = mbar_try_wait(bar, parity);
+  if (gave_up) {
+    *abort = 1;
+    return false;
+  }
+  if (done) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t n = 1;; ++n) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((n & 63u) == 0) {
+      if (*abort) {
+        *abort = 1;
+        return false;
+      }
+      if (globaltimer_ns() - t0 > limit_ns) {
+        *abort = 1;
+        atomicOr(err, kErrTimeout);
+        return false;
+      }
+    }
+  }
+}
+
 __device__ __forceinline__ uint64_t l2_policy_evict_first() {
   uint64_t p;
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
@@ -204,6 +246,12 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
       " [%0], [%1], %2, [%3], %4;" ::"r"(dst),
       "l"(src), "r"(bytes), "r"(bar), "l"(policy)
       : "memory");
+}
+
+// Asks L2 to fetch [src, src + bytes) from global memory (no destination, no
+// completion to wait for). src 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
 }
 
 __device__ __forceinline__ void fence_proxy_async_smem() {
@@ -440,12 +488,17 @@ struct TokenTerms {
   uint8_t flags;
 };
 
-__device__ __forceinline__ TokenTerms token_terms(float logp, float H, float rho, float q,
-                                                  bool has_q, float old, bool has_old,
-                                                  float A, const LossScalars& s) {
-  TokenTerms t;
-  const float base = has_old ? old : rho;
-  const float r = expf(logp - base);
+// The policy-gradient part of a token's objective from its PPO ratio r and
+// its correction ratio rc (Sec. 3.4; rc is ignored without a correction):
+// pg (weighted by the correction), its derivative with respect to logp
+// (weighted) and the clip flags.
+struct PolicyTerms {
+  float pg, gpg;
+  uint8_t flags;
+};
+
+__device__ __forceinline__ PolicyTerms policy_terms(float r, float rc, float A,
+                                                    const LossScalars& s) {
   const float u = -A * r;
   const float cl = fminf(fmaxf(r, 1.0f - s.eps_lo), 1.0f + s.eps_hi);
   const float c = -A * cl;
@@ -460,14 +513,25 @@ __device__ __forceinline__ TokenTerms token_terms(float logp, float H, float rho
     if (d < pg) { pg = d; dual = true; fl |= kFlagDual; }
   }
   float gpg = (clipped || dual) ? 0.0f : -A * r;
-  float rc = 1.0f;
   if (s.corr != RL_CORR_NONE) {
-    rc = expf(old - rho);
     if ((rc < s.corr_lo) || (rc > s.corr_hi)) fl |= kFlagCorrClip;
     const float wt = correction_weight(rc, s);
     pg *= wt;
     gpg *= wt;
   }
+  return PolicyTerms{pg, gpg, fl};
+}
+
+__device__ __forceinline__ TokenTerms token_terms(float logp, float H, float rho, float q,
+                                                  bool has_q, float old, bool has_old,
+                                                  float A, const LossScalars& s) {
+  TokenTerms t;
+  const float base = has_old ? old : rho;
+  const float r = expf(logp - base);
+  // the train/rollout ratio of Sec. 3.4, log pi_train being the given old
+  // log-prob or else this pass's own (then equal to r); a constant weight
+  const float rc = s.corr == RL_CORR_NONE ? 1.0f : (has_old ? expf(old - rho) : r);
+  const PolicyTerms pt = policy_terms(r, rc, A, s);
   float k3 = 0.0f, gkl = 0.0f;
   if (has_q) {
     // expm1 keeps both terms accurate when q is close to logp
@@ -477,19 +541,20 @@ __device__ __forceinline__ TokenTerms token_terms(float logp, float H, float rho
     gkl = -em1;
   }
   t.r = r;
-  t.pg = pg;
+  t.pg = pt.pg;
   t.k3 = k3;
-  t.ell = pg + s.beta * k3 - s.gamma * H;
-  t.G = gpg + s.beta * gkl;
+  t.ell = pt.pg + s.beta * k3 - s.gamma * H;
+  t.G = pt.gpg + s.beta * gkl;
   t.rc = rc;
-  t.flags = fl;
+  t.flags = pt.flags;
   return t;
 }
 
 // Top-K on-policy distillation signal of one row (Sec. 5.2): the sum over
 // the candidate set of w_k (log p_k - teacher_k), with p_k the trainer's
 // probabilities of the candidates (from the row's logits and its lse) and
-// w_k = p_k / sum_j p_j. Candidates outside [0, V) are skipped.
+// w_k = p_k / sum_j p_j. A candidate outside [0, V) marks the row bad (it
+// gets zeros and the call records RL_ERR_TOPK_ID_OUT_OF_RANGE).
 //
 // Since w_k is proportional to exp(z_k / T), the signal is
 //   sum_k w_k (z_k / T - teacher_k) / sum_k w_k  -  lse,
@@ -512,10 +577,12 @@ struct TopKBuf {
 struct TopKLane {
   int id0, id1;  // -1: no candidate (past K or outside [0, V))
   float z0, z1;
+  bool bad;      // one of the lane's ids lies outside [0, V)
 };
 
 struct TopKPart {
   float m, sw, acc;
+  int bad;  // some candidate id of the row lies outside [0, V)
 };
 
 __device__ __forceinline__ void cp_async4(void* dst, const void* src) {
@@ -544,14 +611,14 @@ __device__ __forceinline__ void topk_prefetch(TopKBuf* buf, const int* ids, cons
 
 // The lane's candidate ids of the row (after cp_async_wait_all for its buffer).
 __device__ __forceinline__ TopKLane topk_ids(const TopKBuf* buf, int V, int K, int lane) {
-  TopKLane c{-1, -1, 0.0f, 0.0f};
+  TopKLane c{-1, -1, 0.0f, 0.0f, false};
   if (lane < K) {
     const int id = buf->ids[lane];
-    if (id >= 0 && id < V) c.id0 = id;
+    if (id >= 0 && id < V) c.id0 = id; else c.bad = true;
   }
   if (lane + 32 < K) {
     const int id = buf->ids[lane + 32];
-    if (id >= 0 && id < V) c.id1 = id;
+    if (id >= 0 && id < V) c.id1 = id; else c.bad = true;
   }
   return c;
 }
@@ -570,7 +637,7 @@ __device__ __forceinline__ void topk_gather(TopKLane& c, const void* src, int c0
 __device__ __forceinline__ TopKPart topk_merge_all(const float4* parts, int n) {
   float M = -INFINITY;
   for (int r = 0; r < n; ++r) M = fmaxf(M, parts[r].x);
-  TopKPart p{M, 0.0f, 0.0f};
+  TopKPart p{M, 0.0f, 0.0f, 0};
   if (M == -INFINITY) return p;
   for (int r = 0; r < n; ++r) {
     const float4 e = parts[r];
@@ -589,11 +656,12 @@ template <class Mine>
 __device__ __forceinline__ TopKPart topk_part(const TopKLane& c, const TopKBuf* buf, int lane,
                                               float invT, float k, Mine mine) {
   const bool u0 = c.id0 >= 0 && mine(c.id0), u1 = c.id1 >= 0 && mine(c.id1);
+  const int bad = __any_sync(0xffffffffu, c.bad) ? 1 : 0;
   const float t0 = c.z0 * k, t1 = c.z1 * k;
   float M = fmaxf(u0 ? t0 : -INFINITY, u1 ? t1 : -INFINITY);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-  if (M == -INFINITY) return TopKPart{-INFINITY, 0.0f, 0.0f};
+  if (M == -INFINITY) return TopKPart{-INFINITY, 0.0f, 0.0f, bad};
   const float w0 = u0 ? ex2(t0 - M) : 0.0f, w1 = u1 ? ex2(t1 - M) : 0.0f;
   float sw = w0 + w1;
   float acc = (u0 ? w0 * fmaf(c.z0, invT, -buf->teacher[lane]) : 0.0f) +
@@ -603,7 +671,7 @@ __device__ __forceinline__ TopKPart topk_part(const TopKLane& c, const TopKBuf* 
     sw += __shfl_xor_sync(0xffffffffu, sw, o);
     acc += __shfl_xor_sync(0xffffffffu, acc, o);
   }
-  return TopKPart{M, sw, acc};
+  return TopKPart{M, sw, acc, bad};
 }
 
 // sw >= 1 (the largest candidate contributes 1), so a fast division is exact

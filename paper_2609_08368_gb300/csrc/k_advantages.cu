@@ -170,7 +170,8 @@ __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) 
     const int g = gid[i];
     if (g < 0 || g >= a.n_groups) err |= kErrGroup;
   }
-  if (tid == 0 && (cu[0] != 0 || static_cast<long long>(cu[a.n_traj]) != a.R)) err |= kErrSeqlens;
+  if (tid == 0 && (cu[0] != 0 || static_cast<long long>(cu[a.n_traj]) != a.R_total))
+    err |= kErrSeqlens;
   if (err) atomicOr(&s_err, err);
 
   // ---- group statistics: one warp per group here when there are few
@@ -213,13 +214,21 @@ __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) 
   // training tokens from 16-byte blocks of the mask and fill its row
   // advantages with 16-byte stores, with the one-sample OPD shaping. With
   // invalid row offsets every row gets advantage 0 (plus the shaping) and
-  // only N is counted, row by row.
+  // only N is counted, row by row. A shard sees the part of each trajectory
+  // that falls in its rows [row0, row0 + R) (local indices from 0); given the
+  // counts of every shard (counts_in), it takes N and the trajectories'
+  // counts from them instead of counting.
   const bool lookup = cu_ok && a.n_traj > 0;
   const bool mask_vec = (reinterpret_cast<uintptr_t>(a.mask) & 15u) == 0;
   const bool row_vec = (reinterpret_cast<uintptr_t>(ws.a_row) & 15u) == 0;
   const bool opd_vec = a.teacher && ((reinterpret_cast<uintptr_t>(a.rho) |
                                       reinterpret_cast<uintptr_t>(a.teacher)) & 15u) == 0;
   auto opd = [&](long long t) { return a.teacher ? a.opd_coef * (a.rho[t] - a.teacher[t]) : 0.0f; };
+  // trajectory i's rows in this call, as local indices [lo, hi)
+  auto local_lo = [&](int i) { return max(static_cast<long long>(cu[i]), a.row0) - a.row0; };
+  auto local_hi = [&](int i) {
+    return max(min(static_cast<long long>(cu[i + 1]), a.row0 + a.R) - a.row0, local_lo(i));
+  };
   // With fewer trajectories than warps, wpt warps share each trajectory
   // (warp `sub` of them takes every wpt-th 512-row or 128-row piece).
   const int wpt = a.n_traj > 0 ? max(1, kWarps / a.n_traj) : 1;
@@ -257,10 +266,19 @@ __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) 
     }
   };
   unsigned long long n_tok = 0;
-  if (lookup) {
+  if (lookup && a.counts_in) {
+    for (int i = tid; i < a.n_traj; i += kAdvThreads) {
+      const int c = a.counts_in[i];
+      cnt_i[i] = c;
+      n_tok += static_cast<unsigned long long>(c);
+    }
+    if (!rpp && group < traj_groups)
+      for (int i = group; i < a.n_traj; i += traj_groups) write_rows(local_lo(i), local_hi(i), a_s[i]);
+    __syncthreads();
+  } else if (lookup) {
     if (group < traj_groups) {
       for (int i = group; i < a.n_traj; i += traj_groups) {
-        const long long lo = cu[i], hi = cu[i + 1];
+        const long long lo = local_lo(i), hi = local_hi(i);
         const int c = count_rows(lo, hi);
         if (lane == 0 && c) {
           atomicAdd(&cnt_i[i], c);  // integer: exact in any order
@@ -270,6 +288,8 @@ __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) 
       }
     }
     __syncthreads();  // every trajectory's count complete
+    if (a.counts_out)
+      for (int i = tid; i < a.n_traj; i += kAdvThreads) a.counts_out[i] = cnt_i[i];
   } else {
     for (long long t = tid; t < a.R; t += kAdvThreads) {
       n_tok += a.mask[t] != 0;
@@ -314,7 +334,8 @@ __global__ void __launch_bounds__(kAdvThreads, 1) k_advantages(const AdvArgs a) 
     __syncthreads();
     if (lookup) {
       if (group < traj_groups)
-        for (int i = group; i < a.n_traj; i += traj_groups) write_rows(cu[i], cu[i + 1], a_s[i]);
+        for (int i = group; i < a.n_traj; i += traj_groups)
+          write_rows(local_lo(i), local_hi(i), a_s[i]);
     } else {
       for (long long t = tid; t < a.R; t += kAdvThreads) ws.a_row[t] = -opd(t);
     }

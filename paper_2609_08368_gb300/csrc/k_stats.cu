@@ -102,6 +102,31 @@ __device__ __forceinline__ void final_merge_shfl(Final& f, int o) {
   for (int i = 0; i < 5; ++i) f.c[i] += __shfl_xor_sync(0xffffffffu, f.c[i], o);
 }
 
+// Means over the n = c[0] training tokens; zeros when there are none.
+__device__ rl_loss_stats stats_of(const double* v, const unsigned long long* c, float rmin,
+                                  float rmax) {
+  rl_loss_stats o;
+  const unsigned long long n = c[0];
+  const double inv = n ? 1.0 / static_cast<double>(n) : 0.0;
+  o.loss = v[0] * inv;
+  o.pg_loss_mean = v[1] * inv;
+  o.kl_mean = v[2] * inv;
+  o.entropy_mean = v[3] * inv;
+  o.ratio_mean = v[4] * inv;
+  o.ratio_absdev_mean = v[5] * inv;
+  o.logprob_absdiff_mean = v[6] * inv;
+  o.corr_ratio_mean = v[7] * inv;
+  o.corr_absdev_mean = v[8] * inv;
+  o.ratio_min = n ? rmin : 0.0f;
+  o.ratio_max = n ? rmax : 0.0f;
+  o.n_tokens = static_cast<int64_t>(n);
+  o.n_clip_hi = static_cast<int64_t>(c[1]);
+  o.n_clip_lo = static_cast<int64_t>(c[2]);
+  o.n_dual_clip = static_cast<int64_t>(c[3]);
+  o.n_corr_clip = static_cast<int64_t>(c[4]);
+  return o;
+}
+
 __global__ void __launch_bounds__(kStatThreads) k_stats(const StatArgs a) {
   __shared__ Part sh[kStatThreads / 32];
   __shared__ Final shf[kStatThreads / 32];
@@ -158,32 +183,32 @@ __global__ void __launch_bounds__(kStatThreads) k_stats(const StatArgs a) {
     for (int o = 16; o > 0; o >>= 1) final_merge_shfl(fin, o);
   }
   if (threadIdx.x == 0) {
-    rl_loss_stats o;
-    const unsigned long long n = fin.c[0];
-    const double inv = n ? 1.0 / static_cast<double>(n) : 0.0;
-    o.loss = fin.v[0] * inv;
-    o.pg_loss_mean = fin.v[1] * inv;
-    o.kl_mean = fin.v[2] * inv;
-    o.entropy_mean = fin.v[3] * inv;
-    o.ratio_mean = fin.v[4] * inv;
-    o.ratio_absdev_mean = fin.v[5] * inv;
-    o.logprob_absdiff_mean = fin.v[6] * inv;
-    o.corr_ratio_mean = fin.v[7] * inv;
-    o.corr_absdev_mean = fin.v[8] * inv;
-    o.ratio_min = n ? fin.rmin : 0.0f;
-    o.ratio_max = n ? fin.rmax : 0.0f;
-    o.n_tokens = static_cast<int64_t>(n);
-    o.n_clip_hi = static_cast<int64_t>(fin.c[1]);
-    o.n_clip_lo = static_cast<int64_t>(fin.c[2]);
-    o.n_dual_clip = static_cast<int64_t>(fin.c[3]);
-    o.n_corr_clip = static_cast<int64_t>(fin.c[4]);
-    *a.out = o;
+    if (a.part_out) {
+      rl_loss_partials p;
+      for (int i = 0; i < 9; ++i) p.sum[i] = fin.v[i];
+      for (int i = 0; i < 5; ++i) p.count[i] = static_cast<double>(fin.c[i]);
+      p.max[0] = fin.c[0] ? -static_cast<double>(fin.rmin) : -INFINITY;
+      p.max[1] = fin.c[0] ? static_cast<double>(fin.rmax) : -INFINITY;
+      *a.part_out = p;
+    } else {
+      *a.out = stats_of(fin.v, fin.c, fin.rmin, fin.rmax);
+    }
     ws.hdr->ticket = 0;
   }
+}
+
+// The statistics of a sharded call from its shards' combined partials.
+__global__ void k_finish(const FinishArgs a) {
+  if (threadIdx.x != 0 || blockIdx.x != 0) return;
+  const rl_loss_partials p = *a.part;
+  unsigned long long c[5];
+  for (int i = 0; i < 5; ++i) c[i] = static_cast<unsigned long long>(p.count[i]);
+  *a.out = stats_of(p.sum, c, static_cast<float>(-p.max[0]), static_cast<float>(p.max[1]));
 }
 
 }  // namespace
 
 const void* stats_kernel() { return reinterpret_cast<const void*>(&k_stats); }
+const void* finish_kernel() { return reinterpret_cast<const void*>(&k_finish); }
 
 }  // namespace milesloss

@@ -28,8 +28,6 @@
 //           stores; the sampled token's entry is rewritten during the next
 //           row's epilogue (after a barrier that orders every store before it).
 // Definitions: Sec. 3.4 (ratio), Sec. 2 / 9.1 (advantage), Sec. 2.4 (mask).
-#include <cstdlib>
-#include <string>
 #include <type_traits>
 
 #include "common.cuh"
@@ -196,7 +194,9 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
   TopKPart* tkp = reinterpret_cast<TopKPart*>(bci + 1);         // [2] top-K parts by row parity
   uint64_t* tk_full = reinterpret_cast<uint64_t*>(tkp + 2);     // [2] part written
   uint64_t* tk_empty = tk_full + 2;                             // [2] part read
-  static_assert(2 * kMaxSlots * 8 + (kConsWarps + 3) * 16 + 2 * sizeof(TopKPart) + 4 * 8 <=
+  uint64_t* never = tk_empty + 2;                               // [1] completed by nothing (test hook)
+  volatile int* abort = reinterpret_cast<volatile int*>(never + 1);  // the CTA gave up
+  static_assert(2 * kMaxSlots * 8 + (kConsWarps + 3) * 16 + 2 * sizeof(TopKPart) + 5 * 8 + 16 <=
                     kSweepSmemExtra,
                 "k_stream scratch");
   // [2] top-K candidates of this row and the next (launched with kTopKSmem more)
@@ -211,21 +211,39 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
       mbar_init(smem_u32(&tk_full[b]), 1);
       mbar_init(smem_u32(&tk_empty[b]), 1);
     }
+    mbar_init(smem_u32(never), 1);
+    *abort = 0;
     fence_mbar_init();
   }
   __syncthreads();
 
   WsPtrs ws = a.ws;
+  uint32_t* err = &ws.hdr->err_bits;
   const char* lg = static_cast<const char*>(a.logits);
   const long long rows_mine = (a.R > blockIdx.x) ? (a.R - 1 - blockIdx.x) / gridDim.x + 1 : 0;
 
+  // Every wait below is bounded and, except the producer's waits for its own
+  // copies, also ends as soon as another party of the CTA has given up
+  // (mbar_wait_or_abort). After giving up, a party reads no ring slot it has
+  // not waited for, keeps its arrivals (so no barrier is left short of
+  // them), and the rows still to come are written as zeros.
   if (warp == kConsWarps) {
     // ------------------------------------------------------------ producer
+    // A slot is re-armed only once every reader has released the task the
+    // slot held. A reader that gave up on a wait releases its tasks without
+    // reading them, but it raised the CTA's flag before its release (the
+    // release orders that store before the arrival the producer's wait
+    // observes), so after every completed wait the producer checks the flag
+    // and, when it is up, issues nothing more: no copy is issued over one
+    // still in flight or over data still being read. Before it returns, the
+    // producer waits (bounded) for the last copy issued into each slot,
+    // timeout or not, so no bulk copy lands in this CTA's shared memory after
+    // the CTA exits.
     if (lane == 0) {
       const uint64_t pol_a = l2_policy_evict_last(), pol_b = l2_policy_evict_first();
-      bool dead = false;
+      bool stop = false;
       long long q = 0;
-      for (long long i = 0; i < rows_mine && !dead; ++i) {
+      for (long long i = 0; i < rows_mine && !stop; ++i) {
         const long long row = blockIdx.x + i * gridDim.x;
         const char* src_row = lg + row * a.ld * static_cast<long long>(sizeof(St));
         // a row that does not train has an all-zero gradient: no second read
@@ -237,11 +255,12 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
           // stay in their slots)
           const int c = (t < n_chunks) ? t : 2 * n_chunks - h - 1 - t;
           const int s = static_cast<int>(q % NS);
-          if (q >= NS &&
-              !mbar_wait_bounded(smem_u32(&empty[s]), static_cast<uint32_t>(((q / NS) - 1) & 1),
-                                 kWaitLimitNs)) {
-            dead = true;
-            atomicOr(&ws.hdr->err_bits, kErrTimeout);
+          // every reader has released the task NS back (and none gave up)
+          if (q >= NS && (!mbar_wait_or_abort(smem_u32(&empty[s]),
+                                              static_cast<uint32_t>(((q / NS) - 1) & 1),
+                                              kWaitLimitNs, abort, err) ||
+                          *abort)) {
+            stop = true;
             break;
           }
           const int v0 = cs(c);
@@ -250,17 +269,25 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
           mbar_arrive_expect_tx(bar, bytes);
           bulk_g2s(smem_u32(ring + static_cast<size_t>(s) * CB), src_row + static_cast<size_t>(v0) * 16,
                    bytes, bar, (again && t < n_chunks - h) ? pol_a : pol_b);
+          if (t == n_chunks - 1 && a.prefetch > 0 && i + 1 < rows_mine) {
+            // the row's first pass is issued: ask L2 for the head of the next
+            // row, so that HBM keeps reading while this row is merged
+            const char* nxt = src_row + gridDim.x * a.ld * static_cast<long long>(sizeof(St));
+            const uint32_t total = min(static_cast<uint32_t>(a.prefetch),
+                                       static_cast<uint32_t>(row_vec) * 16u);
+            for (uint32_t off = 0; off < total; off += 32768u)
+              bulk_prefetch_l2(nxt + off, min(32768u, total - off));
+          }
         }
       }
-      // A timeout leaves copies in flight: wait (bounded) for the last one
-      // issued into each slot before the CTA can exit.
-      if (dead) {
-        for (int s = 0; s < NS; ++s) {
-          if (q > s) {
-            const long long last = q - 1 - ((q - 1 - s) % NS);
-            mbar_wait_bounded(smem_u32(&full[s]), static_cast<uint32_t>((last / NS) & 1),
-                              kWaitLimitNs);
-          }
+      // Wait (bounded) for the last copy issued into each slot before the
+      // CTA can exit: returns at once when the readers already waited for it.
+      for (int s = 0; s < NS; ++s) {
+        if (q > s) {
+          const long long last = q - 1 - ((q - 1 - s) % NS);
+          if (!mbar_wait_bounded(smem_u32(&full[s]), static_cast<uint32_t>((last / NS) & 1),
+                                 kWaitLimitNs))
+            atomicOr(err, kErrTimeout);
         }
       }
     }
@@ -279,15 +306,11 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
     // row ahead. (A named barrier synced by both warps once per row cost
     // ~1 us per row on GB300: 6.72 against 6.26 ms on 65,536 x 154,880.) The
     // row's ids and teacher values were copied during the previous row.
-    bool tdead = false;
     auto twait = [&](long long q) {
       const int s = static_cast<int>(q % NS);
-      if (!tdead &&
-          !mbar_wait_bounded(smem_u32(&full[s]), static_cast<uint32_t>((q / NS) & 1), kWaitLimitNs)) {
-        tdead = true;
-        atomicOr(&ws.hdr->err_bits, kErrTimeout);
-      }
-      return reinterpret_cast<const uint4*>(ring + static_cast<size_t>(s) * CB);
+      const bool ok = mbar_wait_or_abort(smem_u32(&full[s]), static_cast<uint32_t>((q / NS) & 1),
+                                         kWaitLimitNs, abort, err);
+      return ok ? reinterpret_cast<const uint4*>(ring + static_cast<size_t>(s) * CB) : nullptr;
     };
     auto tarrive = [&](long long q) {
       __syncwarp();
@@ -312,7 +335,7 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
       for (int c = 0; c < n_chunks; ++c) {
         const uint4* sv = twait(q0 + c);
         const int v0 = cs(c);
-        topk_gather<In>(tk, sv, v0 * V8, (v0 + cn(c)) * V8);
+        if (sv) topk_gather<In>(tk, sv, v0 * V8, (v0 + cn(c)) * V8);
         tarrive(q0 + c);
       }
       if (tail0 < a.V)  // candidates past the last whole vector
@@ -320,12 +343,9 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
                         tail0, a.V);
       const TopKPart p = topk_part(tk, tk_row, lane, a.s.invT, k, [](int) { return true; });
       // the part of row i - 2 (same buffer) has been read
-      if (i >= 2 && !tdead &&
-          !mbar_wait_bounded(smem_u32(&tk_empty[i & 1]), static_cast<uint32_t>(((i >> 1) - 1) & 1),
-                             kWaitLimitNs)) {
-        tdead = true;
-        atomicOr(&ws.hdr->err_bits, kErrTimeout);
-      }
+      if (i >= 2)
+        mbar_wait_or_abort(smem_u32(&tk_empty[i & 1]), static_cast<uint32_t>(((i >> 1) - 1) & 1),
+                           kWaitLimitNs, abort, err);
       if (lane == 0) {
         tkp[i & 1] = p;
         mbar_arrive(smem_u32(&tk_full[i & 1]));
@@ -349,25 +369,33 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
   if (a.grad_loss_dev) g *= *a.grad_loss_dev;
   const float cscale = (N > 0) ? g / static_cast<float>(N) * a.s.invT : 0.0f;
   const float2 k2 = make_float2(k, k);
-  bool dead = false;
   // the sampled token's dLogit of the previous row, written after the next
   // barrier (so after every store of that row)
   char* fix_ptr = nullptr;
   float fix_val = 0.0f;
 
+  // Waits for task q's copy; false: this thread gave up (the CTA's flag is
+  // up). Pass A reads the slot either way (reading shared memory that a copy
+  // may still be writing is harmless, and the epilogue then writes the row
+  // as zeros); pass B writes zeros instead.
   auto wait_slot = [&](long long q) {
-    const int s = static_cast<int>(q % NS);
-    if (!dead &&
-        !mbar_wait_bounded(smem_u32(&full[s]), static_cast<uint32_t>((q / NS) & 1), kWaitLimitNs)) {
-      dead = true;
-      atomicOr(&ws.hdr->err_bits, kErrTimeout);
-    }
-    return reinterpret_cast<const uint4*>(ring + static_cast<size_t>(s) * CB);
+    return mbar_wait_or_abort(smem_u32(&full[q % NS]), static_cast<uint32_t>((q / NS) & 1),
+                              kWaitLimitNs, abort, err);
+  };
+  auto slot = [&](long long q) {
+    return reinterpret_cast<const uint4*>(ring + static_cast<size_t>(q % NS) * CB);
   };
   auto release_slot = [&](long long q) {
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_u32(&empty[q % NS]));
   };
+
+  if (a.stall_ns) {
+    // test hook: a wait on a barrier that nothing completes, before the
+    // first row; it runs out and raises the flag, so every wait after it
+    // gives up at once
+    mbar_wait_or_abort(smem_u32(never), 0u, a.stall_ns, abort, err);
+  }
 
   long long q0 = 0;  // task number of the row's first chunk (same count as the producer's)
   for (long long i = 0; i < rows_mine; ++i) {
@@ -402,36 +430,39 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
     // skipping -inf logits exactly.
     Run run;
     for (int c = 0; c < n_chunks; ++c) {
-      const uint4* sv = wait_slot(q0 + c);
+      wait_slot(q0 + c);
+      const uint4* sv = slot(q0 + c);
       const int v0 = cs(c), nv = cn(c);
-      if (tid == 0 && yv >= v0 && yv < v0 + nv) zy = In::load1(sv, y - v0 * V8);
-      if (run.r == -INFINITY && tid < nv) run.raise(In::vmax(sv[tid]) * k);
-      const Run keep = run;
-      bool redo = run.r == -INFINITY;  // no finite reference yet
-      if (!redo) {
+      {
+        if (tid == 0 && yv >= v0 && yv < v0 + nv) zy = In::load1(sv, y - v0 * V8);
+        if (run.r == -INFINITY && tid < nv) run.raise(In::vmax(sv[tid]) * k);
+        const Run keep = run;
+        bool redo = run.r == -INFINITY;  // no finite reference yet
+        if (!redo) {
 #pragma unroll 4
-        for (int v = tid; v < nv; v += kCons) {
-          float2 f[P];
-          In::unpack2(sv[v], f);
-#pragma unroll
-          for (int e = 0; e < P; ++e) run.add_pair<false>(f[e], k2, (e & 1) ? run.s1 : run.s0,
-                                                          (e & 1) ? run.u1 : run.u0);
-        }
-        const Tri cur = run.tri();
-        redo = !(fabsf(cur.s) < INFINITY) || !(fabsf(cur.u) < INFINITY);  // inf or NaN
-        if (!redo) run.rebase();
-      }
-      if (redo) {
-        typename In::MaxAcc macc = In::kMaxInit;
-        for (int v = tid; v < nv; v += kCons) macc = In::max_acc(macc, sv[v]);
-        run = keep;
-        run.raise(In::max_val(macc) * k);
-        if (run.r != -INFINITY) {
           for (int v = tid; v < nv; v += kCons) {
             float2 f[P];
             In::unpack2(sv[v], f);
 #pragma unroll
-            for (int e = 0; e < P; ++e) run.add_pair<true>(f[e], k2, run.s0, run.u0);
+            for (int e = 0; e < P; ++e) run.add_pair<false>(f[e], k2, (e & 1) ? run.s1 : run.s0,
+                                                            (e & 1) ? run.u1 : run.u0);
+          }
+          const Tri cur = run.tri();
+          redo = !(fabsf(cur.s) < INFINITY) || !(fabsf(cur.u) < INFINITY);  // inf or NaN
+          if (!redo) run.rebase();
+        }
+        if (redo) {
+          typename In::MaxAcc macc = In::kMaxInit;
+          for (int v = tid; v < nv; v += kCons) macc = In::max_acc(macc, sv[v]);
+          run = keep;
+          run.raise(In::max_val(macc) * k);
+          if (run.r != -INFINITY) {
+            for (int v = tid; v < nv; v += kCons) {
+              float2 f[P];
+              In::unpack2(sv[v], f);
+#pragma unroll
+              for (int e = 0; e < P; ++e) run.add_pair<true>(f[e], k2, run.s0, run.u0);
+            }
           }
         }
       }
@@ -472,14 +503,13 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
     // top-K OPD signal (Sec. 5.2), a fixed per-token reward: the top-K warp's
     // part of this row and the row's lse (warp 0)
     float opd = 0.0f;
+    int tk_bad = 0;
     if (kTopK && warp == 0) {
-      if (!dead &&
-          !mbar_wait_bounded(smem_u32(&tk_full[i & 1]), static_cast<uint32_t>((i >> 1) & 1),
-                             kWaitLimitNs)) {
-        dead = true;
-        atomicOr(&ws.hdr->err_bits, kErrTimeout);
+      if (mbar_wait_or_abort(smem_u32(&tk_full[i & 1]), static_cast<uint32_t>((i >> 1) & 1),
+                             kWaitLimitNs, abort, err)) {
+        opd = topk_value(tkp[i & 1], fmaf(t.m, kLn2f, logf(t.s)));
+        tk_bad = tkp[i & 1].bad;
       }
-      opd = topk_value(tkp[i & 1], fmaf(t.m, kLn2f, logf(t.s)));
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&tk_empty[i & 1]));
     }
@@ -489,8 +519,11 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
                              row * a.ld_out * static_cast<long long>(Out::kSize)
                        : nullptr;
     if (tid == 0) {
-      const bool bad = !yok;
-      if (bad) atomicOr(&ws.hdr->err_bits, kErrTarget);
+      // a row read after the CTA gave up, a bad target or a bad top-K
+      // candidate: zeros
+      const bool bad = !yok || tk_bad || *abort;
+      if (!yok) atomicOr(err, kErrTarget);
+      if (tk_bad) atomicOr(err, kErrTopK);
       const float lnS = logf(t.s);
       const float lse = fmaf(t.m, kLn2f, lnS);  // the reference is in log2 units
       float H = lnS - t.u * kLn2f / t.s;
@@ -545,11 +578,7 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
         const long long qq = (j < h) ? q0 + n_chunks - h + j : q0 + n_chunks + (j - h);
         const int nv = cn(c);
         char* dchunk = drow + static_cast<long long>(cs(c)) * V8 * Out::kSize;
-        if (ci.x) {
-          // zero gradient: the chunk's data is not needed; a training row's
-          // chunk was still copied, so its slot is waited on and released to
-          // keep the ring in step with the producer
-          if (trains) wait_slot(qq);
+        auto zero_chunk = [&]() {
           float zf[V8];
 #pragma unroll
           for (int e = 0; e < V8; ++e) zf[e] = 0.0f;
@@ -557,10 +586,22 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
             if (vec_out) Out::template storev<V8>(dchunk + static_cast<size_t>(v) * V8 * Out::kSize, zf, 0u);
             else for (int e = 0; e < V8; ++e) Out::store1(dchunk, v * V8 + e, 0.0f);
           }
+        };
+        if (ci.x) {
+          // zero gradient: the chunk's data is not needed; a training row's
+          // chunk was still copied, so its slot is waited on and released to
+          // keep the ring in step with the producer
+          if (trains) wait_slot(qq);
+          zero_chunk();
           if (trains) release_slot(qq);
           continue;
         }
-        const uint4* sv = wait_slot(qq);
+        if (!wait_slot(qq)) {  // this thread gave up: zeros, not the slot's data
+          zero_chunk();
+          release_slot(qq);
+          continue;
+        }
+        const uint4* sv = slot(qq);
         if (vec_out) {
           if (!ci.y) pass_b_chunk<In, Out, 2>(sv, nv, dchunk, k2, off2, ca2, cb2);
           else if (ci.z) pass_b_chunk<In, Out, 1>(sv, nv, dchunk, k2, off2, ca2, cb2);
@@ -613,15 +654,13 @@ const void* fn(bool topk) {
 // 0.966-0.984 against 0.939-0.959 in clusters, rows of 128-160 KB in
 // clusters 0.94-0.96 against 0.88-0.91 streamed; forward only, rows of
 // 160-310 KB streamed 0.92-1.09 against 0.78-0.88, rows of 96-128 KB in
-// clusters 0.87-0.92 against 0.79. MILESLOSS_SWEEP_KIND=stream|cluster
-// overrides the choice.
+// clusters 0.87-0.92 against 0.79. The sweep_kernel override forces either.
 constexpr long long kStreamMinRowBytes = 192 * 1024;     // fused calls
 constexpr long long kStreamMinRowBytesFwd = 160 * 1024;  // forward-only calls
 
-bool use_stream(long long row_bytes, bool in_bulk, bool grad) {
-  const char* k = std::getenv("MILESLOSS_SWEEP_KIND");
-  if (k && std::string(k) == "cluster") return false;
-  if (k && std::string(k) == "stream") return in_bulk;
+bool use_stream(long long row_bytes, bool in_bulk, bool grad, const rl_launch_overrides& ov) {
+  if (ov.sweep_kernel == 0) return false;
+  if (ov.sweep_kernel == 1) return in_bulk;
   return in_bulk && row_bytes >= (grad ? kStreamMinRowBytes : kStreamMinRowBytesFwd);
 }
 
@@ -631,31 +670,32 @@ bool use_stream(long long row_bytes, bool in_bulk, bool grad) {
 // chunks kept for pass B (0.966-0.984 of the copy peak, against 0.959-0.973
 // with two 112 KB slots); shorter rows with two 112 KB slots and the last
 // chunk kept (200 KB rows: 0.972-0.979, against 0.944 with 74 KB slots). A
-// forward-only call has no pass B: two 112 KB slots. Overridable through
-// MILESLOSS_STREAM_CHUNK / _SLOTS / _HOLD / _SPLIT.
+// forward-only call has no pass B: two 112 KB slots. The stream_* overrides
+// force a chunk size, slot count, kept chunks and split.
 constexpr long long kLongRowBytes = 240 * 1024;
 
-rl_status plan_stream(int dev, int extra, long long row_bytes, bool grad, StreamPlan* out) {
+rl_status plan_stream(int dev, int extra, long long row_bytes, bool grad,
+                      const rl_launch_overrides& ov, StreamPlan* out) {
   int optin = 0;
   if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
     return RL_ERR_CUDA;
   const bool lng = grad && row_bytes >= kLongRowBytes;
-  const int chunk = env_int("MILESLOSS_STREAM_CHUNK", lng ? 75776 : 114688);
+  const int chunk = ov.stream_chunk_bytes > 0 ? ov.stream_chunk_bytes : (lng ? 75776 : 114688);
   if (chunk < 1024 || chunk > 131072 || chunk % 128) return RL_ERR_UNSUPPORTED;
   int slots = (optin - kSweepSmemExtra - extra) / chunk;
   if (slots > kMaxSlots) slots = kMaxSlots;
-  const int forced = env_int("MILESLOSS_STREAM_SLOTS", 0);
-  if (forced) {
-    if (forced < 1 || forced > slots) return RL_ERR_UNSUPPORTED;
-    slots = forced;
+  if (ov.stream_slots > 0) {
+    if (ov.stream_slots > slots) return RL_ERR_UNSUPPORTED;
+    slots = ov.stream_slots;
   }
   if (slots < 1) return RL_ERR_UNSUPPORTED;
-  const int hold = env_int("MILESLOSS_STREAM_HOLD", lng ? 2 : 1);
-  if (hold < 0 || hold > slots) return RL_ERR_UNSUPPORTED;
+  const int hold = ov.stream_hold >= 0 ? ov.stream_hold : (lng ? 2 : 1);
+  if (hold > slots) return RL_ERR_UNSUPPORTED;
   out->chunk = chunk;
   out->slots = slots;
   out->hold = hold;
-  out->split_first = env_int("MILESLOSS_STREAM_SPLIT", lng ? 1 : 0) != 0;
+  out->split_first = ov.stream_split_first >= 0 ? ov.stream_split_first : (lng ? 1 : 0);
+  out->prefetch = ov.stream_prefetch_bytes >= 0 ? ov.stream_prefetch_bytes : 0;
   out->smem = slots * chunk + kSweepSmemExtra + extra;
   return RL_OK;
 }

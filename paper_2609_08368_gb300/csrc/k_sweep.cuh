@@ -183,11 +183,17 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
   float4* red = xch + 4 * kMaxCluster;                         // [kWarps]
   float4* bc = red + kWarps;                                   // [2]
   int4* bci = reinterpret_cast<int4*>(bc + 2);                 // [1]
+  uint64_t* never = reinterpret_cast<uint64_t*>(bci + 1);      // [1] completed by nothing (test hook)
+  volatile int* abort = reinterpret_cast<volatile int*>(never + 1);  // the CTA gave up
+  static_assert(kMaxStages * 8 + 2 * 8 + 4 * kMaxCluster * 16 + (512 / 32 + 3) * 16 + 8 + 16 <=
+                    kSweepSmemExtra,
+                "k_sweep scratch");
   // [2] top-K candidates of this row and the next (launched with kTopKSmem more)
   TopKBuf* tkb = reinterpret_cast<TopKBuf*>(smem + static_cast<size_t>(S) * a.stage_bytes +
                                             kSweepSmemExtra);
 
   WsPtrs ws = a.ws;
+  uint32_t* err = &ws.hdr->err_bits;
   const long long N = ws.hdr->n_tokens;
   float g = a.grad_loss;
   if (a.grad_loss_dev) g *= *a.grad_loss_dev;
@@ -197,6 +203,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
     for (int s = 0; s < S; ++s) mbar_init(smem_u32(&bars[s]), 1);
     mbar_init(smem_u32(&xbar[0]), 1);
     mbar_init(smem_u32(&xbar[1]), 1);
+    mbar_init(smem_u32(never), 1);
+    *abort = 0;
     fence_mbar_init();
   }
   // Peers push into this CTA's exchange slots: all barriers must be
@@ -223,7 +231,14 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
     }
   };
 
-  bool dead = false;
+  // Waits on the ring end early once any thread of the CTA has given up
+  // (mbar_wait_or_abort); thread 0 then issues no more copies, and before
+  // the CTA exits it waits (bounded) for the last copy into every stage, so
+  // no bulk copy lands after the CTA is gone. The row exchange keeps its
+  // own bounded waits (the peers' stores keep coming whatever this CTA
+  // does); after one of them runs out, this CTA leaves the exchange
+  // barriers alone.
+  bool xdead = false;
   if (tid == 0 && bulk_bytes) {
     for (int s = 0; s < S; ++s) {
       const long long row = cl_id + s * n_cl;
@@ -267,10 +282,13 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
       }
     }
 
-    if (bulk_bytes && !dead) {
-      if (!mbar_wait_bounded(smem_u32(&bars[s]), parity, kWaitLimitNs)) {
-        dead = true;
-        atomicOr(&ws.hdr->err_bits, kErrTimeout);
+    bool have = true;  // the stage holds this row's slice (or nothing is copied)
+    if (bulk_bytes) {
+      if (it == 0 && a.stall_ns) {  // test hook: a barrier that nothing completes
+        mbar_wait_or_abort(smem_u32(never), 0u, a.stall_ns, abort, err);
+        have = false;
+      } else {
+        have = mbar_wait_or_abort(smem_u32(&bars[s]), parity, kWaitLimitNs, abort, err);
       }
     }
 
@@ -281,7 +299,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
     // -inf logits exactly. Sums past 2^16 move the reference up by their
     // binary exponent (an exact rescale) before the merge.
     Tri t{-INFINITY, 0.0f, 0.0f};
-    if (tid < n_vec) {
+    if (have && tid < n_vec) {
       const float r = In::vmax(sv[tid]) * k;
       if (r != -INFINITY) {
         float su, uu;
@@ -315,10 +333,10 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
     }
     // top-K OPD candidates in this CTA's columns (warp 0): from the slice in
     // shared memory, past its whole vectors from global memory
-    TopKPart tkp{-INFINITY, 0.0f, 0.0f};
+    TopKPart tkp{-INFINITY, 0.0f, 0.0f, 0};
     if (topk && tid < 32) {
       TopKLane tk = topk_ids(tk_row, a.V, a.s.topk, tid);
-      topk_gather<In>(tk, sb, lo, lo + vec_elems);
+      if (have) topk_gather<In>(tk, sb, lo, lo + vec_elems);
       topk_gather<In>(tk, grow + static_cast<size_t>(vec_elems) * sizeof(St), lo + vec_elems, lo + cnt);
       const int c0 = lo, c1 = lo + cnt;
       tkp = topk_part(tk, tk_row, tid, a.s.invT, k, [c0, c1](int id) { return id >= c0 && id < c1; });
@@ -334,7 +352,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
       float zy = 0.0f;
       if (owner == crank) {
         const int jl = y - lo;
-        zy = (jl < vec_elems) ? In::load1(sb, jl) : In::load1(grow, jl);
+        zy = (jl < vec_elems) ? (have ? In::load1(sb, jl) : 0.0f) : In::load1(grow, jl);
       }
       const int slot = static_cast<int>(it & 1);
       const float4 mine = make_float4(t.m, t.s, t.u, zy);
@@ -352,10 +370,13 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
           st_async_f4(mapa_shared(xaddr, r), mine, mapa_shared(xb, r));
           if (topk) st_async_f4(mapa_shared(taddr, r), mine_tk, mapa_shared(xb, r));
         }
-        mbar_arrive_expect_tx(xb, static_cast<uint32_t>(C - 1) * (topk ? 32u : 16u));
-        if (!dead && !mbar_wait_bounded(xb, static_cast<uint32_t>((it >> 1) & 1), kWaitLimitNs)) {
-          dead = true;
-          atomicOr(&ws.hdr->err_bits, kErrTimeout);
+        if (!xdead) {
+          mbar_arrive_expect_tx(xb, static_cast<uint32_t>(C - 1) * (topk ? 32u : 16u));
+          if (!mbar_wait_bounded(xb, static_cast<uint32_t>((it >> 1) & 1), kWaitLimitNs)) {
+            xdead = true;
+            *abort = 1;
+            atomicOr(err, kErrTimeout);
+          }
         }
         float M = -INFINITY;
         for (int r = 0; r < C; ++r) M = fmaxf(M, xs[r].x);
@@ -369,12 +390,19 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
           }
           if (r == owner) zy_all = e.w;
         }
-        if (topk) tkp = topk_merge_all(xt, C);  // the CTAs' top-K parts
+        if (topk) {  // the CTAs' top-K parts (every CTA read the same ids)
+          const int tk_bad = tkp.bad;
+          tkp = topk_merge_all(xt, C);
+          tkp.bad = tk_bad;
+        }
       }
     }
     if (tid == 0) {
-      const bool bad = !yok;
-      if (bad) atomicOr(&ws.hdr->err_bits, kErrTarget);
+      // a row read after the CTA gave up, a bad target or a bad top-K
+      // candidate: zeros
+      const bool bad = !yok || (topk && tkp.bad) || *abort;
+      if (!yok && crank == 0) atomicOr(err, kErrTarget);
+      if (topk && tkp.bad && crank == 0) atomicOr(err, kErrTopK);
       const float lnS = logf(tot.s);
       const float lse = fmaf(tot.m, kLn2, lnS);  // the reference is in log2 units
       float H = lnS - tot.u * kLn2 / tot.s;
@@ -487,7 +515,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
     }
 
     // Refill this stage with the row S iterations ahead.
-    if (tid == 0 && bulk_bytes && !dead) {
+    if (tid == 0 && bulk_bytes && !*abort) {
       const long long nrow = row + S * n_cl;
       if (nrow < a.R) {
         fence_proxy_async_smem();
@@ -496,12 +524,13 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
     }
   }
 
-  // Copies issued but never waited on exist only after a timeout: wait
-  // (bounded) for the last copy into every stage before leaving.
-  if (dead && tid == 0) {
+  // Wait (bounded) for the last copy into every stage before leaving: at
+  // once unless the CTA gave up with copies in flight.
+  if (tid == 0) {
     for (int s = 0; s < S; ++s)
-      if (iss_any & (1u << s))
-        mbar_wait_bounded(smem_u32(&bars[s]), ((iss_par >> s) & 1u) ^ 1u, kWaitLimitNs);
+      if ((iss_any & (1u << s)) &&
+          !mbar_wait_bounded(smem_u32(&bars[s]), ((iss_par >> s) & 1u) ^ 1u, kWaitLimitNs))
+        atomicOr(err, kErrTimeout);
   }
   // No CTA leaves while a peer's last exchange store into it may be in flight.
   if (C > 1) cluster_sync_all();

@@ -44,6 +44,10 @@ struct SweepArgs {
   const float* grad_loss_dev;
   LossScalars s;
   WsPtrs ws;
+  // Test hook (0 = off): the first wait of every CTA waits instead on a
+  // barrier nothing completes, bounded by this many nanoseconds, so that the
+  // timeout path runs (see rl_launch_overrides).
+  unsigned long long stall_ns;
 };
 
 struct StreamArgs {
@@ -54,6 +58,7 @@ struct StreamArgs {
   int n_slots;      // ring depth
   int n_hold;       // last chunks of a row that pass B reads from shared memory (<= n_slots)
   int split_first;  // 1: the first chunk takes the ragged remainder (rounded up to 128 bytes)
+  int prefetch;     // bytes of the next row to ask L2 for once a row's first pass is issued
   int out_vec;      // dLogits rows are 16-byte aligned: vector stores
   const int* targets;
   const float* rho;
@@ -68,10 +73,16 @@ struct StreamArgs {
   const float* grad_loss_dev;
   LossScalars s;
   WsPtrs ws;
+  unsigned long long stall_ns;  // test hook, as in SweepArgs (the consumers' first wait)
 };
 
 struct AdvArgs {
-  long long R;
+  long long R;          // rows of this call (the local rows of a shard)
+  long long row0;       // global index of local row 0 (0 unless sharded)
+  long long R_total;    // rows of the whole call: cu_seqlens ends here (R unless sharded)
+  const int* counts_in; // sharded calls: every trajectory's training tokens over all
+                        // shards (then N and the per-trajectory counts come from these)
+  int* counts_out;      // sharded calls: this shard's training tokens per trajectory
   int n_traj, n_groups;
   const float* rewards;
   const int* gid;
@@ -105,7 +116,13 @@ struct StatArgs {
   const uint8_t* mask;
   const float* rho;
   rl_loss_stats* out;
+  rl_loss_partials* part_out;  // a shard: its partial sums instead of the statistics
   WsPtrs ws;
+};
+
+struct FinishArgs {
+  const rl_loss_partials* part;
+  rl_loss_stats* out;
 };
 
 struct BwdArgs {
@@ -134,23 +151,23 @@ const void* sweep_kernel(rl_dtype in, rl_dtype out, bool grad, int threads, bool
 const void* sweep_kernel_topk(rl_dtype in, rl_dtype out, bool grad, int threads);
 const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad, bool topk);
 
-// An integer from the environment (tuning overrides), or dflt.
-inline int env_int(const char* name, int dflt) {
-  const char* v = std::getenv(name);
-  if (!v || !*v) return dflt;
-  return std::atoi(v);
-}
+// The process-wide launch-plan overrides set by rl_set_launch_overrides (a
+// copy; every field -1 when none are set).
+rl_launch_overrides current_overrides();
+// The status a workspace's error bits report: the lowest recorded code.
+rl_status status_of_bits(uint32_t bits);
 
 // The streaming kernel's launch plan (defined beside the kernel, k_stream.cu):
 // whether rows of row_bytes go to it, and its ring of shared-memory slots.
 struct StreamPlan {
-  int chunk, slots, hold, split_first, smem;
+  int chunk, slots, hold, split_first, prefetch, smem;
 };
-bool use_stream(long long row_bytes, bool in_bulk, bool grad);
+bool use_stream(long long row_bytes, bool in_bulk, bool grad, const rl_launch_overrides& ov);
 // extra: shared memory beyond the ring and the fixed scratch (kTopKSmem with
 // top-K OPD on, else 0); the ring's shape depends on the row length and on
 // whether the call writes dLogits
-rl_status plan_stream(int dev, int extra, long long row_bytes, bool grad, StreamPlan* out);
+rl_status plan_stream(int dev, int extra, long long row_bytes, bool grad,
+                      const rl_launch_overrides& ov, StreamPlan* out);
 const void* bwd_kernel(rl_dtype in, rl_dtype out);
 const void* adv_kernel();
 const void* groups_kernel();  // one 32-thread block per group (grid-stride)
@@ -160,5 +177,6 @@ constexpr int kMaxGroupBlocks = 65535;
 constexpr int kInlineGroups = 8;
 const void* seq_kernel();
 const void* stats_kernel();
+const void* finish_kernel();  // rl_loss_stats from combined partials (one thread)
 
 }  // namespace milesloss

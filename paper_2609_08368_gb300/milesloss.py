@@ -17,6 +17,9 @@ from . import build as _build
 RL_OK = 0
 RL_BF16, RL_F32 = 0, 1
 RL_PHASE_BEGIN, RL_PHASE_ROWS, RL_PHASE_END, RL_PHASE_ALL = 1, 2, 4, 7
+RL_SHARD_COUNT, RL_SHARD_SWEEP, RL_SHARD_FINISH = 1, 2, 4
+PARTIALS_SUMS = 14   # rl_loss_partials: sum[9] and count[5], combined by addition
+PARTIALS_DOUBLES = 16  # ... then max[2], combined by maximum
 CORRECTIONS = {"none": 0, "tis": 1, "clip_or_pop": 2}
 ESTIMATORS = {"grpo": 0, "reinforcepp": 1, "reinforcepp_baseline": 2, "gspo": 3}
 STATS_BYTES = 128
@@ -60,6 +63,25 @@ def make_params(temperature=1.0, eps_lo=0.2, eps_hi=0.2, dual_clip_c=0.0, kl_coe
                         None if opd_topk_teacher is None else opd_topk_teacher.data_ptr())
 
 
+class RlLaunchOverrides(ctypes.Structure):
+    _fields_ = [
+        ("sweep_kernel", ctypes.c_int32),
+        ("cluster_size", ctypes.c_int32),
+        ("cluster_stages", ctypes.c_int32),
+        ("cluster_threads", ctypes.c_int32),
+        ("cluster_ctas_per_sm", ctypes.c_int32),
+        ("stream_chunk_bytes", ctypes.c_int32),
+        ("stream_slots", ctypes.c_int32),
+        ("stream_hold", ctypes.c_int32),
+        ("stream_split_first", ctypes.c_int32),
+        ("stream_prefetch_bytes", ctypes.c_int32),
+        ("stall_first_wait_ns", ctypes.c_int64),
+    ]
+
+
+SWEEP_KERNELS = {"cluster": 0, "stream": 1}
+
+
 class MilesLossError(RuntimeError):
     def __init__(self, status: int, where: str):
         super().__init__(f"{where}: {status_string(status)} (status {status})")
@@ -98,8 +120,16 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
     lib.rl_status_string.argtypes = [I32]
     lib.rl_status_string.restype = ctypes.c_char_p
     lib.rl_set_sweep_events.argtypes = [P, P]
+    lib.rl_launch_overrides_init.argtypes = [ctypes.POINTER(RlLaunchOverrides)]
+    lib.rl_set_launch_overrides.argtypes = [ctypes.POINTER(RlLaunchOverrides)]
+    lib.rl_loss_fwd_bwd_noalloc.argtypes = fwd_common + [F32, P, P, I32, I64, P]
+    lib.rl_loss_shard_fwd_bwd.argtypes = ([I32, I64, I64] + fwd_common[:-1] + [P, P, P] +
+                                          [F32, P, P, I32, I64, P, SZ, P])
+    lib.rl_loss_noalloc_check_device_error.argtypes = []
     for name in ("rl_loss_workspace_size", "rl_loss_fwd", "rl_loss_fwd_bwd", "rl_loss_fwd_bwd_rows",
-                 "rl_loss_bwd",
+                 "rl_loss_bwd", "rl_loss_fwd_bwd_noalloc", "rl_loss_noalloc_check_device_error",
+                 "rl_loss_shard_fwd_bwd",
+                 "rl_launch_overrides_init", "rl_set_launch_overrides",
                  "rl_loss_check_device_error", "rl_set_sweep_events", "rl_loss_abi_version"):
         getattr(lib, name).restype = ctypes.c_int32
     _lib = lib
@@ -227,6 +257,90 @@ def rl_loss_bwd(logits, targets, loss_mask, params, workspace, dlogits, grad_los
 
 def rl_loss_check_device_error(workspace) -> int:
     return int(load().rl_loss_check_device_error(_ptr(workspace)))
+
+
+def set_launch_overrides(**fields) -> None:
+    """Install process-wide launch-plan overrides (rl_set_launch_overrides);
+    no arguments removes them. ``sweep_kernel`` may be given as "cluster" or
+    "stream"; any other field as in the header."""
+    lib = load()
+    if not fields:
+        _check(lib.rl_set_launch_overrides(None), "rl_set_launch_overrides")
+        return
+    o = RlLaunchOverrides()
+    _check(lib.rl_launch_overrides_init(ctypes.byref(o)), "rl_launch_overrides_init")
+    for k, v in fields.items():
+        if k == "sweep_kernel" and isinstance(v, str):
+            v = SWEEP_KERNELS[v]
+        if not hasattr(o, k):
+            raise TypeError(f"unknown launch override {k!r}")
+        setattr(o, k, int(v))
+    _check(lib.rl_set_launch_overrides(ctypes.byref(o)), "rl_set_launch_overrides")
+
+
+class launch_overrides:
+    """Context manager: the given overrides while the block runs, none after."""
+
+    def __init__(self, **fields):
+        self.fields = fields
+
+    def __enter__(self):
+        set_launch_overrides(**self.fields)
+        return self
+
+    def __exit__(self, *exc):
+        set_launch_overrides()
+        return False
+
+
+def rl_loss_fwd_bwd_noalloc(logits, targets, rollout_logprobs, ref_logprobs, old_logprobs,
+                            teacher_logprobs, rewards, group_id, cu_seqlens, n_groups, loss_mask,
+                            params, token_logprobs, entropy, advantages, group_sizes, stats,
+                            dlogits, grad_loss=1.0, grad_loss_device=None, vocab=None,
+                            stream=None):
+    """rl_loss_fwd_bwd without a workspace (the library's fixed array)."""
+    args = _fwd_args(logits, vocab, targets, rollout_logprobs, ref_logprobs, old_logprobs,
+                     teacher_logprobs, rewards, group_id, cu_seqlens, n_groups, loss_mask, params,
+                     token_logprobs, entropy, advantages, group_sizes, stats)
+    _check(load().rl_loss_fwd_bwd_noalloc(*args, float(grad_loss), _ptr(grad_loss_device),
+                                          _ptr(dlogits), _dtype_code(dlogits),
+                                          int(dlogits.stride(0)), _stream(stream)),
+           "rl_loss_fwd_bwd_noalloc")
+
+
+def rl_loss_shard_fwd_bwd(phase, row_offset, n_rows_total, logits, targets, rollout_logprobs,
+                          ref_logprobs, old_logprobs, teacher_logprobs, rewards, group_id,
+                          cu_seqlens, n_groups, loss_mask, params, token_logprobs, entropy,
+                          advantages, group_sizes, traj_counts, partials, stats, dlogits,
+                          workspace, vocab, n_rows=None, logits_dtype=None, grad_loss=1.0,
+                          grad_loss_device=None, stream=None):
+    """One phase of a shard's part of a row-sharded call. Per-row tensors
+    hold the shard's rows; ``traj_counts`` is int32 [n_traj] and
+    ``partials`` float64 [16] (one rl_loss_partials), both on the device."""
+    import torch
+    n_traj = int(rewards.shape[0]) if rewards is not None else 0
+    if logits is not None:
+        ldt, ld, R = _dtype_code(logits), int(logits.stride(0)), int(logits.shape[0])
+    else:
+        ldt = _dtype_code(torch.empty(0, dtype=logits_dtype or torch.bfloat16))
+        ld, R = int(vocab), int(n_rows if n_rows is not None else targets.shape[0])
+    if dlogits is not None:
+        ddt, ld_out = _dtype_code(dlogits), int(dlogits.stride(0))
+    else:
+        ddt, ld_out = ldt, int(vocab)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(load().rl_loss_shard_fwd_bwd(
+        int(phase), int(row_offset), int(n_rows_total), _ptr(logits), ldt, R, int(vocab), ld,
+        _ptr(targets), _ptr(rollout_logprobs), _ptr(ref_logprobs), _ptr(old_logprobs),
+        _ptr(teacher_logprobs), _ptr(rewards), _ptr(group_id), _ptr(cu_seqlens), n_traj,
+        int(n_groups), _ptr(loss_mask), ctypes.byref(_params(params)), _ptr(token_logprobs),
+        _ptr(entropy), _ptr(advantages), _ptr(group_sizes), _ptr(traj_counts), _ptr(partials),
+        _ptr(stats), float(grad_loss), _ptr(grad_loss_device), _ptr(dlogits), ddt, ld_out,
+        _ptr(workspace), ws_bytes, _stream(stream)), "rl_loss_shard_fwd_bwd")
+
+
+def rl_loss_noalloc_check_device_error() -> int:
+    return int(load().rl_loss_noalloc_check_device_error())
 
 
 def rl_set_sweep_events(begin=None, end=None):
