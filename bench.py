@@ -49,7 +49,8 @@ def parse_args():
     ap.add_argument("--workload", default="glm")
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--e2e-chunk-rows", type=int, default=4096)
-    ap.add_argument("--cpu-sample-rows", type=int, default=3072)
+    ap.add_argument("--cpu-sample-rows", type=int, default=0,
+                    help="time the CPU oracle on this many random rows (0: on every row)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--n-prompts", type=int, default=None,
@@ -239,21 +240,48 @@ def algorithmic_bytes_per_row(w, dl_dtype) -> int:
 
 # ---------------------------------------------------------------- CPU oracle
 
+def _widen_host(a: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns (uint16) or fp32 values as float64."""
+    if a.dtype == np.uint16:
+        return (a.astype(np.uint32) << np.uint32(16)).view(np.float32).astype(np.float64)
+    return a.astype(np.float64)
+
+
 def _oracle_rows_task(task):
-    """One block of sampled rows through the float64 oracle, in a worker
-    process (spawned; it attaches to the parent's shared logits)."""
+    """One block of rows through the float64 oracle, in a worker process
+    (spawned; it attaches to the parent's shared copy of the rows' logits,
+    and of the GPU's dLogits of those rows when it is to compare them).
+    Returns the rows' log-probs, entropies and lse, and for dLogits the count
+    of entries outside 1e-2 relative / 1e-5 absolute and the largest
+    error-to-bound ratio."""
     from multiprocessing import shared_memory
 
     import oracle
 
-    (shm_name, shape, dtype, lo, hi, y, rho, q, A_row, mask, N, params) = task
-    shm = shared_memory.SharedMemory(name=shm_name)
+    (shm_z, shm_dl, shape, zdtype, dldtype, lo, hi, y, rho, q, old, A_row, mask, N, params,
+     grad_loss) = task
+    hz = shared_memory.SharedMemory(name=shm_z)
+    hd = shared_memory.SharedMemory(name=shm_dl) if shm_dl else None
     try:
-        z = np.ndarray(shape, dtype=dtype, buffer=shm.buf)[lo:hi]
-        oracle.rl_loss_rows(z, y, rho, q, A_row, mask, N, oracle.LossParams(**params))
+        z = np.ndarray(shape, dtype=zdtype, buffer=hz.buf)[lo:hi]
+        o = oracle.rl_loss_rows(z, y, rho, q, A_row, mask, N, oracle.LossParams(**params),
+                                grad_loss=grad_loss, old=old)
+        out = dict(lo=lo, logp=o["logp"], H=o["H"], lse=o["lse"], n_bad=0, worst=0.0,
+                   worst_at=None)
+        if hd is not None:
+            got = _widen_host(np.ndarray(shape, dtype=dldtype, buffer=hd.buf)[lo:hi])
+            ref = o["dlogits"]
+            ratio = np.abs(got - ref) / np.maximum(1e-2 * np.abs(ref), 1e-5)
+            ratio[~np.isfinite(got)] = np.inf
+            out["n_bad"] = int((ratio > 1.0).sum())
+            i = np.unravel_index(int(np.argmax(ratio)), ratio.shape)
+            out["worst"] = float(ratio[i])
+            out["worst_at"] = (lo + int(i[0]), int(i[1]), float(got[i]), float(ref[i]))
     finally:
-        shm.close()
-    return hi - lo
+        hz.close()
+        if hd is not None:
+            hd.close()
+    return out
 
 
 def _oracle_worker_init():
@@ -267,8 +295,8 @@ def _oracle_worker_init():
 
 class OraclePool:
     """A pool of spawned worker processes, one per host core this process
-    may run on, that time the oracle on blocks of sampled rows. Started
-    before any sampling, so that no fork follows CUDA initialisation."""
+    may run on, that run the oracle on blocks of rows (spawned, so it may be
+    started after CUDA initialisation)."""
 
     def __init__(self, workers: int | None = None):
         import multiprocessing as mp
@@ -277,12 +305,17 @@ class OraclePool:
         self.pool = (mp.get_context("spawn").Pool(self.workers, initializer=_oracle_worker_init)
                      if self.workers > 1 else None)
         if self.pool is not None:
-            try:  # workers up and importing done; if they cannot start, time in this process
+            try:  # workers up and importing done; if they cannot start, run in this process
                 self.pool.map_async(int, range(self.workers)).get(timeout=300)
             except Exception:  # noqa: BLE001
                 self.pool.terminate()
                 self.pool.join()
                 self.pool, self.workers = None, 1
+
+    def map(self, fn, tasks):
+        if self.pool is None:
+            return [fn(t) for t in tasks]
+        return self.pool.map(fn, tasks, chunksize=1)
 
     def close(self):
         if self.pool is not None:
@@ -290,61 +323,111 @@ class OraclePool:
             self.pool.join()
 
 
-def oracle_sample(w, n_rows: int, seed: int = 7, pool: "OraclePool | None" = None):
-    """Times the float64 CPU oracle on ``n_rows`` rows of the workload (every
-    per-row output and dLogits of those rows, with the call-wide advantages
-    and token count of the whole batch), on the pool's worker processes (one
-    per core) or in this process. Returns (rows/s, seconds, rows, cores)."""
+def _host_rows(t, rows):
+    """Rows of a device tensor as a host numpy array (bf16 as uint16 bits)."""
+    z = t[rows].cpu()
+    if z.dtype == torch.bfloat16:
+        return z.contiguous().view(torch.int16).numpy().view(np.uint16)
+    return z.contiguous().numpy()
+
+
+def oracle_rows(w, pool: OraclePool, rows=None, dlogits=None, grad_loss=1.0, block=2048,
+                task_rows=32):
+    """The float64 oracle over rows of a token-level workload (every row by
+    default), with the call-wide advantages and N of the whole batch: the
+    rows' log-probs, entropies and lse, and dLogits of every row computed
+    (and, when the GPU's ``dlogits`` are given, compared entry by entry in
+    the workers). The logits (and dLogits) go to the workers a block of rows
+    at a time through shared memory. Returns a dict with the per-row arrays,
+    the dLogits check, and ``seconds``: the wall time of the oracle's work
+    (the blocks' host copies excluded)."""
     import oracle
+    from multiprocessing import shared_memory
 
     p = oracle.LossParams(**w.params)
-    rng = np.random.default_rng(seed)
-    rows = np.sort(rng.choice(w.n_rows, size=min(n_rows, w.n_rows), replace=False))
-    idx = torch.from_numpy(rows).to(w.logits.device)
-    z = w.logits[idx, :w.vocab].cpu()
-    z = z.view(torch.int16).numpy().view(np.uint16) if z.dtype == torch.bfloat16 else z.numpy()
 
     def host(t):
         return None if t is None else t.cpu().numpy()
 
-    mask = host(w.loss_mask)
-    y, rho = host(w.targets)[rows], host(w.rollout_logprobs)[rows]
-    q = None if w.ref_logprobs is None else host(w.ref_logprobs)[rows]
-    block = 32
-    if pool is None or pool.pool is None:
-        t0 = time.perf_counter()
-        A, _ = oracle.group_advantages(host(w.rewards), host(w.group_id), w.n_groups, p)
-        A_row = oracle.row_advantages(A, host(w.cu_seqlens), w.n_rows)
-        N = int(mask.astype(bool).sum())
-        for lo in range(0, len(rows), block):
-            hi = min(len(rows), lo + block)
-            oracle.rl_loss_rows(z[lo:hi], y[lo:hi], rho[lo:hi], None if q is None else q[lo:hi],
-                                A_row[rows[lo:hi]], mask[rows[lo:hi]].astype(bool), N, p)
-        dt = time.perf_counter() - t0
-        return len(rows) / dt, dt, len(rows), 1
-    from multiprocessing import shared_memory
-
-    shm = shared_memory.SharedMemory(create=True, size=max(1, z.nbytes))
+    R = w.n_rows
+    rows = np.arange(R) if rows is None else np.asarray(rows)
+    mask = host(w.loss_mask).astype(bool)
+    _, A_row, _ = oracle.estimator_advantages(host(w.rewards), host(w.group_id), w.n_groups,
+                                              host(w.cu_seqlens), mask, p)
+    N = int(mask.sum())
+    y, rho = host(w.targets), host(w.rollout_logprobs)
+    q, old = host(w.ref_logprobs), host(w.old_logprobs)
+    es = w.logits.element_size()
+    blk = min(block, len(rows)) if len(rows) else 1
+    hz = shared_memory.SharedMemory(create=True, size=max(1, blk * w.vocab * es))
+    hd = None
+    if dlogits is not None:
+        hd = shared_memory.SharedMemory(create=True,
+                                        size=max(1, blk * w.vocab * dlogits.element_size()))
+    out = dict(logp=np.zeros(len(rows)), H=np.zeros(len(rows)), lse=np.zeros(len(rows)),
+               n_bad=0, worst=0.0, worst_at=None, seconds=0.0, rows=rows, N=N, A_row=A_row)
     try:
-        zs = np.ndarray(z.shape, dtype=z.dtype, buffer=shm.buf)
-        zs[:] = z
-        t0 = time.perf_counter()
-        A, _ = oracle.group_advantages(host(w.rewards), host(w.group_id), w.n_groups, p)
-        A_row = oracle.row_advantages(A, host(w.cu_seqlens), w.n_rows)
-        N = int(mask.astype(bool).sum())
-        tasks = [(shm.name, z.shape, z.dtype, lo, min(len(rows), lo + block),
-                  y[lo:lo + block], rho[lo:lo + block], None if q is None else q[lo:lo + block],
-                  A_row[rows[lo:lo + block]], mask[rows[lo:lo + block]].astype(bool), N,
-                  dict(w.params))
-                 for lo in range(0, len(rows), block)]
-        done = sum(pool.pool.map(_oracle_rows_task, tasks, chunksize=1))
-        dt = time.perf_counter() - t0
-        del zs
+        for b0 in range(0, len(rows), blk):
+            sel = rows[b0:b0 + blk]
+            n = len(sel)
+            idx = torch.from_numpy(sel).to(w.logits.device)
+            z = _host_rows(w.logits[:, :w.vocab], idx)
+            zs = np.ndarray(z.shape, dtype=z.dtype, buffer=hz.buf)
+            zs[:] = z
+            dl_dtype = None
+            if hd is not None:
+                d = _host_rows(dlogits[:, :w.vocab], idx)
+                ds = np.ndarray(d.shape, dtype=d.dtype, buffer=hd.buf)
+                ds[:] = d
+                dl_dtype = d.dtype
+                del ds
+            del zs
+            tasks = []
+            for lo in range(0, n, task_rows):
+                hi = min(n, lo + task_rows)
+                r = sel[lo:hi]
+                tasks.append((hz.name, None if hd is None else hd.name, z.shape, z.dtype, dl_dtype,
+                              lo, hi, y[r], rho[r], None if q is None else q[r],
+                              None if old is None else old[r], A_row[r], mask[r], N,
+                              dict(w.params), grad_loss))
+            t0 = time.perf_counter()
+            res = pool.map(_oracle_rows_task, tasks)
+            out["seconds"] += time.perf_counter() - t0
+            for o in res:
+                lo = b0 + o["lo"]
+                k = len(o["logp"])
+                for key in ("logp", "H", "lse"):
+                    out[key][lo:lo + k] = o[key]
+                out["n_bad"] += o["n_bad"]
+                if o["worst"] > out["worst"] or out["worst_at"] is None:
+                    out["worst"] = o["worst"]
+                    if o["worst_at"] is not None:
+                        r0, col, g_, r_ = o["worst_at"]  # r0: the row within the block
+                        out["worst_at"] = (int(sel[r0]), col, g_, r_)
     finally:
-        shm.close()
-        shm.unlink()
-    assert done == len(rows)
-    return len(rows) / dt, dt, len(rows), pool.workers
+        hz.close()
+        hz.unlink()
+        if hd is not None:
+            hd.close()
+            hd.unlink()
+    return out
+
+
+def oracle_sample(w, n_rows: int, seed: int = 7, pool: "OraclePool | None" = None):
+    """Times the float64 CPU oracle on ``n_rows`` random rows of the workload
+    (every per-row output and dLogits of those rows, with the call-wide
+    advantages and token count of the whole batch) on the pool's worker
+    processes. Returns (rows/s, seconds, rows, cores)."""
+    rng = np.random.default_rng(seed)
+    rows = np.sort(rng.choice(w.n_rows, size=min(n_rows, w.n_rows), replace=False))
+    own = pool is None
+    pool = pool or OraclePool(workers=1)
+    try:
+        o = oracle_rows(w, pool, rows=rows)
+    finally:
+        if own:
+            pool.close()
+    return len(rows) / o["seconds"], o["seconds"], len(rows), pool.workers
 
 
 def run_reference(args, rank, world):
@@ -402,6 +485,45 @@ def _pinned_copy(w):
                        pin(w.ref_logprobs), pin(w.old_logprobs), pin(w.teacher_logprobs),
                        pin(w.rewards), pin(w.group_id), pin(w.cu_seqlens), pin(w.loss_mask),
                        w.n_groups, dict(w.params))
+
+
+def copy_floor_ms(call, stream, steps: int) -> float:
+    """Milliseconds per step of the pipelined call's logits and dLogits
+    copies alone: per chunk of rows, the host-to-device copy of its logits on
+    the input stream and the device-to-host copy of a dLogits buffer of the
+    same rows on the output stream (after that chunk's input copy, as if the
+    sweep took no time), through the call's own device buffers, so both
+    directions run at once as in the call. What the call takes beyond this
+    is what the sweep and the small copies add."""
+    h = call.host
+    R, V = h.n_rows, h.vocab
+
+    def one():
+        out_done = None
+        for i, r0 in enumerate(range(0, R, call.chunk)):
+            r1 = min(R, r0 + call.chunk)
+            b, n = i % 2, r1 - r0
+            with torch.cuda.stream(call.s_in):
+                call.lg[b][:n].copy_(h.logits[r0:r1, :V], non_blocking=True)
+                in_done = torch.cuda.Event()
+                in_done.record(call.s_in)
+            call.s_out.wait_event(in_done)
+            with torch.cuda.stream(call.s_out):
+                call.out["dlogits"][r0:r1].copy_(call.dl[b][:n], non_blocking=True)
+                out_done = torch.cuda.Event()
+                out_done.record(call.s_out)
+        if out_done is not None:
+            stream.wait_event(out_done)
+
+    one()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        one()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / steps
 
 
 def run_ours(args, rank, world, local):
@@ -497,19 +619,27 @@ def run_ours(args, rank, world, local):
     step_gbs = launch_bytes / (ms_step / 1e3) / 1e9
 
     cpu = None
-    # (the sampled-row oracle timing covers the token-level estimators
-    # without top-K OPD only)
+    # (the oracle's row pass covers the token-level estimators without
+    # top-K OPD only)
     if rank == 0 and world == 1 and not args.no_cpu_baseline and \
             w.params.get("estimator", "grpo") != "gspo" and not args.opd_topk:
         pool = OraclePool()
         try:
-            rps, secs, n, cores = oracle_sample(w, args.cpu_sample_rows, pool=pool)
+            if args.cpu_sample_rows > 0:
+                rps, secs, n, cores = oracle_sample(w, args.cpu_sample_rows, pool=pool)
+                what = f"{n} random rows of the {R} x {V} batch"
+            else:
+                o = oracle_rows(w, pool)
+                n, secs, cores = R, o["seconds"], pool.workers
+                rps = R / secs
+                what = f"all {R} rows of the {R} x {V} batch"
         finally:
             pool.close()
         cpu = {"value": rps, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-               "sample": f"{n} random rows of the {R} x {V} batch (every per-row output and "
-                         f"dLogits of those rows; call-wide advantages and N), {secs:.1f} s "
-                         f"wall on {cores} worker processes"}
+               "sample": f"{what} (every per-row output and dLogits of every row, with the "
+                         f"call-wide advantages and N), {secs:.1f} s wall of oracle work on "
+                         f"{cores} worker processes (the logits reach them through shared "
+                         f"memory a block of rows at a time; those copies are not timed)"}
 
     # end to end through host buffers (pinned), one call per step
     e2e = None
@@ -530,11 +660,17 @@ def run_ours(args, rank, world, local):
         torch.cuda.synchronize()
         barrier(world)
         ms_e2e = max_over_ranks(e0.elapsed_time(e1), world) / args.e2e_steps
+        floor_ms = copy_floor_ms(call, stream, args.e2e_steps)
         e2e = {"value": rows_all / (ms_e2e / 1e3), "unit": "tokens/s",
                "ms_per_step": ms_e2e, "steps": args.e2e_steps,
                "how": f"pinned host buffers, rl_loss_fwd_bwd_rows over chunks of "
                       f"{args.e2e_chunk_rows} rows, copies overlapped with the sweep",
-               "h2d_bytes_per_step": call.bytes_in(), "d2h_bytes_per_step": call.bytes_out()}
+               "h2d_bytes_per_step": call.bytes_in(), "d2h_bytes_per_step": call.bytes_out(),
+               "copy_floor_ms": floor_ms, "frac_of_copy_floor": floor_ms / ms_e2e,
+               "copy_floor_how": "the same logits and dLogits bytes copied alone on this box, "
+                                 "in the same chunks, through the same two device buffers and "
+                                 "copy streams, host-to-device and device-to-host at once "
+                                 "(no sweep)"}
         del call, host_w
 
     # the committed capture is of the default path (GRPO-style fused sweep,

@@ -42,13 +42,13 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert lib.rl_loss_abi_version() == 100
+    assert lib.rl_loss_abi_version() == 110
     seen = set()
-    for code in range(0, 9):
+    for code in range(0, 10):
         s = ml.status_string(code)
         assert s and s != "unknown status"
         seen.add(s)
-    assert len(seen) == 9
+    assert len(seen) == 10
     assert ml.status_string(99) == "unknown status"
 
 
@@ -128,7 +128,6 @@ INVALID = [
     dict(params=dict(kl_coef=-0.1), q=FAKE),
     dict(params=dict(entropy_coef=-1.0)),
     dict(params=dict(std_floor=0.0)),
-    dict(params=dict(correction="tis")),               # no old log-probs
     dict(params=dict(correction="tis", corr_lo=3.0, corr_hi=2.0), old=FAKE),
     dict(params=dict(correction=5), old=FAKE),
     dict(params=dict(opd_coef=0.5)),                   # no teacher log-probs
@@ -203,3 +202,68 @@ def test_chunked_entry_validates(lib):
     assert call(ml.RL_PHASE_ROWS, 0, 8, logits=None) == RL_ERR_INVALID_ARG
     assert call(ml.RL_PHASE_ALL, 0, 8, params=gspo) == 2     # GSPO: whole calls only
     assert call(ml.RL_PHASE_ROWS, 0, 16, params=gspo) == 2
+
+
+def test_launch_overrides_struct_layout_matches_header():
+    text = open(HEADER).read()
+    body = text[text.index("typedef struct {", text.index("Launch-plan overrides")):
+                text.index("} rl_launch_overrides;")]
+    names = re.findall(r"(?:int32_t|int64_t)\s+([a-z_0-9]+)\s*;", body)
+    assert names == [f[0] for f in ml.RlLaunchOverrides._fields_]
+    assert ctypes.sizeof(ml.RlLaunchOverrides) == 48
+
+
+def test_launch_overrides_are_validated_and_cleared(lib):
+    o = ml.RlLaunchOverrides()
+    assert lib.rl_launch_overrides_init(ctypes.byref(o)) == 0
+    assert all(getattr(o, f) == -1 for f, _ in ml.RlLaunchOverrides._fields_)
+    assert lib.rl_launch_overrides_init(None) == RL_ERR_INVALID_ARG
+    try:
+        ml.set_launch_overrides(sweep_kernel="stream", stream_slots=3, stream_hold=2)
+        ml.set_launch_overrides(cluster_size=8, cluster_stages=4, stall_first_wait_ns=1000)
+        for bad in (dict(sweep_kernel=2), dict(cluster_size=16), dict(cluster_stages=0),
+                    dict(stream_chunk_bytes=512), dict(stream_slots=17), dict(stream_hold=-2),
+                    dict(stream_split_first=2), dict(stream_prefetch_bytes=24),
+                    dict(stream_prefetch_bytes=1 << 21), dict(stall_first_wait_ns=-5),
+                    dict(stall_first_wait_ns=10 ** 11)):
+            with pytest.raises(ml.MilesLossError) as e:
+                ml.set_launch_overrides(**bad)
+            assert e.value.status == RL_ERR_INVALID_ARG
+        with pytest.raises(TypeError):
+            ml.set_launch_overrides(no_such_field=1)
+        with ml.launch_overrides(sweep_kernel="cluster"):
+            pass
+    finally:
+        ml.set_launch_overrides()
+    assert lib.rl_set_launch_overrides(None) == 0
+
+
+def test_library_reads_no_environment_variables():
+    """Launch plans come from the library's own rules or the explicit
+    overrides, never from the caller's environment."""
+    csrc = os.path.join(ROOT, "paper_2609_08368_gb300", "csrc")
+    for name in os.listdir(csrc):
+        text = open(os.path.join(csrc, name)).read()
+        assert "getenv" not in text, name
+
+
+def test_sharded_entry_validates(lib):
+    v = ctypes.c_void_p
+    p = ml.make_params()
+    gspo = ml.make_params(estimator="gspo")
+
+    def call(phase, r0=0, total=16, R=16, params=p, counts=FAKE, partials=FAKE, stats=FAKE):
+        return lib.rl_loss_shard_fwd_bwd(
+            phase, r0, total, v(FAKE), 0, R, 64, 64, v(FAKE), v(FAKE), None, None, None,
+            v(FAKE), v(FAKE), v(FAKE), 2, 1, v(FAKE), ctypes.byref(params), v(FAKE), v(FAKE),
+            v(FAKE), v(FAKE), v(counts), v(partials), v(stats), 1.0, None, v(FAKE), 0, 64,
+            v(FAKE * 2), 1 << 30, None)
+    assert call(0) == RL_ERR_INVALID_ARG                      # no phase
+    assert call(3) == RL_ERR_INVALID_ARG                      # one phase per call
+    assert call(ml.RL_SHARD_COUNT, r0=8, total=16, R=9) == RL_ERR_INVALID_ARG  # past the call
+    assert call(ml.RL_SHARD_COUNT, r0=-1) == RL_ERR_INVALID_ARG
+    assert call(ml.RL_SHARD_COUNT, counts=None) == RL_ERR_INVALID_ARG
+    assert call(ml.RL_SHARD_SWEEP, partials=None) == RL_ERR_INVALID_ARG
+    assert call(ml.RL_SHARD_FINISH, partials=None) == RL_ERR_INVALID_ARG
+    assert call(ml.RL_SHARD_FINISH, stats=None) == RL_ERR_INVALID_ARG
+    assert call(ml.RL_SHARD_COUNT, params=gspo) == 2          # GSPO: whole calls only

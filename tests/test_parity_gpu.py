@@ -33,23 +33,25 @@ SHRUNK = {
 
 
 @pytest.fixture(autouse=True)
-def _no_overrides(monkeypatch):
-    monkeypatch.delenv("MILESLOSS_SWEEP_CLUSTER", raising=False)
-    monkeypatch.delenv("MILESLOSS_SWEEP_STAGES", raising=False)
-    monkeypatch.delenv("MILESLOSS_SWEEP_THREADS", raising=False)
-    monkeypatch.delenv("MILESLOSS_SWEEP_CTAS_PER_SM", raising=False)
-    monkeypatch.delenv("MILESLOSS_SWEEP_KIND", raising=False)
-    monkeypatch.delenv("MILESLOSS_STREAM_CHUNK", raising=False)
-    monkeypatch.delenv("MILESLOSS_STREAM_SLOTS", raising=False)
-    monkeypatch.delenv("MILESLOSS_STREAM_HOLD", raising=False)
-    monkeypatch.delenv("MILESLOSS_STREAM_SPLIT", raising=False)
+def ov():
+    """Launch-plan overrides for one test: ``ov(field=value, ...)`` adds to
+    the test's overrides; none are left installed afterwards."""
+    fields = {}
+
+    def set_(**kw):
+        fields.update(kw)
+        ml.set_launch_overrides(**fields)
+    ml.set_launch_overrides()
+    yield set_
+    ml.set_launch_overrides()
 
 
-def _full_check(w, mode="fused", dl_dtype=None, params=None):
+def _full_check(w, mode="fused", dl_dtype=None, params=None, fp32_floor=False):
     g = P.run_gpu(w, mode=mode, dl_dtype=dl_dtype, params=params)
     assert g["err"] == 0, ml.status_string(g["err"])
     o = P.run_oracle(w, params=params)
-    P.compare_forward(w, g, o, params=params)
+    floor = P.fp32_logp_loss_floor(w, o, params) if fp32_floor else 0.0
+    P.compare_forward(w, g, o, params=params, loss_floor=floor)
     if mode != "fwd":
         P.assert_dlogits_close(g["dlogits_t"][:, :w.vocab].float().cpu().numpy(), o["dlogits"])
     return g, o
@@ -62,10 +64,10 @@ def test_parity_fused(name):
 
 @pytest.mark.parametrize("kind", ["cluster", "stream"])
 @pytest.mark.parametrize("name", list(SHRUNK))
-def test_parity_each_sweep_kernel(monkeypatch, kind, name):
+def test_parity_each_sweep_kernel(ov, kind, name):
     """Both vocabulary-sweep kernels (cluster exchange, and one CTA per row
     with an L2-served second read) on every workload."""
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+    ov(sweep_kernel=kind)
     _full_check(wl.make(SHRUNK[name], DEV))
     _full_check(wl.make(SHRUNK[name], DEV), mode="split")
 
@@ -74,15 +76,15 @@ def test_parity_each_sweep_kernel(monkeypatch, kind, name):
     (16384, 14, 1, 0), (16384, 14, 5, 1), (4096, 2, 0, 0), (4096, 2, 2, 1), (12288, 3, 2, 1),
     (12288, 3, 3, 0), (1024, 1, 1, 1), (1024, 1, 0, 0), (65536, 3, 2, 1), (75776, 3, 2, 1),
     (8192, 4, 4, 1)])
-def test_stream_ring_shapes(monkeypatch, chunk, slots, hold, split):
+def test_stream_ring_shapes(ov, chunk, slots, hold, split):
     """The streaming kernel's ring: chunk sizes, slot counts, chunks kept in
     shared memory for pass B (0 to every slot) and the ragged chunk first or
     last, on rows of 2 to 88 chunks."""
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", "stream")
-    monkeypatch.setenv("MILESLOSS_STREAM_CHUNK", str(chunk))
-    monkeypatch.setenv("MILESLOSS_STREAM_SLOTS", str(slots))
-    monkeypatch.setenv("MILESLOSS_STREAM_HOLD", str(hold))
-    monkeypatch.setenv("MILESLOSS_STREAM_SPLIT", str(split))
+    ov(sweep_kernel="stream")
+    ov(stream_chunk_bytes=chunk)
+    ov(stream_slots=slots)
+    ov(stream_hold=hold)
+    ov(stream_split_first=split)
     # ragged rows: 45,003 bf16 columns = 5,625 vectors and a 3-element tail
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=24, vocab=45003,
                     rho_noise=0.3)
@@ -120,26 +122,26 @@ def test_dlogits_relative_error_on_order_p_entries():
 
 
 @pytest.mark.parametrize("cluster", [1, 2, 4, 8])
-def test_every_cluster_size(monkeypatch, cluster):
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", "cluster")
-    monkeypatch.setenv("MILESLOSS_SWEEP_CLUSTER", str(cluster))
+def test_every_cluster_size(ov, cluster):
+    ov(sweep_kernel="cluster")
+    ov(cluster_size=cluster)
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=24, vocab=20000 + 24)
     _full_check(wl.make(rec, DEV))
 
 
 @pytest.mark.parametrize("threads,per_sm", [(256, 4), (256, 5), (512, 2)])
-def test_every_block_shape(monkeypatch, threads, per_sm):
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", "cluster")
-    monkeypatch.setenv("MILESLOSS_SWEEP_THREADS", str(threads))
-    monkeypatch.setenv("MILESLOSS_SWEEP_CTAS_PER_SM", str(per_sm))
+def test_every_block_shape(ov, threads, per_sm):
+    ov(sweep_kernel="cluster")
+    ov(cluster_threads=threads)
+    ov(cluster_ctas_per_sm=per_sm)
     _full_check(wl.make(SHRUNK["glm_noisy"], DEV))
 
 
 @pytest.mark.parametrize("stages", [1, 2, 3, 4])
-def test_every_ring_depth(monkeypatch, stages):
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", "cluster")
-    monkeypatch.setenv("MILESLOSS_SWEEP_CLUSTER", "2")
-    monkeypatch.setenv("MILESLOSS_SWEEP_STAGES", str(stages))
+def test_every_ring_depth(ov, stages):
+    ov(sweep_kernel="cluster")
+    ov(cluster_size=2)
+    ov(cluster_stages=stages)
     rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=1, group_size=4, traj_len=40, vocab=6144)
     _full_check(wl.make(rec, DEV))
 
@@ -197,11 +199,11 @@ def _extreme_rows(w):
 @pytest.mark.parametrize("kind", ["cluster", "stream"])
 @pytest.mark.parametrize("extra", [dict(), dict(entropy_coef=0.01, temperature=0.7),
                                    dict(temperature=0.05)])
-def test_extreme_logits(monkeypatch, kind, extra):
+def test_extreme_logits(ov, kind, extra):
     """Extreme rows (see _extreme_rows) on both sweep kernels, fused and
     split, with and without the entropy term and temperature; a row of 200 KB
     runs in the streaming kernel in two ring chunks."""
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+    ov(sweep_kernel=kind)
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=4, vocab=100000)
     w = wl.make(rec, DEV)
     _extreme_rows(w)
@@ -216,21 +218,27 @@ def test_extreme_logits(monkeypatch, kind, extra):
         w.ref_logprobs.copy_(lp - 0.03)
     if w.old_logprobs is not None:
         w.old_logprobs.copy_(lp + 0.01)
-    g, o = _full_check(w, params=params)
+    # rows shifted to -1000 (and divided by T = 0.05) have |lse| up to ~2e4:
+    # their fp32 log-probs carry errors of ~eps |lse|, which the loss bound
+    # takes as its floor (fp32_logp_loss_floor)
+    g, o = _full_check(w, params=params, fp32_floor=True)
     for k in ("logp", "H"):
         assert np.all(np.isfinite(g[k])), k
     assert abs(float(g["H"][9])) < 1e-6 and abs(float(g["logp"][9])) < 1e-6
-    _full_check(w, mode="split", params=params)
+    # the objective and the reduction alone, on the GPU's own log-probs: 1e-4
+    own = P.stats_on_gpu_logp(w, g, o, P.oracle_params(params))
+    P.assert_loss_close(g["stats"]["loss"], own["loss"], what="loss on the GPU's log-probs")
+    _full_check(w, mode="split", params=params, fp32_floor=True)
 
 
 @pytest.mark.parametrize("kind", ["cluster", "stream"])
 @pytest.mark.parametrize("ld,ld_out", [(100008, 100000), (100003, 100003), (100000, 100011)])
-def test_long_rows_padded_and_misaligned(monkeypatch, kind, ld, ld_out):
+def test_long_rows_padded_and_misaligned(ov, kind, ld, ld_out):
     """Rows of 200 KB on both sweep kernels with a padded row stride, rows
     whose starts are not 16-byte aligned (the cluster kernel's element-wise
     path takes them whatever the kind), and a dLogits stride that is not
     16-byte aligned (scalar stores); fused and split."""
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+    ov(sweep_kernel=kind)
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=6, vocab=100000)
     w = wl.make(rec, DEV, ld=ld)
     for mode in ("fused", "split"):
@@ -290,12 +298,12 @@ def test_ragged_and_empty_trajectories(estimator, n_prompts):
 
 
 @pytest.mark.parametrize("kind", ["cluster", "stream"])
-def test_fused_call_replays_from_a_cuda_graph(monkeypatch, kind):
+def test_fused_call_replays_from_a_cuda_graph(ov, kind):
     """The fused call only enqueues kernels on the caller's stream (no
     allocation, no synchronisation), so it can be captured in a CUDA graph;
     replays give bit-identical results to a direct call, also after the inputs
     change in place."""
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+    ov(sweep_kernel=kind)
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=8, vocab=100000)
     w = wl.make(rec, DEV)
     buf = api.alloc(w.n_rows, int(w.rewards.shape[0]), w.n_groups, DEV, vocab=w.vocab,
@@ -337,6 +345,28 @@ def test_temperature_entropy_kl_correction_opd():
 
 @pytest.mark.parametrize("kind", ["cluster", "stream"])
 @pytest.mark.parametrize("params", [
+    dict(correction="tis", corr_lo=0.0, corr_hi=1.1),
+    dict(correction="clip_or_pop", corr_lo=0.9, corr_hi=1.1, dual_clip_c=2.0, kl_coef=0.05),
+    dict(estimator="gspo", correction="tis", corr_lo=0.0, corr_hi=1.05),
+], ids=["tis", "pop", "gspo_tis"])
+def test_corrections_without_old_logprobs(ov, kind, params):
+    """The corrections of Sec. 3.4 in a single-pass step: no old log-probs,
+    so the correction ratio is the trainer's own log-prob of this pass
+    against the rollout's (held constant) and the PPO ratio is taken against
+    the rollout log-probs; fused and split, both sweep kernels."""
+    ov(sweep_kernel=kind)
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=2, group_size=4, traj_len=32, vocab=9000,
+                    rho_noise=0.25, ref_noise=0.2)
+    w = wl.make(rec, DEV)
+    assert w.old_logprobs is None
+    p = dict(w.params, **params)
+    g, _ = _full_check(w, params=p)
+    assert g["stats"]["n_corr_clip"] > 0
+    _full_check(w, mode="split", params=p)
+
+
+@pytest.mark.parametrize("kind", ["cluster", "stream"])
+@pytest.mark.parametrize("params", [
     dict(estimator="reinforcepp"),
     dict(estimator="reinforcepp_baseline", dual_clip_c=2.0, kl_coef=0.05),
     dict(estimator="reinforcepp", normalize_std=False, unbiased_std=False),
@@ -344,10 +374,10 @@ def test_temperature_entropy_kl_correction_opd():
     dict(estimator="gspo", correction="tis", corr_lo=0.0, corr_hi=1.1, eps_lo=0.1, eps_hi=0.1),
     dict(estimator="gspo", correction="clip_or_pop", corr_lo=0.9, corr_hi=1.1, temperature=0.8),
 ], ids=["rpp", "rpp_base", "rpp_center", "gspo", "gspo_tis", "gspo_pop"])
-def test_advantage_estimators(monkeypatch, kind, params):
+def test_advantage_estimators(ov, kind, params):
     """REINFORCE++ (plain, baseline-relative) and GSPO (Sec. 3.4), fused and
     split, on both sweep kernels; trajectories of unequal training length."""
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+    ov(sweep_kernel=kind)
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=3, group_size=4, traj_len=20, vocab=9000,
                     rho_noise=0.3, ref_noise=0.2, old_noise=0.1, mask="prefix_u0_half")
     w = wl.make(rec, DEV)
@@ -357,10 +387,10 @@ def test_advantage_estimators(monkeypatch, kind, params):
 
 @pytest.mark.parametrize("kind", ["cluster", "stream"])
 @pytest.mark.parametrize("K", [1, 4, 16])
-def test_opd_topk(monkeypatch, kind, K):
+def test_opd_topk(ov, kind, K):
     """The top-K on-policy distillation signal (Sec. 5.2) from candidate sets
     and teacher log-probs, in the sweep epilogue."""
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+    ov(sweep_kernel=kind)
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=2, group_size=4, traj_len=24, vocab=12000,
                     rho_noise=0.3, ref_noise=0.2, topk=K, topk_noise=0.4)
     w = wl.make(rec, DEV)
@@ -372,13 +402,13 @@ def test_opd_topk(monkeypatch, kind, K):
 
 @pytest.mark.parametrize("kind,cluster", [("cluster", 0), ("cluster", 8), ("stream", 0)])
 @pytest.mark.parametrize("K", [4, 64])
-def test_opd_topk_long_rows(monkeypatch, kind, cluster, K):
+def test_opd_topk_long_rows(ov, kind, cluster, K):
     """Top-K OPD on rows of 200 KB: candidates spread over the CTAs of a
     cluster (4 by the plan, 8 forced; their partial sums merge in the row
     exchange) or over the streaming kernel's two ring chunks."""
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+    ov(sweep_kernel=kind)
     if cluster:
-        monkeypatch.setenv("MILESLOSS_SWEEP_CLUSTER", str(cluster))
+        ov(cluster_size=cluster)
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=12, vocab=100000,
                     rho_noise=0.3, ref_noise=0.2, topk=K, topk_noise=0.4)
     w = wl.make(rec, DEV)
@@ -390,16 +420,16 @@ def test_opd_topk_long_rows(monkeypatch, kind, cluster, K):
 @pytest.mark.parametrize("vocab,ring", [
     (45003, (4096, 2, 1, 0)), (45003, (4096, 3, 2, 1)), (45003, (1024, 1, 0, 0)),
     (45003, (16384, 4, 4, 1)), (45003, (75776, 3, 2, 1)), (131072, None)])
-def test_opd_topk_stream_ring_shapes(monkeypatch, vocab, ring):
+def test_opd_topk_stream_ring_shapes(ov, vocab, ring):
     """Top-K OPD in the streaming kernel, whose top-K warp waits on and
     releases every ring slot and hands each row's part to warp 0: chunk
     sizes, slot counts, kept chunks and both splits (rows of 1 to 88 chunks,
     a ragged tail past the last whole vector), and the default plan of
     256 KB rows (three 74 KB slots, two kept)."""
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", "stream")
+    ov(sweep_kernel="stream")
     if ring:
-        for name, v in zip(("CHUNK", "SLOTS", "HOLD", "SPLIT"), ring):
-            monkeypatch.setenv("MILESLOSS_STREAM_" + name, str(v))
+        ov(**dict(zip(("stream_chunk_bytes", "stream_slots", "stream_hold", "stream_split_first"),
+                      ring)))
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=16, vocab=vocab,
                     rho_noise=0.3, ref_noise=0.2, topk=16, topk_noise=0.4)
     w = wl.make(rec, DEV)
@@ -409,8 +439,8 @@ def test_opd_topk_stream_ring_shapes(monkeypatch, vocab, ring):
 
 
 @pytest.mark.parametrize("kind", ["cluster", "stream"])
-def test_no_training_tokens_and_empty_call(monkeypatch, kind):
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+def test_no_training_tokens_and_empty_call(ov, kind):
+    ov(sweep_kernel=kind)
     rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=1, group_size=2, traj_len=8, vocab=300)
     w = wl.make(rec, DEV)
     w.loss_mask.zero_()
@@ -439,8 +469,8 @@ def test_no_training_tokens_and_empty_call(monkeypatch, kind):
 
 
 @pytest.mark.parametrize("kind", ["cluster", "stream"])
-def test_device_errors_are_reported_not_trapped(monkeypatch, kind):
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+def test_device_errors_are_reported_not_trapped(ov, kind):
+    ov(sweep_kernel=kind)
     rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=2, group_size=2, traj_len=8, vocab=256)
     w = wl.make(rec, DEV)
     w.targets[3] = 256                     # outside [0, vocab)
@@ -456,6 +486,71 @@ def test_device_errors_are_reported_not_trapped(monkeypatch, kind):
     assert P.run_gpu(w)["err"] == 7        # RL_ERR_BAD_SEQLENS
     w = wl.make(rec, DEV)
     assert P.run_gpu(w)["err"] == 0        # the error word resets on the next call
+
+
+@pytest.mark.parametrize("kind", ["cluster", "stream"])
+@pytest.mark.parametrize("topk", [0, 4])
+def test_a_wait_that_runs_out_is_reported(ov, kind, topk):
+    """Failure detection on the GPU without a fault. The test hook
+    stall_first_wait_ns makes the first wait for logits of every CTA of the
+    sweep wait on a barrier that nothing completes, bounded by 1 ms; each CTA
+    then gives up as it would on a copy that never arrives (it stops issuing
+    copies, waits for the ones in flight and writes zeros for its rows). The
+    call reports RL_ERR_DEVICE_TIMEOUT with every output finite and zero, and
+    the next call without the hook is RL_OK and matches the oracle."""
+    ov(sweep_kernel=kind)
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=64, vocab=100000,
+                    rho_noise=0.3, ref_noise=0.2, topk=topk, topk_noise=0.4)
+    w = wl.make(rec, DEV)
+    params = dict(w.params, opd_coef=0.5, opd_topk=topk) if topk else None
+    for mode in ("fused", "split"):
+        ov(stall_first_wait_ns=1_000_000)
+        g = P.run_gpu(w, mode=mode, params=params)
+        assert g["err"] == 8, ml.status_string(g["err"])  # RL_ERR_DEVICE_TIMEOUT
+        assert np.all(g["logp"] == 0) and np.all(g["H"] == 0)
+        assert torch.equal(g["dlogits_t"], torch.zeros_like(g["dlogits_t"]))
+        st = g["stats"]
+        assert st["loss"] == 0.0 and st["n_tokens"] == int(w.loss_mask.sum())
+        ov(stall_first_wait_ns=-1)
+        _full_check(w, mode=mode, params=params)
+
+
+@pytest.mark.parametrize("kind,cluster", [("cluster", 0), ("cluster", 4), ("stream", 0)])
+def test_topk_ids_out_of_range_are_reported(ov, kind, cluster):
+    """A top-K OPD candidate id outside [0, vocab) zeros its row (as a bad
+    target does) and the call reports RL_ERR_TOPK_ID_OUT_OF_RANGE; the other
+    rows match the oracle."""
+    ov(sweep_kernel=kind)
+    if cluster:
+        ov(cluster_size=cluster)
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=8, vocab=60000,
+                    rho_noise=0.3, topk=8, topk_noise=0.4)
+    w = wl.make(rec, DEV)
+    params = dict(w.params, opd_coef=0.5, opd_topk=8)
+    bad = [3, 17]
+    w.topk_ids[3, 5] = w.vocab   # one past the end
+    w.topk_ids[17, 0] = -1
+    for mode in ("fused", "split"):
+        g = P.run_gpu(w, mode=mode, params=params)
+        assert g["err"] == 9, ml.status_string(g["err"])  # RL_ERR_TOPK_ID_OUT_OF_RANGE
+        assert all(g["logp"][r] == 0 and g["H"][r] == 0 for r in bad)
+        dl = g["dlogits_t"].float()
+        assert all((dl[r] == 0).all() for r in bad)
+        # the other rows against the oracle on the same call with valid ids
+        # in place of the bad ones (a row's outputs do not depend on another
+        # row's candidates)
+        ids = P.np_(w.topk_ids).copy()
+        ids[3, 5], ids[17, 0] = 0, 1
+        o = oracle.rl_loss(P.host_logits(w), P.np_(w.targets), P.np_(w.rollout_logprobs),
+                           P.np_(w.ref_logprobs), P.np_(w.rewards), P.np_(w.group_id),
+                           P.np_(w.cu_seqlens), w.n_groups, P.np_(w.loss_mask),
+                           P.oracle_params(params), topk_ids=ids,
+                           topk_teacher=P.np_(w.topk_teacher))
+        good = np.setdiff1d(np.arange(w.n_rows), bad)
+        tol = P.logp_tol(w)
+        np.testing.assert_allclose(g["logp"][good], o["logp"][good], atol=tol, rtol=0)
+        np.testing.assert_allclose(g["H"][good], o["H"][good], atol=tol, rtol=0)
+        P.assert_dlogits_close(dl[good][:, :w.vocab].cpu().numpy(), o["dlogits"][good])
 
 
 def test_bitwise_reproducible_and_fwd_matches_fused():
@@ -548,64 +643,55 @@ def test_hand_worked_calls(name):
 
 # ---------------------------------------------------------------- full sizes
 
-FULL = ["qwen", "glm", "agentic", "fp32"]
+FULL = ["glm", "qwen", "agentic", "fp32"]
 
 
-def _sampled_rows(w, n=24, seed=0):
-    rng = np.random.default_rng(seed)
-    R = w.n_rows
-    return np.unique(np.concatenate([[0, R - 1], rng.integers(0, R, size=n)]))
+@pytest.fixture(scope="module")
+def oracle_pool():
+    """The float64 oracle's worker processes (spawned), one per host core."""
+    import bench
+    pool = bench.OraclePool()
+    yield pool
+    pool.close()
 
 
 @pytest.mark.slow
 @pytest.mark.parametrize("name", FULL)
-def test_full_size_sampled_rows(name):
-    """Full-size workloads in the launch configuration the benchmark times:
-    sampled rows against the oracle one by one, and the loss against the
-    oracle's per-token rule applied to the GPU's own log-probs."""
-    rec = wl.RECIPES[name]
-    w = wl.make(rec, DEV)
+def test_full_size_every_row(name, oracle_pool):
+    """Full-size workloads (the headline one first: 65,536 x 154,880 bf16) in
+    the launch configuration the benchmark times, EVERY row against the
+    float64 oracle: the log-prob and entropy of every row, every dLogit
+    (compared entry by entry in the oracle's worker processes at 1e-2
+    relative / 1e-5 absolute), advantages, group sizes and N, the clip counts
+    (exactly, under the oracle's rule on the GPU's log-probs; within the
+    guard band against the oracle's own), the metrics, and the scalar loss
+    to 1e-4 relative of the oracle's."""
+    import bench
+    w = wl.make(wl.RECIPES[name], DEV)
     g = P.run_gpu(w)
-    assert g["err"] == 0
+    assert g["err"] == 0, ml.status_string(g["err"])
+    o_rows = bench.oracle_rows(w, oracle_pool, dlogits=g["dlogits_t"])
+    assert o_rows["n_bad"] == 0, (f"{o_rows['n_bad']} dLogits outside the bound; worst "
+                                  f"(row, col, gpu, oracle) = {o_rows['worst_at']}")
     p = P.oracle_params(w.params)
-    import oracle
-    A_traj, n_g = oracle.group_advantages(P.np_(w.rewards), P.np_(w.group_id), w.n_groups, p)
-    np.testing.assert_allclose(g["A"], A_traj, rtol=1e-6, atol=1e-6)
-    np.testing.assert_array_equal(g["group_sizes"], n_g)
-    A_row = oracle.row_advantages(A_traj, P.np_(w.cu_seqlens), w.n_rows)
-    mask = P.np_(w.loss_mask)
-    N = int(mask.astype(bool).sum())
-    assert g["stats"]["n_tokens"] == N
-    rows = _sampled_rows(w)
-    o = oracle.rl_loss_rows(P.host_logits(w, torch.from_numpy(rows).to(DEV)),
-                            P.np_(w.targets)[rows], P.np_(w.rollout_logprobs)[rows],
-                            None if w.ref_logprobs is None else P.np_(w.ref_logprobs)[rows],
-                            A_row[rows], mask[rows].astype(bool), N, p)
-    tol = P.logp_tol(w)
-    np.testing.assert_allclose(g["logp"][rows], o["logp"], atol=tol, rtol=0)
-    np.testing.assert_allclose(g["H"][rows], o["H"], atol=tol, rtol=0)
-    dl = g["dlogits_t"][torch.from_numpy(rows).to(DEV), :w.vocab].float().cpu().numpy()
-    P.assert_dlogits_close(dl, o["dlogits"])
-    # loss and counts: the oracle's per-token rule on the GPU's log-probs
-    obj = oracle.token_objective(g["logp"].astype(np.float64), P.np_(w.rollout_logprobs),
-                                 P.np_(w.ref_logprobs), A_row, g["H"].astype(np.float64), p)
-    L, _ = oracle.masked_token_mean(obj["ell"], mask)
-    m = mask.astype(bool)
-    scale = np.abs(obj["ell"][m]).mean()
-    assert abs(g["stats"]["loss"] - L) <= 1e-4 * scale
-    counts, band = P.clip_counts(p, g["logp"].astype(np.float64), P.np_(w.rollout_logprobs),
-                                 P.np_(w.ref_logprobs), A_row, g["H"], mask)
-    for k, v in counts.items():
-        assert abs(g["stats"][k] - v) <= band, (k, g["stats"][k], v, band)
-    del g, w
+    mask = P.np_(w.loss_mask).astype(bool)
+    A_traj, A_row, n_g = oracle.estimator_advantages(P.np_(w.rewards), P.np_(w.group_id),
+                                                     w.n_groups, P.np_(w.cu_seqlens), mask, p)
+    obj = oracle.token_objective(o_rows["logp"], P.np_(w.rollout_logprobs), P.np_(w.ref_logprobs),
+                                 A_row, o_rows["H"], p, old=P.np_(w.old_logprobs))
+    stats = oracle.loss_stats(obj, o_rows["logp"], P.np_(w.rollout_logprobs), o_rows["H"], mask)
+    o = dict(obj, logp=o_rows["logp"], H=o_rows["H"], lse=o_rows["lse"], A_traj=A_traj,
+             A_row=A_row, group_sizes=n_g, N=int(mask.sum()), stats=stats)
+    P.compare_forward(w, g, o)
+    del g, w, o_rows
     torch.cuda.empty_cache()
 
 
 @pytest.mark.parametrize("kind", ["cluster", "stream"])
-def test_chunked_call_equals_whole_call(monkeypatch, kind):
+def test_chunked_call_equals_whole_call(ov, kind):
     """BEGIN, ROWS over blocks of rows (ragged last block), END give the same
     bits as one rl_loss_fwd_bwd; a forward-only chunk leaves dLogits alone."""
-    monkeypatch.setenv("MILESLOSS_SWEEP_KIND", kind)
+    ov(sweep_kernel=kind)
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=2, group_size=4, traj_len=40, vocab=20480,
                     rho_noise=0.3, ref_noise=0.2, topk=4)
     w = wl.make(rec, DEV)
@@ -646,3 +732,74 @@ def test_pipelined_host_call_matches_device_call():
         assert torch.equal(out["dlogits"], whole["dlogits_t"].cpu())
         np.testing.assert_array_equal(out["token_logprobs"].numpy(), whole["logp"])
         assert ml.parse_stats(out["stats"].numpy().tobytes()) == whole["stats"]
+
+
+# ---------------------------------------------------------- row-sharded calls
+
+def _shard_of(w, r0, r1):
+    """Rows [r0, r1) of a workload as one shard's workload (the per-trajectory
+    inputs stay those of the whole call)."""
+    sl = slice(r0, r1)
+
+    def rows(t):
+        return None if t is None else t[sl].contiguous()
+    return wl.Workload(w.recipe, rows(w.logits), rows(w.targets), rows(w.rollout_logprobs),
+                       rows(w.ref_logprobs), rows(w.old_logprobs), rows(w.teacher_logprobs),
+                       w.rewards, w.group_id, w.cu_seqlens, rows(w.loss_mask), w.n_groups,
+                       dict(w.params), rows(w.topk_ids), rows(w.topk_teacher))
+
+
+@pytest.mark.parametrize("kind", ["cluster", "stream"])
+@pytest.mark.parametrize("params", [dict(), dict(estimator="reinforcepp", kl_coef=0.05),
+                                    dict(opd_coef=0.3, opd_topk=4, entropy_coef=0.01)],
+                         ids=["grpo", "rpp", "topk"])
+def test_row_sharded_call_equals_whole_call(ov, kind, params):
+    """One call's rows split over shards (2 and 3 shards, trajectories cut at
+    the boundaries, and an empty shard), driven phase by phase with the
+    exchanges done by sums and maxima over the shards' small arrays: every
+    shard's log-probs, entropies and dLogits are those of the whole call bit
+    for bit, the advantages, group sizes and counts equal, the loss within
+    1e-4 relative (its partial sums are added in another order)."""
+    ov(sweep_kernel=kind)
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=2, group_size=4, traj_len=40, vocab=20480,
+                    rho_noise=0.3, ref_noise=0.2, topk=4, mask="prefix_u0_half")
+    w = wl.make(rec, DEV)
+    p = P.gpu_params(w, dict(w.params, **params))
+    whole = P.run_gpu(w, params=p)
+    R, n_traj = w.n_rows, int(w.rewards.shape[0])
+    for cuts in ([0, 137, R], [0, 50, 50, 221, R]):
+        shards = []
+        for r0, r1 in zip(cuts[:-1], cuts[1:]):
+            ws = _shard_of(w, r0, r1)
+            buf = api.alloc(r1 - r0, n_traj, w.n_groups, DEV, vocab=w.vocab,
+                            dlogits_dtype=w.logits.dtype, fill_nan=True)
+            # (the shard's own top-K candidates: params without the whole
+            # call's arrays, so that api.Shard attaches the shard's rows)
+            shards.append(api.Shard(ws, r0, R, buf, params=dict(w.params, **params)))
+        api.sharded_fwd_bwd_local(shards)
+        torch.cuda.synchronize()
+        for sh, (r0, r1) in zip(shards, zip(cuts[:-1], cuts[1:])):
+            b = sh.buf
+            assert ml.rl_loss_check_device_error(b.workspace) == 0
+            assert torch.equal(b.dlogits, whole["dlogits_t"][r0:r1])
+            np.testing.assert_array_equal(b.token_logprobs.cpu().numpy(), whole["logp"][r0:r1])
+            np.testing.assert_array_equal(b.entropy.cpu().numpy(), whole["H"][r0:r1])
+            np.testing.assert_array_equal(b.advantages.cpu().numpy(), whole["A"])
+            np.testing.assert_array_equal(b.group_sizes.cpu().numpy(), whole["group_sizes"])
+            st, ref = b.read_stats(), whole["stats"]
+            for k in ("n_tokens", "n_clip_hi", "n_clip_lo", "n_dual_clip", "n_corr_clip",
+                      "ratio_min", "ratio_max"):
+                assert st[k] == ref[k], k
+            P.assert_loss_close(st["loss"], ref["loss"], what="sharded loss")
+            for k in ("pg_loss_mean", "kl_mean", "entropy_mean", "ratio_mean"):
+                assert abs(st[k] - ref[k]) <= 1e-4 * max(abs(ref[k]), 1e-3), k
+
+
+def test_row_sharded_gspo_is_unsupported():
+    rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=1, group_size=2, traj_len=8, vocab=256)
+    w = wl.make(rec, DEV)
+    buf = api.alloc(w.n_rows, 2, 1, DEV, vocab=256, dlogits_dtype=torch.bfloat16)
+    sh = api.Shard(w, 0, w.n_rows, buf, params=dict(w.params, estimator="gspo"))
+    with pytest.raises(ml.MilesLossError) as e:
+        sh.count()
+    assert e.value.status == 2  # RL_ERR_UNSUPPORTED
