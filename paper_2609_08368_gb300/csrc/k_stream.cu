@@ -83,6 +83,36 @@ __device__ __forceinline__ Tri warp_merge(Tri t) {
   return Tri{M, s, u};
 }
 
+// Merges the consumer warps' partial sums of a row: red[w] = (m, s, u) of
+// warp w, redm[w] = its m again (contiguous, so that every lane takes the
+// maximum with four broadcast reads instead of a shuffle tree). Lanes
+// 0..kConsWarps-1 rescale one warp's sums each and sum them in a fixed order;
+// lane 0 (every lane below kConsWarps) gets the row's sums.
+__device__ __forceinline__ Tri block_merge(const float4* red, const float* redm, int lane) {
+  static_assert(kConsWarps == 16, "four float4 of references, four sum levels");
+  float M = -INFINITY;
+#pragma unroll
+  for (int w = 0; w < kConsWarps / 4; ++w) {
+    const float4 m4 = reinterpret_cast<const float4*>(redm)[w];
+    M = fmaxf(M, fmaxf(fmaxf(m4.x, m4.y), fmaxf(m4.z, m4.w)));
+  }
+  float s = 0.0f, u = 0.0f;
+  if (lane < kConsWarps) {
+    const float4 v = red[lane];
+    if (v.y > 0.0f) {
+      const float d = v.x - M, f = ex2(d);
+      s = f * v.y;
+      u = f * fmaf(d, v.y, v.z);
+    }
+  }
+#pragma unroll
+  for (int o = kConsWarps / 2; o > 0; o >>= 1) {
+    s += __shfl_xor_sync(0xffffffffu, s, o);
+    u += __shfl_xor_sync(0xffffffffu, u, o);
+  }
+  return Tri{M, s, u};
+}
+
 // Running sums of one thread over the chunks of a row. The reference starts
 // at the maximum of the thread's first vector and is moved only by whole
 // powers of two of the sums (rebase), so no per-element maximum is needed.
@@ -189,14 +219,16 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(NS) * CB);
   uint64_t* empty = full + kMaxSlots;
   float4* red = reinterpret_cast<float4*>(empty + kMaxSlots);  // [kConsWarps]
-  float4* bc = red + kConsWarps;                                // [2]
+  float* redm = reinterpret_cast<float*>(red + kConsWarps);     // [kConsWarps]
+  float4* bc = reinterpret_cast<float4*>(redm + kConsWarps);    // [2]
   int4* bci = reinterpret_cast<int4*>(bc + 2);                  // [1]
   TopKPart* tkp = reinterpret_cast<TopKPart*>(bci + 1);         // [2] top-K parts by row parity
   uint64_t* tk_full = reinterpret_cast<uint64_t*>(tkp + 2);     // [2] part written
   uint64_t* tk_empty = tk_full + 2;                             // [2] part read
   uint64_t* never = tk_empty + 2;                               // [1] completed by nothing (test hook)
   volatile int* abort = reinterpret_cast<volatile int*>(never + 1);  // the CTA gave up
-  static_assert(2 * kMaxSlots * 8 + (kConsWarps + 3) * 16 + 2 * sizeof(TopKPart) + 5 * 8 + 16 <=
+  static_assert(2 * kMaxSlots * 8 + (kConsWarps + 3) * 16 + kConsWarps * 4 + 2 * sizeof(TopKPart) +
+                        5 * 8 + 16 <=
                     kSweepSmemExtra,
                 "k_stream scratch");
   // [2] top-K candidates of this row and the next (launched with kTopKSmem more)
@@ -488,18 +520,14 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
 
     // ---------------- merge
     t = warp_merge(t);
-    if (lane == 0) red[warp] = make_float4(t.m, t.s, t.u, 0.0f);
+    if (lane == 0) {
+      red[warp] = make_float4(t.m, t.s, t.u, 0.0f);
+      redm[warp] = t.m;
+    }
     cons_sync();
     if (tid == 0 && fix_ptr) Out::store1(fix_ptr, 0, fix_val);  // previous row's y entry
     fix_ptr = nullptr;
-    if (warp == 0) {
-      Tri x{-INFINITY, 0.0f, 0.0f};
-      if (lane < kConsWarps) {
-        const float4 v = red[lane];
-        x = Tri{v.x, v.y, v.z};
-      }
-      t = warp_merge(x);
-    }
+    if (warp == 0) t = block_merge(red, redm, lane);
     // top-K OPD signal (Sec. 5.2), a fixed per-token reward: the top-K warp's
     // part of this row and the row's lse (warp 0)
     float opd = 0.0f;
@@ -515,23 +543,44 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
     }
 
     // ---------------- epilogue (thread 0)
+    // Only what pass B needs comes before the barrier (the row's statistics,
+    // the per-token objective and the gradient coefficients); the stores of
+    // the row's outputs and the sampled token's entry come after it, while
+    // the other warps start pass B.
     char* drow = kGrad ? static_cast<char*>(a.dlogits) +
                              row * a.ld_out * static_cast<long long>(Out::kSize)
                        : nullptr;
+    bool bad = false;
+    float logp = 0.0f, H = 0.0f, lse = 0.0f, cc = 0.0f;
+    TokenTerms tt{};
     if (tid == 0) {
       // a row read after the CTA gave up, a bad target or a bad top-K
       // candidate: zeros
-      const bool bad = !yok || tk_bad || *abort;
-      if (!yok) atomicOr(err, kErrTarget);
-      if (tk_bad) atomicOr(err, kErrTopK);
+      bad = !yok || tk_bad || *abort;
       const float lnS = logf(t.s);
-      const float lse = fmaf(t.m, kLn2f, lnS);  // the reference is in log2 units
-      float H = lnS - t.u * kLn2f / t.s;
-      float logp = zy * a.s.invT - lse;
+      lse = fmaf(t.m, kLn2f, lnS);  // the reference is in log2 units
+      H = lnS - t.u * kLn2f / t.s;
+      logp = zy * a.s.invT - lse;
       if (bad) { logp = 0.0f; H = 0.0f; }
       if (a.s.topk > 0 && !bad) A -= a.s.opd_coef * opd;
-      TokenTerms tt = token_terms(logp, H, rho, q, a.q != nullptr, old, a.old != nullptr, A, a.s);
+      tt = token_terms(logp, H, rho, q, a.q != nullptr, old, a.old != nullptr, A, a.s);
       if (bad) tt = TokenTerms{0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, kFlagBad};
+      if (kGrad) {
+        cc = (msk && !bad) ? cscale : 0.0f;
+        const float ca = cc * (-tt.G + a.s.gamma * (H - lse));
+        const float cb = cc * a.s.gamma * a.s.invT;
+        const float L2 = t.m + __log2f(t.s);
+        const bool zero = (cc == 0.0f) || (ca == 0.0f && cb == 0.0f);
+        const bool fold = !zero && (cb == 0.0f);
+        const float off = fold ? (__log2f(fabsf(ca)) - L2) : -L2;
+        bc[0] = make_float4(off, ca, cb, 0.0f);
+        bci[0] = make_int4(zero, fold, (fold && ca < 0.0f) ? 1 : 0, 0);
+      }
+    }
+    cons_sync();
+    if (tid == 0) {
+      if (!yok) atomicOr(err, kErrTarget);
+      if (tk_bad) atomicOr(err, kErrTopK);
       if (a.out_logp) a.out_logp[row] = logp;
       if (a.out_H) a.out_H[row] = H;
       ws.logp[row] = logp;
@@ -544,24 +593,14 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
       ws.r[row] = tt.r;
       ws.rc[row] = tt.rc;
       ws.flags[row] = tt.flags;
-      if (kGrad) {
-        const float cc = (msk && !bad) ? cscale : 0.0f;
-        const float ca = cc * (-tt.G + a.s.gamma * (H - lse));
-        const float cb = cc * a.s.gamma * a.s.invT;
-        const float L2 = t.m + __log2f(t.s);
-        const bool zero = (cc == 0.0f) || (ca == 0.0f && cb == 0.0f);
-        const bool fold = !zero && (cb == 0.0f);
-        const float off = fold ? (__log2f(fabsf(ca)) - L2) : -L2;
-        bc[0] = make_float4(off, ca, cb, 0.0f);
-        bci[0] = make_int4(zero, fold, (fold && ca < 0.0f) ? 1 : 0, 0);
-        if (!zero) {
-          // cc [G (1 - p_y) + gamma p_y (log p_y + H)], 1 - p_y = -expm1(logp)
-          fix_ptr = drow + static_cast<long long>(y) * Out::kSize;
-          fix_val = cc * (tt.G * -expm1f(logp) + a.s.gamma * expf(logp) * (logp + H));
-        }
+      if (kGrad && cc != 0.0f && !bci[0].x) {
+        // cc [G (1 - p_y) + gamma p_y (log p_y + H)], 1 - p_y = -expm1(logp);
+        // written after the next row's merge barrier, which orders it after
+        // every store of this row
+        fix_ptr = drow + static_cast<long long>(y) * Out::kSize;
+        fix_val = cc * (tt.G * -expm1f(logp) + a.s.gamma * expf(logp) * (logp + H));
       }
     }
-    cons_sync();
 
     // ---------------- pass B
     if (kGrad) {
