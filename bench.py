@@ -206,13 +206,15 @@ def profiled_traffic(rows_now: int, workload: str, vocab: int):
     return float(tb.group(1)) * rows_now / int(rows.group(1))
 
 
-def sweep_kernel_name(vocab: int, elem_size: int) -> str:
-    """The sweep kernel the library picks for these rows in a fused call
-    (rows of 192 KB and more, 16-byte aligned, stream through one CTA each;
-    shorter rows go to the cluster kernel)."""
-    if vocab * elem_size >= 192 * 1024:
-        return "k_stream (fused fwd+bwd vocabulary sweep, one CTA per row)"
-    return "k_sweep (fused fwd+bwd vocabulary sweep, clusters sharing a row)"
+def sweep_kernel_name(vocab: int, elem_size: int, grad: bool = True) -> str:
+    """The sweep kernel the library picks for these rows (16-byte aligned
+    rows of 192 KB and more in a fused call, of 160 KB and more in a
+    forward-only one, stream through one CTA each; shorter rows go to the
+    cluster kernel)."""
+    kind = "fused fwd+bwd" if grad else "forward-only"
+    if vocab * elem_size >= (192 if grad else 160) * 1024:
+        return f"k_stream ({kind} vocabulary sweep, one CTA per row)"
+    return f"k_sweep ({kind} vocabulary sweep, clusters sharing a row)"
 
 
 def launches_per_call(params: dict, n_groups: int) -> int:
@@ -611,12 +613,19 @@ def run_ours(args, rank, world, local):
     bpr = algorithmic_bytes_per_row(w, dl_dtype)  # before w is released for the e2e leg
     kernel_name = sweep_kernel_name(V, w.logits.element_size())
     w_params, n_groups = dict(w.params), w.n_groups
-    launch_bytes = bpr * R
+    step_bytes = bpr * R
+    launch_bytes = step_bytes
+    if w_params.get("estimator", "grpo") == "gspo":
+        # GSPO's timed sweep is the forward-only one (k_seq and the gradient
+        # sweep k_bwd follow it): it reads the logits and writes no dLogits
+        launch_bytes = (bpr - V * torch.tensor([], dtype=dl_dtype).element_size()) * R
+        kernel_name = sweep_kernel_name(V, w.logits.element_size(), grad=False) + \
+            ", GSPO's first pass (k_bwd reads the logits again for dLogits)"
     sweep_avg = statistics.fmean(sweep_ms)
     peaks, peak_kind = measured_peaks()
     peak = float(peaks["hbm_gbs"])
     achieved = launch_bytes / (sweep_avg / 1e3) / 1e9
-    step_gbs = launch_bytes / (ms_step / 1e3) / 1e9
+    step_gbs = step_bytes / (ms_step / 1e3) / 1e9
 
     cpu = None
     # (the oracle's row pass covers the token-level estimators without
