@@ -343,6 +343,85 @@ rl_status rl_loss_shard_fwd_bwd(int32_t phase, int64_t row_offset, int64_t n_row
                                 rl_dtype dlogits_dtype, int64_t ld_out, void* workspace,
                                 size_t workspace_bytes, rl_stream stream);
 
+/* Phases of rl_loss_vocab_shard_fwd_bwd. */
+enum {
+  RL_VSHARD_COUNT = 1,    /* this shard's training tokens per trajectory        */
+  RL_VSHARD_PARTIAL = 2,  /* advantages; the forward sweep over the shard's
+                             columns, writing each row's partial sums          */
+  RL_VSHARD_SWEEP = 3,    /* merge of the gathered partial sums; dLogits over
+                             the shard's columns; the shard's partial statistics */
+  RL_VSHARD_FINISH = 4    /* the call's statistics from the combined partials   */
+};
+
+/* rl_loss_fwd_bwd with the VOCABULARY of one call split over shards (tensor
+ * parallelism: each rank holds a block of the logits' columns, as the
+ * paper's case study trains with TP 2, Sec. 9.1), optionally combined with
+ * a split of its rows as in rl_loss_shard_fwd_bwd (context / data
+ * parallelism, CP 4 there).
+ *
+ *  col_starts      HOST array of n_col_shards + 1 vocabulary ids: shard k
+ *                  holds columns [col_starts[k], col_starts[k+1]);
+ *                  col_starts[0] = 0, strictly increasing (every shard has a
+ *                  column), col_starts[n_col_shards] = the vocabulary size
+ *                  (<= INT32_MAX). 1 <= n_col_shards <= 64.
+ *  col_shard       this shard's index in col_starts.
+ *  logits          [n_rows, ld] of logits_dtype: this shard's columns of its
+ *                  rows (ld >= its column count); dlogits and ld_out alike.
+ *  targets         vocabulary ids in [0, col_starts[n_col_shards]), the same
+ *                  on every column shard of a row.
+ *  row_offset, n_rows_total, traj_counts, partials, stats: as in
+ *                  rl_loss_shard_fwd_bwd (one column shard of the whole rows:
+ *                  row_offset 0, n_rows_total = n_rows).
+ *  row_partials    [n_rows][4] floats (device, 16-byte aligned), written by
+ *                  PARTIAL: per row, m, s, u and zy, with m a reference in
+ *                  log2 units (a multiple of log2(e)/T of a logit),
+ *                  s = sum_j 2^(z_j log2(e)/T - m) and
+ *                  u = sum_j 2^(z_j log2(e)/T - m) (z_j log2(e)/T - m) over
+ *                  the shard's columns j, zy the target's logit if the target
+ *                  is one of them, else 0. m = NaN marks a row the shard gave
+ *                  up on (RL_ERR_DEVICE_TIMEOUT in its workspace): every
+ *                  shard then writes zeros for that row.
+ *  row_partials_all [n_col_shards][n_rows][4] floats (device, 16-byte
+ *                  aligned), read by SWEEP: every column shard's row_partials
+ *                  of the same rows, in shard order (an all-gather).
+ *
+ * Phases, in order, on one stream, with one workspace
+ * (rl_loss_workspace_size(n_rows, n_traj, n_groups)) per shard:
+ *   1. COUNT writes traj_counts; the caller sums it over the ROW shards.
+ *   2. PARTIAL computes the advantages and N from the summed counts (the
+ *      same on every shard) and writes row_partials. The caller gathers the
+ *      records of the COLUMN shards of its rows into row_partials_all.
+ *   3. SWEEP merges each row's records in shard order (every column shard
+ *      computes the same bits), writes token_logprobs and entropy (the
+ *      same on every column shard), dLogits over the shard's columns
+ *      (dlogits NULL: none) and `partials`. Column shards of the same rows
+ *      write the same partials: the caller combines them over the ROW
+ *      shards only, as rl_loss_partials says.
+ *   4. FINISH writes `stats` from the combined partials.
+ * A shard's log-probs, entropies and dLogits equal the unsharded call's up
+ * to the order of the row's floating-point sums (within the library's
+ * tolerances, not bit for bit). The logits are read twice (PARTIAL and the
+ * gradient in SWEEP), as for the split rl_loss_fwd / rl_loss_bwd pair.
+ * GSPO and top-K OPD return RL_ERR_UNSUPPORTED. A target outside the
+ * vocabulary is reported by SWEEP (RL_ERR_TARGET_OUT_OF_RANGE; the row gets
+ * zeros). Arguments a phase does not read may be NULL (COUNT: logits,
+ * outputs, dlogits, row_partials*, partials, stats; PARTIAL: outputs
+ * other than advantages and group_sizes, row_partials_all, dlogits,
+ * partials, stats; SWEEP: row_partials, stats; FINISH: everything but
+ * partials, stats and the stream). */
+rl_status rl_loss_vocab_shard_fwd_bwd(
+    int32_t phase, int32_t col_shard, int32_t n_col_shards, const int64_t* col_starts,
+    int64_t row_offset, int64_t n_rows_total, const void* logits, rl_dtype logits_dtype,
+    int64_t n_rows, int64_t ld, const int32_t* targets, const float* rollout_logprobs,
+    const float* ref_logprobs, const float* old_logprobs, const float* teacher_logprobs,
+    const float* rewards, const int32_t* group_id, const int32_t* cu_seqlens, int32_t n_traj,
+    int32_t n_groups, const uint8_t* loss_mask, const rl_loss_params* params,
+    float* token_logprobs, float* entropy, float* advantages, int32_t* group_sizes,
+    int32_t* traj_counts, float* row_partials, const float* row_partials_all,
+    rl_loss_partials* partials, rl_loss_stats* stats, float grad_loss,
+    const float* grad_loss_device, void* dlogits, rl_dtype dlogits_dtype, int64_t ld_out,
+    void* workspace, size_t workspace_bytes, rl_stream stream);
+
 /* rl_loss_fwd_bwd for callers that cannot allocate device memory at call
  * time (the paper has no counterpart; this is a deployment convenience).
  * Frameworks that reserve nearly all of HBM for their own pool, plain-C

@@ -302,3 +302,105 @@ def sharded_fwd_bwd_local(shards):
     for s in shards:
         s.partials.copy_(comb)
         s.finish()
+
+
+# ------------------------------------------------------ vocabulary-sharded calls
+
+class VocabShard:
+    """One shard of a vocabulary-sharded fused call
+    (rl_loss_vocab_shard_fwd_bwd): ``w.logits`` holds this shard's columns
+    [col_starts[col_shard], col_starts[col_shard + 1]) of its rows (a view of
+    a wider tensor is fine: its row stride is the ld), ``w.targets`` the
+    vocabulary ids; rows may be sharded as well (``row_offset``,
+    ``n_rows_total``, as in Shard). ``buf.dlogits`` holds the same columns.
+    The phases are ``count``, ``partial``, ``sweep`` and ``finish``; between
+    them the ROW shards' ``counts`` are summed, the COLUMN shards'
+    ``row_partials`` gathered into ``row_partials_all`` (exchange_row_partials)
+    and the ROW shards' ``partials`` combined."""
+
+    def __init__(self, w, col_shard: int, col_starts, buf: Buffers, row_offset: int = 0,
+                 n_rows_total: int | None = None, params=None, grad_loss=1.0):
+        self.w, self.buf = w, buf
+        self.col_shard, self.col_starts = int(col_shard), [int(c) for c in col_starts]
+        self.row_offset = int(row_offset)
+        self.n_rows_total = w.n_rows if n_rows_total is None else int(n_rows_total)
+        self.params = dict(w.params if params is None else params)
+        self.grad_loss = grad_loss
+        dev = w.targets.device
+        R, n_shards = w.n_rows, len(self.col_starts) - 1
+        self.counts = torch.zeros(int(w.rewards.shape[0]), dtype=torch.int32, device=dev)
+        self.row_partials = torch.zeros((R, 4), dtype=torch.float32, device=dev)
+        self.row_partials_all = torch.zeros((n_shards, R, 4), dtype=torch.float32, device=dev)
+        self.partials = torch.zeros(ml.PARTIALS_DOUBLES, dtype=torch.float64, device=dev)
+
+    def _call(self, phase, forward_only=False):
+        w, b = self.w, self.buf
+        ml.rl_loss_vocab_shard_fwd_bwd(
+            phase, self.col_shard, self.col_starts, self.row_offset, self.n_rows_total, w.logits,
+            w.targets, w.rollout_logprobs, w.ref_logprobs, w.old_logprobs, w.teacher_logprobs,
+            w.rewards, w.group_id, w.cu_seqlens, w.n_groups, w.loss_mask, self.params,
+            b.token_logprobs, b.entropy, b.advantages, b.group_sizes, self.counts,
+            self.row_partials, self.row_partials_all, self.partials, b.stats,
+            None if forward_only else b.dlogits, b.workspace, grad_loss=self.grad_loss)
+
+    def count(self):
+        self._call(ml.RL_VSHARD_COUNT)
+
+    def partial(self):
+        self._call(ml.RL_VSHARD_PARTIAL)
+
+    def sweep(self, forward_only=False):
+        self._call(ml.RL_VSHARD_SWEEP, forward_only)
+
+    def finish(self):
+        self._call(ml.RL_VSHARD_FINISH)
+
+
+def exchange_row_partials(row_partials: torch.Tensor, row_partials_all: torch.Tensor,
+                          group=None):
+    """Gather the column shards' per-row records over the ranks of ``group``
+    (rank k of the group holds column shard k): row_partials_all[k] =
+    rank k's row_partials."""
+    import torch.distributed as dist
+    # (rank k's rows land at rows [k R, (k + 1) R) of the flattened output)
+    dist.all_gather_into_tensor(row_partials_all.view(-1, 4), row_partials.contiguous(),
+                                group=group)
+
+
+def vocab_sharded_fwd_bwd(shard: VocabShard, col_group=None, row_group=None):
+    """This rank's shard of a vocabulary-sharded fused call over
+    torch.distributed: ``col_group`` holds the column shards of this rank's
+    rows (in shard order), ``row_group`` the ranks of the same column shard
+    that hold the other rows (None with a single row shard)."""
+    shard.count()
+    if row_group is not None:
+        exchange_counts(shard.counts, row_group)
+    shard.partial()
+    exchange_row_partials(shard.row_partials, shard.row_partials_all, col_group)
+    shard.sweep()
+    if row_group is not None:
+        exchange_partials(shard.partials, row_group)
+    shard.finish()
+
+
+def vocab_sharded_fwd_bwd_local(shards):
+    """Shards of one call driven from one process (for instance on one
+    GPU), ``shards[i][k]`` the column shard k of row shard i: the exchanges
+    are sums, stacks and maxima over the shards' tensors."""
+    flat = [s for row in shards for s in row]
+    for s in flat:
+        s.count()
+    total = torch.stack([row[0].counts for row in shards]).sum(0)
+    for s in flat:
+        s.counts.copy_(total)
+        s.partial()
+    for row in shards:
+        gathered = torch.stack([s.row_partials for s in row])
+        for s in row:
+            s.row_partials_all.copy_(gathered)
+            s.sweep()
+    p = torch.stack([row[0].partials for row in shards])
+    comb = torch.cat([p[:, :ml.PARTIALS_SUMS].sum(0), p[:, ml.PARTIALS_SUMS:].max(0).values])
+    for s in flat:
+        s.partials.copy_(comb)
+        s.finish()

@@ -21,7 +21,7 @@ OUT_DIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(OUT_DIR, "libmilesloss.so")
 
 SOURCES = ["abi.cu", "abi_noalloc.cu", "k_advantages.cu", "k_sweep.cu", "k_sweep_topk.cu", "k_stream.cu",
-           "k_seq.cu", "k_stats.cu", "k_bwd.cu"]
+           "k_seq.cu", "k_stats.cu", "k_bwd.cu", "k_vshard.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
 

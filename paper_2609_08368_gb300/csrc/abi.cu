@@ -325,6 +325,11 @@ struct FwdIn {
   const int* counts_in = nullptr;
   int* counts_out = nullptr;
   rl_loss_partials* part_out = nullptr;
+  // a column shard of a vocabulary-sharded call (rl_loss_vocab_shard_fwd_bwd):
+  // the logits are columns [col0, col0 + V); part_rows receives each row's
+  // partial sums in place of the sweep's epilogue
+  long long col0 = 0;
+  float4* part_rows = nullptr;
 };
 
 rl_status check_fwd(const FwdIn& f, bool need_logits = true) {
@@ -392,7 +397,8 @@ void record(cudaEvent_t ev, cudaStream_t s) {
 }
 
 // The gradient sweep from the per-row state in the workspace (lse, H, G).
-rl_status launch_bwd(const Common& c, const GradOut& go, const WsPtrs& ws, cudaStream_t s) {
+rl_status launch_bwd(const Common& c, const GradOut& go, const WsPtrs& ws, cudaStream_t s,
+                     long long col0 = 0) {
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return RL_ERR_CUDA;
   if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
@@ -415,6 +421,7 @@ rl_status launch_bwd(const Common& c, const GradOut& go, const WsPtrs& ws, cudaS
   b.invT = 1.0f / c.p->temperature;
   b.k = 1.4426950408889634f / c.p->temperature;
   b.gamma = c.p->entropy_coef;
+  b.col0 = col0;
   b.ws = ws;
   // one wave of resident blocks (grid-stride over the tiles): a second,
   // partial wave would run with fewer loads in flight
@@ -548,6 +555,8 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     ta.s = sc;
     ta.ws = ws;
     ta.stall_ns = stall;
+    ta.col0 = f.col0;
+    ta.part_rows = shift(f.part_rows, r0);
     const long long grid = std::min<long long>(ctas, c.R);
     record(t_ev_begin, s);
     st = launch(fn, dim3(static_cast<unsigned>(grid)), dim3(threads), sp.smem, 1, s,
@@ -590,6 +599,8 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     sa.s = sc;
     sa.ws = ws;
     sa.stall_ns = stall;
+    sa.col0 = f.col0;
+    sa.part_rows = shift(f.part_rows, r0);
     record(t_ev_begin, s);
     st = launch(fn, dim3(static_cast<unsigned>(n_cl * pl.C)), dim3(pl.threads), pl.smem, pl.C,
                 s, &sa);
@@ -770,6 +781,124 @@ rl_status rl_loss_shard_fwd_bwd(int32_t phase, int64_t row_offset, int64_t n_row
   return run_fwd(f, grad ? &go : nullptr, s, RL_PHASE_ALL);
 }
 
+rl_status rl_loss_vocab_shard_fwd_bwd(
+    int32_t phase, int32_t col_shard, int32_t n_col_shards, const int64_t* col_starts,
+    int64_t row_offset, int64_t n_rows_total, const void* logits, rl_dtype logits_dtype,
+    int64_t n_rows, int64_t ld, const int32_t* targets, const float* rollout_logprobs,
+    const float* ref_logprobs, const float* old_logprobs, const float* teacher_logprobs,
+    const float* rewards, const int32_t* group_id, const int32_t* cu_seqlens, int32_t n_traj,
+    int32_t n_groups, const uint8_t* loss_mask, const rl_loss_params* params,
+    float* token_logprobs, float* entropy, float* advantages, int32_t* group_sizes,
+    int32_t* traj_counts, float* row_partials, const float* row_partials_all,
+    rl_loss_partials* partials, rl_loss_stats* stats, float grad_loss,
+    const float* grad_loss_device, void* dlogits, rl_dtype dlogits_dtype, int64_t ld_out,
+    void* workspace, size_t workspace_bytes, rl_stream stream) {
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (phase == RL_VSHARD_FINISH) {
+    if (!partials || !stats) return RL_ERR_INVALID_ARG;
+    FinishArgs fa{partials, stats};
+    return launch(finish_kernel(), dim3(1), dim3(32), 0, 1, s, &fa);
+  }
+  if (phase != RL_VSHARD_COUNT && phase != RL_VSHARD_PARTIAL && phase != RL_VSHARD_SWEEP)
+    return RL_ERR_INVALID_ARG;
+  // the column partition: col_starts[0] = 0 < col_starts[1] < ... (every
+  // shard has a column), vocabulary ids fit the int32 targets
+  if (n_col_shards < 1 || n_col_shards > kMaxColShards || !col_starts) return RL_ERR_INVALID_ARG;
+  if (col_shard < 0 || col_shard >= n_col_shards || col_starts[0] != 0) return RL_ERR_INVALID_ARG;
+  for (int k = 0; k < n_col_shards; ++k)
+    if (col_starts[k + 1] <= col_starts[k]) return RL_ERR_INVALID_ARG;
+  if (col_starts[n_col_shards] > INT32_MAX) return RL_ERR_INVALID_ARG;
+  const long long col0 = col_starts[col_shard];
+  const long long vocab = col_starts[col_shard + 1] - col0;
+  if (row_offset < 0 || n_rows < 0 || n_rows_total < 0 || row_offset > n_rows_total - n_rows)
+    return RL_ERR_INVALID_ARG;
+  if (n_traj > 0 && !traj_counts) return RL_ERR_INVALID_ARG;
+  if (!params) return RL_ERR_INVALID_ARG;
+  // GSPO needs whole trajectories before any gradient; top-K OPD candidates
+  // would be spread over the shards
+  if (params->estimator == RL_EST_GSPO || (params->opd_topk > 0 && params->opd_coef != 0.0f))
+    return RL_ERR_UNSUPPORTED;
+  const bool count = phase == RL_VSHARD_COUNT;
+  const bool sweep = phase == RL_VSHARD_SWEEP;
+  FwdIn f{{logits, logits_dtype, n_rows, vocab, ld, targets, loss_mask, params},
+          rollout_logprobs, ref_logprobs, old_logprobs, teacher_logprobs, rewards,
+          group_id, cu_seqlens, n_traj, n_groups, sweep ? token_logprobs : nullptr,
+          sweep ? entropy : nullptr, count ? nullptr : advantages,
+          count ? nullptr : group_sizes, nullptr, workspace, workspace_bytes};
+  f.row0 = row_offset;
+  f.R_total = n_rows_total;
+  f.col0 = col0;
+  if (count) {
+    f.counts_out = traj_counts;
+    rl_status st = check_fwd(f, false);
+    if (st != RL_OK) return st;
+    return run_fwd(f, nullptr, s, RL_PHASE_BEGIN);
+  }
+  if (phase == RL_VSHARD_PARTIAL) {
+    // advantages and N from the summed counts, then the forward sweep over
+    // this shard's columns, writing each row's partial sums
+    if (n_rows > 0 && (!row_partials || !aligned16(row_partials))) return RL_ERR_INVALID_ARG;
+    f.counts_in = traj_counts;
+    f.part_rows = reinterpret_cast<float4*>(row_partials);
+    rl_status st = check_fwd(f, n_rows > 0);
+    if (st != RL_OK) return st;
+    return run_fwd(f, nullptr, s, RL_PHASE_BEGIN | RL_PHASE_ROWS);
+  }
+  // SWEEP: merge the gathered records, dLogits over this shard's columns,
+  // this shard's partial statistics
+  if (!partials) return RL_ERR_INVALID_ARG;
+  if (n_rows > 0 && (!row_partials_all || !aligned16(row_partials_all))) return RL_ERR_INVALID_ARG;
+  rl_status st = check_fwd(f, n_rows > 0 && dlogits != nullptr);
+  if (st != RL_OK) return st;
+  GradOut go{grad_loss, grad_loss_device, dlogits, dlogits_dtype, ld_out};
+  const bool grad = dlogits != nullptr;
+  if (grad) {
+    st = check_grad(f.c, go);
+    if (st != RL_OK) return st;
+  }
+  const WsPtrs ws = WsPtrs::at(workspace, WsLayout::make(n_rows, n_traj, n_groups));
+  if (n_rows > 0) {
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return RL_ERR_CUDA;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return RL_ERR_CUDA;
+    MergeArgs ma;
+    ma.R = n_rows;
+    ma.n_shards = n_col_shards;
+    for (int k = 0; k <= n_col_shards; ++k) ma.col_starts[k] = col_starts[k];
+    ma.all = reinterpret_cast<const float4*>(row_partials_all);
+    ma.targets = targets;
+    ma.rho = rollout_logprobs;
+    ma.q = ref_logprobs;
+    ma.old = old_logprobs;
+    ma.mask = loss_mask;
+    ma.out_logp = token_logprobs;
+    ma.out_H = entropy;
+    ma.s = scalars(params);
+    ma.ws = ws;
+    const long long blocks = std::min<long long>((n_rows + kMergeThreads - 1) / kMergeThreads,
+                                                 static_cast<long long>(sms) * 8);
+    st = launch(merge_kernel(), dim3(static_cast<unsigned>(blocks)), dim3(kMergeThreads), 0, 1,
+                s, &ma);
+    if (st != RL_OK) return st;
+    if (grad) {
+      st = launch_bwd(f.c, go, ws, s, col0);
+      if (st != RL_OK) return st;
+    }
+  }
+  StatArgs ta;
+  ta.R = n_rows;
+  ta.mask = loss_mask;
+  ta.rho = rollout_logprobs;
+  ta.out = nullptr;
+  ta.part_out = partials;
+  ta.ws = ws;
+  long long blocks = (n_rows + kStatThreads - 1) / kStatThreads;
+  blocks = std::max<long long>(1, std::min<long long>(blocks, kMaxStatBlocks));
+  return launch(stats_kernel(), dim3(static_cast<unsigned>(blocks)), dim3(kStatThreads), 0, 1, s,
+                &ta);
+}
+
 rl_status rl_loss_bwd(const void* logits, rl_dtype logits_dtype, int64_t n_rows, int64_t vocab,
                       int64_t ld, const int32_t* targets, const uint8_t* loss_mask,
                       const rl_loss_params* params, float grad_loss,
@@ -853,6 +982,6 @@ rl_status rl_set_launch_overrides(const rl_launch_overrides* o) {
   return RL_OK;
 }
 
-int32_t rl_loss_abi_version(void) { return 110; }
+int32_t rl_loss_abi_version(void) { return 120; }
 
 }  // extern "C"

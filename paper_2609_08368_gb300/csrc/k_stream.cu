@@ -442,13 +442,16 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
     uint8_t msk = 0;
     bool yok = false;
     if (tid == 0) {
-      y = a.targets[row];
+      // the target's column in this call's logits (-1 outside them: a bad
+      // target, or another shard's column in a vocabulary-sharded call)
+      const long long yl = a.targets[row] - a.col0;
+      y = (yl >= 0 && yl < a.V) ? static_cast<int>(yl) : -1;
       rho = a.rho[row];
       if (a.q) q = a.q[row];
       if (a.old) old = a.old[row];
       A = ws.a_row[row];
       msk = a.mask[row];
-      yok = (y >= 0) && (y < a.V);
+      yok = y >= 0;
       if (yok && y >= tail0) zy = In::load1(grow, y);
     }
     const int yv = yok ? y / V8 : -1;  // thread 0 only
@@ -553,7 +556,12 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
     bool bad = false;
     float logp = 0.0f, H = 0.0f, lse = 0.0f, cc = 0.0f;
     TokenTerms tt{};
-    if (tid == 0) {
+    if (tid == 0 && a.part_rows) {
+      // vocabulary-sharded forward: the row's partial sums over this
+      // shard's columns (a row read after the CTA gave up is marked NaN)
+      a.part_rows[row] = *abort ? make_float4(NAN, 0.0f, 0.0f, 0.0f)
+                                : make_float4(t.m, t.s, t.u, yok ? zy : 0.0f);
+    } else if (tid == 0) {
       // a row read after the CTA gave up, a bad target or a bad top-K
       // candidate: zeros
       bad = !yok || tk_bad || *abort;
@@ -578,7 +586,7 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
       }
     }
     cons_sync();
-    if (tid == 0) {
+    if (tid == 0 && !a.part_rows) {
       if (!yok) atomicOr(err, kErrTarget);
       if (tk_bad) atomicOr(err, kErrTopK);
       if (a.out_logp) a.out_logp[row] = logp;

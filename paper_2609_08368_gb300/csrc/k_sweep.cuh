@@ -264,7 +264,10 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
     float rho = 0.0f, q = 0.0f, old = 0.0f, A = 0.0f;
     uint8_t msk = 0;
     if (tid == 0) {
-      y = a.targets[row];
+      // the target's column in this call's logits (-1 outside them: a bad
+      // target, or another shard's column in a vocabulary-sharded call)
+      const long long yl = a.targets[row] - a.col0;
+      y = (yl >= 0 && yl < a.V) ? static_cast<int>(yl) : -1;
       rho = a.rho[row];
       if (a.q) q = a.q[row];
       if (a.old) old = a.old[row];
@@ -344,7 +347,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
     t = block_merge<kWarps>(t, red);
 
     // ---------------- exchange and epilogue (thread 0)
-    const bool yok = (tid == 0) && (y >= 0) && (y < a.V);
+    const bool yok = (tid == 0) && (y >= 0);
     const int owner = yok ? y / slice : -1;
     Tri tot{t.m, t.s, t.u};  // the row's statistics (thread 0)
     float zy_all = 0.0f;
@@ -397,7 +400,13 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
         }
       }
     }
-    if (tid == 0) {
+    if (tid == 0 && a.part_rows) {
+      // vocabulary-sharded forward: the row's partial sums over this
+      // shard's columns (a row read after the CTA gave up is marked NaN)
+      if (crank == 0)
+        a.part_rows[row] = *abort ? make_float4(NAN, 0.0f, 0.0f, 0.0f)
+                                  : make_float4(tot.m, tot.s, tot.u, yok ? zy_all : 0.0f);
+    } else if (tid == 0) {
       // a row read after the CTA gave up, a bad target or a bad top-K
       // candidate: zeros
       const bool bad = !yok || (topk && tkp.bad) || *abort;

@@ -48,6 +48,12 @@ struct SweepArgs {
   // barrier nothing completes, bounded by this many nanoseconds, so that the
   // timeout path runs (see rl_launch_overrides).
   unsigned long long stall_ns;
+  // A vocabulary-sharded call (forward only): the logits are columns
+  // [col0, col0 + V) of the vocabulary, a target outside them is another
+  // shard's, and each row's partial sums go to part_rows (RowPartial) in
+  // place of the epilogue. Unsharded calls: 0 and null.
+  long long col0;
+  float4* part_rows;
 };
 
 struct StreamArgs {
@@ -74,6 +80,8 @@ struct StreamArgs {
   LossScalars s;
   WsPtrs ws;
   unsigned long long stall_ns;  // test hook, as in SweepArgs (the consumers' first wait)
+  long long col0;               // vocabulary-sharded calls, as in SweepArgs
+  float4* part_rows;
 };
 
 struct AdvArgs {
@@ -139,6 +147,29 @@ struct BwdArgs {
   float grad_loss;
   const float* grad_loss_dev;
   float invT, k, gamma;
+  long long col0;  // the logits are columns [col0, col0 + V) of the vocabulary
+  WsPtrs ws;
+};
+
+// The merge of a vocabulary-sharded call: each row's partial sums from every
+// column shard (RowPartial, shard-major: all[k * R + row]) in shard order,
+// then the row's statistics and per-token objective, as the fused sweep's
+// epilogue writes them.
+constexpr int kMaxColShards = 64;
+constexpr int kMergeThreads = 256;
+struct MergeArgs {
+  long long R;
+  int n_shards;
+  long long col_starts[kMaxColShards + 1];
+  const float4* all;
+  const int* targets;  // vocabulary ids
+  const float* rho;
+  const float* q;
+  const float* old;
+  const uint8_t* mask;
+  float* out_logp;
+  float* out_H;
+  LossScalars s;
   WsPtrs ws;
 };
 
@@ -176,6 +207,7 @@ constexpr int kMaxGroupBlocks = 65535;
 // (a launch costs more than their double arithmetic on one SM).
 constexpr int kInlineGroups = 8;
 const void* seq_kernel();
+const void* merge_kernel();   // vocabulary-sharded calls: k_vmerge
 const void* stats_kernel();
 const void* finish_kernel();  // rl_loss_stats from combined partials (one thread)
 

@@ -18,6 +18,7 @@ RL_OK = 0
 RL_BF16, RL_F32 = 0, 1
 RL_PHASE_BEGIN, RL_PHASE_ROWS, RL_PHASE_END, RL_PHASE_ALL = 1, 2, 4, 7
 RL_SHARD_COUNT, RL_SHARD_SWEEP, RL_SHARD_FINISH = 1, 2, 4
+RL_VSHARD_COUNT, RL_VSHARD_PARTIAL, RL_VSHARD_SWEEP, RL_VSHARD_FINISH = 1, 2, 3, 4
 PARTIALS_SUMS = 14   # rl_loss_partials: sum[9] and count[5], combined by addition
 PARTIALS_DOUBLES = 16  # ... then max[2], combined by maximum
 CORRECTIONS = {"none": 0, "tis": 1, "clip_or_pop": 2}
@@ -125,10 +126,13 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
     lib.rl_loss_fwd_bwd_noalloc.argtypes = fwd_common + [F32, P, P, I32, I64, P]
     lib.rl_loss_shard_fwd_bwd.argtypes = ([I32, I64, I64] + fwd_common[:-1] + [P, P, P] +
                                           [F32, P, P, I32, I64, P, SZ, P])
+    lib.rl_loss_vocab_shard_fwd_bwd.argtypes = (
+        [I32, I32, I32, P, I64, I64, P, I32, I64, I64] + fwd_common[5:-1] + [P, P, P, P, P] +
+        [F32, P, P, I32, I64, P, SZ, P])
     lib.rl_loss_noalloc_check_device_error.argtypes = []
     for name in ("rl_loss_workspace_size", "rl_loss_fwd", "rl_loss_fwd_bwd", "rl_loss_fwd_bwd_rows",
                  "rl_loss_bwd", "rl_loss_fwd_bwd_noalloc", "rl_loss_noalloc_check_device_error",
-                 "rl_loss_shard_fwd_bwd",
+                 "rl_loss_shard_fwd_bwd", "rl_loss_vocab_shard_fwd_bwd",
                  "rl_launch_overrides_init", "rl_set_launch_overrides",
                  "rl_loss_check_device_error", "rl_set_sweep_events", "rl_loss_abi_version"):
         getattr(lib, name).restype = ctypes.c_int32
@@ -337,6 +341,46 @@ def rl_loss_shard_fwd_bwd(phase, row_offset, n_rows_total, logits, targets, roll
         _ptr(entropy), _ptr(advantages), _ptr(group_sizes), _ptr(traj_counts), _ptr(partials),
         _ptr(stats), float(grad_loss), _ptr(grad_loss_device), _ptr(dlogits), ddt, ld_out,
         _ptr(workspace), ws_bytes, _stream(stream)), "rl_loss_shard_fwd_bwd")
+
+
+def rl_loss_vocab_shard_fwd_bwd(phase, col_shard, col_starts, row_offset, n_rows_total, logits,
+                                targets, rollout_logprobs, ref_logprobs, old_logprobs,
+                                teacher_logprobs, rewards, group_id, cu_seqlens, n_groups,
+                                loss_mask, params, token_logprobs, entropy, advantages,
+                                group_sizes, traj_counts, row_partials, row_partials_all,
+                                partials, stats, dlogits, workspace, n_rows=None,
+                                logits_dtype=None, grad_loss=1.0, grad_loss_device=None,
+                                stream=None):
+    """One phase of a column shard's part of a vocabulary-sharded call.
+    ``col_starts`` is a host sequence of n_col_shards + 1 vocabulary ids;
+    ``logits`` / ``dlogits`` hold this shard's columns of its rows;
+    ``row_partials`` is float32 [n_rows, 4] and ``row_partials_all`` float32
+    [n_col_shards, n_rows, 4] (device)."""
+    import torch
+    cs = [int(c) for c in col_starts]
+    n_shards = len(cs) - 1
+    c_arr = (ctypes.c_int64 * len(cs))(*cs)
+    V = cs[col_shard + 1] - cs[col_shard] if 0 <= col_shard < n_shards else 1
+    n_traj = int(rewards.shape[0]) if rewards is not None else 0
+    if logits is not None:
+        ldt, ld, R = _dtype_code(logits), int(logits.stride(0)), int(logits.shape[0])
+    else:
+        ldt = _dtype_code(torch.empty(0, dtype=logits_dtype or torch.bfloat16))
+        ld, R = V, int(n_rows if n_rows is not None else targets.shape[0])
+    if dlogits is not None:
+        ddt, ld_out = _dtype_code(dlogits), int(dlogits.stride(0))
+    else:
+        ddt, ld_out = ldt, V
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(load().rl_loss_vocab_shard_fwd_bwd(
+        int(phase), int(col_shard), n_shards, ctypes.cast(c_arr, ctypes.c_void_p),
+        int(row_offset), int(n_rows_total), _ptr(logits), ldt, R, ld, _ptr(targets),
+        _ptr(rollout_logprobs), _ptr(ref_logprobs), _ptr(old_logprobs), _ptr(teacher_logprobs),
+        _ptr(rewards), _ptr(group_id), _ptr(cu_seqlens), n_traj, int(n_groups), _ptr(loss_mask),
+        ctypes.byref(_params(params)), _ptr(token_logprobs), _ptr(entropy), _ptr(advantages),
+        _ptr(group_sizes), _ptr(traj_counts), _ptr(row_partials), _ptr(row_partials_all),
+        _ptr(partials), _ptr(stats), float(grad_loss), _ptr(grad_loss_device), _ptr(dlogits), ddt,
+        ld_out, _ptr(workspace), ws_bytes, _stream(stream)), "rl_loss_vocab_shard_fwd_bwd")
 
 
 def rl_loss_noalloc_check_device_error() -> int:

@@ -42,7 +42,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert lib.rl_loss_abi_version() == 110
+    assert lib.rl_loss_abi_version() == 120
     seen = set()
     for code in range(0, 10):
         s = ml.status_string(code)
@@ -267,3 +267,47 @@ def test_sharded_entry_validates(lib):
     assert call(ml.RL_SHARD_FINISH, partials=None) == RL_ERR_INVALID_ARG
     assert call(ml.RL_SHARD_FINISH, stats=None) == RL_ERR_INVALID_ARG
     assert call(ml.RL_SHARD_COUNT, params=gspo) == 2          # GSPO: whole calls only
+
+
+def test_vocab_sharded_entry_validates(lib):
+    """Every argument error of rl_loss_vocab_shard_fwd_bwd is caught on the
+    host, before anything is enqueued (no GPU is needed)."""
+    v = ctypes.c_void_p
+    p = ml.make_params()
+
+    def call(phase, shard=0, starts=(0, 40, 64), r0=0, total=16, R=16, params=p, counts=FAKE,
+             rp=FAKE, rp_all=FAKE, partials=FAKE, stats=FAKE, ld=40, starts_ptr=True):
+        arr = (ctypes.c_int64 * len(starts))(*starts)
+        return lib.rl_loss_vocab_shard_fwd_bwd(
+            phase, shard, len(starts) - 1, ctypes.cast(arr, v) if starts_ptr else None, r0, total,
+            v(FAKE), 0, R, ld, v(FAKE), v(FAKE), None, None, None, v(FAKE), v(FAKE), v(FAKE), 2, 1,
+            v(FAKE), ctypes.byref(params), v(FAKE), v(FAKE), v(FAKE), v(FAKE), v(counts), v(rp),
+            v(rp_all), v(partials), v(stats), 1.0, None, v(FAKE), 0, 64, v(FAKE * 2), 1 << 30,
+            None)
+    C, PA, SW, FI = (ml.RL_VSHARD_COUNT, ml.RL_VSHARD_PARTIAL, ml.RL_VSHARD_SWEEP,
+                     ml.RL_VSHARD_FINISH)
+    assert call(0) == RL_ERR_INVALID_ARG                               # no phase
+    assert call(5) == RL_ERR_INVALID_ARG
+    assert call(C, starts_ptr=False) == RL_ERR_INVALID_ARG             # no column partition
+    assert call(C, starts=(1, 40, 64)) == RL_ERR_INVALID_ARG           # does not start at 0
+    assert call(C, starts=(0, 40, 40)) == RL_ERR_INVALID_ARG           # an empty shard
+    assert call(C, starts=(0, 50, 40)) == RL_ERR_INVALID_ARG           # decreasing
+    assert call(C, starts=(0, 40, 1 << 31)) == RL_ERR_INVALID_ARG      # ids past int32
+    assert call(C, starts=tuple(range(66))) == RL_ERR_INVALID_ARG      # 65 shards
+    assert call(C, shard=2) == RL_ERR_INVALID_ARG                      # no such shard
+    assert call(C, shard=-1) == RL_ERR_INVALID_ARG
+    assert call(PA, ld=39) == RL_ERR_INVALID_ARG                       # ld below the shard's 40 columns
+    assert call(C, r0=8, total=16, R=9) == RL_ERR_INVALID_ARG          # rows past the call
+    assert call(C, counts=None) == RL_ERR_INVALID_ARG
+    assert call(PA, rp=None) == RL_ERR_INVALID_ARG
+    assert call(PA, rp=FAKE + 4) == RL_ERR_INVALID_ARG                 # records not 16-byte aligned
+    assert call(SW, rp_all=None) == RL_ERR_INVALID_ARG
+    assert call(SW, rp_all=FAKE + 8) == RL_ERR_INVALID_ARG
+    assert call(SW, partials=None) == RL_ERR_INVALID_ARG
+    assert call(FI, partials=None) == RL_ERR_INVALID_ARG
+    assert call(FI, stats=None) == RL_ERR_INVALID_ARG
+    assert call(C, params=ml.make_params(estimator="gspo")) == 2       # RL_ERR_UNSUPPORTED
+    tk = ml.make_params(opd_coef=0.5, opd_topk=4, opd_topk_ids=_Ptr(FAKE),
+                        opd_topk_teacher=_Ptr(FAKE))
+    assert call(PA, params=tk) == 2
+    assert call(PA, params=ml.make_params(temperature=0.0)) == RL_ERR_INVALID_ARG
