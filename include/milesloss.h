@@ -299,8 +299,11 @@ rl_status rl_loss_fwd_bwd_rows(int32_t phase, int64_t row_begin, int64_t row_end
 enum {
   RL_SHARD_COUNT = 1,  /* this shard's training tokens per trajectory        */
   RL_SHARD_SWEEP = 2,  /* advantages, the sweep over the shard's rows, dLogits
-                          and the shard's partial statistics                 */
-  RL_SHARD_FINISH = 4  /* the call's statistics from the combined partials   */
+                          and the shard's partial statistics (GSPO: the
+                          forward sweep and the per-trajectory sums)          */
+  RL_SHARD_FINISH = 4, /* the call's statistics from the combined partials   */
+  RL_SHARD_SEQ = 8     /* GSPO only, after SWEEP: the trajectories' terms from
+                          the added sums, dLogits, partial statistics        */
 };
 
 /* rl_loss_fwd_bwd with the rows of one call spread over several shards (one
@@ -320,13 +323,21 @@ enum {
  *      N, dLogits (dlogits NULL: forward only) and writes `partials`. The
  *      caller combines the shards' partials as rl_loss_partials says.
  *   3. RL_SHARD_FINISH writes `stats` from the combined partials.
+ * GSPO (a token's gradient needs its whole trajectory's sequence ratio) takes
+ * one more exchange: SWEEP runs the forward sweep and writes
+ * traj_sums[n_traj][2] (double, device): per trajectory, the sums over this
+ * shard's training tokens of (log-prob - base log-prob) and of the
+ * correction weight. The caller adds traj_sums over the shards in place;
+ * RL_SHARD_SEQ then computes each trajectory's sequence ratio and terms,
+ * dLogits and `partials`; FINISH as above.
  * Each shard's outputs for its rows (log-probs, entropies, dLogits) are those
- * of the unsharded call; the statistics differ from it only in the order of
- * their floating-point sums. Every phase of a shard uses the same
- * workspace (rl_loss_workspace_size(n_rows, n_traj, n_groups)), in order, on
- * one stream. GSPO, whose gradient needs whole trajectories, returns
- * RL_ERR_UNSUPPORTED. Arguments a phase does not read may be NULL (COUNT:
- * logits, outputs, dlogits, partials, stats; FINISH: everything but
+ * of the unsharded call (GSPO: up to the order of the per-trajectory sums);
+ * the statistics differ from it only in the order of their floating-point
+ * sums. Every phase of a shard uses the same workspace
+ * (rl_loss_workspace_size(n_rows, n_traj, n_groups)), in order, on one
+ * stream. Arguments a phase does not read may be NULL (COUNT: logits,
+ * outputs, dlogits, traj_sums, partials, stats; SWEEP without GSPO:
+ * traj_sums; GSPO's SWEEP: dlogits, partials, stats; FINISH: everything but
  * partials, stats and the stream). */
 rl_status rl_loss_shard_fwd_bwd(int32_t phase, int64_t row_offset, int64_t n_rows_total,
                                 const void* logits, rl_dtype logits_dtype, int64_t n_rows,
@@ -337,7 +348,7 @@ rl_status rl_loss_shard_fwd_bwd(int32_t phase, int64_t row_offset, int64_t n_row
                                 const int32_t* cu_seqlens, int32_t n_traj, int32_t n_groups,
                                 const uint8_t* loss_mask, const rl_loss_params* params,
                                 float* token_logprobs, float* entropy, float* advantages,
-                                int32_t* group_sizes, int32_t* traj_counts,
+                                int32_t* group_sizes, int32_t* traj_counts, double* traj_sums,
                                 rl_loss_partials* partials, rl_loss_stats* stats,
                                 float grad_loss, const float* grad_loss_device, void* dlogits,
                                 rl_dtype dlogits_dtype, int64_t ld_out, void* workspace,
@@ -350,7 +361,9 @@ enum {
                              columns, writing each row's partial sums          */
   RL_VSHARD_SWEEP = 3,    /* merge of the gathered partial sums; dLogits over
                              the shard's columns; the shard's partial statistics */
-  RL_VSHARD_FINISH = 4    /* the call's statistics from the combined partials   */
+  RL_VSHARD_FINISH = 4,   /* the call's statistics from the combined partials   */
+  RL_VSHARD_SEQ = 5       /* GSPO only, after SWEEP: the trajectories' terms from
+                             the added sums, dLogits, partial statistics       */
 };
 
 /* rl_loss_fwd_bwd with the VOCABULARY of one call split over shards (tensor
@@ -369,9 +382,9 @@ enum {
  *                  rows (ld >= its column count); dlogits and ld_out alike.
  *  targets         vocabulary ids in [0, col_starts[n_col_shards]), the same
  *                  on every column shard of a row.
- *  row_offset, n_rows_total, traj_counts, partials, stats: as in
- *                  rl_loss_shard_fwd_bwd (one column shard of the whole rows:
- *                  row_offset 0, n_rows_total = n_rows).
+ *  row_offset, n_rows_total, traj_counts, traj_sums, partials, stats: as
+ *                  in rl_loss_shard_fwd_bwd (one column shard of the whole
+ *                  rows: row_offset 0, n_rows_total = n_rows).
  *  row_partials    [n_rows][4] floats (device, 16-byte aligned), written by
  *                  PARTIAL: per row, m, s, u and zy, with m a reference in
  *                  log2 units (a multiple of log2(e)/T of a logit),
@@ -398,17 +411,24 @@ enum {
  *      write the same partials: the caller combines them over the ROW
  *      shards only, as rl_loss_partials says.
  *   4. FINISH writes `stats` from the combined partials.
+ * GSPO: SWEEP stops after the merge with the shard's per-trajectory sums in
+ * traj_sums (as in rl_loss_shard_fwd_bwd); the caller adds them over the ROW
+ * shards (column shards of the same rows hold the same sums), then SEQ
+ * writes dLogits over the shard's columns and `partials`, and FINISH
+ * follows.
  * A shard's log-probs, entropies and dLogits equal the unsharded call's up
  * to the order of the row's floating-point sums (within the library's
  * tolerances, not bit for bit). The logits are read twice (PARTIAL and the
- * gradient in SWEEP), as for the split rl_loss_fwd / rl_loss_bwd pair.
- * GSPO and top-K OPD return RL_ERR_UNSUPPORTED. A target outside the
+ * gradient in SWEEP or SEQ), as for the split rl_loss_fwd / rl_loss_bwd
+ * pair. Top-K OPD returns RL_ERR_UNSUPPORTED. A target outside the
  * vocabulary is reported by SWEEP (RL_ERR_TARGET_OUT_OF_RANGE; the row gets
  * zeros). Arguments a phase does not read may be NULL (COUNT: logits,
- * outputs, dlogits, row_partials*, partials, stats; PARTIAL: outputs
- * other than advantages and group_sizes, row_partials_all, dlogits,
- * partials, stats; SWEEP: row_partials, stats; FINISH: everything but
- * partials, stats and the stream). */
+ * outputs, dlogits, traj_sums, row_partials*, partials, stats; PARTIAL:
+ * outputs other than advantages and group_sizes, traj_sums,
+ * row_partials_all, dlogits, partials, stats; SWEEP: row_partials, stats,
+ * traj_sums without GSPO, and dlogits and partials with it; SEQ:
+ * row_partials*, stats; FINISH: everything but partials, stats and the
+ * stream). */
 rl_status rl_loss_vocab_shard_fwd_bwd(
     int32_t phase, int32_t col_shard, int32_t n_col_shards, const int64_t* col_starts,
     int64_t row_offset, int64_t n_rows_total, const void* logits, rl_dtype logits_dtype,
@@ -417,7 +437,7 @@ rl_status rl_loss_vocab_shard_fwd_bwd(
     const float* rewards, const int32_t* group_id, const int32_t* cu_seqlens, int32_t n_traj,
     int32_t n_groups, const uint8_t* loss_mask, const rl_loss_params* params,
     float* token_logprobs, float* entropy, float* advantages, int32_t* group_sizes,
-    int32_t* traj_counts, float* row_partials, const float* row_partials_all,
+    int32_t* traj_counts, double* traj_sums, float* row_partials, const float* row_partials_all,
     rl_loss_partials* partials, rl_loss_stats* stats, float grad_loss,
     const float* grad_loss_device, void* dlogits, rl_dtype dlogits_dtype, int64_t ld_out,
     void* workspace, size_t workspace_bytes, rl_stream stream);

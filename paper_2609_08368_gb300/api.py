@@ -240,8 +240,14 @@ class Shard:
         self.params = _params(w, params)
         self.grad_loss = grad_loss
         dev = w.targets.device
-        self.counts = torch.zeros(int(w.rewards.shape[0]), dtype=torch.int32, device=dev)
+        n_traj = int(w.rewards.shape[0])
+        self.counts = torch.zeros(n_traj, dtype=torch.int32, device=dev)
+        self.traj_sums = torch.zeros((n_traj, 2), dtype=torch.float64, device=dev)
         self.partials = torch.zeros(ml.PARTIALS_DOUBLES, dtype=torch.float64, device=dev)
+
+    @property
+    def gspo(self) -> bool:
+        return self.params.get("estimator", "grpo") == "gspo"
 
     def _call(self, phase, forward_only=False):
         w, b = self.w, self.buf
@@ -251,13 +257,18 @@ class Shard:
                                  w.n_groups, w.loss_mask, self.params, b.token_logprobs,
                                  b.entropy, b.advantages, b.group_sizes, self.counts,
                                  self.partials, b.stats, None if forward_only else b.dlogits,
-                                 b.workspace, w.vocab, grad_loss=self.grad_loss)
+                                 b.workspace, w.vocab, grad_loss=self.grad_loss,
+                                 traj_sums=self.traj_sums)
 
     def count(self):
         self._call(ml.RL_SHARD_COUNT)
 
     def sweep(self, forward_only=False):
         self._call(ml.RL_SHARD_SWEEP, forward_only)
+
+    def seq(self, forward_only=False):
+        """GSPO only: after the shards' traj_sums have been added."""
+        self._call(ml.RL_SHARD_SEQ, forward_only)
 
     def finish(self):
         self._call(ml.RL_SHARD_FINISH)
@@ -268,6 +279,13 @@ def exchange_counts(counts: torch.Tensor, group=None):
     ``group`` (in place)."""
     import torch.distributed as dist
     dist.all_reduce(counts, op=dist.ReduceOp.SUM, group=group)
+
+
+def exchange_traj_sums(traj_sums: torch.Tensor, group=None):
+    """GSPO: add the shards' per-trajectory sums over the ranks of ``group``
+    (in place)."""
+    import torch.distributed as dist
+    dist.all_reduce(traj_sums, op=dist.ReduceOp.SUM, group=group)
 
 
 def exchange_partials(partials: torch.Tensor, group=None):
@@ -284,6 +302,9 @@ def sharded_fwd_bwd(shard: Shard, group=None):
     shard.count()
     exchange_counts(shard.counts, group)
     shard.sweep()
+    if shard.gspo:
+        exchange_traj_sums(shard.traj_sums, group)
+        shard.seq()
     exchange_partials(shard.partials, group)
     shard.finish()
 
@@ -297,6 +318,11 @@ def sharded_fwd_bwd_local(shards):
     for s in shards:
         s.counts.copy_(total)
         s.sweep()
+    if shards and shards[0].gspo:
+        sums = torch.stack([s.traj_sums for s in shards]).sum(0)
+        for s in shards:
+            s.traj_sums.copy_(sums)
+            s.seq()
     p = torch.stack([s.partials for s in shards])
     comb = torch.cat([p[:, :ml.PARTIALS_SUMS].sum(0), p[:, ml.PARTIALS_SUMS:].max(0).values])
     for s in shards:
@@ -329,6 +355,8 @@ class VocabShard:
         dev = w.targets.device
         R, n_shards = w.n_rows, len(self.col_starts) - 1
         self.counts = torch.zeros(int(w.rewards.shape[0]), dtype=torch.int32, device=dev)
+        self.traj_sums = torch.zeros((int(w.rewards.shape[0]), 2), dtype=torch.float64,
+                                     device=dev)
         self.row_partials = torch.zeros((R, 4), dtype=torch.float32, device=dev)
         self.row_partials_all = torch.zeros((n_shards, R, 4), dtype=torch.float32, device=dev)
         self.partials = torch.zeros(ml.PARTIALS_DOUBLES, dtype=torch.float64, device=dev)
@@ -341,7 +369,12 @@ class VocabShard:
             w.rewards, w.group_id, w.cu_seqlens, w.n_groups, w.loss_mask, self.params,
             b.token_logprobs, b.entropy, b.advantages, b.group_sizes, self.counts,
             self.row_partials, self.row_partials_all, self.partials, b.stats,
-            None if forward_only else b.dlogits, b.workspace, grad_loss=self.grad_loss)
+            None if forward_only else b.dlogits, b.workspace, grad_loss=self.grad_loss,
+            traj_sums=self.traj_sums)
+
+    @property
+    def gspo(self) -> bool:
+        return self.params.get("estimator", "grpo") == "gspo"
 
     def count(self):
         self._call(ml.RL_VSHARD_COUNT)
@@ -351,6 +384,10 @@ class VocabShard:
 
     def sweep(self, forward_only=False):
         self._call(ml.RL_VSHARD_SWEEP, forward_only)
+
+    def seq(self, forward_only=False):
+        """GSPO only: after the row shards' traj_sums have been added."""
+        self._call(ml.RL_VSHARD_SEQ, forward_only)
 
     def finish(self):
         self._call(ml.RL_VSHARD_FINISH)
@@ -378,6 +415,10 @@ def vocab_sharded_fwd_bwd(shard: VocabShard, col_group=None, row_group=None):
     shard.partial()
     exchange_row_partials(shard.row_partials, shard.row_partials_all, col_group)
     shard.sweep()
+    if shard.gspo:
+        if row_group is not None:
+            exchange_traj_sums(shard.traj_sums, row_group)
+        shard.seq()
     if row_group is not None:
         exchange_partials(shard.partials, row_group)
     shard.finish()
@@ -399,6 +440,11 @@ def vocab_sharded_fwd_bwd_local(shards):
         for s in row:
             s.row_partials_all.copy_(gathered)
             s.sweep()
+    if flat and flat[0].gspo:
+        sums = torch.stack([row[0].traj_sums for row in shards]).sum(0)
+        for s in flat:
+            s.traj_sums.copy_(sums)
+            s.seq()
     p = torch.stack([row[0].partials for row in shards])
     comb = torch.cat([p[:, :ml.PARTIALS_SUMS].sum(0), p[:, ml.PARTIALS_SUMS:].max(0).values])
     for s in flat:

@@ -330,6 +330,9 @@ struct FwdIn {
   // partial sums in place of the sweep's epilogue
   long long col0 = 0;
   float4* part_rows = nullptr;
+  // a shard of a sharded GSPO call: the per-trajectory sums over its rows go
+  // here (k_seq's first half) and the call stops before the statistics
+  double* seq_sums_out = nullptr;
 };
 
 rl_status check_fwd(const FwdIn& f, bool need_logits = true) {
@@ -432,6 +435,41 @@ rl_status launch_bwd(const Common& c, const GradOut& go, const WsPtrs& ws, cudaS
   const long long grid =
       std::min<long long>(b.n_tiles, static_cast<long long>(sms) * std::max(per_sm, 1));
   return launch(fn, dim3(static_cast<unsigned>(grid)), dim3(kBwdThreads), 0, 1, s, &b);
+}
+
+// GSPO's per-trajectory pass over a call's rows (k_seq), whole or one half
+// of a sharded call's (sums_out: the shard's sums only; sums_in: apply the
+// sums added over the shards).
+rl_status launch_seq(const FwdIn& f, double* sums_out, const double* sums_in, cudaStream_t s) {
+  SeqArgs qa;
+  qa.cu = f.cu;
+  qa.rho = f.rho;
+  qa.old = f.old;
+  qa.q = f.q;
+  qa.mask = f.c.mask;
+  qa.row0 = f.row0;
+  qa.R = f.c.R;
+  qa.sums_out = sums_out;
+  qa.sums_in = sums_in;
+  qa.s = scalars(f.c.p);
+  qa.ws = WsPtrs::at(f.ws, WsLayout::make(f.c.R, f.n_traj, f.n_groups));
+  return launch(seq_kernel(), dim3(static_cast<unsigned>(f.n_traj)), dim3(kSeqThreads), 0, 1, s,
+                &qa);
+}
+
+// A shard's partial statistics over its rows (k_stats into `partials`).
+rl_status launch_shard_stats(const FwdIn& f, rl_loss_partials* partials, cudaStream_t s) {
+  StatArgs ta;
+  ta.R = f.c.R;
+  ta.mask = f.c.mask;
+  ta.rho = f.rho;
+  ta.out = nullptr;
+  ta.part_out = partials;
+  ta.ws = WsPtrs::at(f.ws, WsLayout::make(f.c.R, f.n_traj, f.n_groups));
+  long long blocks = (f.c.R + kStatThreads - 1) / kStatThreads;
+  blocks = std::max<long long>(1, std::min<long long>(blocks, kMaxStatBlocks));
+  return launch(stats_kernel(), dim3(static_cast<unsigned>(blocks)), dim3(kStatThreads), 0, 1, s,
+                &ta);
 }
 
 // phase: RL_PHASE_BEGIN (advantages, N), RL_PHASE_ROWS (the sweep over rows
@@ -608,17 +646,8 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     if (st != RL_OK) return st;
   }
 
-  if (gspo && (phase & RL_PHASE_ROWS) && call.R > 0 && f.n_traj > 0) {
-    SeqArgs qa;
-    qa.cu = f.cu;
-    qa.rho = f.rho;
-    qa.old = f.old;
-    qa.q = f.q;
-    qa.mask = call.mask;
-    qa.s = scalars(call.p);
-    qa.ws = ws_all;
-    st = launch(seq_kernel(), dim3(static_cast<unsigned>(f.n_traj)), dim3(kSeqThreads), 0, 1, s,
-                &qa);
+  if (gspo && (phase & RL_PHASE_ROWS) && (call.R > 0 || f.seq_sums_out) && f.n_traj > 0) {
+    st = launch_seq(f, f.seq_sums_out, nullptr, s);
     if (st != RL_OK) return st;
   }
 
@@ -737,7 +766,7 @@ rl_status rl_loss_shard_fwd_bwd(int32_t phase, int64_t row_offset, int64_t n_row
                                 const int32_t* cu_seqlens, int32_t n_traj, int32_t n_groups,
                                 const uint8_t* loss_mask, const rl_loss_params* params,
                                 float* token_logprobs, float* entropy, float* advantages,
-                                int32_t* group_sizes, int32_t* traj_counts,
+                                int32_t* group_sizes, int32_t* traj_counts, double* traj_sums,
                                 rl_loss_partials* partials, rl_loss_stats* stats,
                                 float grad_loss, const float* grad_loss_device, void* dlogits,
                                 rl_dtype dlogits_dtype, int64_t ld_out, void* workspace,
@@ -748,11 +777,18 @@ rl_status rl_loss_shard_fwd_bwd(int32_t phase, int64_t row_offset, int64_t n_row
     FinishArgs fa{partials, stats};
     return launch(finish_kernel(), dim3(1), dim3(32), 0, 1, s, &fa);
   }
-  if (phase != RL_SHARD_COUNT && phase != RL_SHARD_SWEEP) return RL_ERR_INVALID_ARG;
+  if (phase != RL_SHARD_COUNT && phase != RL_SHARD_SWEEP && phase != RL_SHARD_SEQ)
+    return RL_ERR_INVALID_ARG;
   if (row_offset < 0 || n_rows < 0 || n_rows_total < 0 || row_offset > n_rows_total - n_rows)
     return RL_ERR_INVALID_ARG;
   if (n_traj > 0 && !traj_counts) return RL_ERR_INVALID_ARG;
-  if (params && params->estimator == RL_EST_GSPO) return RL_ERR_UNSUPPORTED;
+  if (!params) return RL_ERR_INVALID_ARG;
+  // GSPO: a trajectory's sequence ratio needs its rows on every shard, so
+  // its sweep stops at the per-trajectory sums, which the caller adds over
+  // the shards before SEQ
+  const bool gspo = params->estimator == RL_EST_GSPO;
+  if (phase == RL_SHARD_SEQ && !gspo) return RL_ERR_INVALID_ARG;
+  if (gspo && phase != RL_SHARD_COUNT && n_traj > 0 && !traj_sums) return RL_ERR_INVALID_ARG;
   const bool count = phase == RL_SHARD_COUNT;
   FwdIn f{{logits, logits_dtype, n_rows, vocab, ld, targets, loss_mask, params},
           rollout_logprobs, ref_logprobs, old_logprobs, teacher_logprobs, rewards,
@@ -767,18 +803,44 @@ rl_status rl_loss_shard_fwd_bwd(int32_t phase, int64_t row_offset, int64_t n_row
     if (st != RL_OK) return st;
     return run_fwd(f, nullptr, s, RL_PHASE_BEGIN);
   }
-  if (!partials) return RL_ERR_INVALID_ARG;
   f.counts_in = traj_counts;
-  f.part_out = partials;
-  rl_status st = check_fwd(f, n_rows > 0);
-  if (st != RL_OK) return st;
+  if (phase == RL_SHARD_SWEEP && gspo) {
+    // advantages, the forward sweep and the shard's per-trajectory sums
+    f.seq_sums_out = traj_sums;
+    rl_status st = check_fwd(f, n_rows > 0);
+    if (st != RL_OK) return st;
+    return run_fwd(f, nullptr, s, RL_PHASE_BEGIN | RL_PHASE_ROWS);
+  }
+  if (!partials) return RL_ERR_INVALID_ARG;
   GradOut go{grad_loss, grad_loss_device, dlogits, dlogits_dtype, ld_out};
   const bool grad = dlogits != nullptr;
+  if (phase == RL_SHARD_SWEEP) {
+    f.part_out = partials;
+    rl_status st = check_fwd(f, n_rows > 0);
+    if (st != RL_OK) return st;
+    if (grad) {
+      st = check_grad(f.c, go);
+      if (st != RL_OK) return st;
+    }
+    return run_fwd(f, grad ? &go : nullptr, s, RL_PHASE_ALL);
+  }
+  // SEQ (GSPO): the trajectories' terms from the added sums, the shard's
+  // partial statistics, dLogits over its rows
+  rl_status st = check_fwd(f, n_rows > 0 && grad);
+  if (st != RL_OK) return st;
   if (grad) {
     st = check_grad(f.c, go);
     if (st != RL_OK) return st;
   }
-  return run_fwd(f, grad ? &go : nullptr, s, RL_PHASE_ALL);
+  if (n_traj > 0) {
+    st = launch_seq(f, nullptr, traj_sums, s);
+    if (st != RL_OK) return st;
+  }
+  st = launch_shard_stats(f, partials, s);
+  if (st != RL_OK) return st;
+  if (grad && n_rows > 0)
+    return launch_bwd(f.c, go, WsPtrs::at(workspace, WsLayout::make(n_rows, n_traj, n_groups)), s);
+  return RL_OK;
 }
 
 rl_status rl_loss_vocab_shard_fwd_bwd(
@@ -789,7 +851,7 @@ rl_status rl_loss_vocab_shard_fwd_bwd(
     const float* rewards, const int32_t* group_id, const int32_t* cu_seqlens, int32_t n_traj,
     int32_t n_groups, const uint8_t* loss_mask, const rl_loss_params* params,
     float* token_logprobs, float* entropy, float* advantages, int32_t* group_sizes,
-    int32_t* traj_counts, float* row_partials, const float* row_partials_all,
+    int32_t* traj_counts, double* traj_sums, float* row_partials, const float* row_partials_all,
     rl_loss_partials* partials, rl_loss_stats* stats, float grad_loss,
     const float* grad_loss_device, void* dlogits, rl_dtype dlogits_dtype, int64_t ld_out,
     void* workspace, size_t workspace_bytes, rl_stream stream) {
@@ -799,7 +861,8 @@ rl_status rl_loss_vocab_shard_fwd_bwd(
     FinishArgs fa{partials, stats};
     return launch(finish_kernel(), dim3(1), dim3(32), 0, 1, s, &fa);
   }
-  if (phase != RL_VSHARD_COUNT && phase != RL_VSHARD_PARTIAL && phase != RL_VSHARD_SWEEP)
+  if (phase != RL_VSHARD_COUNT && phase != RL_VSHARD_PARTIAL && phase != RL_VSHARD_SWEEP &&
+      phase != RL_VSHARD_SEQ)
     return RL_ERR_INVALID_ARG;
   // the column partition: col_starts[0] = 0 < col_starts[1] < ... (every
   // shard has a column), vocabulary ids fit the int32 targets
@@ -814,12 +877,16 @@ rl_status rl_loss_vocab_shard_fwd_bwd(
     return RL_ERR_INVALID_ARG;
   if (n_traj > 0 && !traj_counts) return RL_ERR_INVALID_ARG;
   if (!params) return RL_ERR_INVALID_ARG;
-  // GSPO needs whole trajectories before any gradient; top-K OPD candidates
-  // would be spread over the shards
-  if (params->estimator == RL_EST_GSPO || (params->opd_topk > 0 && params->opd_coef != 0.0f))
-    return RL_ERR_UNSUPPORTED;
+  // top-K OPD candidates would be spread over the column shards
+  if (params->opd_topk > 0 && params->opd_coef != 0.0f) return RL_ERR_UNSUPPORTED;
+  // GSPO: SWEEP stops at the per-trajectory sums over the shard's rows, which
+  // the caller adds over the row shards before SEQ
+  const bool gspo = params->estimator == RL_EST_GSPO;
+  if (phase == RL_VSHARD_SEQ && !gspo) return RL_ERR_INVALID_ARG;
+  if (gspo && (phase == RL_VSHARD_SWEEP || phase == RL_VSHARD_SEQ) && n_traj > 0 && !traj_sums)
+    return RL_ERR_INVALID_ARG;
   const bool count = phase == RL_VSHARD_COUNT;
-  const bool sweep = phase == RL_VSHARD_SWEEP;
+  const bool sweep = phase == RL_VSHARD_SWEEP || phase == RL_VSHARD_SEQ;
   FwdIn f{{logits, logits_dtype, n_rows, vocab, ld, targets, loss_mask, params},
           rollout_logprobs, ref_logprobs, old_logprobs, teacher_logprobs, rewards,
           group_id, cu_seqlens, n_traj, n_groups, sweep ? token_logprobs : nullptr,
@@ -845,18 +912,31 @@ rl_status rl_loss_vocab_shard_fwd_bwd(
     return run_fwd(f, nullptr, s, RL_PHASE_BEGIN | RL_PHASE_ROWS);
   }
   // SWEEP: merge the gathered records, dLogits over this shard's columns,
-  // this shard's partial statistics
-  if (!partials) return RL_ERR_INVALID_ARG;
-  if (n_rows > 0 && (!row_partials_all || !aligned16(row_partials_all))) return RL_ERR_INVALID_ARG;
-  rl_status st = check_fwd(f, n_rows > 0 && dlogits != nullptr);
-  if (st != RL_OK) return st;
+  // this shard's partial statistics (GSPO: the merge and the shard's
+  // per-trajectory sums; SEQ: the rest)
+  if (!partials && !(gspo && phase == RL_VSHARD_SWEEP)) return RL_ERR_INVALID_ARG;
+  if (phase == RL_VSHARD_SWEEP && n_rows > 0 &&
+      (!row_partials_all || !aligned16(row_partials_all)))
+    return RL_ERR_INVALID_ARG;
   GradOut go{grad_loss, grad_loss_device, dlogits, dlogits_dtype, ld_out};
-  const bool grad = dlogits != nullptr;
+  const bool grad = dlogits != nullptr && !(gspo && phase == RL_VSHARD_SWEEP);
+  rl_status st = check_fwd(f, n_rows > 0 && grad);
+  if (st != RL_OK) return st;
   if (grad) {
     st = check_grad(f.c, go);
     if (st != RL_OK) return st;
   }
   const WsPtrs ws = WsPtrs::at(workspace, WsLayout::make(n_rows, n_traj, n_groups));
+  if (phase == RL_VSHARD_SEQ) {
+    if (n_traj > 0) {
+      st = launch_seq(f, nullptr, traj_sums, s);
+      if (st != RL_OK) return st;
+    }
+    st = launch_shard_stats(f, partials, s);
+    if (st != RL_OK) return st;
+    if (grad && n_rows > 0) return launch_bwd(f.c, go, ws, s, col0);
+    return RL_OK;
+  }
   if (n_rows > 0) {
     int dev = 0, sms = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return RL_ERR_CUDA;
@@ -881,22 +961,13 @@ rl_status rl_loss_vocab_shard_fwd_bwd(
     st = launch(merge_kernel(), dim3(static_cast<unsigned>(blocks)), dim3(kMergeThreads), 0, 1,
                 s, &ma);
     if (st != RL_OK) return st;
-    if (grad) {
-      st = launch_bwd(f.c, go, ws, s, col0);
-      if (st != RL_OK) return st;
-    }
   }
-  StatArgs ta;
-  ta.R = n_rows;
-  ta.mask = loss_mask;
-  ta.rho = rollout_logprobs;
-  ta.out = nullptr;
-  ta.part_out = partials;
-  ta.ws = ws;
-  long long blocks = (n_rows + kStatThreads - 1) / kStatThreads;
-  blocks = std::max<long long>(1, std::min<long long>(blocks, kMaxStatBlocks));
-  return launch(stats_kernel(), dim3(static_cast<unsigned>(blocks)), dim3(kStatThreads), 0, 1, s,
-                &ta);
+  if (gspo) return n_traj > 0 ? launch_seq(f, traj_sums, nullptr, s) : RL_OK;
+  if (grad && n_rows > 0) {
+    st = launch_bwd(f.c, go, ws, s, col0);
+    if (st != RL_OK) return st;
+  }
+  return launch_shard_stats(f, partials, s);
 }
 
 rl_status rl_loss_bwd(const void* logits, rl_dtype logits_dtype, int64_t n_rows, int64_t vocab,
@@ -982,6 +1053,6 @@ rl_status rl_set_launch_overrides(const rl_launch_overrides* o) {
   return RL_OK;
 }
 
-int32_t rl_loss_abi_version(void) { return 120; }
+int32_t rl_loss_abi_version(void) { return 130; }
 
 }  // extern "C"

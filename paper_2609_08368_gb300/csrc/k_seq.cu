@@ -13,7 +13,11 @@
 //
 // Runs after the forward sweep (which left logp, H, k3 and the correction
 // ratio of every row in the workspace) and before the gradient sweep: one
-// block per trajectory, sums in a fixed order in double precision.
+// block per trajectory, sums in a fixed order in double precision. In a
+// row-sharded call a trajectory's rows may lie on several shards: each shard
+// first writes its part of the two sums (sums_out), the caller adds them
+// over the shards, and each shard then applies the trajectory's terms to its
+// own rows from the added sums (sums_in).
 #include "common.cuh"
 #include "kernels.h"
 
@@ -28,19 +32,26 @@ __global__ void __launch_bounds__(kThreads) k_seq(const SeqArgs a) {
   __shared__ double s_a[kWarps], s_b[kWarps];
   __shared__ float s_out[4];  // s_i, scale * pg_i, scale * mean_w * (-A s_i) or 0, flags
   WsPtrs ws = a.ws;
-  if (ws.hdr->err_bits & kErrSeqlens) return;  // rows cannot be attributed to trajectories
   const int i = blockIdx.x;
-  const int lo = a.cu[i], hi = a.cu[i + 1];
+  if (ws.hdr->err_bits & kErrSeqlens) {  // rows cannot be attributed to trajectories
+    if (a.sums_out && threadIdx.x == 0) a.sums_out[2 * i] = a.sums_out[2 * i + 1] = 0.0;
+    return;
+  }
+  // the trajectory's rows in this call, as local indices [lo, hi)
+  const long long lo = max(static_cast<long long>(a.cu[i]), a.row0) - a.row0;
+  const long long hi = max(min(static_cast<long long>(a.cu[i + 1]), a.row0 + a.R) - a.row0, lo);
   const int n_i = ws.traj_n[i];
   const LossScalars& s = a.s;
 
   // sums over the trajectory's training tokens: log-ratio and correction weight
   double sl = 0.0, sw = 0.0;
-  for (int t = lo + threadIdx.x; t < hi; t += kThreads) {
-    if (!a.mask[t]) continue;
-    const float base = a.old ? a.old[t] : a.rho[t];
-    sl += static_cast<double>(ws.logp[t]) - static_cast<double>(base);
-    sw += correction_weight(ws.rc[t], s);
+  if (!a.sums_in) {
+    for (long long t = lo + threadIdx.x; t < hi; t += kThreads) {
+      if (!a.mask[t]) continue;
+      const float base = a.old ? a.old[t] : a.rho[t];
+      sl += static_cast<double>(ws.logp[t]) - static_cast<double>(base);
+      sw += correction_weight(ws.rc[t], s);
+    }
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -53,6 +64,14 @@ __global__ void __launch_bounds__(kThreads) k_seq(const SeqArgs a) {
   if (threadIdx.x == 0) {
     double tl = 0.0, tw = 0.0;
     for (int w = 0; w < kWarps; ++w) { tl += s_a[w]; tw += s_b[w]; }
+    if (a.sums_in) {
+      tl = a.sums_in[2 * i];
+      tw = a.sums_in[2 * i + 1];
+    }
+    if (a.sums_out) {
+      a.sums_out[2 * i] = tl;
+      a.sums_out[2 * i + 1] = tw;
+    }
     float si = 1.0f, pg = 0.0f, gp = 0.0f;
     uint8_t fl = 0;
     if (n_i > 0) {
@@ -81,9 +100,10 @@ __global__ void __launch_bounds__(kThreads) k_seq(const SeqArgs a) {
     s_out[3] = static_cast<float>(fl);
   }
   __syncthreads();
+  if (a.sums_out) return;  // the shard's part of the sums only
   const float si = s_out[0], pg_i = s_out[1], gp = s_out[2];
   const uint8_t seq_flags = static_cast<uint8_t>(s_out[3]);
-  for (int t = lo + threadIdx.x; t < hi; t += kThreads) {
+  for (long long t = lo + threadIdx.x; t < hi; t += kThreads) {
     const uint8_t keep = ws.flags[t] & (kFlagCorrClip | kFlagBad);
     if (keep & kFlagBad) continue;  // a row with a bad target keeps its zeros
     const float wt = correction_weight(ws.rc[t], s);

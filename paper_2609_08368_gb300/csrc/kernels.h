@@ -110,11 +110,18 @@ struct AdvArgs {
 };
 
 struct SeqArgs {
-  const int* cu;
-  const float* rho;
+  const int* cu;        // row offsets of the whole call
+  const float* rho;     // per-row arrays: this call's rows (local indices)
   const float* old;
   const float* q;
   const uint8_t* mask;
+  long long row0, R;    // the call's rows are [row0, row0 + R) of the whole call
+  // Sharded calls: sums_out receives, per trajectory, the sums over this
+  // call's rows (sum of logp - base, sum of correction weights; [n_traj][2])
+  // and nothing else is written; sums_in gives those sums added over every
+  // shard, in place of the kernel's own.
+  double* sums_out;
+  const double* sums_in;
   LossScalars s;
   WsPtrs ws;
 };

@@ -17,8 +17,8 @@ from . import build as _build
 RL_OK = 0
 RL_BF16, RL_F32 = 0, 1
 RL_PHASE_BEGIN, RL_PHASE_ROWS, RL_PHASE_END, RL_PHASE_ALL = 1, 2, 4, 7
-RL_SHARD_COUNT, RL_SHARD_SWEEP, RL_SHARD_FINISH = 1, 2, 4
-RL_VSHARD_COUNT, RL_VSHARD_PARTIAL, RL_VSHARD_SWEEP, RL_VSHARD_FINISH = 1, 2, 3, 4
+RL_SHARD_COUNT, RL_SHARD_SWEEP, RL_SHARD_FINISH, RL_SHARD_SEQ = 1, 2, 4, 8
+RL_VSHARD_COUNT, RL_VSHARD_PARTIAL, RL_VSHARD_SWEEP, RL_VSHARD_FINISH, RL_VSHARD_SEQ = 1, 2, 3, 4, 5
 PARTIALS_SUMS = 14   # rl_loss_partials: sum[9] and count[5], combined by addition
 PARTIALS_DOUBLES = 16  # ... then max[2], combined by maximum
 CORRECTIONS = {"none": 0, "tis": 1, "clip_or_pop": 2}
@@ -124,10 +124,10 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
     lib.rl_launch_overrides_init.argtypes = [ctypes.POINTER(RlLaunchOverrides)]
     lib.rl_set_launch_overrides.argtypes = [ctypes.POINTER(RlLaunchOverrides)]
     lib.rl_loss_fwd_bwd_noalloc.argtypes = fwd_common + [F32, P, P, I32, I64, P]
-    lib.rl_loss_shard_fwd_bwd.argtypes = ([I32, I64, I64] + fwd_common[:-1] + [P, P, P] +
+    lib.rl_loss_shard_fwd_bwd.argtypes = ([I32, I64, I64] + fwd_common[:-1] + [P, P, P, P] +
                                           [F32, P, P, I32, I64, P, SZ, P])
     lib.rl_loss_vocab_shard_fwd_bwd.argtypes = (
-        [I32, I32, I32, P, I64, I64, P, I32, I64, I64] + fwd_common[5:-1] + [P, P, P, P, P] +
+        [I32, I32, I32, P, I64, I64, P, I32, I64, I64] + fwd_common[5:-1] + [P, P, P, P, P, P] +
         [F32, P, P, I32, I64, P, SZ, P])
     lib.rl_loss_noalloc_check_device_error.argtypes = []
     for name in ("rl_loss_workspace_size", "rl_loss_fwd", "rl_loss_fwd_bwd", "rl_loss_fwd_bwd_rows",
@@ -317,10 +317,11 @@ def rl_loss_shard_fwd_bwd(phase, row_offset, n_rows_total, logits, targets, roll
                           cu_seqlens, n_groups, loss_mask, params, token_logprobs, entropy,
                           advantages, group_sizes, traj_counts, partials, stats, dlogits,
                           workspace, vocab, n_rows=None, logits_dtype=None, grad_loss=1.0,
-                          grad_loss_device=None, stream=None):
+                          grad_loss_device=None, stream=None, traj_sums=None):
     """One phase of a shard's part of a row-sharded call. Per-row tensors
-    hold the shard's rows; ``traj_counts`` is int32 [n_traj] and
-    ``partials`` float64 [16] (one rl_loss_partials), both on the device."""
+    hold the shard's rows; ``traj_counts`` is int32 [n_traj], ``partials``
+    float64 [16] (one rl_loss_partials) and ``traj_sums`` (GSPO) float64
+    [n_traj, 2], all on the device."""
     import torch
     n_traj = int(rewards.shape[0]) if rewards is not None else 0
     if logits is not None:
@@ -338,9 +339,9 @@ def rl_loss_shard_fwd_bwd(phase, row_offset, n_rows_total, logits, targets, roll
         _ptr(targets), _ptr(rollout_logprobs), _ptr(ref_logprobs), _ptr(old_logprobs),
         _ptr(teacher_logprobs), _ptr(rewards), _ptr(group_id), _ptr(cu_seqlens), n_traj,
         int(n_groups), _ptr(loss_mask), ctypes.byref(_params(params)), _ptr(token_logprobs),
-        _ptr(entropy), _ptr(advantages), _ptr(group_sizes), _ptr(traj_counts), _ptr(partials),
-        _ptr(stats), float(grad_loss), _ptr(grad_loss_device), _ptr(dlogits), ddt, ld_out,
-        _ptr(workspace), ws_bytes, _stream(stream)), "rl_loss_shard_fwd_bwd")
+        _ptr(entropy), _ptr(advantages), _ptr(group_sizes), _ptr(traj_counts), _ptr(traj_sums),
+        _ptr(partials), _ptr(stats), float(grad_loss), _ptr(grad_loss_device), _ptr(dlogits), ddt,
+        ld_out, _ptr(workspace), ws_bytes, _stream(stream)), "rl_loss_shard_fwd_bwd")
 
 
 def rl_loss_vocab_shard_fwd_bwd(phase, col_shard, col_starts, row_offset, n_rows_total, logits,
@@ -350,7 +351,7 @@ def rl_loss_vocab_shard_fwd_bwd(phase, col_shard, col_starts, row_offset, n_rows
                                 group_sizes, traj_counts, row_partials, row_partials_all,
                                 partials, stats, dlogits, workspace, n_rows=None,
                                 logits_dtype=None, grad_loss=1.0, grad_loss_device=None,
-                                stream=None):
+                                stream=None, traj_sums=None):
     """One phase of a column shard's part of a vocabulary-sharded call.
     ``col_starts`` is a host sequence of n_col_shards + 1 vocabulary ids;
     ``logits`` / ``dlogits`` hold this shard's columns of its rows;
@@ -378,7 +379,8 @@ def rl_loss_vocab_shard_fwd_bwd(phase, col_shard, col_starts, row_offset, n_rows
         _ptr(rollout_logprobs), _ptr(ref_logprobs), _ptr(old_logprobs), _ptr(teacher_logprobs),
         _ptr(rewards), _ptr(group_id), _ptr(cu_seqlens), n_traj, int(n_groups), _ptr(loss_mask),
         ctypes.byref(_params(params)), _ptr(token_logprobs), _ptr(entropy), _ptr(advantages),
-        _ptr(group_sizes), _ptr(traj_counts), _ptr(row_partials), _ptr(row_partials_all),
+        _ptr(group_sizes), _ptr(traj_counts), _ptr(traj_sums), _ptr(row_partials),
+        _ptr(row_partials_all),
         _ptr(partials), _ptr(stats), float(grad_loss), _ptr(grad_loss_device), _ptr(dlogits), ddt,
         ld_out, _ptr(workspace), ws_bytes, _stream(stream)), "rl_loss_vocab_shard_fwd_bwd")
 

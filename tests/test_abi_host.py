@@ -42,7 +42,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert lib.rl_loss_abi_version() == 120
+    assert lib.rl_loss_abi_version() == 130
     seen = set()
     for code in range(0, 10):
         s = ml.status_string(code)
@@ -252,21 +252,25 @@ def test_sharded_entry_validates(lib):
     p = ml.make_params()
     gspo = ml.make_params(estimator="gspo")
 
-    def call(phase, r0=0, total=16, R=16, params=p, counts=FAKE, partials=FAKE, stats=FAKE):
+    def call(phase, r0=0, total=16, R=16, params=p, counts=FAKE, partials=FAKE, stats=FAKE,
+             sums=FAKE):
         return lib.rl_loss_shard_fwd_bwd(
             phase, r0, total, v(FAKE), 0, R, 64, 64, v(FAKE), v(FAKE), None, None, None,
             v(FAKE), v(FAKE), v(FAKE), 2, 1, v(FAKE), ctypes.byref(params), v(FAKE), v(FAKE),
-            v(FAKE), v(FAKE), v(counts), v(partials), v(stats), 1.0, None, v(FAKE), 0, 64,
-            v(FAKE * 2), 1 << 30, None)
+            v(FAKE), v(FAKE), v(counts), v(sums), v(partials), v(stats), 1.0, None, v(FAKE), 0,
+            64, v(FAKE * 2), 1 << 30, None)
     assert call(0) == RL_ERR_INVALID_ARG                      # no phase
     assert call(3) == RL_ERR_INVALID_ARG                      # one phase per call
+    assert call(ml.RL_SHARD_SEQ) == RL_ERR_INVALID_ARG        # SEQ is GSPO's only
+    assert call(ml.RL_SHARD_SWEEP, params=gspo, sums=None) == RL_ERR_INVALID_ARG
+    assert call(ml.RL_SHARD_SEQ, params=gspo, sums=None) == RL_ERR_INVALID_ARG
+    assert call(ml.RL_SHARD_SEQ, params=gspo, partials=None) == RL_ERR_INVALID_ARG
     assert call(ml.RL_SHARD_COUNT, r0=8, total=16, R=9) == RL_ERR_INVALID_ARG  # past the call
     assert call(ml.RL_SHARD_COUNT, r0=-1) == RL_ERR_INVALID_ARG
     assert call(ml.RL_SHARD_COUNT, counts=None) == RL_ERR_INVALID_ARG
     assert call(ml.RL_SHARD_SWEEP, partials=None) == RL_ERR_INVALID_ARG
     assert call(ml.RL_SHARD_FINISH, partials=None) == RL_ERR_INVALID_ARG
     assert call(ml.RL_SHARD_FINISH, stats=None) == RL_ERR_INVALID_ARG
-    assert call(ml.RL_SHARD_COUNT, params=gspo) == 2          # GSPO: whole calls only
 
 
 def test_vocab_sharded_entry_validates(lib):
@@ -276,18 +280,19 @@ def test_vocab_sharded_entry_validates(lib):
     p = ml.make_params()
 
     def call(phase, shard=0, starts=(0, 40, 64), r0=0, total=16, R=16, params=p, counts=FAKE,
-             rp=FAKE, rp_all=FAKE, partials=FAKE, stats=FAKE, ld=40, starts_ptr=True):
+             rp=FAKE, rp_all=FAKE, partials=FAKE, stats=FAKE, ld=40, starts_ptr=True, sums=FAKE):
         arr = (ctypes.c_int64 * len(starts))(*starts)
         return lib.rl_loss_vocab_shard_fwd_bwd(
             phase, shard, len(starts) - 1, ctypes.cast(arr, v) if starts_ptr else None, r0, total,
             v(FAKE), 0, R, ld, v(FAKE), v(FAKE), None, None, None, v(FAKE), v(FAKE), v(FAKE), 2, 1,
-            v(FAKE), ctypes.byref(params), v(FAKE), v(FAKE), v(FAKE), v(FAKE), v(counts), v(rp),
-            v(rp_all), v(partials), v(stats), 1.0, None, v(FAKE), 0, 64, v(FAKE * 2), 1 << 30,
-            None)
+            v(FAKE), ctypes.byref(params), v(FAKE), v(FAKE), v(FAKE), v(FAKE), v(counts), v(sums),
+            v(rp), v(rp_all), v(partials), v(stats), 1.0, None, v(FAKE), 0, 64, v(FAKE * 2),
+            1 << 30, None)
     C, PA, SW, FI = (ml.RL_VSHARD_COUNT, ml.RL_VSHARD_PARTIAL, ml.RL_VSHARD_SWEEP,
                      ml.RL_VSHARD_FINISH)
     assert call(0) == RL_ERR_INVALID_ARG                               # no phase
-    assert call(5) == RL_ERR_INVALID_ARG
+    assert call(6) == RL_ERR_INVALID_ARG
+    assert call(ml.RL_VSHARD_SEQ) == RL_ERR_INVALID_ARG                # SEQ is GSPO's only
     assert call(C, starts_ptr=False) == RL_ERR_INVALID_ARG             # no column partition
     assert call(C, starts=(1, 40, 64)) == RL_ERR_INVALID_ARG           # does not start at 0
     assert call(C, starts=(0, 40, 40)) == RL_ERR_INVALID_ARG           # an empty shard
@@ -306,7 +311,10 @@ def test_vocab_sharded_entry_validates(lib):
     assert call(SW, partials=None) == RL_ERR_INVALID_ARG
     assert call(FI, partials=None) == RL_ERR_INVALID_ARG
     assert call(FI, stats=None) == RL_ERR_INVALID_ARG
-    assert call(C, params=ml.make_params(estimator="gspo")) == 2       # RL_ERR_UNSUPPORTED
+    gspo = ml.make_params(estimator="gspo")
+    assert call(SW, params=gspo, sums=None) == RL_ERR_INVALID_ARG     # GSPO writes its sums
+    assert call(ml.RL_VSHARD_SEQ, params=gspo, sums=None) == RL_ERR_INVALID_ARG
+    assert call(ml.RL_VSHARD_SEQ, params=gspo, partials=None) == RL_ERR_INVALID_ARG
     tk = ml.make_params(opd_coef=0.5, opd_topk=4, opd_topk_ids=_Ptr(FAKE),
                         opd_topk_teacher=_Ptr(FAKE))
     assert call(PA, params=tk) == 2

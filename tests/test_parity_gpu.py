@@ -795,11 +795,41 @@ def test_row_sharded_call_equals_whole_call(ov, kind, params):
                 assert abs(st[k] - ref[k]) <= 1e-4 * max(abs(ref[k]), 1e-3), k
 
 
-def test_row_sharded_gspo_is_unsupported():
-    rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=1, group_size=2, traj_len=8, vocab=256)
+@pytest.mark.parametrize("kind", ["cluster", "stream"])
+@pytest.mark.parametrize("params", [dict(estimator="gspo"),
+                                    dict(estimator="gspo", correction="tis", corr_lo=0.0,
+                                         corr_hi=1.5, entropy_coef=0.01, kl_coef=0.05)],
+                         ids=["gspo", "gspo_tis_ent_kl"])
+def test_row_sharded_gspo_matches_the_oracle(ov, kind, params):
+    """GSPO over row shards (trajectories cut at the boundaries, an empty
+    shard): the forward sweep, the exchange of per-trajectory sums, then each
+    shard's sequence terms and dLogits. The assembled outputs match the
+    float64 oracle at the stated tolerances, and the shards' log-probs are
+    the whole call's bit for bit (the sequence sums only change the
+    gradient's scalars)."""
+    ov(sweep_kernel=kind)
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=2, group_size=4, traj_len=40, vocab=20480,
+                    rho_noise=0.3, ref_noise=0.2, mask="prefix_u0_half")
     w = wl.make(rec, DEV)
-    buf = api.alloc(w.n_rows, 2, 1, DEV, vocab=256, dlogits_dtype=torch.bfloat16)
-    sh = api.Shard(w, 0, w.n_rows, buf, params=dict(w.params, estimator="gspo"))
-    with pytest.raises(ml.MilesLossError) as e:
-        sh.count()
-    assert e.value.status == 2  # RL_ERR_UNSUPPORTED
+    p = dict(w.params, **params)
+    whole = P.run_gpu(w, params=p)
+    R, n_traj = w.n_rows, int(w.rewards.shape[0])
+    for cuts in ([0, 137, R], [0, 50, 50, 221, R]):
+        shards = []
+        for r0, r1 in zip(cuts[:-1], cuts[1:]):
+            buf = api.alloc(r1 - r0, n_traj, w.n_groups, DEV, vocab=w.vocab,
+                            dlogits_dtype=w.logits.dtype, fill_nan=True)
+            shards.append(api.Shard(_shard_of(w, r0, r1), r0, R, buf, params=p))
+        api.sharded_fwd_bwd_local(shards)
+        torch.cuda.synchronize()
+        dl = torch.cat([sh.buf.dlogits for sh in shards])
+        for sh in shards:
+            assert ml.rl_loss_check_device_error(sh.buf.workspace) == 0
+        g = dict(logp=np.concatenate([P.np_(sh.buf.token_logprobs) for sh in shards]),
+                 H=np.concatenate([P.np_(sh.buf.entropy) for sh in shards]),
+                 A=P.np_(shards[0].buf.advantages), group_sizes=P.np_(shards[0].buf.group_sizes),
+                 stats=shards[0].buf.read_stats())
+        np.testing.assert_array_equal(g["logp"], whole["logp"])
+        o = P.run_oracle(w, params=p)
+        P.compare_forward(w, g, o, params=p)
+        P.assert_dlogits_close(dl.float().cpu().numpy(), o["dlogits"])

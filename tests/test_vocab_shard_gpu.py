@@ -106,6 +106,7 @@ PARAMS = {
     "rpp_kl": dict(estimator="reinforcepp", kl_coef=0.05),
     "opd_ent_tis": dict(opd_coef=0.3, entropy_coef=0.01, temperature=0.7, correction="tis",
                         corr_lo=0.0, corr_hi=2.0),
+    "gspo_tis": dict(estimator="gspo", correction="tis", corr_lo=0.0, corr_hi=1.5),
 }
 
 
@@ -195,16 +196,15 @@ def test_vocab_sharded_bad_target_is_reported():
     P.assert_dlogits_close(g["dlogits_t"][good].float().cpu().numpy(), o["dlogits"][good])
 
 
-def test_vocab_sharded_gspo_and_topk_are_unsupported():
+def test_vocab_sharded_topk_is_unsupported():
     w = _workload()
-    for params in (dict(w.params, estimator="gspo"),
-                   dict(w.params, opd_coef=0.5, opd_topk=4,
-                        opd_topk_ids=torch.zeros((w.n_rows, 4), dtype=torch.int32, device=DEV),
-                        opd_topk_teacher=torch.zeros((w.n_rows, 4), device=DEV))):
-        s = run_sharded(w, [0, 10240, V], [0, w.n_rows], params, drive=False)[0][0]
-        with pytest.raises(ml.MilesLossError) as e:
-            s.count()
-        assert e.value.status == 2  # RL_ERR_UNSUPPORTED
+    params = dict(w.params, opd_coef=0.5, opd_topk=4,
+                  opd_topk_ids=torch.zeros((w.n_rows, 4), dtype=torch.int32, device=DEV),
+                  opd_topk_teacher=torch.zeros((w.n_rows, 4), device=DEV))
+    s = run_sharded(w, [0, 10240, V], [0, w.n_rows], params, drive=False)[0][0]
+    with pytest.raises(ml.MilesLossError) as e:
+        s.count()
+    assert e.value.status == 2  # RL_ERR_UNSUPPORTED
 
 
 @pytest.mark.slow
