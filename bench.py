@@ -528,6 +528,47 @@ def copy_floor_ms(call, stream, steps: int) -> float:
     return e0.elapsed_time(e1) / steps
 
 
+def vocab_tp2_timing(w, dev, dl_dtype, stream, reps: int = 10) -> dict:
+    """The call as two column shards of its vocabulary (tensor parallelism 2,
+    rl_loss_vocab_shard_fwd_bwd), both run one after the other on this GPU
+    with the record exchange done on the device: each of two GPUs would
+    spend about half of that (plus an all-gather of 16 B per row). Median of
+    ``reps`` whole calls after 3 warm-ups."""
+    from paper_2609_08368_gb300 import api, milesloss as ml, workloads as wl
+    R, V, n_traj = w.n_rows, w.vocab, int(w.rewards.shape[0])
+    half = (V // 2 + 7) // 8 * 8  # keeps the second shard's rows 16-byte aligned
+    cols = [0, half, V]
+    row = []
+    for k in range(2):
+        c0, c1 = cols[k], cols[k + 1]
+        wk = wl.Workload(w.recipe, w.logits[:, c0:c1], w.targets, w.rollout_logprobs,
+                         w.ref_logprobs, w.old_logprobs, w.teacher_logprobs, w.rewards,
+                         w.group_id, w.cu_seqlens, w.loss_mask, w.n_groups, dict(w.params))
+        b = api.alloc(R, n_traj, w.n_groups, dev, vocab=c1 - c0, dlogits_dtype=dl_dtype)
+        row.append(api.VocabShard(wk, k, cols, b))
+    shards = [row]
+    for _ in range(3):
+        api.vocab_sharded_fwd_bwd_local(shards)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(reps)]
+    for b_, e_ in evs:
+        b_.record(stream)
+        api.vocab_sharded_fwd_bwd_local(shards)
+        e_.record(stream)
+    torch.cuda.synchronize()
+    for s in row:
+        err = ml.rl_loss_check_device_error(s.buf.workspace)
+        if err:
+            raise RuntimeError(f"device error (vocabulary shards): {ml.status_string(err)}")
+    ms = statistics.median(b_.elapsed_time(e_) for b_, e_ in evs)
+    del shards, row
+    torch.cuda.empty_cache()
+    return {"vocab_tp2_ms_per_shard": ms / 2,
+            "vocab_tp2_how": "two column shards of the vocabulary, both on this GPU one after "
+                             "the other; per shard: partial sweep, merge, gradient sweep, "
+                             "statistics (the logits read twice, as in the split pair)"}
+
+
 def run_ours(args, rank, world, local):
     from paper_2609_08368_gb300 import api, milesloss as ml, workloads as wl
 
@@ -606,6 +647,8 @@ def run_ours(args, rank, world, local):
     err = ml.rl_loss_check_device_error(buf.workspace)
     if err:
         raise RuntimeError(f"device error: {ml.status_string(err)}")
+    if w.params.get("estimator", "grpo") != "gspo" and not args.opd_topk:
+        also.update(vocab_tp2_timing(w, dev, dl_dtype, stream))
     logit_bytes = R * V * w.logits.element_size()
     also["fwd_only_read_gbs"] = logit_bytes / (also["fwd_only_ms"] / 1e3) / 1e9
     also["split_fwd_bwd_tokens_per_s"] = R / (also["split_fwd_bwd_ms"] / 1e3)

@@ -424,7 +424,7 @@ rl_status launch_bwd(const Common& c, const GradOut& go, const WsPtrs& ws, cudaS
   b.invT = 1.0f / c.p->temperature;
   b.k = 1.4426950408889634f / c.p->temperature;
   b.gamma = c.p->entropy_coef;
-  b.col0 = col0;
+  b.col0 = static_cast<int>(col0);  // vocabulary ids fit int32
   b.ws = ws;
   // one wave of resident blocks (grid-stride over the tiles): a second,
   // partial wave would run with fewer loads in flight

@@ -77,9 +77,9 @@ __global__ void __launch_bounds__(kBwdThreads) k_bwd(const BwdArgs a) {
     const float ca = cc * (-G + a.gamma * (H - lse));
     const float cb = cc * a.gamma * a.invT;
     const float L2 = lse * 1.4426950408889634f;
-    // the target's column in this call's logits (-1: another shard's)
-    const long long yl = a.targets[row] - a.col0;
-    const int y = (yl >= 0 && yl < a.V) ? static_cast<int>(yl) : -1;
+    // the target's column in this call's logits (outside [0, V): another
+    // shard's, which no tile of this row holds)
+    const int y = a.targets[row] - a.col0;
     const bool has_y = y >= j0 && y < j1;
     // The sampled token's entry (only in the tile that holds it):
     // cc [G (1 - p_y) + gamma p_y (log p_y + H)] with 1 - p_y = -expm1(logp),

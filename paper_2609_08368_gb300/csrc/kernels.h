@@ -154,7 +154,7 @@ struct BwdArgs {
   float grad_loss;
   const float* grad_loss_dev;
   float invT, k, gamma;
-  long long col0;  // the logits are columns [col0, col0 + V) of the vocabulary
+  int col0;  // the logits are columns [col0, col0 + V) of the vocabulary
   WsPtrs ws;
 };
 
