@@ -208,11 +208,11 @@ def profiled_traffic(rows_now: int, workload: str, vocab: int):
 
 def sweep_kernel_name(vocab: int, elem_size: int, grad: bool = True) -> str:
     """The sweep kernel the library picks for these rows (16-byte aligned
-    rows of 192 KB and more in a fused call, of 160 KB and more in a
+    rows of 192 KB and more in a fused call, of 148 KB and more in a
     forward-only one, stream through one CTA each; shorter rows go to the
     cluster kernel)."""
     kind = "fused fwd+bwd" if grad else "forward-only"
-    if vocab * elem_size >= (192 if grad else 160) * 1024:
+    if vocab * elem_size >= (192 if grad else 148) * 1024:
         return f"k_stream ({kind} vocabulary sweep, one CTA per row)"
     return f"k_sweep ({kind} vocabulary sweep, clusters sharing a row)"
 

@@ -695,15 +695,18 @@ const void* fn(bool topk) {
 
 // Rows with 16-byte aligned starts go to the streaming kernel (one CTA per
 // row, second read served by L2 or shared memory) from 192 KB in a fused
-// call and from 160 KB in a forward-only one; shorter or unaligned rows to
+// call and from 148 KB in a forward-only one; shorter or unaligned rows to
 // the cluster kernel, which keeps them on chip. Measured on GB300 (bf16,
 // fractions of the copy peak): fused, rows of 200-310 KB streamed
 // 0.966-0.984 against 0.939-0.959 in clusters, rows of 128-160 KB in
 // clusters 0.94-0.96 against 0.88-0.91 streamed; forward only, rows of
-// 160-310 KB streamed 0.92-1.09 against 0.78-0.88, rows of 96-128 KB in
-// clusters 0.87-0.92 against 0.79. The sweep_kernel override forces either.
+// 148-310 KB streamed 0.92-1.09 against 0.78-0.88, rows of 96-144 KB in
+// clusters 0.87-0.94 against 0.79-0.92. The forward plan's clusters of two
+// stop fitting a third of the SM's shared memory past 148 KB rows, and
+// clusters of four ran 0.78-0.81 there. The sweep_kernel override forces
+// either.
 constexpr long long kStreamMinRowBytes = 192 * 1024;     // fused calls
-constexpr long long kStreamMinRowBytesFwd = 160 * 1024;  // forward-only calls
+constexpr long long kStreamMinRowBytesFwd = 148 * 1024;  // forward-only calls
 
 bool use_stream(long long row_bytes, bool in_bulk, bool grad, const rl_launch_overrides& ov) {
   if (ov.sweep_kernel == 0) return false;

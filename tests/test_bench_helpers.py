@@ -30,10 +30,10 @@ def test_sweep_kernel_name_follows_the_fused_threshold():
     assert bench.sweep_kernel_name(98303, 2).startswith("k_sweep")
     assert bench.sweep_kernel_name(32768, 4).startswith("k_sweep")
     assert bench.sweep_kernel_name(49152, 4).startswith("k_stream")
-    # forward-only calls stream from 160 KB
-    assert bench.sweep_kernel_name(81920, 2, grad=False).startswith("k_stream")
+    # forward-only calls stream from 148 KB
+    assert bench.sweep_kernel_name(75776, 2, grad=False).startswith("k_stream")
     assert bench.sweep_kernel_name(81920, 2).startswith("k_sweep")
-    assert bench.sweep_kernel_name(81919, 2, grad=False).startswith("k_sweep")
+    assert bench.sweep_kernel_name(75775, 2, grad=False).startswith("k_sweep")
 
 
 def test_profiled_traffic_only_for_its_workload_and_sources():
