@@ -49,6 +49,8 @@ def parse_args():
     ap.add_argument("--workload", default="glm")
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--e2e-chunk-rows", type=int, default=4096)
+    ap.add_argument("--e2e-depth", type=int, default=2,
+                    help="device chunk buffers of the pipelined host-buffer call")
     ap.add_argument("--cpu-sample-rows", type=int, default=0,
                     help="time the CPU oracle on this many random rows (0: on every row)")
     ap.add_argument("--no-e2e", action="store_true")
@@ -504,7 +506,7 @@ def copy_floor_ms(call, stream, steps: int) -> float:
         out_done = None
         for i, r0 in enumerate(range(0, R, call.chunk)):
             r1 = min(R, r0 + call.chunk)
-            b, n = i % 2, r1 - r0
+            b, n = i % len(call.lg), r1 - r0
             with torch.cuda.stream(call.s_in):
                 call.lg[b][:n].copy_(h.logits[r0:r1, :V], non_blocking=True)
                 in_done = torch.cuda.Event()
@@ -699,7 +701,8 @@ def run_ours(args, rank, world, local):
         host_w = _pinned_copy(w)
         del w, buf  # the pipelined call keeps its own two chunk buffers
         torch.cuda.empty_cache()
-        call = api.PipelinedHostCall(host_w, dev, chunk_rows=args.e2e_chunk_rows)
+        call = api.PipelinedHostCall(host_w, dev, chunk_rows=args.e2e_chunk_rows,
+                                     depth=args.e2e_depth)
         call()
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -716,7 +719,8 @@ def run_ours(args, rank, world, local):
         e2e = {"value": rows_all / (ms_e2e / 1e3), "unit": "tokens/s",
                "ms_per_step": ms_e2e, "steps": args.e2e_steps,
                "how": f"pinned host buffers, rl_loss_fwd_bwd_rows over chunks of "
-                      f"{args.e2e_chunk_rows} rows, copies overlapped with the sweep",
+                      f"{args.e2e_chunk_rows} rows through {args.e2e_depth} device chunk "
+                      f"buffers, copies overlapped with the sweep",
                "h2d_bytes_per_step": call.bytes_in(), "d2h_bytes_per_step": call.bytes_out(),
                "copy_floor_ms": floor_ms, "frac_of_copy_floor": floor_ms / ms_e2e,
                "copy_floor_how": "the same logits and dLogits bytes copied alone on this box, "

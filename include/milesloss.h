@@ -385,16 +385,21 @@ enum {
  *  row_offset, n_rows_total, traj_counts, traj_sums, partials, stats: as
  *                  in rl_loss_shard_fwd_bwd (one column shard of the whole
  *                  rows: row_offset 0, n_rows_total = n_rows).
- *  row_partials    [n_rows][4] floats (device, 16-byte aligned), written by
+ *  row_partials    [n_rows][8] floats (device, 16-byte aligned), written by
  *                  PARTIAL: per row, m, s, u and zy, with m a reference in
- *                  log2 units (a multiple of log2(e)/T of a logit),
- *                  s = sum_j 2^(z_j log2(e)/T - m) and
- *                  u = sum_j 2^(z_j log2(e)/T - m) (z_j log2(e)/T - m) over
- *                  the shard's columns j, zy the target's logit if the target
- *                  is one of them, else 0. m = NaN marks a row the shard gave
- *                  up on (RL_ERR_DEVICE_TIMEOUT in its workspace): every
- *                  shard then writes zeros for that row.
- *  row_partials_all [n_col_shards][n_rows][4] floats (device, 16-byte
+ *                  log2 units (a multiple of k = log2(e)/T of a logit),
+ *                  s = sum_j 2^(z_j k - m) and u = sum_j 2^(z_j k - m)
+ *                  (z_j k - m) over the shard's columns j, zy the target's
+ *                  logit if the target is one of them, else 0; then, with
+ *                  top-K OPD, the part of the row's candidates c in the
+ *                  shard's columns: mt = max z_c k, sw = sum_c 2^(z_c k - mt),
+ *                  acc = sum_c 2^(z_c k - mt) (z_c / T - teacher_c), and 1 if
+ *                  a candidate id lies outside the vocabulary (else 0);
+ *                  (-inf, 0, 0, 0) without candidates there or without
+ *                  top-K. m = NaN marks a row the shard gave up on
+ *                  (RL_ERR_DEVICE_TIMEOUT in its workspace): every shard
+ *                  then writes zeros for that row.
+ *  row_partials_all [n_col_shards][n_rows][8] floats (device, 16-byte
  *                  aligned), read by SWEEP: every column shard's row_partials
  *                  of the same rows, in shard order (an all-gather).
  *
@@ -420,9 +425,12 @@ enum {
  * to the order of the row's floating-point sums (within the library's
  * tolerances, not bit for bit). The logits are read twice (PARTIAL and the
  * gradient in SWEEP or SEQ), as for the split rl_loss_fwd / rl_loss_bwd
- * pair. Top-K OPD returns RL_ERR_UNSUPPORTED. A target outside the
- * vocabulary is reported by SWEEP (RL_ERR_TARGET_OUT_OF_RANGE; the row gets
- * zeros). Arguments a phase does not read may be NULL (COUNT: logits,
+ * pair. With top-K OPD the candidate ids and teacher log-probs
+ * (rl_loss_params.opd_topk_ids / opd_topk_teacher, [n_rows][K]) are the
+ * shard's rows' whole candidate lists, as vocabulary ids, on every column
+ * shard. A target outside the vocabulary is reported by SWEEP
+ * (RL_ERR_TARGET_OUT_OF_RANGE; the row gets zeros), a candidate id outside
+ * it likewise (RL_ERR_TOPK_ID_OUT_OF_RANGE). Arguments a phase does not read may be NULL (COUNT: logits,
  * outputs, dlogits, traj_sums, row_partials*, partials, stats; PARTIAL:
  * outputs other than advantages and group_sizes, traj_sums,
  * row_partials_all, dlogits, partials, stats; SWEEP: row_partials, stats,

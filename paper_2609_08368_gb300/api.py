@@ -132,19 +132,24 @@ def fwd_bwd_chunked(w, buf: Buffers, chunk_rows: int, params=None, grad_loss=1.0
 
 class PipelinedHostCall:
     """The fused call with logits and dLogits in pinned HOST memory, streamed
-    through two device chunk buffers: per chunk of rows, the host-to-device
-    copy (one stream), the vocabulary sweep (the caller's stream) and the
-    device-to-host copy of dLogits (a third stream) overlap with the other
-    chunks'. The small per-row inputs go to the device whole before the sweep
-    (BEGIN needs all of them)."""
+    through ``depth`` device chunk buffers: per chunk of rows, the
+    host-to-device copy (one stream), the vocabulary sweep (the caller's
+    stream) and the device-to-host copy of dLogits (a third stream) overlap
+    with the other chunks'. A chunk's input copy waits only for the sweep
+    ``depth`` chunks back, so the two copy directions can drift apart by that
+    many chunks when the host link's rate varies. The small per-row inputs go
+    to the device whole before the sweep (BEGIN needs all of them)."""
 
     SMALL = ("targets", "rollout_logprobs", "ref_logprobs", "old_logprobs", "teacher_logprobs",
              "rewards", "group_id", "cu_seqlens", "loss_mask", "topk_ids", "topk_teacher")
 
-    def __init__(self, host_w, device, chunk_rows=4096, dlogits_dtype=None):
+    def __init__(self, host_w, device, chunk_rows=4096, dlogits_dtype=None, depth=2):
         from . import workloads as wl
         self.host = host_w
         self.chunk = chunk_rows
+        self.depth = int(depth)
+        if self.depth < 2:
+            raise ValueError("depth must be at least 2")
         R, V = host_w.n_rows, host_w.vocab
         self.dl_dtype = dlogits_dtype or host_w.logits.dtype
 
@@ -157,8 +162,10 @@ class PipelinedHostCall:
                                dev(host_w.loss_mask), host_w.n_groups, dict(host_w.params),
                                dev(host_w.topk_ids), dev(host_w.topk_teacher))
         n = min(chunk_rows, R)
-        self.lg = [torch.empty((n, V), dtype=host_w.logits.dtype, device=device) for _ in range(2)]
-        self.dl = [torch.empty((n, V), dtype=self.dl_dtype, device=device) for _ in range(2)]
+        self.lg = [torch.empty((n, V), dtype=host_w.logits.dtype, device=device)
+                   for _ in range(self.depth)]
+        self.dl = [torch.empty((n, V), dtype=self.dl_dtype, device=device)
+                   for _ in range(self.depth)]
         self.buf = alloc(R, int(host_w.rewards.shape[0]), host_w.n_groups, device, vocab=V)
         pin = dict(pin_memory=True)
         self.out = dict(
@@ -190,12 +197,12 @@ class PipelinedHostCall:
             if getattr(h, k) is not None:
                 getattr(d, k).copy_(getattr(h, k), non_blocking=True)
         _rows_call(d, self.buf, ml.RL_PHASE_BEGIN, 0, R, None, None, self.params, grad_loss)
-        comp_done = [None, None]
-        out_done = [None, None]
+        comp_done = [None] * self.depth
+        out_done = [None] * self.depth
         for i, r0 in enumerate(range(0, R, self.chunk)):
             r1 = min(R, r0 + self.chunk)
-            b, n = i % 2, r1 - r0
-            if comp_done[b] is not None:   # the sweep two chunks back read lg[b]
+            b, n = i % self.depth, r1 - r0
+            if comp_done[b] is not None:   # the sweep `depth` chunks back read lg[b]
                 self.s_in.wait_event(comp_done[b])
             with torch.cuda.stream(self.s_in):
                 self.lg[b][:n].copy_(h.logits[r0:r1, :V], non_blocking=True)
@@ -350,15 +357,15 @@ class VocabShard:
         self.col_shard, self.col_starts = int(col_shard), [int(c) for c in col_starts]
         self.row_offset = int(row_offset)
         self.n_rows_total = w.n_rows if n_rows_total is None else int(n_rows_total)
-        self.params = dict(w.params if params is None else params)
+        self.params = _params(w, params)
         self.grad_loss = grad_loss
         dev = w.targets.device
         R, n_shards = w.n_rows, len(self.col_starts) - 1
         self.counts = torch.zeros(int(w.rewards.shape[0]), dtype=torch.int32, device=dev)
         self.traj_sums = torch.zeros((int(w.rewards.shape[0]), 2), dtype=torch.float64,
                                      device=dev)
-        self.row_partials = torch.zeros((R, 4), dtype=torch.float32, device=dev)
-        self.row_partials_all = torch.zeros((n_shards, R, 4), dtype=torch.float32, device=dev)
+        self.row_partials = torch.zeros((R, 8), dtype=torch.float32, device=dev)
+        self.row_partials_all = torch.zeros((n_shards, R, 8), dtype=torch.float32, device=dev)
         self.partials = torch.zeros(ml.PARTIALS_DOUBLES, dtype=torch.float64, device=dev)
 
     def _call(self, phase, forward_only=False):
@@ -400,8 +407,8 @@ def exchange_row_partials(row_partials: torch.Tensor, row_partials_all: torch.Te
     rank k's row_partials."""
     import torch.distributed as dist
     # (rank k's rows land at rows [k R, (k + 1) R) of the flattened output)
-    dist.all_gather_into_tensor(row_partials_all.view(-1, 4), row_partials.contiguous(),
-                                group=group)
+    dist.all_gather_into_tensor(row_partials_all.view(-1, row_partials.shape[-1]),
+                                row_partials.contiguous(), group=group)
 
 
 def vocab_sharded_fwd_bwd(shard: VocabShard, col_group=None, row_group=None):

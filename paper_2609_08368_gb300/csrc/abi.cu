@@ -329,6 +329,7 @@ struct FwdIn {
   // the logits are columns [col0, col0 + V); part_rows receives each row's
   // partial sums in place of the sweep's epilogue
   long long col0 = 0;
+  int vocab_total = 0;  // the vocabulary's size (0: V)
   float4* part_rows = nullptr;
   // a shard of a sharded GSPO call: the per-trajectory sums over its rows go
   // here (k_seq's first half) and the call stops before the statistics
@@ -594,7 +595,8 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     ta.ws = ws;
     ta.stall_ns = stall;
     ta.col0 = f.col0;
-    ta.part_rows = shift(f.part_rows, r0);
+    ta.vocab_total = f.vocab_total > 0 ? f.vocab_total : ta.V;
+    ta.part_rows = shift(f.part_rows, 2 * r0);
     const long long grid = std::min<long long>(ctas, c.R);
     record(t_ev_begin, s);
     st = launch(fn, dim3(static_cast<unsigned>(grid)), dim3(threads), sp.smem, 1, s,
@@ -638,7 +640,8 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     sa.ws = ws;
     sa.stall_ns = stall;
     sa.col0 = f.col0;
-    sa.part_rows = shift(f.part_rows, r0);
+    sa.vocab_total = f.vocab_total > 0 ? f.vocab_total : sa.V;
+    sa.part_rows = shift(f.part_rows, 2 * r0);
     record(t_ev_begin, s);
     st = launch(fn, dim3(static_cast<unsigned>(n_cl * pl.C)), dim3(pl.threads), pl.smem, pl.C,
                 s, &sa);
@@ -877,8 +880,6 @@ rl_status rl_loss_vocab_shard_fwd_bwd(
     return RL_ERR_INVALID_ARG;
   if (n_traj > 0 && !traj_counts) return RL_ERR_INVALID_ARG;
   if (!params) return RL_ERR_INVALID_ARG;
-  // top-K OPD candidates would be spread over the column shards
-  if (params->opd_topk > 0 && params->opd_coef != 0.0f) return RL_ERR_UNSUPPORTED;
   // GSPO: SWEEP stops at the per-trajectory sums over the shard's rows, which
   // the caller adds over the row shards before SEQ
   const bool gspo = params->estimator == RL_EST_GSPO;
@@ -895,6 +896,7 @@ rl_status rl_loss_vocab_shard_fwd_bwd(
   f.row0 = row_offset;
   f.R_total = n_rows_total;
   f.col0 = col0;
+  f.vocab_total = static_cast<int>(col_starts[n_col_shards]);
   if (count) {
     f.counts_out = traj_counts;
     rl_status st = check_fwd(f, false);

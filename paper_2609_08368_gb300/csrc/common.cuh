@@ -609,16 +609,23 @@ __device__ __forceinline__ void topk_prefetch(TopKBuf* buf, const int* ids, cons
   cp_async_commit();
 }
 
-// The lane's candidate ids of the row (after cp_async_wait_all for its buffer).
-__device__ __forceinline__ TopKLane topk_ids(const TopKBuf* buf, int V, int K, int lane) {
+// The lane's candidate ids of the row (after cp_async_wait_all for its
+// buffer), as columns of this call's logits, which are the vocabulary's
+// columns [col0, col0 + V) of a vocabulary of V_total (col0 = 0, V_total = V
+// unless the call is a vocabulary shard): -1 for a candidate in another
+// shard's columns; an id outside [0, V_total) marks the row bad.
+__device__ __forceinline__ TopKLane topk_ids(const TopKBuf* buf, int col0, int V, int V_total,
+                                             int K, int lane) {
   TopKLane c{-1, -1, 0.0f, 0.0f, false};
   if (lane < K) {
     const int id = buf->ids[lane];
-    if (id >= 0 && id < V) c.id0 = id; else c.bad = true;
+    if (id < 0 || id >= V_total) c.bad = true;
+    else if (id - col0 >= 0 && id - col0 < V) c.id0 = id - col0;
   }
   if (lane + 32 < K) {
     const int id = buf->ids[lane + 32];
-    if (id >= 0 && id < V) c.id1 = id; else c.bad = true;
+    if (id < 0 || id >= V_total) c.bad = true;
+    else if (id - col0 >= 0 && id - col0 < V) c.id1 = id - col0;
   }
   return c;
 }

@@ -359,7 +359,7 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
       const int h = (kGrad && trains && n_chunks > 0) ? min(a.n_hold, n_chunks) : 0;
       const TopKBuf* tk_row = &tkb[i & 1];
       cp_async_wait_all();
-      TopKLane tk = topk_ids(tk_row, a.V, K, lane);
+      TopKLane tk = topk_ids(tk_row, static_cast<int>(a.col0), a.V, a.vocab_total, K, lane);
       if (i + 1 < rows_mine) {
         const long long o = (row + gridDim.x) * K;
         topk_prefetch(&tkb[(i + 1) & 1], a.s.topk_ids + o, a.s.topk_teacher + o, K, lane);
@@ -535,11 +535,13 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
     // part of this row and the row's lse (warp 0)
     float opd = 0.0f;
     int tk_bad = 0;
+    TopKPart part{-INFINITY, 0.0f, 0.0f, 0};  // (kept for a vocabulary shard's record)
     if (kTopK && warp == 0) {
       if (mbar_wait_or_abort(smem_u32(&tk_full[i & 1]), static_cast<uint32_t>((i >> 1) & 1),
                              kWaitLimitNs, abort, err)) {
-        opd = topk_value(tkp[i & 1], fmaf(t.m, kLn2f, logf(t.s)));
-        tk_bad = tkp[i & 1].bad;
+        part = tkp[i & 1];
+        opd = topk_value(part, fmaf(t.m, kLn2f, logf(t.s)));
+        tk_bad = part.bad;
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&tk_empty[i & 1]));
@@ -558,9 +560,11 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
     TokenTerms tt{};
     if (tid == 0 && a.part_rows) {
       // vocabulary-sharded forward: the row's partial sums over this
-      // shard's columns (a row read after the CTA gave up is marked NaN)
-      a.part_rows[row] = *abort ? make_float4(NAN, 0.0f, 0.0f, 0.0f)
-                                : make_float4(t.m, t.s, t.u, yok ? zy : 0.0f);
+      // shard's columns and its top-K candidates' part (a row read after
+      // the CTA gave up is marked NaN)
+      a.part_rows[2 * row] = *abort ? make_float4(NAN, 0.0f, 0.0f, 0.0f)
+                                    : make_float4(t.m, t.s, t.u, yok ? zy : 0.0f);
+      a.part_rows[2 * row + 1] = make_float4(part.m, part.sw, part.acc, part.bad ? 1.0f : 0.0f);
     } else if (tid == 0) {
       // a row read after the CTA gave up, a bad target or a bad top-K
       // candidate: zeros

@@ -338,7 +338,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
     // shared memory, past its whole vectors from global memory
     TopKPart tkp{-INFINITY, 0.0f, 0.0f, 0};
     if (topk && tid < 32) {
-      TopKLane tk = topk_ids(tk_row, a.V, a.s.topk, tid);
+      TopKLane tk = topk_ids(tk_row, static_cast<int>(a.col0), a.V, a.vocab_total, a.s.topk, tid);
       if (have) topk_gather<In>(tk, sb, lo, lo + vec_elems);
       topk_gather<In>(tk, grow + static_cast<size_t>(vec_elems) * sizeof(St), lo + vec_elems, lo + cnt);
       const int c0 = lo, c1 = lo + cnt;
@@ -403,9 +403,12 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) k_sweep(const SweepArgs 
     if (tid == 0 && a.part_rows) {
       // vocabulary-sharded forward: the row's partial sums over this
       // shard's columns (a row read after the CTA gave up is marked NaN)
-      if (crank == 0)
-        a.part_rows[row] = *abort ? make_float4(NAN, 0.0f, 0.0f, 0.0f)
-                                  : make_float4(tot.m, tot.s, tot.u, yok ? zy_all : 0.0f);
+      if (crank == 0) {
+        a.part_rows[2 * row] = *abort ? make_float4(NAN, 0.0f, 0.0f, 0.0f)
+                                      : make_float4(tot.m, tot.s, tot.u, yok ? zy_all : 0.0f);
+        a.part_rows[2 * row + 1] = topk ? make_float4(tkp.m, tkp.sw, tkp.acc, tkp.bad ? 1.0f : 0.0f)
+                                        : make_float4(-INFINITY, 0.0f, 0.0f, 0.0f);
+      }
     } else if (tid == 0) {
       // a row read after the CTA gave up, a bad target or a bad top-K
       // candidate: zeros

@@ -49,10 +49,12 @@ struct SweepArgs {
   // timeout path runs (see rl_launch_overrides).
   unsigned long long stall_ns;
   // A vocabulary-sharded call (forward only): the logits are columns
-  // [col0, col0 + V) of the vocabulary, a target outside them is another
-  // shard's, and each row's partial sums go to part_rows (RowPartial) in
-  // place of the epilogue. Unsharded calls: 0 and null.
+  // [col0, col0 + V) of a vocabulary of vocab_total ids, a target or top-K
+  // candidate outside them is another shard's, and each row's partial sums
+  // go to part_rows (two float4 per row, see k_vshard.cu) in place of the
+  // epilogue. Unsharded calls: col0 0, vocab_total V, part_rows null.
   long long col0;
+  int vocab_total;
   float4* part_rows;
 };
 
@@ -81,6 +83,7 @@ struct StreamArgs {
   WsPtrs ws;
   unsigned long long stall_ns;  // test hook, as in SweepArgs (the consumers' first wait)
   long long col0;               // vocabulary-sharded calls, as in SweepArgs
+  int vocab_total;
   float4* part_rows;
 };
 
@@ -158,10 +161,10 @@ struct BwdArgs {
   WsPtrs ws;
 };
 
-// The merge of a vocabulary-sharded call: each row's partial sums from every
-// column shard (RowPartial, shard-major: all[k * R + row]) in shard order,
-// then the row's statistics and per-token objective, as the fused sweep's
-// epilogue writes them.
+// The merge of a vocabulary-sharded call: each row's record from every
+// column shard (two float4, shard-major: all[2 (k R + row)] and the one after
+// it) in shard order, then the row's statistics and per-token objective, as
+// the fused sweep's epilogue writes them.
 constexpr int kMaxColShards = 64;
 constexpr int kMergeThreads = 256;
 struct MergeArgs {

@@ -355,8 +355,8 @@ def rl_loss_vocab_shard_fwd_bwd(phase, col_shard, col_starts, row_offset, n_rows
     """One phase of a column shard's part of a vocabulary-sharded call.
     ``col_starts`` is a host sequence of n_col_shards + 1 vocabulary ids;
     ``logits`` / ``dlogits`` hold this shard's columns of its rows;
-    ``row_partials`` is float32 [n_rows, 4] and ``row_partials_all`` float32
-    [n_col_shards, n_rows, 4] (device)."""
+    ``row_partials`` is float32 [n_rows, 8] and ``row_partials_all`` float32
+    [n_col_shards, n_rows, 8] (device)."""
     import torch
     cs = [int(c) for c in col_starts]
     n_shards = len(cs) - 1

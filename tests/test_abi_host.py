@@ -315,7 +315,9 @@ def test_vocab_sharded_entry_validates(lib):
     assert call(SW, params=gspo, sums=None) == RL_ERR_INVALID_ARG     # GSPO writes its sums
     assert call(ml.RL_VSHARD_SEQ, params=gspo, sums=None) == RL_ERR_INVALID_ARG
     assert call(ml.RL_VSHARD_SEQ, params=gspo, partials=None) == RL_ERR_INVALID_ARG
-    tk = ml.make_params(opd_coef=0.5, opd_topk=4, opd_topk_ids=_Ptr(FAKE),
-                        opd_topk_teacher=_Ptr(FAKE))
-    assert call(PA, params=tk) == 2
+    tk = ml.make_params(opd_coef=0.5, opd_topk=4, opd_topk_ids=_Ptr(FAKE + 2),
+                        opd_topk_teacher=_Ptr(FAKE))                   # ids not 4-byte aligned
+    assert call(PA, params=tk) == RL_ERR_INVALID_ARG
+    tk = ml.make_params(opd_coef=0.5, opd_topk=4)                      # no candidate arrays
+    assert call(PA, params=tk) == RL_ERR_INVALID_ARG
     assert call(PA, params=ml.make_params(temperature=0.0)) == RL_ERR_INVALID_ARG

@@ -43,7 +43,7 @@ def _view(w, r0, r1, c0, c1):
     return wl.Workload(w.recipe, w.logits[sl, c0:c1], rows(w.targets), rows(w.rollout_logprobs),
                        rows(w.ref_logprobs), rows(w.old_logprobs), rows(w.teacher_logprobs),
                        w.rewards, w.group_id, w.cu_seqlens, rows(w.loss_mask), w.n_groups,
-                       dict(w.params))
+                       dict(w.params), rows(w.topk_ids), rows(w.topk_teacher))
 
 
 def run_sharded(w, col_starts, row_cuts, params, dl_dtype=None, drive=True):
@@ -107,12 +107,14 @@ PARAMS = {
     "opd_ent_tis": dict(opd_coef=0.3, entropy_coef=0.01, temperature=0.7, correction="tis",
                         corr_lo=0.0, corr_hi=2.0),
     "gspo_tis": dict(estimator="gspo", correction="tis", corr_lo=0.0, corr_hi=1.5),
+    "topk_ent": dict(opd_coef=0.3, opd_topk=8, entropy_coef=0.01),
 }
 
 
 def _workload():
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=2, group_size=4, traj_len=40, vocab=V,
-                    rho_noise=0.3, ref_noise=0.2, teacher_noise=0.4, mask="prefix_u0_half")
+                    rho_noise=0.3, ref_noise=0.2, teacher_noise=0.4, mask="prefix_u0_half",
+                    topk=8, topk_noise=0.4)
     return wl.make(rec, DEV)
 
 
@@ -196,15 +198,30 @@ def test_vocab_sharded_bad_target_is_reported():
     P.assert_dlogits_close(g["dlogits_t"][good].float().cpu().numpy(), o["dlogits"][good])
 
 
-def test_vocab_sharded_topk_is_unsupported():
+@pytest.mark.parametrize("kind", ["cluster", "stream"])
+def test_vocab_sharded_topk_ids_out_of_range_are_reported(ov, kind):
+    """A top-K candidate id outside the vocabulary: SWEEP on every column
+    shard reports RL_ERR_TOPK_ID_OUT_OF_RANGE and writes zeros for that row;
+    the other rows match the oracle (with a valid id in its place)."""
+    ov(sweep_kernel=kind)
     w = _workload()
-    params = dict(w.params, opd_coef=0.5, opd_topk=4,
-                  opd_topk_ids=torch.zeros((w.n_rows, 4), dtype=torch.int32, device=DEV),
-                  opd_topk_teacher=torch.zeros((w.n_rows, 4), device=DEV))
-    s = run_sharded(w, [0, 10240, V], [0, w.n_rows], params, drive=False)[0][0]
-    with pytest.raises(ml.MilesLossError) as e:
-        s.count()
-    assert e.value.status == 2  # RL_ERR_UNSUPPORTED
+    params = dict(w.params, opd_coef=0.3, opd_topk=8)
+    bad = [5, 33]
+    ids_ok = w.topk_ids.clone()
+    w.topk_ids[5, 3] = V        # one past the end
+    w.topk_ids[33, 0] = -1
+    cols, cuts = [0, 10240, V], [0, w.n_rows]
+    g = assemble(w, run_sharded(w, cols, cuts, params), cols, cuts, expect_err=9)
+    for r in bad:
+        assert g["logp"][r] == 0 and g["H"][r] == 0
+        assert (g["dlogits_t"][r].float() == 0).all()
+    w.topk_ids.copy_(ids_ok)
+    o = P.run_oracle(w, params=params)
+    good = np.setdiff1d(np.arange(w.n_rows), bad)
+    tol = P.logp_tol(w)
+    np.testing.assert_allclose(g["logp"][good], o["logp"][good], atol=tol, rtol=0)
+    np.testing.assert_allclose(g["H"][good], o["H"][good], atol=tol, rtol=0)
+    P.assert_dlogits_close(g["dlogits_t"][good].float().cpu().numpy(), o["dlogits"][good])
 
 
 @pytest.mark.slow
