@@ -47,7 +47,7 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="glm")
-    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--e2e-steps", type=int, default=4)
     ap.add_argument("--e2e-chunk-rows", type=int, default=4096)
     ap.add_argument("--e2e-depth", type=int, default=2,
                     help="device chunk buffers of the pipelined host-buffer call")
@@ -491,7 +491,7 @@ def _pinned_copy(w):
                        w.n_groups, dict(w.params))
 
 
-def copy_floor_ms(call, stream, steps: int) -> float:
+def copy_floor_ms(call, stream, steps: int, warm: bool = True) -> float:
     """Milliseconds per step of the pipelined call's logits and dLogits
     copies alone: per chunk of rows, the host-to-device copy of its logits on
     the input stream and the device-to-host copy of a dLogits buffer of the
@@ -519,7 +519,8 @@ def copy_floor_ms(call, stream, steps: int) -> float:
         if out_done is not None:
             stream.wait_event(out_done)
 
-    one()
+    if warm:
+        one()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
@@ -704,29 +705,38 @@ def run_ours(args, rank, world, local):
         call = api.PipelinedHostCall(host_w, dev, chunk_rows=args.e2e_chunk_rows,
                                      depth=args.e2e_depth)
         call()
+        copy_floor_ms(call, stream, 1)
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        # each timed step of the call is followed by one step of its copies
+        # alone, so that a change in the host link's rate during the
+        # measurement (other processes on the host) falls on both
+        call_ms, floor_steps = [], []
         barrier(world)
-        torch.cuda.synchronize()
-        e0.record(stream)
         for _ in range(args.e2e_steps):
+            torch.cuda.synchronize()
+            e0.record(stream)
             call()
-        e1.record(stream)
-        torch.cuda.synchronize()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            call_ms.append(e0.elapsed_time(e1))
+            floor_steps.append(copy_floor_ms(call, stream, 1, warm=False))
         barrier(world)
-        ms_e2e = max_over_ranks(e0.elapsed_time(e1), world) / args.e2e_steps
-        floor_ms = copy_floor_ms(call, stream, args.e2e_steps)
+        ms_e2e = max_over_ranks(statistics.fmean(call_ms), world)
+        floor_ms = statistics.fmean(floor_steps)
         e2e = {"value": rows_all / (ms_e2e / 1e3), "unit": "tokens/s",
                "ms_per_step": ms_e2e, "steps": args.e2e_steps,
+               "ms_per_step_each": call_ms, "copy_floor_ms_each": floor_steps,
                "how": f"pinned host buffers, rl_loss_fwd_bwd_rows over chunks of "
                       f"{args.e2e_chunk_rows} rows through {args.e2e_depth} device chunk "
                       f"buffers, copies overlapped with the sweep",
                "h2d_bytes_per_step": call.bytes_in(), "d2h_bytes_per_step": call.bytes_out(),
                "copy_floor_ms": floor_ms, "frac_of_copy_floor": floor_ms / ms_e2e,
                "copy_floor_how": "the same logits and dLogits bytes copied alone on this box, "
-                                 "in the same chunks, through the same two device buffers and "
+                                 "in the same chunks, through the same device buffers and "
                                  "copy streams, host-to-device and device-to-host at once "
-                                 "(no sweep)"}
+                                 "(no sweep); one such step after each timed step of the "
+                                 "call"}
         del call, host_w
 
     # the committed capture is of the default path (GRPO-style fused sweep,
