@@ -224,6 +224,43 @@ def test_vocab_sharded_topk_ids_out_of_range_are_reported(ov, kind):
     P.assert_dlogits_close(g["dlogits_t"][good].float().cpu().numpy(), o["dlogits"][good])
 
 
+@pytest.mark.parametrize("kind", ["cluster", "stream"])
+def test_vocab_shard_that_gives_up_zeroes_its_rows_everywhere(ov, kind):
+    """Failure detection across shards, without a fault: the test hook makes
+    every CTA of shard 0's partial sweep give up on its first wait (bounded
+    by 1 ms). Shard 0 reports RL_ERR_DEVICE_TIMEOUT; its records carry the
+    give-up mark, so the merge on EVERY shard writes zeros for those rows
+    (finite outputs, zero dLogits) and shard 1's own error word stays clean.
+    The next call without the hook matches the oracle."""
+    ov(sweep_kernel=kind)
+    w = _workload()
+    cols, cuts = [0, 10240, V], [0, w.n_rows]
+    shards = run_sharded(w, cols, cuts, dict(w.params), drive=False)
+    s0, s1 = shards[0]
+    for s in (s0, s1):
+        s.count()
+    ov(stall_first_wait_ns=1_000_000)
+    s0.partial()
+    ov(stall_first_wait_ns=-1)
+    s1.partial()
+    gathered = torch.stack([s0.row_partials, s1.row_partials])
+    for s in (s0, s1):
+        s.row_partials_all.copy_(gathered)
+        s.sweep()
+        s.finish()
+    torch.cuda.synchronize()
+    assert ml.rl_loss_check_device_error(s0.buf.workspace) == 8  # RL_ERR_DEVICE_TIMEOUT
+    assert ml.rl_loss_check_device_error(s1.buf.workspace) == 0
+    for s in (s0, s1):
+        assert (s.buf.token_logprobs == 0).all() and (s.buf.entropy == 0).all()
+        assert torch.equal(s.buf.dlogits, torch.zeros_like(s.buf.dlogits))
+        assert s.buf.read_stats()["loss"] == 0.0
+    g = assemble(w, run_sharded(w, cols, cuts, dict(w.params)), cols, cuts)
+    o = P.run_oracle(w)
+    P.compare_forward(w, g, o)
+    P.assert_dlogits_close(g["dlogits_t"].float().cpu().numpy(), o["dlogits"])
+
+
 @pytest.mark.slow
 def test_full_size_two_column_shards_equal_the_whole_call():
     """The headline batch (65,536 x 154,880 bf16) split into two column
