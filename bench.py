@@ -491,6 +491,24 @@ def _pinned_copy(w):
                        w.n_groups, dict(w.params))
 
 
+def e2e_host_memory_check(bytes_per_rank: int, ranks_on_host: int):
+    """None if this host's available memory holds every local rank's pinned
+    host buffers with a tenth to spare, else the reason to skip the e2e
+    leg (pinning more than the host has would take the machine down)."""
+    try:
+        with open("/proc/meminfo") as f:
+            avail = next(int(line.split()[1]) * 1024 for line in f
+                         if line.startswith("MemAvailable:"))
+    except (OSError, StopIteration, ValueError):
+        return None
+    need = bytes_per_rank * max(1, ranks_on_host)
+    if need * 1.1 > avail:
+        return (f"the e2e leg would pin {need / 1e9:.1f} GB of host memory for "
+                f"{ranks_on_host} local rank(s), more than 0.9 x the {avail / 1e9:.1f} GB "
+                f"available")
+    return None
+
+
 def copy_floor_ms(call, stream, steps: int, warm: bool = True) -> float:
     """Milliseconds per step of the pipelined call's logits and dLogits
     copies alone: per chunk of rows, the host-to-device copy of its logits on
@@ -698,7 +716,11 @@ def run_ours(args, rank, world, local):
 
     # end to end through host buffers (pinned), one call per step
     e2e = None
-    if not args.no_e2e and args.e2e_steps > 0:
+    host_need = 2 * R * V * w.logits.element_size()  # pinned logits in, dLogits out
+    host_skip = e2e_host_memory_check(host_need, int(os.environ.get("LOCAL_WORLD_SIZE", "1")))
+    if host_skip and not args.no_e2e:
+        e2e = {"skipped": host_skip}
+    elif not args.no_e2e and args.e2e_steps > 0:
         host_w = _pinned_copy(w)
         del w, buf  # the pipelined call keeps its own two chunk buffers
         torch.cuda.empty_cache()

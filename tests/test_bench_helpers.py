@@ -63,3 +63,12 @@ def test_api_attaches_top_k_inputs():
     p = api._params(w, dict(w.params, opd_topk=4, opd_coef=0.5))
     assert p["opd_topk_ids"] is w.topk_ids and p["opd_topk_teacher"] is w.topk_teacher
     assert "opd_topk_ids" not in api._params(w, None)
+
+
+def test_e2e_leg_is_skipped_when_the_host_cannot_pin_its_buffers():
+    avail = next(int(line.split()[1]) * 1024 for line in open("/proc/meminfo")
+                 if line.startswith("MemAvailable:"))
+    assert bench.e2e_host_memory_check(avail // 4, 1) is None
+    reason = bench.e2e_host_memory_check(avail, 1)
+    assert reason and "host memory" in reason
+    assert bench.e2e_host_memory_check(avail // 4, 8) is not None  # eight local ranks
