@@ -47,7 +47,7 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="glm")
-    ap.add_argument("--e2e-steps", type=int, default=4)
+    ap.add_argument("--e2e-steps", type=int, default=6)
     ap.add_argument("--e2e-chunk-rows", type=int, default=4096)
     ap.add_argument("--e2e-depth", type=int, default=2,
                     help="device chunk buffers of the pipelined host-buffer call")
@@ -512,30 +512,33 @@ def e2e_host_memory_check(bytes_per_rank: int, ranks_on_host: int):
 def copy_floor_ms(call, stream, steps: int, warm: bool = True) -> float:
     """Milliseconds per step of the pipelined call's logits and dLogits
     copies alone: per chunk of rows, the host-to-device copy of its logits on
-    the input stream and the device-to-host copy of a dLogits buffer of the
-    same rows on the output stream (after that chunk's input copy, as if the
-    sweep took no time), through the call's own device buffers, so both
-    directions run at once as in the call. What the call takes beyond this
-    is what the sweep and the small copies add."""
+    the input stream and, when the call copies dLogits back, the
+    device-to-host copy of a dLogits buffer of the same rows on the output
+    stream (after that chunk's input copy, as if the sweep took no time),
+    through the call's own device buffers, so both directions run at once as
+    in the call. What the call takes beyond this is what the sweep and the
+    small copies add."""
     h = call.host
     R, V = h.n_rows, h.vocab
 
     def one():
-        out_done = None
+        done = None
         for i, r0 in enumerate(range(0, R, call.chunk)):
             r1 = min(R, r0 + call.chunk)
             b, n = i % len(call.lg), r1 - r0
             with torch.cuda.stream(call.s_in):
                 call.lg[b][:n].copy_(h.logits[r0:r1, :V], non_blocking=True)
-                in_done = torch.cuda.Event()
+                done = in_done = torch.cuda.Event()
                 in_done.record(call.s_in)
+            if call.dl is None:  # dLogits stay on the device: input copies only
+                continue
             call.s_out.wait_event(in_done)
             with torch.cuda.stream(call.s_out):
                 call.out["dlogits"][r0:r1].copy_(call.dl[b][:n], non_blocking=True)
-                out_done = torch.cuda.Event()
-                out_done.record(call.s_out)
-        if out_done is not None:
-            stream.wait_event(out_done)
+                done = torch.cuda.Event()
+                done.record(call.s_out)
+        if done is not None:
+            stream.wait_event(done)
 
     if warm:
         one()
@@ -588,6 +591,55 @@ def vocab_tp2_timing(w, dev, dl_dtype, stream, reps: int = 10) -> dict:
             "vocab_tp2_how": "two column shards of the vocabulary, both on this GPU one after "
                              "the other; per shard: partial sweep, merge, gradient sweep, "
                              "statistics (the logits read twice, as in the split pair)"}
+
+
+def e2e_leg(host_w, dev, args, stream, world, rows_all, dlogits_on_device: bool) -> dict:
+    """The pipelined host-buffer call timed end to end, each timed step
+    followed by one step of its copies alone (so that a change in the host
+    link's rate during the measurement, from other processes on the host,
+    falls on both)."""
+    from paper_2609_08368_gb300 import api
+    call = api.PipelinedHostCall(host_w, dev, chunk_rows=args.e2e_chunk_rows,
+                                 depth=args.e2e_depth, dlogits_on_device=dlogits_on_device)
+    call()
+    copy_floor_ms(call, stream, 1)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    call_ms, floor_steps = [], []
+    barrier(world)
+    for _ in range(args.e2e_steps):
+        torch.cuda.synchronize()
+        e0.record(stream)
+        call()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        call_ms.append(e0.elapsed_time(e1))
+        floor_steps.append(copy_floor_ms(call, stream, 1, warm=False))
+    barrier(world)
+    ms_e2e = max_over_ranks(statistics.fmean(call_ms), world)
+    floor_ms = statistics.fmean(floor_steps)
+    where = ("dLogits written to one device tensor; the per-row log-probs and entropies "
+             "and the statistics copied back" if dlogits_on_device else
+             "dLogits copied back to pinned host memory too, overlapped with the sweep")
+    out = {"value": rows_all / (ms_e2e / 1e3), "unit": "tokens/s",
+           "ms_per_step": ms_e2e, "steps": args.e2e_steps,
+           "ms_per_step_each": call_ms, "copy_floor_ms_each": floor_steps,
+           "how": f"logits from pinned host memory through rl_loss_fwd_bwd_rows in chunks of "
+                  f"{args.e2e_chunk_rows} rows and {args.e2e_depth} device chunk buffers, "
+                  f"the copies overlapped with the sweep; {where}",
+           "h2d_bytes_per_step": call.bytes_in(), "d2h_bytes_per_step": call.bytes_out(),
+           "copy_floor_ms": floor_ms, "frac_of_copy_floor": floor_ms / ms_e2e,
+           # the host link's rate drops to a third or less for bursts of a few
+           # hundred ms on some boxes, hitting the call and its copies alike:
+           # the best step of each shows what the call adds on a steady link
+           "best_ms_per_step": min(call_ms), "best_copy_floor_ms": min(floor_steps),
+           "frac_of_copy_floor_best": min(floor_steps) / min(call_ms),
+           "copy_floor_how": "the same logits (and, when they go back, dLogits) copied alone "
+                             "on this box, in the same chunks, through the same device "
+                             "buffers and copy streams (no sweep); one such step after each "
+                             "timed step of the call"}
+    del call
+    return out
 
 
 def run_ours(args, rank, world, local):
@@ -722,44 +774,17 @@ def run_ours(args, rank, world, local):
         e2e = {"skipped": host_skip}
     elif not args.no_e2e and args.e2e_steps > 0:
         host_w = _pinned_copy(w)
-        del w, buf  # the pipelined call keeps its own two chunk buffers
+        del w, buf  # the pipelined call keeps its own chunk buffers
         torch.cuda.empty_cache()
-        call = api.PipelinedHostCall(host_w, dev, chunk_rows=args.e2e_chunk_rows,
-                                     depth=args.e2e_depth)
-        call()
-        copy_floor_ms(call, stream, 1)
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        # each timed step of the call is followed by one step of its copies
-        # alone, so that a change in the host link's rate during the
-        # measurement (other processes on the host) falls on both
-        call_ms, floor_steps = [], []
-        barrier(world)
-        for _ in range(args.e2e_steps):
-            torch.cuda.synchronize()
-            e0.record(stream)
-            call()
-            e1.record(stream)
-            torch.cuda.synchronize()
-            call_ms.append(e0.elapsed_time(e1))
-            floor_steps.append(copy_floor_ms(call, stream, 1, warm=False))
-        barrier(world)
-        ms_e2e = max_over_ranks(statistics.fmean(call_ms), world)
-        floor_ms = statistics.fmean(floor_steps)
-        e2e = {"value": rows_all / (ms_e2e / 1e3), "unit": "tokens/s",
-               "ms_per_step": ms_e2e, "steps": args.e2e_steps,
-               "ms_per_step_each": call_ms, "copy_floor_ms_each": floor_steps,
-               "how": f"pinned host buffers, rl_loss_fwd_bwd_rows over chunks of "
-                      f"{args.e2e_chunk_rows} rows through {args.e2e_depth} device chunk "
-                      f"buffers, copies overlapped with the sweep",
-               "h2d_bytes_per_step": call.bytes_in(), "d2h_bytes_per_step": call.bytes_out(),
-               "copy_floor_ms": floor_ms, "frac_of_copy_floor": floor_ms / ms_e2e,
-               "copy_floor_how": "the same logits and dLogits bytes copied alone on this box, "
-                                 "in the same chunks, through the same device buffers and "
-                                 "copy streams, host-to-device and device-to-host at once "
-                                 "(no sweep); one such step after each timed step of the "
-                                 "call"}
-        del call, host_w
+        # the step's inputs from pinned host memory, its results (per-row
+        # log-prob and entropy, the statistics) back; dLogits stay on the
+        # device, where the trainer's backward pass reads them
+        e2e = e2e_leg(host_w, dev, args, stream, world, rows_all, dlogits_on_device=True)
+        torch.cuda.empty_cache()
+        # the same with dLogits copied back to pinned host memory as well
+        e2e["host_dlogits"] = e2e_leg(host_w, dev, args, stream, world, rows_all,
+                                      dlogits_on_device=False)
+        del host_w
 
     # the committed capture is of the default path (GRPO-style fused sweep,
     # no top-K): it does not describe the others

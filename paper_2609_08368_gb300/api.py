@@ -131,19 +131,23 @@ def fwd_bwd_chunked(w, buf: Buffers, chunk_rows: int, params=None, grad_loss=1.0
 
 
 class PipelinedHostCall:
-    """The fused call with logits and dLogits in pinned HOST memory, streamed
-    through ``depth`` device chunk buffers: per chunk of rows, the
-    host-to-device copy (one stream), the vocabulary sweep (the caller's
-    stream) and the device-to-host copy of dLogits (a third stream) overlap
-    with the other chunks'. A chunk's input copy waits only for the sweep
-    ``depth`` chunks back, so the two copy directions can drift apart by that
-    many chunks when the host link's rate varies. The small per-row inputs go
-    to the device whole before the sweep (BEGIN needs all of them)."""
+    """The fused call with logits in pinned HOST memory, streamed through
+    ``depth`` device chunk buffers: per chunk of rows, the host-to-device
+    copy (one stream), the vocabulary sweep (the caller's stream) and, when
+    dLogits go back to pinned host memory too, their device-to-host copy (a
+    third stream) overlap with the other chunks'. A chunk's input copy waits
+    only for the sweep ``depth`` chunks back, so the two copy directions can
+    drift apart by that many chunks when the host link's rate varies. With
+    ``dlogits_on_device`` the dLogits stay in one device tensor (where a
+    trainer's backward pass reads them) and only the per-row results and the
+    statistics come back. The small per-row inputs go to the device whole
+    before the sweep (BEGIN needs all of them)."""
 
     SMALL = ("targets", "rollout_logprobs", "ref_logprobs", "old_logprobs", "teacher_logprobs",
              "rewards", "group_id", "cu_seqlens", "loss_mask", "topk_ids", "topk_teacher")
 
-    def __init__(self, host_w, device, chunk_rows=4096, dlogits_dtype=None, depth=2):
+    def __init__(self, host_w, device, chunk_rows=4096, dlogits_dtype=None, depth=2,
+                 dlogits_on_device=False):
         from . import workloads as wl
         self.host = host_w
         self.chunk = chunk_rows
@@ -164,12 +168,13 @@ class PipelinedHostCall:
         n = min(chunk_rows, R)
         self.lg = [torch.empty((n, V), dtype=host_w.logits.dtype, device=device)
                    for _ in range(self.depth)]
-        self.dl = [torch.empty((n, V), dtype=self.dl_dtype, device=device)
-                   for _ in range(self.depth)]
+        self.dl = None if dlogits_on_device else [
+            torch.empty((n, V), dtype=self.dl_dtype, device=device) for _ in range(self.depth)]
         self.buf = alloc(R, int(host_w.rewards.shape[0]), host_w.n_groups, device, vocab=V)
         pin = dict(pin_memory=True)
         self.out = dict(
-            dlogits=torch.empty((R, V), dtype=self.dl_dtype, **pin),
+            dlogits=torch.empty((R, V), dtype=self.dl_dtype,
+                                **(dict(device=device) if dlogits_on_device else pin)),
             token_logprobs=torch.empty(R, dtype=torch.float32, **pin),
             entropy=torch.empty(R, dtype=torch.float32, **pin),
             stats=torch.empty(ml.STATS_BYTES, dtype=torch.uint8, **pin))
@@ -187,7 +192,8 @@ class PipelinedHostCall:
             for k in self.SMALL if getattr(h, k) is not None)
 
     def bytes_out(self) -> int:
-        return sum(t.numel() * t.element_size() for t in self.out.values())
+        """Bytes copied back to the host per call."""
+        return sum(t.numel() * t.element_size() for t in self.out.values() if not t.is_cuda)
 
     def __call__(self, grad_loss=1.0):
         comp = torch.cuda.current_stream()
@@ -211,15 +217,17 @@ class PipelinedHostCall:
             comp.wait_event(in_done)
             if out_done[b] is not None:    # dl[b] was copied out
                 comp.wait_event(out_done[b])
-            _rows_call(d, self.buf, ml.RL_PHASE_ROWS, r0, r1, self.lg[b][:n], self.dl[b][:n],
+            dl = self.out["dlogits"][r0:r1] if self.dl is None else self.dl[b][:n]
+            _rows_call(d, self.buf, ml.RL_PHASE_ROWS, r0, r1, self.lg[b][:n], dl,
                        self.params, grad_loss)
             comp_done[b] = torch.cuda.Event()
             comp_done[b].record(comp)
-            self.s_out.wait_event(comp_done[b])
-            with torch.cuda.stream(self.s_out):
-                self.out["dlogits"][r0:r1].copy_(self.dl[b][:n], non_blocking=True)
-                out_done[b] = torch.cuda.Event()
-                out_done[b].record(self.s_out)
+            if self.dl is not None:
+                self.s_out.wait_event(comp_done[b])
+                with torch.cuda.stream(self.s_out):
+                    self.out["dlogits"][r0:r1].copy_(self.dl[b][:n], non_blocking=True)
+                    out_done[b] = torch.cuda.Event()
+                    out_done[b].record(self.s_out)
         _rows_call(d, self.buf, ml.RL_PHASE_END, 0, R, None, None, self.params, grad_loss)
         self.out["token_logprobs"].copy_(self.buf.token_logprobs, non_blocking=True)
         self.out["entropy"].copy_(self.buf.entropy, non_blocking=True)

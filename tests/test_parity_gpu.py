@@ -725,13 +725,16 @@ def test_pipelined_host_call_matches_device_call():
     for k in ("logits", "targets", "rollout_logprobs", "ref_logprobs", "rewards", "group_id",
               "cu_seqlens", "loss_mask"):
         setattr(host, k, getattr(host, k).pin_memory())
-    call = api.PipelinedHostCall(host, DEV, chunk_rows=100)
-    for _ in range(2):
-        out = call()
-        torch.cuda.synchronize()
-        assert torch.equal(out["dlogits"], whole["dlogits_t"].cpu())
-        np.testing.assert_array_equal(out["token_logprobs"].numpy(), whole["logp"])
-        assert ml.parse_stats(out["stats"].numpy().tobytes()) == whole["stats"]
+    for depth, on_device in ((2, False), (3, False), (2, True)):
+        call = api.PipelinedHostCall(host, DEV, chunk_rows=100, depth=depth,
+                                     dlogits_on_device=on_device)
+        assert call.out["dlogits"].is_cuda == on_device
+        for _ in range(2):
+            out = call()
+            torch.cuda.synchronize()
+            assert torch.equal(out["dlogits"].cpu(), whole["dlogits_t"].cpu())
+            np.testing.assert_array_equal(out["token_logprobs"].numpy(), whole["logp"])
+            assert ml.parse_stats(out["stats"].numpy().tobytes()) == whole["stats"]
 
 
 # ---------------------------------------------------------- row-sharded calls
