@@ -100,6 +100,8 @@ LAYOUTS = {
     "tp3_unaligned": ([0, 7001, 13000, V], None),     # column starts off 16-byte boundaries
     "tp2_cp2": ([0, 10240, V], [0, 137]),
     "tp4_cp3": ([0, 5000, 10240, 15003, V], [0, 50, 50]),  # with an empty row shard
+    "tp1": ([0, V], None),                               # one column shard: the whole vocabulary
+    "tp8_uneven": ([0, 8, 1000, 1024, 9000, 9001, 15000, 20000, V], [0, 200]),
 }
 PARAMS = {
     "grpo": dict(),
