@@ -47,7 +47,7 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="glm")
-    ap.add_argument("--e2e-steps", type=int, default=6)
+    ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--e2e-chunk-rows", type=int, default=4096)
     ap.add_argument("--e2e-depth", type=int, default=2,
                     help="device chunk buffers of the pipelined host-buffer call")
