@@ -275,11 +275,17 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
       const uint64_t pol_a = l2_policy_evict_last(), pol_b = l2_policy_evict_first();
       bool stop = false;
       long long q = 0;
+      // each row's mask byte is loaded one row ahead, so that its latency
+      // (often a DRAM access: a CTA's rows are gridDim.x bytes apart) never
+      // delays the row it decides
+      uint8_t mask_next = rows_mine > 0 ? a.mask[blockIdx.x] : 0;
       for (long long i = 0; i < rows_mine && !stop; ++i) {
         const long long row = blockIdx.x + i * gridDim.x;
         const char* src_row = lg + row * a.ld * static_cast<long long>(sizeof(St));
+        const uint8_t msk_row = mask_next;
+        if (i + 1 < rows_mine) mask_next = a.mask[row + gridDim.x];
         // a row that does not train has an all-zero gradient: no second read
-        const bool again = kGrad && a.mask[row] && n_chunks > 0;
+        const bool again = kGrad && msk_row && n_chunks > 0;
         const int h = again ? min(a.n_hold, n_chunks) : 0;
         const int tasks = again ? 2 * n_chunks - h : n_chunks;
         for (int t = 0; t < tasks; ++t, ++q) {
@@ -353,9 +359,11 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
       topk_prefetch(&tkb[0], a.s.topk_ids + static_cast<long long>(blockIdx.x) * K,
                     a.s.topk_teacher + static_cast<long long>(blockIdx.x) * K, K, lane);
     long long q0 = 0;
+    uint8_t mask_next = rows_mine > 0 ? a.mask[blockIdx.x] : 0;  // one row ahead
     for (long long i = 0; i < rows_mine; ++i) {
       const long long row = blockIdx.x + i * gridDim.x;
-      const bool trains = a.mask[row] != 0;
+      const bool trains = mask_next != 0;
+      if (i + 1 < rows_mine) mask_next = a.mask[row + gridDim.x];
       const int h = (kGrad && trains && n_chunks > 0) ? min(a.n_hold, n_chunks) : 0;
       const TopKBuf* tk_row = &tkb[i & 1];
       cp_async_wait_all();
@@ -430,10 +438,12 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
   }
 
   long long q0 = 0;  // task number of the row's first chunk (same count as the producer's)
+  uint8_t mask_next = rows_mine > 0 ? a.mask[blockIdx.x] : 0;  // one row ahead
   for (long long i = 0; i < rows_mine; ++i) {
     const long long row = blockIdx.x + i * gridDim.x;
     const char* grow = lg + row * a.ld * static_cast<long long>(sizeof(St));
-    const bool trains = a.mask[row] != 0;
+    const bool trains = mask_next != 0;
+    if (i + 1 < rows_mine) mask_next = a.mask[row + gridDim.x];
     // pass B takes the last h chunks from the slots pass A left them in
     const int h = (kGrad && trains && n_chunks > 0) ? min(a.n_hold, n_chunks) : 0;
 
@@ -450,7 +460,7 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
       if (a.q) q = a.q[row];
       if (a.old) old = a.old[row];
       A = ws.a_row[row];
-      msk = a.mask[row];
+      msk = trains ? 1 : 0;
       yok = y >= 0;
       if (yok && y >= tail0) zy = In::load1(grow, y);
     }
