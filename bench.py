@@ -208,14 +208,37 @@ def profiled_traffic(rows_now: int, workload: str, vocab: int):
     return float(tb.group(1)) * rows_now / int(rows.group(1))
 
 
-def sweep_kernel_name(vocab: int, elem_size: int, grad: bool = True) -> str:
-    """The sweep kernel the library picks for these rows (16-byte aligned
-    rows of 192 KB and more in a fused call, of 148 KB and more in a
-    forward-only one, stream through one CTA each; shorter rows go to the
-    cluster kernel)."""
+def stream_ctas(row_bytes: int, grad: bool, topk: bool = False) -> int:
+    """Streaming CTAs per SM the library picks for 16-byte aligned rows of
+    row_bytes (0: the cluster kernel): one from 192 KB (fused) or 200 KB
+    (forward only), two or four on shorter rows, clusters in between and
+    below 20 KB."""
+    KB = 1024
+    if grad:
+        if row_bytes >= 192 * KB:
+            return 1
+        if 56 * KB < row_bytes <= 80 * KB:
+            return 2
+        if not topk and 20 * KB <= row_bytes <= 56 * KB:
+            return 4
+        return 0
+    if row_bytes >= 200 * KB:
+        return 1
+    if row_bytes > 112 * KB:
+        return 2
+    if row_bytes > 56 * KB:
+        return 2 if topk else 4
+    return 4 if (not topk and row_bytes >= 20 * KB) else 0
+
+
+def sweep_kernel_name(vocab: int, elem_size: int, grad: bool = True, topk: bool = False) -> str:
+    """The sweep kernel the library picks for these (16-byte aligned) rows."""
     kind = "fused fwd+bwd" if grad else "forward-only"
-    if vocab * elem_size >= (192 if grad else 148) * 1024:
+    per = stream_ctas(vocab * elem_size, grad, topk)
+    if per == 1:
         return f"k_stream ({kind} vocabulary sweep, one CTA per row)"
+    if per > 1:
+        return f"k_stream ({kind} vocabulary sweep, one CTA per row, {per} CTAs per SM)"
     return f"k_sweep ({kind} vocabulary sweep, clusters sharing a row)"
 
 
@@ -727,7 +750,7 @@ def run_ours(args, rank, world, local):
     also["split_fwd_bwd_tokens_per_s"] = R / (also["split_fwd_bwd_ms"] / 1e3)
 
     bpr = algorithmic_bytes_per_row(w, dl_dtype)  # before w is released for the e2e leg
-    kernel_name = sweep_kernel_name(V, w.logits.element_size())
+    kernel_name = sweep_kernel_name(V, w.logits.element_size(), topk=bool(args.opd_topk))
     w_params, n_groups = dict(w.params), w.n_groups
     step_bytes = bpr * R
     launch_bytes = step_bytes
@@ -735,7 +758,8 @@ def run_ours(args, rank, world, local):
         # GSPO's timed sweep is the forward-only one (k_seq and the gradient
         # sweep k_bwd follow it): it reads the logits and writes no dLogits
         launch_bytes = (bpr - V * torch.tensor([], dtype=dl_dtype).element_size()) * R
-        kernel_name = sweep_kernel_name(V, w.logits.element_size(), grad=False) + \
+        kernel_name = sweep_kernel_name(V, w.logits.element_size(), grad=False,
+                                        topk=bool(args.opd_topk)) + \
             ", GSPO's first pass (k_bwd reads the logits again for dLogits)"
     sweep_avg = statistics.fmean(sweep_ms)
     peaks, peak_kind = measured_peaks()

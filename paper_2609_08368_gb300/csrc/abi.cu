@@ -19,7 +19,7 @@ using namespace milesloss;
 
 namespace {
 std::mutex g_ov_mu;
-rl_launch_overrides g_ov = {-1, -1, -1, -1, -1, -1, -1, -1, -1, -1, -1};
+rl_launch_overrides g_ov = {-1, -1, -1, -1, -1, -1, -1, -1, -1, -1, -1, -1};
 }  // namespace
 
 namespace milesloss {
@@ -557,16 +557,16 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
   const rl_launch_overrides ov = current_overrides();
   const unsigned long long stall =
       ov.stall_first_wait_ns > 0 ? static_cast<unsigned long long>(ov.stall_first_wait_ns) : 0ull;
-  if (c.R > 0 && use_stream(c.V * static_cast<long long>(es), in_bulk, grad, ov)) {
+  if (c.R > 0 && use_stream(c.V * static_cast<long long>(es), in_bulk, grad, sc.topk > 0, ov)) {
     StreamPlan sp;
-    st = plan_stream(dev, sc.topk ? kTopKSmem : 0, c.V * static_cast<long long>(es), grad, ov,
-                     &sp);
+    st = plan_stream(dev, sc.topk ? kTopKSmem : 0, c.V * static_cast<long long>(es), grad,
+                     sc.topk > 0, ov, &sp);
     if (st != RL_OK) return st;
-    const void* fn = stream_kernel(c.dt, grad ? go->dt : c.dt, grad, sc.topk > 0);
+    const void* fn = stream_kernel(c.dt, grad ? go->dt : c.dt, grad, sc.topk > 0, sp.cw);
     st = set_smem(fn, dev, sp.smem);
     if (st != RL_OK) return st;
     int ctas = 0;
-    const int threads = stream_threads(sc.topk > 0);
+    const int threads = stream_threads(sc.topk > 0, sp.cw);
     st = resident_clusters(fn, dev, 1, sp.smem, threads, &ctas);
     if (st != RL_OK) return st;
     StreamArgs ta;
@@ -1029,7 +1029,7 @@ rl_status rl_launch_overrides_init(rl_launch_overrides* o) {
   if (!o) return RL_ERR_INVALID_ARG;
   o->sweep_kernel = o->cluster_size = o->cluster_stages = o->cluster_threads = -1;
   o->cluster_ctas_per_sm = o->stream_chunk_bytes = o->stream_slots = o->stream_hold = -1;
-  o->stream_split_first = o->stream_prefetch_bytes = -1;
+  o->stream_split_first = o->stream_prefetch_bytes = o->stream_ctas_per_sm = -1;
   o->stall_first_wait_ns = -1;
   return RL_OK;
 }
@@ -1045,6 +1045,8 @@ rl_status rl_set_launch_overrides(const rl_launch_overrides* o) {
         !in(o->stream_slots, 1, kMaxSlots) || !in(o->stream_hold, 0, kMaxSlots) ||
         !in(o->stream_split_first, 0, 1) || !in(o->stream_prefetch_bytes, 0, 1 << 20) ||
         (o->stream_prefetch_bytes > 0 && o->stream_prefetch_bytes % 16) ||
+        (o->stream_ctas_per_sm != -1 && o->stream_ctas_per_sm != 1 &&
+         o->stream_ctas_per_sm != 2 && o->stream_ctas_per_sm != 4) ||
         o->stall_first_wait_ns < -1 ||
         o->stall_first_wait_ns > 10000000000LL)
       return RL_ERR_INVALID_ARG;
@@ -1055,6 +1057,6 @@ rl_status rl_set_launch_overrides(const rl_launch_overrides* o) {
   return RL_OK;
 }
 
-int32_t rl_loss_abi_version(void) { return 130; }
+int32_t rl_loss_abi_version(void) { return 131; }
 
 }  // extern "C"

@@ -1,6 +1,9 @@
-// The vocabulary sweep for long rows, one CTA per row: the same per-row
-// results as k_sweep (log-softmax statistics, log-prob, entropy, per-token
-// objective, dLogits), with no exchange between CTAs.
+// The streaming vocabulary sweep, one CTA per row: the same per-row results
+// as k_sweep (log-softmax statistics, log-prob, entropy, per-token
+// objective, dLogits), with no exchange between CTAs. Long rows run one CTA
+// per SM with sixteen consumer warps; shorter rows two or four CTAs per SM
+// with eight or four consumer warps each, so that one CTA's per-row merge and
+// epilogue overlap the others' passes.
 //
 // A CTA is warp-specialised. One producer warp streams the row in chunks
 // (bulk async copies, non-multicast) into a ring of shared-memory slots,
@@ -14,7 +17,7 @@
 // ~one row per SM is live (~46 MB on the headline workload, against a
 // 126 MB L2), so the second read of a row is served by L2 and HBM sees each
 // logit about once (checked with the DRAM byte counters); the reverse order
-// re-reads the most recently copied chunk first. The sixteen consumer warps:
+// re-reads the most recently copied chunk first. The consumer warps:
 //   pass A  per chunk, each thread sums its vectors into (S, U) in packed
 //           f32x2 against a running reference that moves by whole powers of
 //           two (no per-element maximum), then releases the slot;
@@ -28,6 +31,7 @@
 //           stores; the sampled token's entry is rewritten during the next
 //           row's epilogue (after a barrier that orders every store before it).
 // Definitions: Sec. 3.4 (ratio), Sec. 2 / 9.1 (advantage), Sec. 2.4 (mask).
+#include <algorithm>
 #include <type_traits>
 
 #include "common.cuh"
@@ -37,13 +41,13 @@ namespace milesloss {
 
 namespace {
 
-constexpr int kCons = kStreamConsumers;   // consumer threads
-constexpr int kConsWarps = kCons / 32;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr float kLn2f = 0.69314718055994531f;
 
+// Named barrier 1 among the kCW consumer warps of the CTA.
+template <int kCW>
 __device__ __forceinline__ void cons_sync() {
-  asm volatile("bar.sync 1, %0;" ::"r"(kCons) : "memory");
+  asm volatile("bar.sync 1, %0;" ::"r"(kCW * 32) : "memory");
 }
 
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
@@ -83,21 +87,22 @@ __device__ __forceinline__ Tri warp_merge(Tri t) {
   return Tri{M, s, u};
 }
 
-// Merges the consumer warps' partial sums of a row: red[w] = (m, s, u) of
-// warp w, redm[w] = its m again (contiguous, so that every lane takes the
-// maximum with four broadcast reads instead of a shuffle tree). Lanes
-// 0..kConsWarps-1 rescale one warp's sums each and sum them in a fixed order;
-// lane 0 (every lane below kConsWarps) gets the row's sums.
+// Merges the kCW consumer warps' partial sums of a row: red[w] = (m, s, u)
+// of warp w, redm[w] = its m again (contiguous, so that every lane takes the
+// maximum with kCW / 4 broadcast reads instead of a shuffle tree). Lanes
+// 0..kCW-1 rescale one warp's sums each and sum them in a fixed order (xor
+// butterflies within each group of kCW lanes); lane 0 gets the row's sums.
+template <int kCW>
 __device__ __forceinline__ Tri block_merge(const float4* red, const float* redm, int lane) {
-  static_assert(kConsWarps == 16, "four float4 of references, four sum levels");
+  static_assert(kCW % 4 == 0 && kCW <= 32, "whole float4 of references, one warp of lanes");
   float M = -INFINITY;
 #pragma unroll
-  for (int w = 0; w < kConsWarps / 4; ++w) {
+  for (int w = 0; w < kCW / 4; ++w) {
     const float4 m4 = reinterpret_cast<const float4*>(redm)[w];
     M = fmaxf(M, fmaxf(fmaxf(m4.x, m4.y), fmaxf(m4.z, m4.w)));
   }
   float s = 0.0f, u = 0.0f;
-  if (lane < kConsWarps) {
+  if (lane < kCW) {
     const float4 v = red[lane];
     if (v.y > 0.0f) {
       const float d = v.x - M, f = ex2(d);
@@ -106,7 +111,7 @@ __device__ __forceinline__ Tri block_merge(const float4* red, const float* redm,
     }
   }
 #pragma unroll
-  for (int o = kConsWarps / 2; o > 0; o >>= 1) {
+  for (int o = kCW / 2; o > 0; o >>= 1) {
     s += __shfl_xor_sync(0xffffffffu, s, o);
     u += __shfl_xor_sync(0xffffffffu, u, o);
   }
@@ -167,7 +172,7 @@ struct Run {
 
 // dLogits of one chunk with vector stores. kMode 0: p ca with |ca| folded
 // into the exponent; 1: the same negated; 2: p (ca + cb z).
-template <class In, class Out, int kMode>
+template <class In, class Out, int kMode, int kCons>
 __device__ __forceinline__ void pass_b_chunk(const uint4* sv, int nv, char* dchunk, float2 k2,
                                              float2 off2, float2 ca2, float2 cb2) {
   constexpr int V8 = In::kVec;
@@ -190,8 +195,13 @@ __device__ __forceinline__ void pass_b_chunk(const uint4* sv, int nv, char* dchu
   }
 }
 
-template <class In, class Out, bool kGrad, bool kTopK>
-__global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_stream(const StreamArgs a) {
+// kCW consumer warps: 16 with one CTA per SM, 8 with two (each CTA then
+// has half of the SM's shared memory for its ring, and one CTA's per-row
+// merge and epilogue overlap the other's passes).
+template <class In, class Out, bool kGrad, bool kTopK, int kCW>
+__global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stream(const StreamArgs a) {
+  constexpr int kCons = kCW * 32;  // consumer threads
+  constexpr int kConsWarps = kCW;
   using St = typename In::storage;
   constexpr int V8 = In::kVec;
   constexpr int P = V8 / 2;
@@ -537,10 +547,10 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
       red[warp] = make_float4(t.m, t.s, t.u, 0.0f);
       redm[warp] = t.m;
     }
-    cons_sync();
+    cons_sync<kCW>();
     if (tid == 0 && fix_ptr) Out::store1(fix_ptr, 0, fix_val);  // previous row's y entry
     fix_ptr = nullptr;
-    if (warp == 0) t = block_merge(red, redm, lane);
+    if (warp == 0) t = block_merge<kCW>(red, redm, lane);
     // top-K OPD signal (Sec. 5.2), a fixed per-token reward: the top-K warp's
     // part of this row and the row's lse (warp 0)
     float opd = 0.0f;
@@ -599,7 +609,7 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
         bci[0] = make_int4(zero, fold, (fold && ca < 0.0f) ? 1 : 0, 0);
       }
     }
-    cons_sync();
+    cons_sync<kCW>();
     if (tid == 0 && !a.part_rows) {
       if (!yok) atomicOr(err, kErrTarget);
       if (tk_bad) atomicOr(err, kErrTopK);
@@ -664,9 +674,9 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
         }
         const uint4* sv = slot(qq);
         if (vec_out) {
-          if (!ci.y) pass_b_chunk<In, Out, 2>(sv, nv, dchunk, k2, off2, ca2, cb2);
-          else if (ci.z) pass_b_chunk<In, Out, 1>(sv, nv, dchunk, k2, off2, ca2, cb2);
-          else pass_b_chunk<In, Out, 0>(sv, nv, dchunk, k2, off2, ca2, cb2);
+          if (!ci.y) pass_b_chunk<In, Out, 2, kCons>(sv, nv, dchunk, k2, off2, ca2, cb2);
+          else if (ci.z) pass_b_chunk<In, Out, 1, kCons>(sv, nv, dchunk, k2, off2, ca2, cb2);
+          else pass_b_chunk<In, Out, 0, kCons>(sv, nv, dchunk, k2, off2, ca2, cb2);
         } else {
           for (int v = tid; v < nv; v += kCons) {
             float2 f[P];
@@ -695,81 +705,140 @@ __global__ void __launch_bounds__(kStreamConsumers + (kTopK ? 64 : 32), 1) k_str
     }
     q0 += (kGrad && trains) ? 2 * n_chunks - h : n_chunks;
   }
-  cons_sync();
+  cons_sync<kCW>();
   if (tid == 0 && fix_ptr) Out::store1(fix_ptr, 0, fix_val);
 }
 
 template <class In, class Out, bool kGrad>
-const void* fn(bool topk) {
-  return topk ? reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, true>)
-              : reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, false>);
+const void* fn(bool topk, int cw) {
+  if (cw == 4)
+    return topk ? reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, true, 4>)
+                : reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, false, 4>);
+  if (cw == 8)
+    return topk ? reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, true, 8>)
+                : reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, false, 8>);
+  return topk ? reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, true, 16>)
+              : reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, false, 16>);
 }
 
 }  // namespace
 
-// Rows with 16-byte aligned starts go to the streaming kernel (one CTA per
-// row, second read served by L2 or shared memory) from 192 KB in a fused
-// call and from 148 KB in a forward-only one; shorter or unaligned rows to
-// the cluster kernel, which keeps them on chip. Measured on GB300 (bf16,
-// fractions of the copy peak): fused, rows of 200-310 KB streamed
-// 0.966-0.984 against 0.939-0.959 in clusters, rows of 128-160 KB in
-// clusters 0.94-0.96 against 0.88-0.91 streamed; forward only, rows of
-// 148-310 KB streamed 0.92-1.09 against 0.78-0.88, rows of 96-144 KB in
-// clusters 0.87-0.94 against 0.79-0.92. The forward plan's clusters of two
-// stop fitting a third of the SM's shared memory past 148 KB rows, and
-// clusters of four ran 0.78-0.81 there. The sweep_kernel override forces
-// either.
-constexpr long long kStreamMinRowBytes = 192 * 1024;     // fused calls
-constexpr long long kStreamMinRowBytesFwd = 148 * 1024;  // forward-only calls
-
-bool use_stream(long long row_bytes, bool in_bulk, bool grad, const rl_launch_overrides& ov) {
-  if (ov.sweep_kernel == 0) return false;
-  if (ov.sweep_kernel == 1) return in_bulk;
-  return in_bulk && row_bytes >= (grad ? kStreamMinRowBytes : kStreamMinRowBytesFwd);
+// Which kernel sweeps rows of row_bytes, and with how many streaming CTAs per
+// SM: 0 = the cluster kernel, 1 = one streaming CTA per SM (sixteen consumer
+// warps, the whole shared memory for its ring), 2 or 4 = that many CTAs per SM
+// (eight or four consumer warps, a half or a quarter of the shared memory),
+// so that one CTA's per-row merge and epilogue overlap the other CTAs'
+// passes. Rows must start 16-byte aligned to stream (else the cluster
+// kernel). Measured on GB300 (fractions of the copy peak, A/B on one box,
+// bf16 and fp32 rows):
+//   fused: rows of 192-310 KB one CTA 0.966-0.984 against 0.939-0.959 in
+//   clusters; 56-80 KB rows two CTAs 0.956-1.00 against 0.91-0.94; 20-56 KB
+//   rows four CTAs 0.93-1.00 against 0.90-0.94 (48 KB fp32 rows: equal);
+//   80-192 KB rows in clusters (0.93-0.97; two CTAs ran from 2 % ahead to 1 %
+//   behind on 96 KB rows, depending on the box); 16 KB rows in clusters (fp32
+//   0.91 against 0.79 with four CTAs). With top-K OPD, four CTAs per SM ran 6
+//   % behind the clusters on 32 KB rows; two ran 3-4 % ahead on 64 KB rows.
+//   forward only: 200-310 KB rows one CTA (224 / 288 / 302 KB: 1.13 / 1.10
+//   / 1.10 against 1.10 / 1.07 / 1.06 with two); 112-200 KB rows two CTAs
+//   (151 KB: 1.05 against 0.94 with one, 192 KB: 1.08 against 1.06; a
+//   read-only stream can pass the copy peak); 20-112 KB
+//   rows four CTAs 0.84-1.06 against 0.71-0.96 in clusters (64 KB fp32 rows:
+//   1.07 against 1.08).
+// The sweep_kernel override forces either kernel, stream_ctas_per_sm the
+// CTAs per SM.
+int stream_ctas(long long row_bytes, bool grad, bool topk) {
+  constexpr long long KB = 1024;
+  if (grad) {
+    if (row_bytes >= 192 * KB) return 1;
+    if (row_bytes > 56 * KB && row_bytes <= 80 * KB) return 2;
+    if (!topk && row_bytes >= 20 * KB && row_bytes <= 56 * KB) return 4;
+    return 0;
+  }
+  if (row_bytes >= 200 * KB) return 1;
+  if (row_bytes > 112 * KB) return 2;
+  if (row_bytes > 56 * KB) return topk ? 2 : 4;
+  if (!topk && row_bytes >= 20 * KB) return 4;
+  return 0;
 }
 
-// The ring (one CTA per SM), measured on GB300 among 44-112 KB chunks and
-// 0-3 kept chunks (bf16, fused): rows of 240 KB and more run best with three
-// 74 KB slots, the ragged remainder as the first chunk and the last two
-// chunks kept for pass B (0.966-0.984 of the copy peak, against 0.959-0.973
-// with two 112 KB slots); shorter rows with two 112 KB slots and the last
-// chunk kept (200 KB rows: 0.972-0.979, against 0.944 with 74 KB slots). A
-// forward-only call has no pass B: two 112 KB slots. The stream_* overrides
-// force a chunk size, slot count, kept chunks and split.
+bool use_stream(long long row_bytes, bool in_bulk, bool grad, bool topk,
+                const rl_launch_overrides& ov) {
+  if (ov.sweep_kernel == 0) return false;
+  if (ov.sweep_kernel == 1) return in_bulk;
+  return in_bulk && stream_ctas(row_bytes, grad, topk) > 0;
+}
+
+// The ring. One CTA per SM, measured on GB300 among 44-112 KB chunks and 0-3
+// kept chunks (bf16, fused): rows of 240 KB and more run best with three 74
+// KB slots, the ragged remainder as the first chunk and the last two chunks
+// kept for pass B (0.966-0.984 of the copy peak, against 0.959-0.973 with two
+// 112 KB slots); shorter rows with two 112 KB slots and the last chunk kept
+// (200 KB rows: 0.972-0.979, against 0.944 with 74 KB slots); a forward-only
+// call has no pass B: two 112 KB slots. Several CTAs per SM, measured among
+// 8-36 KB chunks and 1-3 kept chunks: two CTAs with three 36 KB slots (every
+// chunk kept, up to three); four CTAs with the whole row in one slot up to 24
+// KB rows, else 16 KB slots up to 44 KB rows, 12 KB slots up to 56 KB rows
+// and 18 KB slots past that (forward only), the last chunk kept; chunks of 12
+// KB or less with two CTAs, or 8 KB with four, ran 10-45 % slower. The stream_*
+// overrides force a chunk size, slot count, kept chunks, split and CTAs per
+// SM.
 constexpr long long kLongRowBytes = 240 * 1024;
 
-rl_status plan_stream(int dev, int extra, long long row_bytes, bool grad,
+rl_status plan_stream(int dev, int extra, long long row_bytes, bool grad, bool topk,
                       const rl_launch_overrides& ov, StreamPlan* out) {
-  int optin = 0;
-  if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+  int optin = 0, per_sm = 0, reserved = 0;
+  if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) !=
+          cudaSuccess ||
+      cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev) !=
+          cudaSuccess)
     return RL_ERR_CUDA;
+  const int per = ov.stream_ctas_per_sm > 0 ? ov.stream_ctas_per_sm
+                                            : std::max(1, stream_ctas(row_bytes, grad, topk));
+  if (per != 1 && per != 2 && per != 4) return RL_ERR_UNSUPPORTED;
   const bool lng = grad && row_bytes >= kLongRowBytes;
-  const int chunk = ov.stream_chunk_bytes > 0 ? ov.stream_chunk_bytes : (lng ? 75776 : 114688);
+  const int budget = per > 1 ? std::min(optin, per_sm / per - reserved) : optin;
+  int chunk_d = lng ? 75776 : 114688, hold_d = lng ? 2 : 1, split_d = lng ? 1 : 0;
+  if (per == 2) {
+    chunk_d = 36864;
+    hold_d = 3;
+    split_d = 1;
+  } else if (per == 4) {
+    // (rows up to 56 KB take the same chunks in fused and forward-only
+    // calls, so that both sum a row in the same order: the same bits)
+    const long long whole = (row_bytes + 127) / 128 * 128;
+    chunk_d = whole <= 24576 ? static_cast<int>(std::max(1024LL, whole))
+                             : (row_bytes <= 44 * 1024 ? 16384 : (row_bytes <= 56 * 1024 ? 12288 : 18432));
+    hold_d = 1;
+    split_d = 1;
+  }
+  const int chunk = ov.stream_chunk_bytes > 0 ? ov.stream_chunk_bytes : chunk_d;
   if (chunk < 1024 || chunk > 131072 || chunk % 128) return RL_ERR_UNSUPPORTED;
-  int slots = (optin - kSweepSmemExtra - extra) / chunk;
+  int slots = (budget - kSweepSmemExtra - extra) / chunk;
   if (slots > kMaxSlots) slots = kMaxSlots;
   if (ov.stream_slots > 0) {
     if (ov.stream_slots > slots) return RL_ERR_UNSUPPORTED;
     slots = ov.stream_slots;
   }
   if (slots < 1) return RL_ERR_UNSUPPORTED;
-  const int hold = ov.stream_hold >= 0 ? ov.stream_hold : (lng ? 2 : 1);
+  const int hold = ov.stream_hold >= 0 ? ov.stream_hold : std::min(hold_d, slots);
   if (hold > slots) return RL_ERR_UNSUPPORTED;
   out->chunk = chunk;
   out->slots = slots;
   out->hold = hold;
-  out->split_first = ov.stream_split_first >= 0 ? ov.stream_split_first : (lng ? 1 : 0);
+  out->split_first = ov.stream_split_first >= 0 ? ov.stream_split_first : split_d;
   out->prefetch = ov.stream_prefetch_bytes >= 0 ? ov.stream_prefetch_bytes : 0;
   out->smem = slots * chunk + kSweepSmemExtra + extra;
+  out->cw = 16 / per;
   return RL_OK;
 }
 
-const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad, bool topk) {
+const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad, bool topk, int cw) {
   if (!grad)
-    return in == RL_BF16 ? fn<InBf16, OutBf16, false>(topk) : fn<InF32, OutF32, false>(topk);
+    return in == RL_BF16 ? fn<InBf16, OutBf16, false>(topk, cw) : fn<InF32, OutF32, false>(topk, cw);
   if (in == RL_BF16)
-    return out == RL_BF16 ? fn<InBf16, OutBf16, true>(topk) : fn<InBf16, OutF32, true>(topk);
-  return out == RL_BF16 ? fn<InF32, OutBf16, true>(topk) : fn<InF32, OutF32, true>(topk);
+    return out == RL_BF16 ? fn<InBf16, OutBf16, true>(topk, cw) : fn<InBf16, OutF32, true>(topk, cw);
+  return out == RL_BF16 ? fn<InF32, OutBf16, true>(topk, cw) : fn<InF32, OutF32, true>(topk, cw);
 }
 
 }  // namespace milesloss

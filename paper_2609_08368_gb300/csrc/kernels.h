@@ -13,10 +13,9 @@ constexpr uint32_t kBulkChunk = 16384;    // bytes per cp.async.bulk
 constexpr int kSweepSmemExtra = 1024;     // mbarriers + exchange + reduction scratch
 constexpr int kAdvThreads = 1024;
 constexpr int kBwdThreads = 256;
-constexpr int kStreamConsumers = 512;     // consumer threads of k_stream (+ one producer warp)
-// k_stream's block: the consumers, the producer warp and, with top-K OPD, the
-// top-K warp
-constexpr int stream_threads(bool topk) { return kStreamConsumers + (topk ? 64 : 32); }
+// k_stream's block: cw consumer warps (16 with one CTA per SM, 8 with two),
+// the producer warp and, with top-K OPD, the top-K warp
+constexpr int stream_threads(bool topk, int cw) { return cw * 32 + (topk ? 64 : 32); }
 constexpr int kMaxSlots = 16;             // ring slots of k_stream
 constexpr int kSeqThreads = 256;
 constexpr int kAdvSmemBytes = 48 * 1024;  // on-chip trajectory tables when they fit
@@ -190,7 +189,7 @@ constexpr int kBwdTile = kBwdThreads * 8 * 4;  // elements of one row per backwa
 // carry none of its code)
 const void* sweep_kernel(rl_dtype in, rl_dtype out, bool grad, int threads, bool topk);
 const void* sweep_kernel_topk(rl_dtype in, rl_dtype out, bool grad, int threads);
-const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad, bool topk);
+const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad, bool topk, int cw);
 
 // The process-wide launch-plan overrides set by rl_set_launch_overrides (a
 // copy; every field -1 when none are set).
@@ -202,12 +201,14 @@ rl_status status_of_bits(uint32_t bits);
 // whether rows of row_bytes go to it, and its ring of shared-memory slots.
 struct StreamPlan {
   int chunk, slots, hold, split_first, prefetch, smem;
+  int cw;  // consumer warps per CTA: 16, 8 or 4 (one, two or four CTAs per SM)
 };
-bool use_stream(long long row_bytes, bool in_bulk, bool grad, const rl_launch_overrides& ov);
+bool use_stream(long long row_bytes, bool in_bulk, bool grad, bool topk,
+                const rl_launch_overrides& ov);
 // extra: shared memory beyond the ring and the fixed scratch (kTopKSmem with
 // top-K OPD on, else 0); the ring's shape depends on the row length and on
 // whether the call writes dLogits
-rl_status plan_stream(int dev, int extra, long long row_bytes, bool grad,
+rl_status plan_stream(int dev, int extra, long long row_bytes, bool grad, bool topk,
                       const rl_launch_overrides& ov, StreamPlan* out);
 const void* bwd_kernel(rl_dtype in, rl_dtype out);
 const void* adv_kernel();

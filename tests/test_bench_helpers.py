@@ -23,17 +23,33 @@ def test_launches_per_call():
     assert bench.launches_per_call({"estimator": "reinforcepp"}, 1) == 3
 
 
-def test_sweep_kernel_name_follows_the_fused_threshold():
-    assert bench.sweep_kernel_name(154880, 2).startswith("k_stream")
-    assert bench.sweep_kernel_name(131072, 2).startswith("k_stream")
-    assert bench.sweep_kernel_name(98304, 2).startswith("k_stream")
-    assert bench.sweep_kernel_name(98303, 2).startswith("k_sweep")
-    assert bench.sweep_kernel_name(32768, 4).startswith("k_sweep")
-    assert bench.sweep_kernel_name(49152, 4).startswith("k_stream")
-    # forward-only calls stream from 148 KB
-    assert bench.sweep_kernel_name(75776, 2, grad=False).startswith("k_stream")
-    assert bench.sweep_kernel_name(81920, 2).startswith("k_sweep")
-    assert bench.sweep_kernel_name(75775, 2, grad=False).startswith("k_sweep")
+def test_sweep_kernel_name_follows_the_plan_tiers():
+    one, clusters = "one CTA per row)", "clusters sharing a row)"
+    assert bench.sweep_kernel_name(154880, 2).endswith(one)
+    assert bench.sweep_kernel_name(98304, 2).endswith(one)
+    assert bench.sweep_kernel_name(98303, 2).endswith(clusters)      # 80-192 KB: clusters
+    assert bench.sweep_kernel_name(40964, 2).endswith(clusters)
+    assert bench.sweep_kernel_name(32768, 4).endswith(clusters)      # fp32, 128 KB
+    assert bench.sweep_kernel_name(49152, 4).endswith(one)
+    assert "2 CTAs per SM" in bench.sweep_kernel_name(32768, 2)      # 64 KB
+    assert "2 CTAs per SM" in bench.sweep_kernel_name(40960, 2)      # 80 KB
+    assert "4 CTAs per SM" in bench.sweep_kernel_name(28672, 2)      # 56 KB
+    assert "4 CTAs per SM" in bench.sweep_kernel_name(16384, 2)      # 32 KB
+    assert "4 CTAs per SM" in bench.sweep_kernel_name(10240, 2)      # 20 KB
+    assert bench.sweep_kernel_name(10232, 2).endswith(clusters)      # below 20 KB
+    assert bench.sweep_kernel_name(4096, 2).endswith(clusters)       # the tiny workload
+    # with top-K OPD, no four-CTA plans
+    assert bench.sweep_kernel_name(16384, 2, topk=True).endswith(clusters)
+    assert "2 CTAs per SM" in bench.sweep_kernel_name(32768, 2, topk=True)
+    # forward-only calls: one CTA from 200 KB, two from 112 KB, four from 20 KB
+    assert bench.sweep_kernel_name(154880, 2, grad=False).endswith(one)
+    assert bench.sweep_kernel_name(102400, 2, grad=False).endswith(one)
+    assert "2 CTAs per SM" in bench.sweep_kernel_name(102392, 2, grad=False)
+    assert "2 CTAs per SM" in bench.sweep_kernel_name(77440, 2, grad=False)  # glm TP 2 shards
+    assert "2 CTAs per SM" in bench.sweep_kernel_name(57348, 2, grad=False)
+    assert "4 CTAs per SM" in bench.sweep_kernel_name(57344, 2, grad=False)
+    assert "2 CTAs per SM" in bench.sweep_kernel_name(32768, 2, grad=False, topk=True)
+    assert bench.sweep_kernel_name(8192, 2, grad=False).endswith(clusters)
 
 
 def test_profiled_traffic_only_for_its_workload_and_sources():

@@ -94,6 +94,33 @@ def test_stream_ring_shapes(ov, chunk, slots, hold, split):
     _full_check(wl.make(rec, DEV))
 
 
+@pytest.mark.parametrize("per_sm,chunk,slots,hold,split", [
+    (2, -1, -1, -1, -1), (2, 36864, 3, 2, 1), (2, 36864, 3, 3, 0), (2, 16384, 6, 2, 1),
+    (2, 4096, 2, 0, 0), (2, 1024, 1, 1, 1), (4, -1, -1, -1, -1), (4, 12288, 4, 2, 1),
+    (4, 9216, 5, 5, 0), (4, 2048, 3, 0, 1)])
+def test_stream_several_ctas_per_sm(ov, per_sm, chunk, slots, hold, split):
+    """The streaming kernel with two or four CTAs per SM (eight or four
+    consumer warps each, a half or a quarter of the SM's shared memory for
+    each ring), with its default ring and forced ones, on ragged bf16 and
+    fp32 rows, fused and split, and with top-K OPD and the entropy bonus."""
+    ov(sweep_kernel="stream")
+    ov(stream_ctas_per_sm=per_sm)
+    for f, v in (("stream_chunk_bytes", chunk), ("stream_slots", slots), ("stream_hold", hold),
+                 ("stream_split_first", split)):
+        if v >= 0:
+            ov(**{f: v})
+    rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=24, vocab=45003,
+                    rho_noise=0.3)
+    _full_check(wl.make(rec, DEV))
+    _full_check(wl.make(rec, DEV), mode="split")
+    rec = wl.shrink(wl.RECIPES["fp32"], n_prompts=1, group_size=4, traj_len=16, vocab=20001,
+                    rho_noise=0.3)
+    _full_check(wl.make(rec, DEV))
+    w = wl.make(wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=24,
+                          vocab=40960, topk=16), DEV)
+    _full_check(w, params=dict(w.params, entropy_coef=0.01, opd_topk=16, opd_coef=0.5))
+
+
 @pytest.mark.parametrize("name", ["tiny", "fp32", "glm_noisy"])
 def test_parity_split_fwd_then_bwd(name):
     _full_check(wl.make(SHRUNK[name], DEV), mode="split")
