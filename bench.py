@@ -59,6 +59,9 @@ def parse_args():
                     help="fewer groups (a smaller case of the same workload, for profiling)")
     ap.add_argument("--traj-len", type=int, default=None,
                     help="shorter trajectories (a smaller case, for profiling)")
+    ap.add_argument("--vocab", type=int, default=None,
+                    help="another vocabulary size (other row lengths, for profiling the "
+                         "launch plans)")
     ap.add_argument("--estimator", default=None,
                     choices=["grpo", "reinforcepp", "reinforcepp_baseline", "gspo"],
                     help="another advantage estimator than the workload's (for profiling "
@@ -671,7 +674,7 @@ def run_ours(args, rank, world, local):
     ml.load()
     dev = torch.device("cuda", local)
     rec = wl.RECIPES[args.workload]
-    rec = wl.shrink(rec, n_prompts=args.n_prompts, traj_len=args.traj_len,
+    rec = wl.shrink(rec, n_prompts=args.n_prompts, traj_len=args.traj_len, vocab=args.vocab,
                     seed=rec.seed + 1000 * rank)  # each replica has its own batch
     if args.estimator:
         rec = dataclasses.replace(rec, params=dict(rec.params, estimator=args.estimator))
@@ -824,7 +827,8 @@ def run_ours(args, rank, world, local):
                    "rows": R, "vocab": V, "parallelism": f"replicas x{world}",
                    **({"estimator": args.estimator} if args.estimator else {}),
                    **({"opd_topk": args.opd_topk} if args.opd_topk else {}),
-                   "l2": "inputs larger than L2 (20+ GB per step), no flush"},
+                   "l2": f"inputs larger than L2 ({step_bytes / 1e9:.1f} GB per step), "
+                         "no flush"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "kernel": kernel_name,
