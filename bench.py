@@ -185,10 +185,16 @@ def measured_peaks():
 
 
 def sweep_source_hash() -> str:
+    """Hash of the sweep kernel's code and launch plan, comments and
+    whitespace left out (a comment edit does not change what was captured;
+    none of these files has a comment marker inside a string literal)."""
     h = hashlib.sha256()
     for name in SWEEP_SOURCES:
-        with open(os.path.join(ROOT, "paper_2609_08368_gb300", "csrc", name), "rb") as f:
-            h.update(f.read())
+        with open(os.path.join(ROOT, "paper_2609_08368_gb300", "csrc", name)) as f:
+            text = f.read()
+        text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", " ", text)
+        h.update(" ".join(text.split()).encode())
     return h.hexdigest()[:16]
 
 

@@ -518,8 +518,9 @@ const char* rl_status_string(rl_status status);
  *  stream_prefetch_bytes bytes of the next row the streaming kernel asks L2
  *                       to fetch once a row's first-pass copies are issued
  *                       (0 = none; a multiple of 16)
- *  stream_ctas_per_sm   streaming kernel: 1 (sixteen consumer warps per
- *                       CTA) or 2 (eight each, half the shared memory)
+ *  stream_ctas_per_sm   streaming kernel: CTAs per SM, 1 (sixteen consumer
+ *                       warps per CTA), 2 (eight each, half of the shared
+ *                       memory each) or 4 (four each, a quarter)
  *  stall_first_wait_ns  TEST HOOK, > 0: in each CTA of the vocabulary sweep,
  *                       the first wait for logits waits instead on a barrier
  *                       that nothing completes, bounded by this many

@@ -195,9 +195,9 @@ __device__ __forceinline__ void pass_b_chunk(const uint4* sv, int nv, char* dchu
   }
 }
 
-// kCW consumer warps: 16 with one CTA per SM, 8 with two (each CTA then
-// has half of the SM's shared memory for its ring, and one CTA's per-row
-// merge and epilogue overlap the other's passes).
+// kCW consumer warps: 16 with one CTA per SM, 8 with two, 4 with four (each
+// CTA then has a half or a quarter of the SM's shared memory for its ring,
+// and one CTA's per-row merge and epilogue overlap the others' passes).
 template <class In, class Out, bool kGrad, bool kTopK, int kCW>
 __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stream(const StreamArgs a) {
   constexpr int kCons = kCW * 32;  // consumer threads

@@ -13,7 +13,8 @@ constexpr uint32_t kBulkChunk = 16384;    // bytes per cp.async.bulk
 constexpr int kSweepSmemExtra = 1024;     // mbarriers + exchange + reduction scratch
 constexpr int kAdvThreads = 1024;
 constexpr int kBwdThreads = 256;
-// k_stream's block: cw consumer warps (16 with one CTA per SM, 8 with two),
+// k_stream's block: cw consumer warps (16 with one CTA per SM, 8 with two, 4
+// with four),
 // the producer warp and, with top-K OPD, the top-K warp
 constexpr int stream_threads(bool topk, int cw) { return cw * 32 + (topk ? 64 : 32); }
 constexpr int kMaxSlots = 16;             // ring slots of k_stream
