@@ -66,6 +66,9 @@ def parse_args():
                     choices=["grpo", "reinforcepp", "reinforcepp_baseline", "gspo"],
                     help="another advantage estimator than the workload's (for profiling "
                          "the kernels of that path)")
+    ap.add_argument("--sweep-kernel", choices=["cluster", "stream"], default=None,
+                    help="force the vocabulary-sweep kernel (a launch-plan override, for "
+                         "profiling the kernel the library would not pick)")
     ap.add_argument("--opd-topk", type=int, default=0,
                     help="top-K on-policy distillation with K candidates per row, coefficient "
                          "0.5 (for profiling the sweeps' top-K instantiations)")
@@ -217,7 +220,7 @@ def profiled_traffic(rows_now: int, workload: str, vocab: int):
     return float(tb.group(1)) * rows_now / int(rows.group(1))
 
 
-def stream_ctas(row_bytes: int, grad: bool, topk: bool = False) -> int:
+def stream_ctas(row_bytes: int, grad: bool, topk: bool = False, elem_size: int = 2) -> int:
     """Streaming CTAs per SM the library picks for 16-byte aligned rows of
     row_bytes (0: the cluster kernel): one from 192 KB (fused) or 200 KB
     (forward only), two or four on shorter rows, clusters in between and
@@ -226,6 +229,8 @@ def stream_ctas(row_bytes: int, grad: bool, topk: bool = False) -> int:
     if grad:
         if row_bytes >= 192 * KB:
             return 1
+        if elem_size == 4 and not topk and 120 * KB < row_bytes <= 136 * KB:
+            return 2  # fp32 rows of 120-136 KB
         if 56 * KB < row_bytes <= 80 * KB:
             return 2
         if not topk and 20 * KB <= row_bytes <= 56 * KB:
@@ -240,10 +245,16 @@ def stream_ctas(row_bytes: int, grad: bool, topk: bool = False) -> int:
     return 4 if (not topk and row_bytes >= 20 * KB) else 0
 
 
-def sweep_kernel_name(vocab: int, elem_size: int, grad: bool = True, topk: bool = False) -> str:
-    """The sweep kernel the library picks for these (16-byte aligned) rows."""
+def sweep_kernel_name(vocab: int, elem_size: int, grad: bool = True, topk: bool = False,
+                      forced: str | None = None) -> str:
+    """The sweep kernel the library picks for these (16-byte aligned) rows,
+    or the one the sweep_kernel override forces."""
     kind = "fused fwd+bwd" if grad else "forward-only"
-    per = stream_ctas(vocab * elem_size, grad, topk)
+    per = stream_ctas(vocab * elem_size, grad, topk, elem_size)
+    if forced == "cluster":
+        per = 0
+    elif forced == "stream":
+        per = max(per, 1)
     if per == 1:
         return f"k_stream ({kind} vocabulary sweep, one CTA per row)"
     if per > 1:
@@ -678,6 +689,8 @@ def run_ours(args, rank, world, local):
     from paper_2609_08368_gb300 import api, milesloss as ml, workloads as wl
 
     ml.load()
+    if args.sweep_kernel:
+        ml.set_launch_overrides(sweep_kernel=args.sweep_kernel)
     dev = torch.device("cuda", local)
     rec = wl.RECIPES[args.workload]
     rec = wl.shrink(rec, n_prompts=args.n_prompts, traj_len=args.traj_len, vocab=args.vocab,
@@ -759,7 +772,8 @@ def run_ours(args, rank, world, local):
     also["split_fwd_bwd_tokens_per_s"] = R / (also["split_fwd_bwd_ms"] / 1e3)
 
     bpr = algorithmic_bytes_per_row(w, dl_dtype)  # before w is released for the e2e leg
-    kernel_name = sweep_kernel_name(V, w.logits.element_size(), topk=bool(args.opd_topk))
+    kernel_name = sweep_kernel_name(V, w.logits.element_size(), topk=bool(args.opd_topk),
+                                    forced=args.sweep_kernel)
     w_params, n_groups = dict(w.params), w.n_groups
     step_bytes = bpr * R
     launch_bytes = step_bytes
@@ -768,7 +782,7 @@ def run_ours(args, rank, world, local):
         # sweep k_bwd follow it): it reads the logits and writes no dLogits
         launch_bytes = (bpr - V * torch.tensor([], dtype=dl_dtype).element_size()) * R
         kernel_name = sweep_kernel_name(V, w.logits.element_size(), grad=False,
-                                        topk=bool(args.opd_topk)) + \
+                                        topk=bool(args.opd_topk), forced=args.sweep_kernel) + \
             ", GSPO's first pass (k_bwd reads the logits again for dLogits)"
     sweep_avg = statistics.fmean(sweep_ms)
     peaks, peak_kind = measured_peaks()
@@ -821,7 +835,8 @@ def run_ours(args, rank, world, local):
 
     # the committed capture is of the default path (GRPO-style fused sweep,
     # no top-K): it does not describe the others
-    traffic = None if (args.estimator or args.opd_topk) else profiled_traffic(R, args.workload, V)
+    traffic = None if (args.estimator or args.opd_topk or args.sweep_kernel) \
+        else profiled_traffic(R, args.workload, V)
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True,
@@ -833,6 +848,7 @@ def run_ours(args, rank, world, local):
                    "rows": R, "vocab": V, "parallelism": f"replicas x{world}",
                    **({"estimator": args.estimator} if args.estimator else {}),
                    **({"opd_topk": args.opd_topk} if args.opd_topk else {}),
+                   **({"sweep_kernel": args.sweep_kernel} if args.sweep_kernel else {}),
                    "l2": f"inputs larger than L2 ({step_bytes / 1e9:.1f} GB per step), "
                          "no flush"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",

@@ -557,10 +557,11 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
   const rl_launch_overrides ov = current_overrides();
   const unsigned long long stall =
       ov.stall_first_wait_ns > 0 ? static_cast<unsigned long long>(ov.stall_first_wait_ns) : 0ull;
-  if (c.R > 0 && use_stream(c.V * static_cast<long long>(es), in_bulk, grad, sc.topk > 0, ov)) {
+  if (c.R > 0 &&
+      use_stream(c.V * static_cast<long long>(es), static_cast<int>(es), in_bulk, grad, sc.topk > 0, ov)) {
     StreamPlan sp;
-    st = plan_stream(dev, sc.topk ? kTopKSmem : 0, c.V * static_cast<long long>(es), grad,
-                     sc.topk > 0, ov, &sp);
+    st = plan_stream(dev, sc.topk ? kTopKSmem : 0, c.V * static_cast<long long>(es),
+                     static_cast<int>(es), grad, sc.topk > 0, ov, &sp);
     if (st != RL_OK) return st;
     const void* fn = stream_kernel(c.dt, grad ? go->dt : c.dt, grad, sc.topk > 0, sp.cw);
     st = set_smem(fn, dev, sp.smem);

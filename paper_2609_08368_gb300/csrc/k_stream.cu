@@ -746,10 +746,19 @@ const void* fn(bool topk, int cw) {
 //   1.07 against 1.08).
 // The sweep_kernel override forces either kernel, stream_ctas_per_sm the
 // CTAs per SM.
-int stream_ctas(long long row_bytes, bool grad, bool topk) {
+// fp32 rows of 120-136 KB (the fp32 workload's 32,768 columns), fused: two
+// CTAs per SM with 18 KB chunks, 0.976 / 0.979 / 0.983 against 0.970 / 0.960
+// / 0.969 in clusters on three boxes (bf16 rows of that length with those
+// chunks: 0.87; with 24-36 KB chunks equal to the clusters).
+bool fp32_mid_row(long long row_bytes, int es, bool grad, bool topk) {
+  return grad && !topk && es == 4 && row_bytes > 120 * 1024 && row_bytes <= 136 * 1024;
+}
+
+int stream_ctas(long long row_bytes, int es, bool grad, bool topk) {
   constexpr long long KB = 1024;
   if (grad) {
     if (row_bytes >= 192 * KB) return 1;
+    if (fp32_mid_row(row_bytes, es, grad, topk)) return 2;
     if (row_bytes > 56 * KB && row_bytes <= 80 * KB) return 2;
     if (!topk && row_bytes >= 20 * KB && row_bytes <= 56 * KB) return 4;
     return 0;
@@ -761,11 +770,11 @@ int stream_ctas(long long row_bytes, bool grad, bool topk) {
   return 0;
 }
 
-bool use_stream(long long row_bytes, bool in_bulk, bool grad, bool topk,
+bool use_stream(long long row_bytes, int es, bool in_bulk, bool grad, bool topk,
                 const rl_launch_overrides& ov) {
   if (ov.sweep_kernel == 0) return false;
   if (ov.sweep_kernel == 1) return in_bulk;
-  return in_bulk && stream_ctas(row_bytes, grad, topk) > 0;
+  return in_bulk && stream_ctas(row_bytes, es, grad, topk) > 0;
 }
 
 // The ring. One CTA per SM, measured on GB300 among 44-112 KB chunks and 0-3
@@ -776,7 +785,8 @@ bool use_stream(long long row_bytes, bool in_bulk, bool grad, bool topk,
 // (200 KB rows: 0.972-0.979, against 0.944 with 74 KB slots); a forward-only
 // call has no pass B: two 112 KB slots. Several CTAs per SM, measured among
 // 8-36 KB chunks and 1-3 kept chunks: two CTAs with three 36 KB slots (every
-// chunk kept, up to three); four CTAs with the whole row in one slot up to 24
+// chunk kept, up to three; six 18 KB slots for the fp32 rows above, three
+// kept); four CTAs with the whole row in one slot up to 24
 // KB rows, else 16 KB slots up to 44 KB rows, 12 KB slots up to 56 KB rows
 // and 18 KB slots past that (forward only), the last chunk kept; chunks of 12
 // KB or less with two CTAs, or 8 KB with four, ran 10-45 % slower. The stream_*
@@ -784,7 +794,7 @@ bool use_stream(long long row_bytes, bool in_bulk, bool grad, bool topk,
 // SM.
 constexpr long long kLongRowBytes = 240 * 1024;
 
-rl_status plan_stream(int dev, int extra, long long row_bytes, bool grad, bool topk,
+rl_status plan_stream(int dev, int extra, long long row_bytes, int es, bool grad, bool topk,
                       const rl_launch_overrides& ov, StreamPlan* out) {
   int optin = 0, per_sm = 0, reserved = 0;
   if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
@@ -794,13 +804,13 @@ rl_status plan_stream(int dev, int extra, long long row_bytes, bool grad, bool t
           cudaSuccess)
     return RL_ERR_CUDA;
   const int per = ov.stream_ctas_per_sm > 0 ? ov.stream_ctas_per_sm
-                                            : std::max(1, stream_ctas(row_bytes, grad, topk));
+                                            : std::max(1, stream_ctas(row_bytes, es, grad, topk));
   if (per != 1 && per != 2 && per != 4) return RL_ERR_UNSUPPORTED;
   const bool lng = grad && row_bytes >= kLongRowBytes;
   const int budget = per > 1 ? std::min(optin, per_sm / per - reserved) : optin;
   int chunk_d = lng ? 75776 : 114688, hold_d = lng ? 2 : 1, split_d = lng ? 1 : 0;
   if (per == 2) {
-    chunk_d = 36864;
+    chunk_d = fp32_mid_row(row_bytes, es, grad, topk) ? 18432 : 36864;
     hold_d = 3;
     split_d = 1;
   } else if (per == 4) {

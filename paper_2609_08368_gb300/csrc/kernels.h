@@ -204,12 +204,12 @@ struct StreamPlan {
   int chunk, slots, hold, split_first, prefetch, smem;
   int cw;  // consumer warps per CTA: 16, 8 or 4 (one, two or four CTAs per SM)
 };
-bool use_stream(long long row_bytes, bool in_bulk, bool grad, bool topk,
+bool use_stream(long long row_bytes, int es, bool in_bulk, bool grad, bool topk,
                 const rl_launch_overrides& ov);
 // extra: shared memory beyond the ring and the fixed scratch (kTopKSmem with
 // top-K OPD on, else 0); the ring's shape depends on the row length and on
 // whether the call writes dLogits
-rl_status plan_stream(int dev, int extra, long long row_bytes, bool grad, bool topk,
+rl_status plan_stream(int dev, int extra, long long row_bytes, int es, bool grad, bool topk,
                       const rl_launch_overrides& ov, StreamPlan* out);
 const void* bwd_kernel(rl_dtype in, rl_dtype out);
 const void* adv_kernel();

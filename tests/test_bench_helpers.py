@@ -29,7 +29,10 @@ def test_sweep_kernel_name_follows_the_plan_tiers():
     assert bench.sweep_kernel_name(98304, 2).endswith(one)
     assert bench.sweep_kernel_name(98303, 2).endswith(clusters)      # 80-192 KB: clusters
     assert bench.sweep_kernel_name(40964, 2).endswith(clusters)
-    assert bench.sweep_kernel_name(32768, 4).endswith(clusters)      # fp32, 128 KB
+    assert "2 CTAs per SM" in bench.sweep_kernel_name(32768, 4)      # fp32, 128 KB
+    assert bench.sweep_kernel_name(65536, 2).endswith(clusters)      # bf16, 128 KB
+    assert bench.sweep_kernel_name(32768, 4, topk=True).endswith(clusters)
+    assert bench.sweep_kernel_name(36864, 4).endswith(clusters)      # fp32, 144 KB
     assert bench.sweep_kernel_name(49152, 4).endswith(one)
     assert "2 CTAs per SM" in bench.sweep_kernel_name(32768, 2)      # 64 KB
     assert "2 CTAs per SM" in bench.sweep_kernel_name(40960, 2)      # 80 KB
@@ -50,6 +53,9 @@ def test_sweep_kernel_name_follows_the_plan_tiers():
     assert "4 CTAs per SM" in bench.sweep_kernel_name(57344, 2, grad=False)
     assert "2 CTAs per SM" in bench.sweep_kernel_name(32768, 2, grad=False, topk=True)
     assert bench.sweep_kernel_name(8192, 2, grad=False).endswith(clusters)
+    # the sweep_kernel override
+    assert bench.sweep_kernel_name(32768, 4, forced="cluster").endswith(clusters)
+    assert bench.sweep_kernel_name(65536, 2, forced="stream").endswith(one)
 
 
 def test_profiled_traffic_only_for_its_workload_and_sources():
