@@ -229,6 +229,8 @@ def stream_ctas(row_bytes: int, grad: bool, topk: bool = False, elem_size: int =
     if grad:
         if row_bytes >= 192 * KB:
             return 1
+        if elem_size == 4 and 136 * KB <= row_bytes:
+            return 1  # fp32 rows in two equal chunks
         if elem_size == 4 and not topk and 120 * KB < row_bytes <= 136 * KB:
             return 2  # fp32 rows of 120-136 KB
         if 56 * KB < row_bytes <= 80 * KB:

@@ -734,8 +734,11 @@ const void* fn(bool topk, int cw) {
 //   fused: rows of 192-310 KB one CTA 0.966-0.984 against 0.939-0.959 in
 //   clusters; 56-80 KB rows two CTAs 0.956-1.00 against 0.91-0.94; 20-56 KB
 //   rows four CTAs 0.93-1.00 against 0.90-0.94 (48 KB fp32 rows: equal);
-//   80-192 KB rows in clusters (0.93-0.97; two CTAs ran from 2 % ahead to 1 %
-//   behind on 96 KB rows, depending on the box); 16 KB rows in clusters (fp32
+//   80-192 KB rows in clusters (0.93-0.99 by box; two CTAs ran from 2 % ahead
+//   to 1 % behind on 96 KB rows, and one CTA with equal chunks from 3 % ahead
+//   to 2 % behind on 136-184 KB bf16 rows, depending on the box), except fp32
+//   rows of 120-136 KB (fp32_mid_row) and 136-192 KB (halves_row); 16 KB rows
+//   in clusters (fp32
 //   0.91 against 0.79 with four CTAs). With top-K OPD, four CTAs per SM ran 6
 //   % behind the clusters on 32 KB rows; two ran 3-4 % ahead on 64 KB rows.
 //   forward only: 200-310 KB rows one CTA (224 / 288 / 302 KB: 1.13 / 1.10
@@ -754,10 +757,21 @@ bool fp32_mid_row(long long row_bytes, int es, bool grad, bool topk) {
   return grad && !topk && es == 4 && row_bytes > 120 * 1024 && row_bytes <= 136 * 1024;
 }
 
+// Fused fp32 rows of 136-192 KB: one CTA per SM with the row in two equal
+// chunks (three ring slots up to 150 KB rows, two above), neither kept:
+// against the clusters, rows of 136 / 144 / 152 / 160 / 176 KB ran +0.3 /
+// +2.9 / +1.8 / +1.7 / +1.3 % on one box, 144 / 160 KB +4.1 / +3.5 % on
+// another. (bf16 rows of that length: from 3 % ahead on one box to 2 % behind
+// on another, where the clusters ran 0.96-0.99; they stay in clusters.)
+bool halves_row(long long row_bytes, int es, bool grad) {
+  constexpr long long KB = 1024;
+  return grad && es == 4 && row_bytes >= 136 * KB && row_bytes < 192 * KB;
+}
+
 int stream_ctas(long long row_bytes, int es, bool grad, bool topk) {
   constexpr long long KB = 1024;
   if (grad) {
-    if (row_bytes >= 192 * KB) return 1;
+    if (row_bytes >= 192 * KB || halves_row(row_bytes, es, grad)) return 1;
     if (fp32_mid_row(row_bytes, es, grad, topk)) return 2;
     if (row_bytes > 56 * KB && row_bytes <= 80 * KB) return 2;
     if (!topk && row_bytes >= 20 * KB && row_bytes <= 56 * KB) return 4;
@@ -809,7 +823,11 @@ rl_status plan_stream(int dev, int extra, long long row_bytes, int es, bool grad
   const bool lng = grad && row_bytes >= kLongRowBytes;
   const int budget = per > 1 ? std::min(optin, per_sm / per - reserved) : optin;
   int chunk_d = lng ? 75776 : 114688, hold_d = lng ? 2 : 1, split_d = lng ? 1 : 0;
-  if (per == 2) {
+  if (per == 1 && halves_row(row_bytes, es, grad)) {
+    chunk_d = static_cast<int>(((row_bytes + 1) / 2 + 127) / 128 * 128);
+    hold_d = 0;
+    split_d = 1;
+  } else if (per == 2) {
     chunk_d = fp32_mid_row(row_bytes, es, grad, topk) ? 18432 : 36864;
     hold_d = 3;
     split_d = 1;

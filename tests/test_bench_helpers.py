@@ -27,12 +27,17 @@ def test_sweep_kernel_name_follows_the_plan_tiers():
     one, clusters = "one CTA per row)", "clusters sharing a row)"
     assert bench.sweep_kernel_name(154880, 2).endswith(one)
     assert bench.sweep_kernel_name(98304, 2).endswith(one)
-    assert bench.sweep_kernel_name(98303, 2).endswith(clusters)      # 80-192 KB: clusters
+    assert bench.sweep_kernel_name(98303, 2).endswith(clusters)      # bf16 80-192 KB
+    assert bench.sweep_kernel_name(69632, 2).endswith(clusters)
+    assert bench.sweep_kernel_name(34816, 4).endswith(one)           # fp32 136 KB: halves
+    assert bench.sweep_kernel_name(38912, 4).endswith(one)           # fp32 152 KB
+    assert bench.sweep_kernel_name(49151, 4).endswith(one)
     assert bench.sweep_kernel_name(40964, 2).endswith(clusters)
     assert "2 CTAs per SM" in bench.sweep_kernel_name(32768, 4)      # fp32, 128 KB
     assert bench.sweep_kernel_name(65536, 2).endswith(clusters)      # bf16, 128 KB
     assert bench.sweep_kernel_name(32768, 4, topk=True).endswith(clusters)
-    assert bench.sweep_kernel_name(36864, 4).endswith(clusters)      # fp32, 144 KB
+    assert bench.sweep_kernel_name(36864, 4).endswith(one)           # fp32, 144 KB
+    assert bench.sweep_kernel_name(57344, 2).endswith(clusters)      # bf16, 112 KB
     assert bench.sweep_kernel_name(49152, 4).endswith(one)
     assert "2 CTAs per SM" in bench.sweep_kernel_name(32768, 2)      # 64 KB
     assert "2 CTAs per SM" in bench.sweep_kernel_name(40960, 2)      # 80 KB

@@ -121,6 +121,17 @@ def test_stream_several_ctas_per_sm(ov, per_sm, chunk, slots, hold, split):
     _full_check(w, params=dict(w.params, entropy_coef=0.01, opd_topk=16, opd_coef=0.5))
 
 
+@pytest.mark.parametrize("vocab", [34816, 36864, 45000])
+def test_fp32_rows_in_two_equal_chunks(vocab):
+    """The launch plan of fused fp32 rows of 136-192 KB: one streaming CTA
+    per SM, the row in two equal chunks (a ragged last vector for 45,000
+    columns), neither kept for pass B."""
+    rec = wl.shrink(wl.RECIPES["fp32"], n_prompts=1, group_size=4, traj_len=16, vocab=vocab,
+                    rho_noise=0.3)
+    _full_check(wl.make(rec, DEV))
+    _full_check(wl.make(rec, DEV), mode="split")
+
+
 @pytest.mark.parametrize("name", ["tiny", "fp32", "glm_noisy"])
 def test_parity_split_fwd_then_bwd(name):
     _full_check(wl.make(SHRUNK[name], DEV), mode="split")
