@@ -124,8 +124,9 @@ def test_stream_several_ctas_per_sm(ov, per_sm, chunk, slots, hold, split):
 @pytest.mark.parametrize("vocab", [34816, 36864, 45000])
 def test_fp32_rows_in_two_equal_chunks(vocab):
     """The launch plan of fused fp32 rows of 136-192 KB: one streaming CTA
-    per SM, the row in two equal chunks (a ragged last vector for 45,000
-    columns), neither kept for pass B."""
+    per SM, the row in two (nearly) equal chunks, neither kept for pass B:
+    three 68 / 72 KB slots, or two of 88 KB for 45,000 columns (chunks of
+    5,624 and 5,626 vectors)."""
     rec = wl.shrink(wl.RECIPES["fp32"], n_prompts=1, group_size=4, traj_len=16, vocab=vocab,
                     rho_noise=0.3)
     _full_check(wl.make(rec, DEV))
