@@ -527,7 +527,7 @@ def test_device_errors_are_reported_not_trapped(ov, kind):
     assert P.run_gpu(w)["err"] == 0        # the error word resets on the next call
 
 
-@pytest.mark.parametrize("kind", ["cluster", "stream"])
+@pytest.mark.parametrize("kind", ["cluster", "stream", "stream2", "stream4"])
 @pytest.mark.parametrize("topk", [0, 4])
 def test_a_wait_that_runs_out_is_reported(ov, kind, topk):
     """Failure detection on the GPU without a fault. The test hook
@@ -536,8 +536,12 @@ def test_a_wait_that_runs_out_is_reported(ov, kind, topk):
     then gives up as it would on a copy that never arrives (it stops issuing
     copies, waits for the ones in flight and writes zeros for its rows). The
     call reports RL_ERR_DEVICE_TIMEOUT with every output finite and zero, and
-    the next call without the hook is RL_OK and matches the oracle."""
-    ov(sweep_kernel=kind)
+    the next call without the hook is RL_OK and matches the oracle. The
+    streaming kernel runs with one CTA per SM, or two or four ("stream2",
+    "stream4")."""
+    ov(sweep_kernel=kind[:6])
+    if len(kind) > 6:
+        ov(stream_ctas_per_sm=int(kind[6:]))
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=64, vocab=100000,
                     rho_noise=0.3, ref_noise=0.2, topk=topk, topk_noise=0.4)
     w = wl.make(rec, DEV)
