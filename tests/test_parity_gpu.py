@@ -539,9 +539,9 @@ def test_a_wait_that_runs_out_is_reported(ov, kind, topk):
     the next call without the hook is RL_OK and matches the oracle. The
     streaming kernel runs with one CTA per SM, or two or four ("stream2",
     "stream4")."""
-    ov(sweep_kernel=kind[:6])
-    if len(kind) > 6:
-        ov(stream_ctas_per_sm=int(kind[6:]))
+    ov(sweep_kernel=kind.rstrip("24"))
+    if kind[-1] in "24":
+        ov(stream_ctas_per_sm=int(kind[-1]))
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=64, vocab=100000,
                     rho_noise=0.3, ref_noise=0.2, topk=topk, topk_noise=0.4)
     w = wl.make(rec, DEV)
