@@ -37,7 +37,7 @@ METRIC = "RL-loss fwd+bwd tokens/sec at vocab 154,880 bf16; achieved HBM GB/s vs
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "stream_kernel_glm.md")
-SWEEP_SOURCES = ["k_stream.cu", "common.cuh", "kernels.h"]  # the kernel and its launch plan
+SWEEP_SOURCES = ["k_stream.cu", "stream_plan.h", "common.cuh", "kernels.h"]  # the kernel and its launch plan
 
 
 def parse_args():

@@ -4,20 +4,19 @@
 #include <cstdlib>
 
 #include "common.cuh"
+#include "stream_plan.h"
 
 namespace milesloss {
 
 constexpr int kMaxStages = 4;
 constexpr int kMaxCluster = 8;
 constexpr uint32_t kBulkChunk = 16384;    // bytes per cp.async.bulk
-constexpr int kSweepSmemExtra = 1024;     // mbarriers + exchange + reduction scratch
 constexpr int kAdvThreads = 1024;
 constexpr int kBwdThreads = 256;
 // k_stream's block: cw consumer warps (16 with one CTA per SM, 8 with two, 4
 // with four),
 // the producer warp and, with top-K OPD, the top-K warp
 constexpr int stream_threads(bool topk, int cw) { return cw * 32 + (topk ? 64 : 32); }
-constexpr int kMaxSlots = 16;             // ring slots of k_stream
 constexpr int kSeqThreads = 256;
 constexpr int kAdvSmemBytes = 48 * 1024;  // on-chip trajectory tables when they fit
 constexpr int kTopKSmem = 2 * (2 * kMaxTopK * 4);  // two rows of top-K ids + teacher values
@@ -198,12 +197,9 @@ rl_launch_overrides current_overrides();
 // The status a workspace's error bits report: the lowest recorded code.
 rl_status status_of_bits(uint32_t bits);
 
-// The streaming kernel's launch plan (defined beside the kernel, k_stream.cu):
-// whether rows of row_bytes go to it, and its ring of shared-memory slots.
-struct StreamPlan {
-  int chunk, slots, hold, split_first, prefetch, smem;
-  int cw;  // consumer warps per CTA: 16, 8 or 4 (one, two or four CTAs per SM)
-};
+// The streaming kernel's launch plan (k_stream.cu, from the pure plan in
+// stream_plan.h): whether rows of row_bytes go to it, and its ring of
+// shared-memory slots.
 bool use_stream(long long row_bytes, int es, bool in_bulk, bool grad, bool topk,
                 const rl_launch_overrides& ov);
 // extra: shared memory beyond the ring and the fixed scratch (kTopKSmem with
