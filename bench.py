@@ -69,6 +69,9 @@ def parse_args():
     ap.add_argument("--sweep-kernel", choices=["cluster", "stream"], default=None,
                     help="force the vocabulary-sweep kernel (a launch-plan override, for "
                          "profiling the kernel the library would not pick)")
+    ap.add_argument("--stream-cluster", type=int, default=None,
+                    help="measurement aid: CTAs per row of the streaming kernel (1, 2, 4, 8; "
+                         "fused calls without top-K)")
     ap.add_argument("--opd-topk", type=int, default=0,
                     help="top-K on-policy distillation with K candidates per row, coefficient "
                          "0.5 (for profiling the sweeps' top-K instantiations)")
@@ -247,16 +250,32 @@ def stream_ctas(row_bytes: int, grad: bool, topk: bool = False, elem_size: int =
     return 4 if (not topk and row_bytes >= 20 * KB) else 0
 
 
+def stream_cluster(row_bytes: int, grad: bool, topk: bool = False) -> int:
+    """CTAs per row of the streaming kernel the library picks (a cluster of
+    them on rows of 480 KB and more in fused calls without top-K)."""
+    KB = 1024
+    if not grad or topk:
+        return 1
+    if row_bytes >= 1280 * KB:
+        return 4
+    return 2 if row_bytes >= 480 * KB else 1
+
+
 def sweep_kernel_name(vocab: int, elem_size: int, grad: bool = True, topk: bool = False,
-                      forced: str | None = None) -> str:
+                      forced: str | None = None, forced_cluster: int | None = None) -> str:
     """The sweep kernel the library picks for these (16-byte aligned) rows,
-    or the one the sweep_kernel override forces."""
+    or the one the sweep_kernel / stream_cluster overrides force."""
     kind = "fused fwd+bwd" if grad else "forward-only"
     per = stream_ctas(vocab * elem_size, grad, topk, elem_size)
     if forced == "cluster":
         per = 0
     elif forced == "stream":
         per = max(per, 1)
+    clu = stream_cluster(vocab * elem_size, grad, topk)
+    if forced_cluster and grad and not topk:
+        clu = forced_cluster
+    if per == 1 and clu > 1:
+        return f"k_stream ({kind} vocabulary sweep, a cluster of {clu} CTAs per row)"
     if per == 1:
         return f"k_stream ({kind} vocabulary sweep, one CTA per row)"
     if per > 1:
@@ -691,8 +710,13 @@ def run_ours(args, rank, world, local):
     from paper_2609_08368_gb300 import api, milesloss as ml, workloads as wl
 
     ml.load()
+    ov = {}
     if args.sweep_kernel:
-        ml.set_launch_overrides(sweep_kernel=args.sweep_kernel)
+        ov["sweep_kernel"] = args.sweep_kernel
+    if args.stream_cluster:
+        ov["stream_cluster"] = args.stream_cluster
+    if ov:
+        ml.set_launch_overrides(**ov)
     dev = torch.device("cuda", local)
     rec = wl.RECIPES[args.workload]
     rec = wl.shrink(rec, n_prompts=args.n_prompts, traj_len=args.traj_len, vocab=args.vocab,
@@ -775,7 +799,7 @@ def run_ours(args, rank, world, local):
 
     bpr = algorithmic_bytes_per_row(w, dl_dtype)  # before w is released for the e2e leg
     kernel_name = sweep_kernel_name(V, w.logits.element_size(), topk=bool(args.opd_topk),
-                                    forced=args.sweep_kernel)
+                                    forced=args.sweep_kernel, forced_cluster=args.stream_cluster)
     w_params, n_groups = dict(w.params), w.n_groups
     step_bytes = bpr * R
     launch_bytes = step_bytes
@@ -837,7 +861,7 @@ def run_ours(args, rank, world, local):
 
     # the committed capture is of the default path (GRPO-style fused sweep,
     # no top-K): it does not describe the others
-    traffic = None if (args.estimator or args.opd_topk or args.sweep_kernel) \
+    traffic = None if (args.estimator or args.opd_topk or args.sweep_kernel or args.stream_cluster) \
         else profiled_traffic(R, args.workload, V)
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
@@ -851,6 +875,7 @@ def run_ours(args, rank, world, local):
                    **({"estimator": args.estimator} if args.estimator else {}),
                    **({"opd_topk": args.opd_topk} if args.opd_topk else {}),
                    **({"sweep_kernel": args.sweep_kernel} if args.sweep_kernel else {}),
+                   **({"stream_cluster": args.stream_cluster} if args.stream_cluster else {}),
                    "l2": f"inputs larger than L2 ({step_bytes / 1e9:.1f} GB per step), "
                          "no flush"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",

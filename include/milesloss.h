@@ -521,6 +521,10 @@ const char* rl_status_string(rl_status status);
  *  stream_ctas_per_sm   streaming kernel: CTAs per SM, 1 (sixteen consumer
  *                       warps per CTA), 2 (eight each, half of the shared
  *                       memory each) or 4 (four each, a quarter)
+ *  stream_cluster       streaming kernel, fused calls without top-K (other
+ *                       calls ignore it): CTAs per row, 1 (each row on one
+ *                       CTA) or 2, 4 or 8 (a cluster of that many CTAs per
+ *                       row, each streaming a slice of it; one CTA per SM)
  *  stall_first_wait_ns  TEST HOOK, > 0: in each CTA of the vocabulary sweep,
  *                       the first wait for logits waits instead on a barrier
  *                       that nothing completes, bounded by this many
@@ -545,6 +549,7 @@ typedef struct {
   int32_t stream_prefetch_bytes;
   int32_t stream_ctas_per_sm;
   int64_t stall_first_wait_ns;
+  int32_t stream_cluster;
 } rl_launch_overrides;
 
 /* Sets every field of *o to -1 (no override). */

@@ -19,7 +19,7 @@ using namespace milesloss;
 
 namespace {
 std::mutex g_ov_mu;
-rl_launch_overrides g_ov = {-1, -1, -1, -1, -1, -1, -1, -1, -1, -1, -1, -1};
+rl_launch_overrides g_ov = {-1, -1, -1, -1, -1, -1, -1, -1, -1, -1, -1, -1, -1};
 }  // namespace
 
 namespace milesloss {
@@ -561,14 +561,16 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
       use_stream(c.V * static_cast<long long>(es), static_cast<int>(es), in_bulk, grad, sc.topk > 0, ov)) {
     StreamPlan sp;
     st = plan_stream(dev, sc.topk ? kTopKSmem : 0, c.V * static_cast<long long>(es),
-                     static_cast<int>(es), grad, sc.topk > 0, ov, &sp);
+                     static_cast<int>(es), grad, sc.topk > 0, f.part_rows == nullptr, ov, &sp);
     if (st != RL_OK) return st;
-    const void* fn = stream_kernel(c.dt, grad ? go->dt : c.dt, grad, sc.topk > 0, sp.cw);
+    const void* fn = stream_kernel(c.dt, grad ? go->dt : c.dt, grad, sc.topk > 0, sp.cw,
+                                   sp.cluster > 1);
+    if (!fn) return RL_ERR_UNSUPPORTED;
     st = set_smem(fn, dev, sp.smem);
     if (st != RL_OK) return st;
-    int ctas = 0;
+    int ctas = 0;  // resident CTAs, or clusters of sp.cluster CTAs
     const int threads = stream_threads(sc.topk > 0, sp.cw);
-    st = resident_clusters(fn, dev, 1, sp.smem, threads, &ctas);
+    st = resident_clusters(fn, dev, sp.cluster, sp.smem, threads, &ctas);
     if (st != RL_OK) return st;
     StreamArgs ta;
     ta.logits = c.logits;
@@ -581,6 +583,7 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     ta.split_first = sp.split_first;
     ta.prefetch = sp.prefetch;
     ta.out_vec = out_vec;
+    ta.slice_vec = sp.slice_vec;
     ta.targets = c.targets;
     ta.rho = fr.rho;
     ta.q = fr.q;
@@ -598,9 +601,9 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
     ta.col0 = f.col0;
     ta.vocab_total = f.vocab_total > 0 ? f.vocab_total : ta.V;
     ta.part_rows = shift(f.part_rows, 2 * r0);
-    const long long grid = std::min<long long>(ctas, c.R);
+    const long long grid = std::min<long long>(ctas, c.R) * sp.cluster;
     record(t_ev_begin, s);
-    st = launch(fn, dim3(static_cast<unsigned>(grid)), dim3(threads), sp.smem, 1, s,
+    st = launch(fn, dim3(static_cast<unsigned>(grid)), dim3(threads), sp.smem, sp.cluster, s,
                 &ta);
     record(t_ev_end, s);
     if (st != RL_OK) return st;
@@ -1032,6 +1035,7 @@ rl_status rl_launch_overrides_init(rl_launch_overrides* o) {
   o->cluster_ctas_per_sm = o->stream_chunk_bytes = o->stream_slots = o->stream_hold = -1;
   o->stream_split_first = o->stream_prefetch_bytes = o->stream_ctas_per_sm = -1;
   o->stall_first_wait_ns = -1;
+  o->stream_cluster = -1;
   return RL_OK;
 }
 
@@ -1049,7 +1053,9 @@ rl_status rl_set_launch_overrides(const rl_launch_overrides* o) {
         (o->stream_ctas_per_sm != -1 && o->stream_ctas_per_sm != 1 &&
          o->stream_ctas_per_sm != 2 && o->stream_ctas_per_sm != 4) ||
         o->stall_first_wait_ns < -1 ||
-        o->stall_first_wait_ns > 10000000000LL)
+        o->stall_first_wait_ns > 10000000000LL ||
+        (o->stream_cluster != -1 && o->stream_cluster != 1 && o->stream_cluster != 2 &&
+         o->stream_cluster != 4 && o->stream_cluster != 8))
       return RL_ERR_INVALID_ARG;
     v = *o;
   }

@@ -3,7 +3,9 @@
 // objective, dLogits), with no exchange between CTAs. Long rows run one CTA
 // per SM with sixteen consumer warps; shorter rows two or four CTAs per SM
 // with eight or four consumer warps each, so that one CTA's per-row merge and
-// epilogue overlap the others' passes.
+// epilogue overlap the others' passes. Rows of 480 KB and more (fused calls
+// without top-K) run on a cluster of two or four CTAs per row, each streaming
+// a slice, so that fewer rows are live in L2 at once (kClu below).
 //
 // A CTA is warp-specialised. One producer warp streams the row in chunks
 // (bulk async copies, non-multicast) into a ring of shared-memory slots,
@@ -199,8 +201,22 @@ __device__ __forceinline__ void pass_b_chunk(const uint4* sv, int nv, char* dchu
 // kCW consumer warps: 16 with one CTA per SM, 8 with two, 4 with four (each
 // CTA then has a half or a quarter of the SM's shared memory for its ring,
 // and one CTA's per-row merge and epilogue overlap the others' passes).
-template <class In, class Out, bool kGrad, bool kTopK, int kCW>
+//
+// kClu (fused calls, sixteen consumer warps, no top-K, no vocabulary-shard
+// records): the kernel runs in clusters of C CTAs, one cluster per row, CTA
+// crank streaming the vectors [crank slice_vec, (crank + 1) slice_vec) of the
+// row (the last CTA also the elements past the last whole vector) through its
+// own ring. After pass A each CTA's thread 0 pushes the CTA's (m, s, u, z_y)
+// into every peer's shared memory (st.async, counted on the peer's mbarrier
+// for that row parity) and merges the C entries in rank order, so every CTA
+// of the cluster holds the same row statistics and gradient coefficients;
+// then each CTA writes its part of the row's dLogits. With C CTAs per row,
+// C times fewer rows are live at once, so a long row's second read still
+// comes from L2 (one CTA per SM keeps 152 rows live: 78 MB of 512 KB rows,
+// 304 MB of 2 MB rows, against a 126 MB L2).
+template <class In, class Out, bool kGrad, bool kTopK, int kCW, bool kClu>
 __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stream(const StreamArgs a) {
+  static_assert(!kClu || (kGrad && !kTopK && kCW == 16), "clusters: fused calls without top-K");
   constexpr int kCons = kCW * 32;  // consumer threads
   constexpr int kConsWarps = kCW;
   using St = typename In::storage;
@@ -212,8 +228,16 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
   const int NS = a.n_slots;
   const int CB = a.chunk_bytes;
   const int CV = CB / 16;                        // vectors per full chunk
-  const int row_vec = a.V / V8;                  // whole 16-byte vectors per row
-  const int tail0 = row_vec * V8;                // first element not in a vector
+  // rows are visited by one CTA each (cl_id = the CTA) or by one cluster each
+  const int C = kClu ? static_cast<int>(cluster_nctarank()) : 1;
+  const int crank = kClu ? static_cast<int>(cluster_ctarank()) : 0;
+  const long long cl_id = kClu ? blockIdx.x / C : blockIdx.x;
+  const long long n_cl = kClu ? gridDim.x / C : gridDim.x;
+  const int all_vec = a.V / V8;                  // whole 16-byte vectors per row
+  const int lo_v = kClu ? min(all_vec, crank * a.slice_vec) : 0;  // this CTA's first vector
+  const int row_vec = kClu ? min(all_vec - lo_v, a.slice_vec) : all_vec;  // ... and count
+  const int tail0 = all_vec * V8;                // first element not in a vector
+  const int my_tail0 = (crank == C - 1) ? tail0 : a.V;  // this CTA's part of those
   const int n_chunks = (row_vec + CV - 1) / CV;
   // Chunk c starts at vector cs(c) and holds cn(c) vectors. With
   // split_first the first chunk takes the remainder, rounded up to a multiple
@@ -238,8 +262,11 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
   uint64_t* tk_empty = tk_full + 2;                             // [2] part read
   uint64_t* never = tk_empty + 2;                               // [1] completed by nothing (test hook)
   volatile int* abort = reinterpret_cast<volatile int*>(never + 1);  // the CTA gave up
+  uint64_t* xbar = never + 2;                                   // [2] exchange barriers (kClu)
+  float4* xch = reinterpret_cast<float4*>(
+      (reinterpret_cast<uintptr_t>(xbar + 2) + 15) & ~static_cast<uintptr_t>(15));  // [2][kMaxCluster]
   static_assert(2 * kMaxSlots * 8 + (kConsWarps + 3) * 16 + kConsWarps * 4 + 2 * sizeof(TopKPart) +
-                        5 * 8 + 16 <=
+                        6 * 8 + 2 * 8 + 8 + 2 * kMaxCluster * 16 <=
                     kSweepSmemExtra,
                 "k_stream scratch");
   // [2] top-K candidates of this row and the next (launched with kTopKSmem more)
@@ -255,15 +282,22 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
       mbar_init(smem_u32(&tk_empty[b]), 1);
     }
     mbar_init(smem_u32(never), 1);
+    if (kClu) {
+      mbar_init(smem_u32(&xbar[0]), 1);
+      mbar_init(smem_u32(&xbar[1]), 1);
+    }
     *abort = 0;
     fence_mbar_init();
   }
-  __syncthreads();
+  // (peers push into this CTA's exchange slots: every barrier of the cluster
+  // is initialised before any CTA goes on)
+  if constexpr (kClu) cluster_sync_all();
+  else __syncthreads();
 
   WsPtrs ws = a.ws;
   uint32_t* err = &ws.hdr->err_bits;
   const char* lg = static_cast<const char*>(a.logits);
-  const long long rows_mine = (a.R > blockIdx.x) ? (a.R - 1 - blockIdx.x) / gridDim.x + 1 : 0;
+  const long long rows_mine = (a.R > cl_id) ? (a.R - 1 - cl_id) / n_cl + 1 : 0;
 
   // Every wait below is bounded and, except the producer's waits for its own
   // copies, also ends as soon as another party of the CTA has given up
@@ -287,14 +321,15 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
       bool stop = false;
       long long q = 0;
       // each row's mask byte is loaded one row ahead, so that its latency
-      // (often a DRAM access: a CTA's rows are gridDim.x bytes apart) never
+      // (often a DRAM access: a CTA's rows are n_cl bytes apart) never
       // delays the row it decides
-      uint8_t mask_next = rows_mine > 0 ? a.mask[blockIdx.x] : 0;
+      uint8_t mask_next = rows_mine > 0 ? a.mask[cl_id] : 0;
       for (long long i = 0; i < rows_mine && !stop; ++i) {
-        const long long row = blockIdx.x + i * gridDim.x;
-        const char* src_row = lg + row * a.ld * static_cast<long long>(sizeof(St));
+        const long long row = cl_id + i * n_cl;
+        const char* src_row = lg + row * a.ld * static_cast<long long>(sizeof(St)) +
+                              static_cast<long long>(lo_v) * 16;
         const uint8_t msk_row = mask_next;
-        if (i + 1 < rows_mine) mask_next = a.mask[row + gridDim.x];
+        if (i + 1 < rows_mine) mask_next = a.mask[row + n_cl];
         // a row that does not train has an all-zero gradient: no second read
         const bool again = kGrad && msk_row && n_chunks > 0;
         const int h = again ? min(a.n_hold, n_chunks) : 0;
@@ -321,7 +356,7 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
           if (t == n_chunks - 1 && a.prefetch > 0 && i + 1 < rows_mine) {
             // the row's first pass is issued: ask L2 for the head of the next
             // row, so that HBM keeps reading while this row is merged
-            const char* nxt = src_row + gridDim.x * a.ld * static_cast<long long>(sizeof(St));
+            const char* nxt = src_row + n_cl * a.ld * static_cast<long long>(sizeof(St));
             const uint32_t total = min(static_cast<uint32_t>(a.prefetch),
                                        static_cast<uint32_t>(row_vec) * 16u);
             for (uint32_t off = 0; off < total; off += 32768u)
@@ -339,6 +374,10 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
             atomicOr(err, kErrTimeout);
         }
       }
+    }
+    if constexpr (kClu) {  // the cluster's closing barrier (every thread of every CTA)
+      __syncwarp();
+      cluster_sync_all();
     }
     return;
   }
@@ -367,20 +406,19 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
     };
     const int K = a.s.topk;
     if (rows_mine > 0)
-      topk_prefetch(&tkb[0], a.s.topk_ids + static_cast<long long>(blockIdx.x) * K,
-                    a.s.topk_teacher + static_cast<long long>(blockIdx.x) * K, K, lane);
+      topk_prefetch(&tkb[0], a.s.topk_ids + cl_id * K, a.s.topk_teacher + cl_id * K, K, lane);
     long long q0 = 0;
-    uint8_t mask_next = rows_mine > 0 ? a.mask[blockIdx.x] : 0;  // one row ahead
+    uint8_t mask_next = rows_mine > 0 ? a.mask[cl_id] : 0;  // one row ahead
     for (long long i = 0; i < rows_mine; ++i) {
-      const long long row = blockIdx.x + i * gridDim.x;
+      const long long row = cl_id + i * n_cl;
       const bool trains = mask_next != 0;
-      if (i + 1 < rows_mine) mask_next = a.mask[row + gridDim.x];
+      if (i + 1 < rows_mine) mask_next = a.mask[row + n_cl];
       const int h = (kGrad && trains && n_chunks > 0) ? min(a.n_hold, n_chunks) : 0;
       const TopKBuf* tk_row = &tkb[i & 1];
       cp_async_wait_all();
       TopKLane tk = topk_ids(tk_row, static_cast<int>(a.col0), a.V, a.vocab_total, K, lane);
       if (i + 1 < rows_mine) {
-        const long long o = (row + gridDim.x) * K;
+        const long long o = (row + n_cl) * K;
         topk_prefetch(&tkb[(i + 1) & 1], a.s.topk_ids + o, a.s.topk_teacher + o, K, lane);
       }
       for (int c = 0; c < n_chunks; ++c) {
@@ -449,12 +487,13 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
   }
 
   long long q0 = 0;  // task number of the row's first chunk (same count as the producer's)
-  uint8_t mask_next = rows_mine > 0 ? a.mask[blockIdx.x] : 0;  // one row ahead
+  bool xdead = false;  // (kClu, thread 0) an exchange wait of this CTA ran out
+  uint8_t mask_next = rows_mine > 0 ? a.mask[cl_id] : 0;  // one row ahead
   for (long long i = 0; i < rows_mine; ++i) {
-    const long long row = blockIdx.x + i * gridDim.x;
+    const long long row = cl_id + i * n_cl;
     const char* grow = lg + row * a.ld * static_cast<long long>(sizeof(St));
     const bool trains = mask_next != 0;
-    if (i + 1 < rows_mine) mask_next = a.mask[row + gridDim.x];
+    if (i + 1 < rows_mine) mask_next = a.mask[row + n_cl];
     // pass B takes the last h chunks from the slots pass A left them in
     const int h = (kGrad && trains && n_chunks > 0) ? min(a.n_hold, n_chunks) : 0;
 
@@ -473,9 +512,12 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
       A = ws.a_row[row];
       msk = trains ? 1 : 0;
       yok = y >= 0;
-      if (yok && y >= tail0) zy = In::load1(grow, y);
+      if (yok && y >= my_tail0) zy = In::load1(grow, y);
     }
-    const int yv = yok ? y / V8 : -1;  // thread 0 only
+    // the target's vector within this CTA's vectors, and (kClu) the CTA
+    // whose part of the row holds the target (thread 0 only)
+    const int yv = yok ? y / V8 - lo_v : -1;
+    const int owner = (!kClu || !yok) ? 0 : (y >= tail0 ? C - 1 : min(C - 1, (y / V8) / a.slice_vec));
 
     // ---------------- pass A
     // One sweep of each chunk in shared memory against the thread's running
@@ -490,7 +532,7 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
       const uint4* sv = slot(q0 + c);
       const int v0 = cs(c), nv = cn(c);
       {
-        if (tid == 0 && yv >= v0 && yv < v0 + nv) zy = In::load1(sv, y - v0 * V8);
+        if (tid == 0 && yv >= v0 && yv < v0 + nv) zy = In::load1(sv, y - (lo_v + v0) * V8);
         if (run.r == -INFINITY && tid < nv) run.raise(In::vmax(sv[tid]) * k);
         const Run keep = run;
         bool redo = run.r == -INFINITY;  // no finite reference yet
@@ -525,7 +567,7 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
       if (c < n_chunks - h) release_slot(q0 + c);
     }
     Tri t = run.tri();
-    for (int j = tail0 + tid; j < a.V; j += kCons) {
+    for (int j = my_tail0 + tid; j < a.V; j += kCons) {
       const float z = In::load1(grow, j);
       if (z == -INFINITY) continue;
       const float zk = z * k;
@@ -552,6 +594,47 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
     if (tid == 0 && fix_ptr) Out::store1(fix_ptr, 0, fix_val);  // previous row's y entry
     fix_ptr = nullptr;
     if (warp == 0) t = block_merge<kCW>(red, redm, lane);
+    bool cl_bad = false;  // (kClu, thread 0) a CTA of the cluster gave up before this row
+    if constexpr (kClu) {
+      if (tid == 0) {
+        // the cluster's row statistics: this CTA's (m, s, u, z_y) into every
+        // peer's slot for this row parity, then the C entries merged in rank
+        // order (the same bits in every CTA). A CTA whose wait ran out keeps
+        // pushing but waits no more (its rows are written as zeros).
+        const int slot = static_cast<int>(i & 1);
+        float4* xs = xch + slot * kMaxCluster;
+        // (s = -1, which no row's sums take, marks a CTA that gave up)
+        const float4 mine = make_float4(t.m, *abort ? -1.0f : t.s, t.u, zy);
+        xs[crank] = mine;
+        const uint32_t xaddr = smem_u32(&xs[crank]), xb = smem_u32(&xbar[slot]);
+        for (int r = 0; r < C; ++r)
+          if (r != crank) st_async_f4(mapa_shared(xaddr, r), mine, mapa_shared(xb, r));
+        if (!xdead) {
+          mbar_arrive_expect_tx(xb, static_cast<uint32_t>(C - 1) * 16u);
+          if (!mbar_wait_bounded(xb, static_cast<uint32_t>((i >> 1) & 1), kWaitLimitNs)) {
+            xdead = true;
+            *abort = 1;
+            atomicOr(err, kErrTimeout);
+          }
+        }
+        float M = -INFINITY;
+        for (int r = 0; r < C; ++r) {
+          M = fmaxf(M, xs[r].x);
+          cl_bad |= xs[r].y < 0.0f;
+        }
+        Tri tot{M, 0.0f, 0.0f};
+        for (int r = 0; r < C; ++r) {
+          const float4 e = xs[r];
+          if (e.y > 0.0f) {
+            const float d = e.x - M, f = ex2(d);
+            tot.s += f * e.y;
+            tot.u += f * fmaf(d, e.y, e.z);
+          }
+        }
+        zy = xs[owner].w;
+        t = tot;
+      }
+    }
     // top-K OPD signal (Sec. 5.2), a fixed per-token reward: the top-K warp's
     // part of this row and the row's lse (warp 0)
     float opd = 0.0f;
@@ -589,7 +672,7 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
     } else if (tid == 0) {
       // a row read after the CTA gave up, a bad target or a bad top-K
       // candidate: zeros
-      bad = !yok || tk_bad || *abort;
+      bad = !yok || tk_bad || *abort || cl_bad;
       const float lnS = logf(t.s);
       lse = fmaf(t.m, kLn2f, lnS);  // the reference is in log2 units
       H = lnS - t.u * kLn2f / t.s;
@@ -612,21 +695,24 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
     }
     cons_sync<kCW>();
     if (tid == 0 && !a.part_rows) {
-      if (!yok) atomicOr(err, kErrTarget);
-      if (tk_bad) atomicOr(err, kErrTopK);
-      if (a.out_logp) a.out_logp[row] = logp;
-      if (a.out_H) a.out_H[row] = H;
-      ws.logp[row] = logp;
-      ws.H[row] = H;
-      ws.lse[row] = lse;
-      ws.G[row] = tt.G;
-      ws.ell[row] = tt.ell;
-      ws.pg[row] = tt.pg;
-      ws.k3[row] = tt.k3;
-      ws.r[row] = tt.r;
-      ws.rc[row] = tt.rc;
-      ws.flags[row] = tt.flags;
-      if (kGrad && cc != 0.0f && !bci[0].x) {
+      if (crank == 0) {  // (one CTA of a cluster writes the row's results)
+        if (!yok) atomicOr(err, kErrTarget);
+        if (tk_bad) atomicOr(err, kErrTopK);
+        if (a.out_logp) a.out_logp[row] = logp;
+        if (a.out_H) a.out_H[row] = H;
+        ws.logp[row] = logp;
+        ws.H[row] = H;
+        ws.lse[row] = lse;
+        ws.G[row] = tt.G;
+        ws.ell[row] = tt.ell;
+        ws.pg[row] = tt.pg;
+        ws.k3[row] = tt.k3;
+        ws.r[row] = tt.r;
+        ws.rc[row] = tt.rc;
+        ws.flags[row] = tt.flags;
+      }
+      // (the CTA whose part of the row holds the target)
+      if (kGrad && owner == crank && cc != 0.0f && !bci[0].x) {
         // cc [G (1 - p_y) + gamma p_y (log p_y + H)], 1 - p_y = -expm1(logp);
         // written after the next row's merge barrier, which orders it after
         // every store of this row
@@ -649,7 +735,7 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
         const int c = (j < h) ? n_chunks - h + j : n_chunks - 1 - j;
         const long long qq = (j < h) ? q0 + n_chunks - h + j : q0 + n_chunks + (j - h);
         const int nv = cn(c);
-        char* dchunk = drow + static_cast<long long>(cs(c)) * V8 * Out::kSize;
+        char* dchunk = drow + static_cast<long long>(lo_v + cs(c)) * V8 * Out::kSize;
         auto zero_chunk = [&]() {
           float zf[V8];
 #pragma unroll
@@ -694,7 +780,7 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
         }
         release_slot(qq);
       }
-      for (int j = tail0 + tid; j < a.V; j += kCons) {
+      for (int j = my_tail0 + tid; j < a.V; j += kCons) {
         const float z = In::load1(grow, j);
         float x = 0.0f;
         if (!ci.x) {
@@ -708,18 +794,27 @@ __global__ void __launch_bounds__(kCW * 32 + (kTopK ? 64 : 32), 16 / kCW) k_stre
   }
   cons_sync<kCW>();
   if (tid == 0 && fix_ptr) Out::store1(fix_ptr, 0, fix_val);
+  if constexpr (kClu) {  // no CTA leaves while a peer's last exchange store into it may be in flight
+    __syncwarp();
+    cluster_sync_all();
+  }
 }
 
 template <class In, class Out, bool kGrad>
-const void* fn(bool topk, int cw) {
+const void* fn(bool topk, int cw, bool clu) {
+  if constexpr (kGrad) {
+    if (clu) return topk ? nullptr : reinterpret_cast<const void*>(&k_stream<In, Out, true, false, 16, true>);
+  } else {
+    if (clu) return nullptr;
+  }
   if (cw == 4)
-    return topk ? reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, true, 4>)
-                : reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, false, 4>);
+    return topk ? reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, true, 4, false>)
+                : reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, false, 4, false>);
   if (cw == 8)
-    return topk ? reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, true, 8>)
-                : reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, false, 8>);
-  return topk ? reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, true, 16>)
-              : reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, false, 16>);
+    return topk ? reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, true, 8, false>)
+                : reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, false, 8, false>);
+  return topk ? reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, true, 16, false>)
+              : reinterpret_cast<const void*>(&k_stream<In, Out, kGrad, false, 16, false>);
 }
 
 }  // namespace
@@ -732,7 +827,7 @@ bool use_stream(long long row_bytes, int es, bool in_bulk, bool grad, bool topk,
 }
 
 rl_status plan_stream(int dev, int extra, long long row_bytes, int es, bool grad, bool topk,
-                      const rl_launch_overrides& ov, StreamPlan* out) {
+                      bool can_cluster, const rl_launch_overrides& ov, StreamPlan* out) {
   int optin = 0, per_sm = 0, reserved = 0;
   if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) !=
@@ -740,17 +835,21 @@ rl_status plan_stream(int dev, int extra, long long row_bytes, int es, bool grad
       cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev) !=
           cudaSuccess)
     return RL_ERR_CUDA;
-  return plan_ring(row_bytes, es, grad, topk, SmemLimits{optin, per_sm, reserved}, extra, ov, out)
+  return plan_stream_rows(row_bytes, es, grad, topk, can_cluster,
+                          SmemLimits{optin, per_sm, reserved}, extra, ov, out)
              ? RL_OK
              : RL_ERR_UNSUPPORTED;
 }
 
-const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad, bool topk, int cw) {
+const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad, bool topk, int cw, bool clu) {
   if (!grad)
-    return in == RL_BF16 ? fn<InBf16, OutBf16, false>(topk, cw) : fn<InF32, OutF32, false>(topk, cw);
+    return in == RL_BF16 ? fn<InBf16, OutBf16, false>(topk, cw, clu)
+                         : fn<InF32, OutF32, false>(topk, cw, clu);
   if (in == RL_BF16)
-    return out == RL_BF16 ? fn<InBf16, OutBf16, true>(topk, cw) : fn<InBf16, OutF32, true>(topk, cw);
-  return out == RL_BF16 ? fn<InF32, OutBf16, true>(topk, cw) : fn<InF32, OutF32, true>(topk, cw);
+    return out == RL_BF16 ? fn<InBf16, OutBf16, true>(topk, cw, clu)
+                          : fn<InBf16, OutF32, true>(topk, cw, clu);
+  return out == RL_BF16 ? fn<InF32, OutBf16, true>(topk, cw, clu)
+                        : fn<InF32, OutF32, true>(topk, cw, clu);
 }
 
 }  // namespace milesloss

@@ -67,6 +67,8 @@ struct StreamArgs {
   int split_first;  // 1: the first chunk takes the ragged remainder (rounded up to 128 bytes)
   int prefetch;     // bytes of the next row to ask L2 for once a row's first pass is issued
   int out_vec;      // dLogits rows are 16-byte aligned: vector stores
+  int slice_vec;    // launched in clusters (one per row): whole vectors of a row per CTA, a
+                    // multiple of 8 (the cluster's last CTA may take fewer, or none)
   const int* targets;
   const float* rho;
   const float* q;
@@ -189,7 +191,9 @@ constexpr int kBwdTile = kBwdThreads * 8 * 4;  // elements of one row per backwa
 // carry none of its code)
 const void* sweep_kernel(rl_dtype in, rl_dtype out, bool grad, int threads, bool topk);
 const void* sweep_kernel_topk(rl_dtype in, rl_dtype out, bool grad, int threads);
-const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad, bool topk, int cw);
+// clu: the instantiation that runs in clusters of CTAs per row (fused
+// calls without top-K only; nullptr otherwise)
+const void* stream_kernel(rl_dtype in, rl_dtype out, bool grad, bool topk, int cw, bool clu);
 
 // The process-wide launch-plan overrides set by rl_set_launch_overrides (a
 // copy; every field -1 when none are set).
@@ -205,8 +209,9 @@ bool use_stream(long long row_bytes, int es, bool in_bulk, bool grad, bool topk,
 // extra: shared memory beyond the ring and the fixed scratch (kTopKSmem with
 // top-K OPD on, else 0); the ring's shape depends on the row length and on
 // whether the call writes dLogits
+// (can_cluster: the call may run a row over a cluster of CTAs)
 rl_status plan_stream(int dev, int extra, long long row_bytes, int es, bool grad, bool topk,
-                      const rl_launch_overrides& ov, StreamPlan* out);
+                      bool can_cluster, const rl_launch_overrides& ov, StreamPlan* out);
 const void* bwd_kernel(rl_dtype in, rl_dtype out);
 const void* adv_kernel();
 const void* groups_kernel();  // one 32-thread block per group (grid-stride)

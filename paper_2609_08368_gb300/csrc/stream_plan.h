@@ -100,11 +100,41 @@ struct SmemLimits {
 };
 
 // The streaming kernel's launch plan (ring slots, kept chunks, split, shared
-// memory per CTA, consumer warps).
+// memory per CTA, consumer warps, CTAs per row).
 struct StreamPlan {
   int chunk, slots, hold, split_first, prefetch, smem;
-  int cw;  // consumer warps per CTA: 16, 8 or 4 (one, two or four CTAs per SM)
+  int cw;         // consumer warps per CTA: 16, 8 or 4 (one, two or four CTAs per SM)
+  int cluster;    // CTAs per row: 1, or a cluster of 2, 4 or 8 (one CTA per SM)
+  int slice_vec;  // with a cluster: whole 16-byte vectors of a row per CTA
 };
+
+// Fused calls without top-K: how many CTAs share a row (a thread-block
+// cluster, each CTA streaming one slice of the row through its own ring, one
+// CTA per SM). With one CTA per row and per SM, 152 rows are live at once and
+// the second read of each row comes from L2 only while they fit in it; each
+// row of a cluster costs one exchange between its CTAs, which short slices
+// do not repay, and clusters of 4 or 8 leave some SMs idle. Measured on
+// GB300 (fractions of the copy peak, the glm recipe's rows with the
+// vocabulary shown; one CTA / two / four per row):
+//   bf16 400 KB 0.972 / 0.903, 448 KB 0.965 / 0.946, 512 KB 0.916 / 0.934 /
+//   0.740, 1 MB - / 0.939 / 0.861, 1.5 MB - / 0.850 / 0.933, 2 MB 0.751 /
+//   0.815 / 0.943 (eight: 0.724); fp32 400 KB 0.957 / 0.964, 620 KB 0.899 /
+//   0.935 / 0.836; 310 KB (the glm rows) 0.978 / 0.831.
+inline int stream_cluster(long long row_bytes, int es, bool grad, bool topk) {
+  (void)es;
+  constexpr long long KB = 1024;
+  if (!grad || topk) return 1;
+  if (row_bytes >= 1280 * KB) return 4;
+  if (row_bytes >= 480 * KB) return 2;
+  return 1;
+}
+
+// The whole 16-byte vectors of a row each CTA of a cluster of C takes: an
+// even split rounded up to a multiple of 8 (every slice starts 128-byte
+// aligned; the last CTA takes the rest, possibly nothing).
+inline int slice_vectors(long long row_vec, int C) {
+  return static_cast<int>(std::max(8LL, ((row_vec + C - 1) / C + 7) / 8 * 8));
+}
 
 // The plan for rows of row_bytes (elements of es bytes), given the SM's
 // shared-memory limits, the extra shared memory beyond the ring and the
@@ -154,6 +184,33 @@ inline bool plan_ring(long long row_bytes, int es, bool grad, bool topk, const S
   out->prefetch = ov.stream_prefetch_bytes >= 0 ? ov.stream_prefetch_bytes : 0;
   out->smem = slots * chunk + kSweepSmemExtra + extra;
   out->cw = 16 / per;
+  out->cluster = 1;
+  out->slice_vec = 0;
+  return true;
+}
+
+// The plan with the row's CTAs: one (plan_ring over the whole row), or a
+// cluster of C, whose CTAs each run plan_ring's one-CTA ring over their
+// slice. Only fused calls without top-K run in clusters, and only when
+// can_cluster (a call that writes the row's own results, not a vocabulary
+// shard's records); other calls take one CTA per row whatever the
+// stream_cluster override says. False when a forced value does not fit.
+inline bool plan_stream_rows(long long row_bytes, int es, bool grad, bool topk, bool can_cluster,
+                             const SmemLimits& lim, int extra, const rl_launch_overrides& ov,
+                             StreamPlan* out) {
+  const bool can = can_cluster && grad && !topk;
+  const int C = !can ? 1
+                     : (ov.stream_cluster > 0 ? ov.stream_cluster
+                                              : stream_cluster(row_bytes, es, grad, topk));
+  if (C == 1) return plan_ring(row_bytes, es, grad, topk, lim, extra, ov, out);
+  if (C != 2 && C != 4 && C != 8) return false;
+  if (ov.stream_ctas_per_sm > 1) return false;
+  const int sv = slice_vectors(row_bytes / 16, C);
+  rl_launch_overrides one = ov;
+  one.stream_ctas_per_sm = 1;
+  if (!plan_ring(static_cast<long long>(sv) * 16, es, grad, topk, lim, extra, one, out)) return false;
+  out->cluster = C;
+  out->slice_vec = sv;
   return true;
 }
 

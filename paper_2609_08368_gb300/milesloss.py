@@ -78,6 +78,7 @@ class RlLaunchOverrides(ctypes.Structure):
         ("stream_prefetch_bytes", ctypes.c_int32),
         ("stream_ctas_per_sm", ctypes.c_int32),
         ("stall_first_wait_ns", ctypes.c_int64),
+        ("stream_cluster", ctypes.c_int32),
     ]
 
 

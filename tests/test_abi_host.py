@@ -210,8 +210,9 @@ def test_launch_overrides_struct_layout_matches_header():
                 text.index("} rl_launch_overrides;")]
     names = re.findall(r"(?:int32_t|int64_t)\s+([a-z_0-9]+)\s*;", body)
     assert names == [f[0] for f in ml.RlLaunchOverrides._fields_]
-    # eleven int32 fields, four bytes of padding, one int64
-    assert ctypes.sizeof(ml.RlLaunchOverrides) == 56
+    # eleven int32 fields, four bytes of padding, one int64, one int32 and
+    # four bytes of tail padding
+    assert ctypes.sizeof(ml.RlLaunchOverrides) == 64
 
 
 def test_launch_overrides_are_validated_and_cleared(lib):
@@ -223,12 +224,14 @@ def test_launch_overrides_are_validated_and_cleared(lib):
         ml.set_launch_overrides(sweep_kernel="stream", stream_slots=3, stream_hold=2)
         ml.set_launch_overrides(cluster_size=8, cluster_stages=4, stall_first_wait_ns=1000)
         ml.set_launch_overrides(sweep_kernel="stream", stream_ctas_per_sm=2)
+        ml.set_launch_overrides(sweep_kernel="stream", stream_cluster=4)
         for bad in (dict(sweep_kernel=2), dict(cluster_size=16), dict(cluster_stages=0),
                     dict(stream_chunk_bytes=512), dict(stream_slots=17), dict(stream_hold=-2),
                     dict(stream_split_first=2), dict(stream_prefetch_bytes=24),
                     dict(stream_prefetch_bytes=1 << 21), dict(stall_first_wait_ns=-5),
                     dict(stall_first_wait_ns=10 ** 11), dict(stream_ctas_per_sm=0),
-                    dict(stream_ctas_per_sm=3)):
+                    dict(stream_ctas_per_sm=3), dict(stream_cluster=0), dict(stream_cluster=3),
+                    dict(stream_cluster=16)):
             with pytest.raises(ml.MilesLossError) as e:
                 ml.set_launch_overrides(**bad)
             assert e.value.status == RL_ERR_INVALID_ARG

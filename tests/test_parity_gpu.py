@@ -317,6 +317,59 @@ def test_long_row_plan_shapes(logits, vocab, ld, dl_dtype, ld_out):
             assert torch.isnan(g["dlogits_t"][:, vocab:]).all()
 
 
+@pytest.mark.parametrize("logits,vocab,ld,topk", [
+    ("bf16", 262144, 262144, 0),       # 512 KB rows (a 256K vocabulary)
+    ("bf16", 256000, 256000, 16),      # with top-K OPD
+    ("bf16", 1000003, 1000008, 0),     # ~2 MB rows, elements past the last whole vector
+    ("f32", 200003, 200004, 0)])       # ~800 KB fp32 rows
+def test_very_long_rows(logits, vocab, ld, topk):
+    """Rows far longer than the headline's (up to ~2 MB, tens of ring chunks
+    per row, most of pass B's second read from L2): fused and split calls
+    against the oracle, the padding of each row left untouched."""
+    base = wl.RECIPES["glm" if logits == "bf16" else "fp32"]
+    rec = wl.shrink(base, n_prompts=1, group_size=4, traj_len=6, vocab=vocab, rho_noise=0.3,
+                    topk=topk)
+    w = wl.make(rec, DEV, ld=ld)
+    params = dict(w.params, opd_coef=0.3, opd_topk=topk) if topk else None
+    for mode in ("fused", "split"):
+        g = P.run_gpu(w, mode=mode, ld_out=ld, params=params)
+        assert g["err"] == 0, ml.status_string(g["err"])
+        o = P.run_oracle(w, params=params)
+        P.compare_forward(w, g, o, params=params)
+        P.assert_dlogits_close(g["dlogits_t"][:, :vocab].float().cpu().numpy(), o["dlogits"])
+        if ld > vocab:
+            assert torch.isnan(g["dlogits_t"][:, vocab:]).all()
+
+
+@pytest.mark.parametrize("C", [2, 4, 8])
+@pytest.mark.parametrize("logits,vocab,ld,dl_dtype,traj", [
+    ("bf16", 262144, 262144, None, 60),        # 512 KB rows, several rows per cluster
+    ("bf16", 100003, 100008, torch.float32, 60),  # elements past the last whole vector
+    ("f32", 200003, 200004, None, 30),         # ~800 KB fp32 rows
+    ("bf16", 100, 104, None, 8)])              # CTAs whose slice holds no vector of the row
+def test_stream_clusters(ov, C, logits, vocab, ld, dl_dtype, traj):
+    """The streaming kernel with a cluster of C CTAs per row (each CTA
+    streams one slice of the row, the CTAs exchange their row sums and merge
+    them in rank order): every output against the oracle, every CTA's part of
+    dLogits, the row padding untouched, and bit-identical reruns."""
+    ov(sweep_kernel="stream", stream_cluster=C)
+    base = wl.RECIPES["glm" if logits == "bf16" else "fp32"]
+    rec = wl.shrink(base, n_prompts=1, group_size=4, traj_len=traj, vocab=vocab, rho_noise=0.3,
+                    ref_noise=0.2)
+    w = wl.make(rec, DEV, ld=ld)
+    params = dict(w.params, entropy_coef=0.01, kl_coef=0.05)
+    g = P.run_gpu(w, dl_dtype=dl_dtype, ld_out=ld, params=params)
+    assert g["err"] == 0, ml.status_string(g["err"])
+    o = P.run_oracle(w, params=params)
+    P.compare_forward(w, g, o, params=params)
+    P.assert_dlogits_close(g["dlogits_t"][:, :vocab].float().cpu().numpy(), o["dlogits"])
+    if ld > vocab:
+        assert torch.isnan(g["dlogits_t"][:, vocab:]).all()
+    again = P.run_gpu(w, dl_dtype=dl_dtype, ld_out=ld, params=params)
+    assert torch.equal(again["dlogits_t"].view(torch.uint8), g["dlogits_t"].view(torch.uint8))
+    np.testing.assert_array_equal(again["logp"], g["logp"])
+
+
 @pytest.mark.parametrize("estimator", ["grpo", "reinforcepp", "gspo"])
 @pytest.mark.parametrize("n_prompts", [8, 1200])
 def test_ragged_and_empty_trajectories(estimator, n_prompts):
@@ -527,8 +580,8 @@ def test_device_errors_are_reported_not_trapped(ov, kind):
     assert P.run_gpu(w)["err"] == 0        # the error word resets on the next call
 
 
-@pytest.mark.parametrize("kind", ["cluster", "stream", "stream2", "stream4"])
-@pytest.mark.parametrize("topk", [0, 4])
+@pytest.mark.parametrize("kind,topk", [(k, t) for k in ("cluster", "stream", "stream2", "stream4")
+                                       for t in (0, 4)] + [("streamC2", 0), ("streamC8", 0)])
 def test_a_wait_that_runs_out_is_reported(ov, kind, topk):
     """Failure detection on the GPU without a fault. The test hook
     stall_first_wait_ns makes the first wait for logits of every CTA of the
@@ -538,10 +591,15 @@ def test_a_wait_that_runs_out_is_reported(ov, kind, topk):
     call reports RL_ERR_DEVICE_TIMEOUT with every output finite and zero, and
     the next call without the hook is RL_OK and matches the oracle. The
     streaming kernel runs with one CTA per SM, or two or four ("stream2",
-    "stream4")."""
-    ov(sweep_kernel=kind.rstrip("24"))
-    if kind[-1] in "24":
-        ov(stream_ctas_per_sm=int(kind[-1]))
+    "stream4"), or with a cluster of two or eight CTAs per row ("streamC2",
+    "streamC8": the CTAs still exchange their row sums, which carry the
+    give-up mark)."""
+    if kind.startswith("streamC"):
+        ov(sweep_kernel="stream", stream_cluster=int(kind[-1]))
+    else:
+        ov(sweep_kernel=kind.rstrip("24"))
+        if kind[-1] in "24":
+            ov(stream_ctas_per_sm=int(kind[-1]))
     rec = wl.shrink(wl.RECIPES["glm"], n_prompts=1, group_size=4, traj_len=64, vocab=100000,
                     rho_noise=0.3, ref_noise=0.2, topk=topk, topk_noise=0.4)
     w = wl.make(rec, DEV)

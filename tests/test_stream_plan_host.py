@@ -1,9 +1,11 @@
 """The streaming kernel's launch plan, checked on the host: stream_plan.h is
 plain C++, so a small program built with the host compiler prints the plan
-for every row length from 1 to 320 KB (and 16 bytes either side of each KB),
-both element sizes, fused and forward-only calls, top-K OPD on and off, at one
-GB300 SM's shared-memory limits. The plan must fit the SM, keep no more
-chunks than it has slots, and match the tiers bench.py names its kernel by."""
+for every row length from 1 to 320 KB (and 16 bytes either side of each KB)
+and on to 4 MB in steps of 32 KB, both element sizes, fused and forward-only
+calls, top-K OPD on and off, at one GB300 SM's shared-memory limits. The plan
+must fit the SM, keep no more chunks than it has slots, split long rows over a
+cluster in whole 128-byte slices, and match the tiers bench.py names its
+kernel by."""
 
 import os
 import shutil
@@ -29,12 +31,12 @@ def table(tmp_path_factory):
                     os.path.join(ROOT, "tests", "stream_plan_table.cpp"), "-o", exe], check=True)
     out = subprocess.run([exe], check=True, capture_output=True, text=True).stdout
     keys = ("es", "grad", "topk", "row", "ctas", "ok", "chunk", "slots", "hold", "split",
-            "smem", "cw")
+            "smem", "cw", "cluster", "slice_vec")
     return [dict(zip(keys, map(int, line.split()))) for line in out.splitlines()]
 
 
 def test_every_default_plan_fits_one_sm(table):
-    assert len(table) == 2 * 2 * 2 * 320 * 3
+    assert len(table) == 2 * 2 * 2 * (320 + 118) * 3
     for p in table:
         assert p["ok"] == 1, p
         per = max(1, p["ctas"])
@@ -52,6 +54,28 @@ def test_tiers_match_the_bench_names(table):
     for p in table:
         want = bench.stream_ctas(p["row"], bool(p["grad"]), bool(p["topk"]), p["es"])
         assert p["ctas"] == want, p
+        assert p["cluster"] == bench.stream_cluster(p["row"], bool(p["grad"]), bool(p["topk"])), p
+
+
+def test_long_rows_split_over_clusters_in_whole_slices(table):
+    """Rows of 480 KB and more in fused calls without top-K run on a cluster
+    of two (four from 1.25 MB) CTAs, one per SM, each with a slice of the row
+    that starts on a 128-byte boundary; the slices cover the row's whole
+    vectors and each CTA's ring is the one-CTA ring of its slice's length."""
+    seen = set()
+    for p in table:
+        C = p["cluster"]
+        if not p["grad"] or p["topk"] or p["row"] < 480 * 1024:
+            assert C == 1, p
+            continue
+        assert C == (4 if p["row"] >= 1280 * 1024 else 2), p
+        seen.add(C)
+        vec = p["row"] // 16
+        sv = p["slice_vec"]
+        assert sv % 8 == 0 and sv * C >= vec and sv * (C - 1) < vec, p
+        assert p["cw"] == 16, p
+        assert p["chunk"] == (75776 if sv * 16 >= 240 * 1024 else 114688), p
+    assert seen == {2, 4}
 
 
 def _plan(table, es, grad, topk, row):

@@ -521,3 +521,162 @@ def test_give_up_model_catches_a_faulty_producer(variant):
                 assert ("copies in flight" in str(e)) == (variant != "no_flag_check"), str(e)
                 caught += 1
     assert caught > 0
+
+
+# ------------------------------------------- the row exchange of a cluster
+
+class XBar:
+    """An mbarrier as the exchange uses it: one pending arrival per phase
+    (the CTA's own arrive.expect_tx) and a transaction count that the peers'
+    st.async stores decrement, possibly before the arrival raised it."""
+
+    def __init__(self):
+        self.phase, self.pending, self.tx = 0, 1, 0
+
+    def _maybe_complete(self):
+        if self.pending == 0 and self.tx == 0:
+            self.phase += 1
+            self.pending = 1
+
+    def complete_tx(self, n):
+        self.tx -= n
+        self._maybe_complete()
+
+    def arrive_expect_tx(self, n):
+        self.tx += n
+        self.pending -= 1
+        assert self.pending == 0, "more arrivals than the barrier expects in one phase"
+        self._maybe_complete()
+
+
+def run_exchange(C, rows, seed, give_up=None):
+    """C CTAs of one cluster exchange their row sums for `rows` rows (k_stream's
+    kClu path): per row, write the own entry, push it to every peer (data and
+    a 16-byte complete_tx on the peer's barrier for the row's parity), arrive
+    with expect_tx (C - 1) x 16 unless the CTA gave up, wait for the phase,
+    read the C entries. give_up = (cta, row): that CTA's wait on that row runs
+    out (it stops waiting from then on). Random interleavings; returns what
+    each CTA read per row."""
+    rng = random.Random(seed)
+    xs = [[[None] * C for _ in range(2)] for _ in range(C)]
+    bars = [[XBar(), XBar()] for _ in range(C)]
+    state = [dict(row=0, step="push", dead=False, read={}) for _ in range(C)]
+    in_flight = []  # st.async stores not yet landed: (dst, slot, src, value)
+
+    def runnable(c):
+        s = state[c]
+        if s["row"] >= rows:
+            return False
+        if s["step"] == "wait":
+            slot = s["row"] & 1
+            return s["dead"] or bars[c][slot].phase > (s["row"] >> 1)
+        return True
+
+    for _ in range(10 ** 6):
+        choices = [("cta", c) for c in range(C) if runnable(c)]
+        choices += [("land", k) for k in range(len(in_flight))]
+        if not choices:
+            break
+        kind, k = rng.choice(choices)
+        if kind == "land":
+            dst, slot, src, value = in_flight.pop(k)
+            xs[dst][slot][src] = value
+            bars[dst][slot].complete_tx(16)
+            continue
+        s = state[k]
+        i, slot = s["row"], s["row"] & 1
+        if s["step"] == "push":
+            value = (k, i)
+            xs[k][slot][k] = value
+            for r in range(C):
+                if r != k:
+                    in_flight.append((r, slot, k, value))
+            if s["dead"]:
+                s["step"] = "read"
+            else:
+                bars[k][slot].arrive_expect_tx(16 * (C - 1))
+                s["step"] = "wait"
+        elif s["step"] == "wait":
+            if give_up == (k, i) and bars[k][slot].phase <= (i >> 1):
+                s["dead"] = True
+            s["step"] = "read"
+        else:  # read the C entries of the row, then the next row
+            s["read"][i] = list(xs[k][slot])
+            s["row"] += 1
+            s["step"] = "push"
+    assert all(s["row"] == rows for s in state), "a CTA never finished its rows"
+    return state
+
+
+@pytest.mark.parametrize("C", [2, 4, 8])
+@pytest.mark.parametrize("seed", range(40))
+def test_cluster_exchange_reads_every_peers_entry_of_the_same_row(C, seed):
+    rows = 7
+    state = run_exchange(C, rows, seed)
+    for c in range(C):
+        for i in range(rows):
+            assert state[c]["read"][i] == [(r, i) for r in range(C)], (c, i)
+
+
+@pytest.mark.parametrize("C", [2, 8])
+@pytest.mark.parametrize("seed", range(20))
+def test_cluster_exchange_with_a_cta_that_gave_up_still_ends(C, seed):
+    """A CTA whose exchange wait ran out keeps pushing but waits no more:
+    every CTA still finishes its rows (what a CTA that gave up reads is not
+    used; its rows are written as zeros), and the others read correct
+    entries up to the row where the peer gave up."""
+    rows = 6
+    gave_up = (seed % C, seed % rows)
+    state = run_exchange(C, rows, seed, give_up=gave_up)
+    for c in range(C):
+        if c == gave_up[0]:
+            continue
+        for i in range(rows):
+            assert state[c]["read"][i] == [(r, i) for r in range(C)], (c, i)
+
+
+def test_cluster_exchange_model_catches_a_single_buffer():
+    """The same model with one exchange slot per CTA (no row-parity double
+    buffer) lets a fast peer's next row overwrite an entry before it is read:
+    some interleaving reads a wrong row."""
+    def run_single(C, rows, seed):
+        rng = random.Random(seed)
+        xs = [[None] * C for _ in range(C)]
+        bars = [XBar() for _ in range(C)]
+        st = [dict(row=0, step="push", read={}) for _ in range(C)]
+        fl = []
+        for _ in range(10 ** 5):
+            ch = [("cta", c) for c in range(C) if st[c]["row"] < rows and
+                  (st[c]["step"] != "wait" or bars[c].phase > st[c]["row"])]
+            ch += [("land", k) for k in range(len(fl))]
+            if not ch:
+                break
+            kind, k = rng.choice(ch)
+            if kind == "land":
+                d, s_, v = fl.pop(k)
+                xs[d][s_] = v
+                bars[d].complete_tx(16)
+                continue
+            s = st[k]
+            if s["step"] == "push":
+                xs[k][k] = (k, s["row"])
+                fl += [(r, k, (k, s["row"])) for r in range(C) if r != k]
+                bars[k].arrive_expect_tx(16 * (C - 1))
+                s["step"] = "wait"
+            elif s["step"] == "wait":
+                s["step"] = "read"
+            else:
+                s["read"][s["row"]] = list(xs[k])
+                s["row"] += 1
+                s["step"] = "push"
+        return st
+    wrong = 0
+    for seed in range(200):
+        try:
+            st = run_single(2, 5, seed)
+        except AssertionError:
+            wrong += 1
+            continue
+        wrong += any(st[c]["read"].get(i) != [(r, i) for r in range(2)]
+                     for c in range(2) for i in range(5))
+    assert wrong > 0
