@@ -14,8 +14,9 @@ with GUARD bytes before and after it:
   writes none of them).
 
 The cases cover every sweep kernel and launch plan the library picks (the
-streaming kernel with one, two and four CTAs per SM, the fp32 two-chunk
-plan, clusters of 1, 2, 4 and 8 CTAs), top-K OPD in both kernels, the split
+streaming kernel with one, two and four CTAs per SM and with a cluster of two
+or four CTAs per row, the fp32 two-chunk plan, clusters of 1, 2, 4 and 8
+CTAs), top-K OPD in both kernels, the split
 forward / backward pair, GSPO, the chunked row call, ragged and padded rows,
 and the row- and vocabulary-sharded calls with their exchange buffers."""
 
@@ -176,6 +177,12 @@ CASES = {
                   dict(sweep_kernel=0, cluster_size=4), "fused", {}, None, None),
     "cluster_8": (_rec("glm", n_prompts=2, group_size=4, traj_len=40, vocab=20480),
                   dict(sweep_kernel=0, cluster_size=8), "fused", {}, None, None),
+    "stream_cluster_of_two": (_rec("glm", vocab=262144, n_prompts=1, group_size=4, traj_len=40),
+                              {}, "fused", {}, None, None),
+    "stream_cluster_of_four_ragged": (_rec("glm", vocab=100003, n_prompts=1, group_size=4,
+                                           traj_len=40),
+                                      dict(sweep_kernel=1, stream_cluster=4), "fused", {},
+                                      100008, 100016),
     "ragged_vocab": (_rec("tiny", n_prompts=1, group_size=3, traj_len=50, vocab=12345), {},
                      "fused", {}, None, None),
     "misaligned_rows": (_rec("tiny", n_prompts=1, group_size=2, traj_len=24, vocab=1000), {},

@@ -560,9 +560,15 @@ def test_no_training_tokens_and_empty_call(ov, kind):
     np.testing.assert_allclose(buf.advantages.cpu().numpy(), [-2 ** -0.5, 2 ** -0.5], rtol=1e-6)
 
 
-@pytest.mark.parametrize("kind", ["cluster", "stream"])
+@pytest.mark.parametrize("kind", ["cluster", "stream", "streamC4"])
 def test_device_errors_are_reported_not_trapped(ov, kind):
-    ov(sweep_kernel=kind)
+    """Bad inputs that the kernels' own checks turn into error codes (no
+    trap); "streamC4": the streaming kernel with a cluster of four CTAs per
+    row, every CTA of which writes its part of a bad row as zeros."""
+    if kind.startswith("streamC"):
+        ov(sweep_kernel="stream", stream_cluster=int(kind[-1]))
+    else:
+        ov(sweep_kernel=kind)
     rec = wl.shrink(wl.RECIPES["tiny"], n_prompts=2, group_size=2, traj_len=8, vocab=256)
     w = wl.make(rec, DEV)
     w.targets[3] = 256                     # outside [0, vocab)
@@ -570,6 +576,9 @@ def test_device_errors_are_reported_not_trapped(ov, kind):
     assert g["err"] == 5                   # RL_ERR_TARGET_OUT_OF_RANGE
     assert g["logp"][3] == 0.0 and (g["dlogits_t"][3] == 0).all()
     assert np.isfinite(g["logp"]).all()
+    good = [r for r in range(w.n_rows) if r != 3]  # the other rows as in a clean call
+    g2 = P.run_gpu(wl.make(rec, DEV))
+    np.testing.assert_array_equal(g["logp"][good], g2["logp"][good])
     w = wl.make(rec, DEV)
     w.group_id[1] = 9
     assert P.run_gpu(w)["err"] == 6        # RL_ERR_GROUP_OUT_OF_RANGE
