@@ -1,6 +1,7 @@
 // The streaming vocabulary sweep, one CTA per row: the same per-row results
 // as k_sweep (log-softmax statistics, log-prob, entropy, per-token
-// objective, dLogits), with no exchange between CTAs. Long rows run one CTA
+// objective, dLogits), with no exchange between CTAs (except in the cluster
+// instantiation for the longest rows, below). Long rows run one CTA
 // per SM with sixteen consumer warps; shorter rows two or four CTAs per SM
 // with eight or four consumer warps each, so that one CTA's per-row merge and
 // epilogue overlap the others' passes. Rows of 480 KB and more (fused calls
