@@ -61,6 +61,16 @@ def test_sweep_kernel_name_follows_the_plan_tiers():
     # the sweep_kernel override
     assert bench.sweep_kernel_name(32768, 4, forced="cluster").endswith(clusters)
     assert bench.sweep_kernel_name(65536, 2, forced="stream").endswith(one)
+    # rows of 480 KB and more (fused, no top-K): a cluster of two, from 1.25 MB four
+    assert bench.sweep_kernel_name(245759, 2).endswith(one)
+    assert "a cluster of 2 CTAs per row" in bench.sweep_kernel_name(245760, 2)
+    assert "a cluster of 2 CTAs per row" in bench.sweep_kernel_name(154880, 4)  # fp32, 620 KB
+    assert "a cluster of 4 CTAs per row" in bench.sweep_kernel_name(655360, 2)
+    assert bench.sweep_kernel_name(262144, 2, topk=True).endswith(one)
+    assert bench.sweep_kernel_name(262144, 2, grad=False).endswith(one)
+    # the stream_cluster override (fused calls without top-K only)
+    assert "a cluster of 4 CTAs per row" in bench.sweep_kernel_name(154880, 2, forced_cluster=4)
+    assert bench.sweep_kernel_name(154880, 2, topk=True, forced_cluster=4).endswith(one)
 
 
 def test_profiled_traffic_only_for_its_workload_and_sources():
