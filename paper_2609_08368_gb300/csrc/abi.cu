@@ -560,18 +560,29 @@ rl_status run_fwd(const FwdIn& f, const GradOut* go, cudaStream_t s, int phase =
   if (c.R > 0 &&
       use_stream(c.V * static_cast<long long>(es), static_cast<int>(es), in_bulk, grad, sc.topk > 0, ov)) {
     StreamPlan sp;
-    st = plan_stream(dev, sc.topk ? kTopKSmem : 0, c.V * static_cast<long long>(es),
-                     static_cast<int>(es), grad, sc.topk > 0, f.part_rows == nullptr, ov, &sp);
-    if (st != RL_OK) return st;
-    const void* fn = stream_kernel(c.dt, grad ? go->dt : c.dt, grad, sc.topk > 0, sp.cw,
-                                   sp.cluster > 1);
-    if (!fn) return RL_ERR_UNSUPPORTED;
-    st = set_smem(fn, dev, sp.smem);
-    if (st != RL_OK) return st;
+    const void* fn = nullptr;
     int ctas = 0;  // resident CTAs, or clusters of sp.cluster CTAs
-    const int threads = stream_threads(sc.topk > 0, sp.cw);
-    st = resident_clusters(fn, dev, sp.cluster, sp.smem, threads, &ctas);
-    if (st != RL_OK) return st;
+    int threads = 0;
+    rl_launch_overrides pov = ov;
+    for (;;) {
+      st = plan_stream(dev, sc.topk ? kTopKSmem : 0, c.V * static_cast<long long>(es),
+                       static_cast<int>(es), grad, sc.topk > 0, f.part_rows == nullptr, pov, &sp);
+      if (st != RL_OK) return st;
+      fn = stream_kernel(c.dt, grad ? go->dt : c.dt, grad, sc.topk > 0, sp.cw, sp.cluster > 1);
+      if (!fn) return RL_ERR_UNSUPPORTED;
+      st = set_smem(fn, dev, sp.smem);
+      if (st != RL_OK) return st;
+      threads = stream_threads(sc.topk > 0, sp.cw);
+      st = resident_clusters(fn, dev, sp.cluster, sp.smem, threads, &ctas);
+      // no cluster of the plan fits the device (a partition with too few SMs
+      // together): one CTA per row instead, unless the override forced it
+      if (st == RL_ERR_UNSUPPORTED && sp.cluster > 1 && ov.stream_cluster <= 0) {
+        pov.stream_cluster = 1;
+        continue;
+      }
+      if (st != RL_OK) return st;
+      break;
+    }
     StreamArgs ta;
     ta.logits = c.logits;
     ta.ld = c.ld;
