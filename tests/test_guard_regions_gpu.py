@@ -1,5 +1,5 @@
 """Guard regions around every buffer a call touches: a stand-in for a memory
-checker (compute-sanitizer is not available on this machine).
+checker, which these tests do not run.
 
 Each input and output of a call is placed inside a larger device allocation,
 with GUARD bytes before and after it:
