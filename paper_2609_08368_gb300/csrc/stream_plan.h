@@ -194,14 +194,16 @@ inline bool plan_ring(long long row_bytes, int es, bool grad, bool topk, const S
 // slice. Only fused calls without top-K run in clusters, and only when
 // can_cluster (a call that writes the row's own results, not a vocabulary
 // shard's records); other calls take one CTA per row whatever the
-// stream_cluster override says. False when a forced value does not fit.
+// stream_cluster override says, and so does a row whose CTAs per SM are
+// forced above one (unless stream_cluster is forced too: no plan). False
+// when a forced value does not fit.
 inline bool plan_stream_rows(long long row_bytes, int es, bool grad, bool topk, bool can_cluster,
                              const SmemLimits& lim, int extra, const rl_launch_overrides& ov,
                              StreamPlan* out) {
   const bool can = can_cluster && grad && !topk;
-  const int C = !can ? 1
-                     : (ov.stream_cluster > 0 ? ov.stream_cluster
-                                              : stream_cluster(row_bytes, es, grad, topk));
+  int C = 1;
+  if (can && ov.stream_cluster > 0) C = ov.stream_cluster;
+  else if (can && ov.stream_ctas_per_sm <= 1) C = stream_cluster(row_bytes, es, grad, topk);
   if (C == 1) return plan_ring(row_bytes, es, grad, topk, lim, extra, ov, out);
   if (C != 2 && C != 4 && C != 8) return false;
   if (ov.stream_ctas_per_sm > 1) return false;

@@ -8,7 +8,7 @@
 
 #include "stream_plan.h"
 
-int main() {
+int main(int argc, char** argv) {
   using namespace milesloss;
   const SmemLimits lim{232448, 233472, 1024};
   rl_launch_overrides none;
@@ -17,6 +17,23 @@ int main() {
   none.stream_split_first = none.stream_prefetch_bytes = none.stream_ctas_per_sm = -1;
   none.stall_first_wait_ns = -1;
   none.stream_cluster = -1;
+  if (argc > 1) {
+    // forced plans of a fused bf16 row of 512 KB: "per clu topk" per line,
+    // printed as "ok cluster cw"
+    const int cases[][3] = {{-1, -1, 0}, {2, -1, 0}, {4, -1, 0}, {1, -1, 0}, {-1, 4, 0},
+                            {1, 8, 0}, {2, 2, 0}, {-1, 4, 1}, {-1, 1, 0}};
+    for (const auto& c : cases) {
+      rl_launch_overrides o = none;
+      o.stream_ctas_per_sm = c[0];
+      o.stream_cluster = c[1];
+      StreamPlan p{};
+      const bool ok = plan_stream_rows(512 * 1024, 2, true, c[2] != 0, true, lim,
+                                       c[2] ? 1024 : 0, o, &p);
+      std::printf("%d %d %d %d %d %d\n", c[0], c[1], c[2], ok ? 1 : 0, ok ? p.cluster : 0,
+                  ok ? p.cw : 0);
+    }
+    return 0;
+  }
   for (int es = 2; es <= 4; es += 2)
     for (int grad = 0; grad <= 1; ++grad)
       for (int topk = 0; topk <= 1; ++topk)

@@ -115,3 +115,30 @@ def test_fused_and_forward_rows_up_to_56kb_take_the_same_chunks(table):
         if p["grad"] == 1 and p["topk"] == 0 and p["ctas"] == 4:
             q = _plan(table, p["es"], 0, 0, p["row"])
             assert q["ctas"] == 4 and q["chunk"] == p["chunk"] and q["split"] == p["split"], (p, q)
+
+
+def test_forced_plans_of_a_long_row(tmp_path):
+    """A 512 KB fused bf16 row (a cluster of two by default) under the
+    overrides: forced CTAs per SM above one give one CTA per row (not an
+    error), a forced cluster size is taken, forcing both is refused, and a
+    top-K call stays on one CTA per row whatever the cluster override."""
+    cxx = shutil.which("g++") or shutil.which("c++")
+    if cxx is None:
+        pytest.skip("no host C++ compiler")
+    exe = str(tmp_path / "stream_plan_table")
+    subprocess.run([cxx, "-std=c++17", "-O1", "-Wall", "-Werror",
+                    "-I", os.path.join(ROOT, "paper_2609_08368_gb300", "csrc"),
+                    "-I", os.path.join(ROOT, "include"),
+                    os.path.join(ROOT, "tests", "stream_plan_table.cpp"), "-o", exe], check=True)
+    out = subprocess.run([exe, "forced"], check=True, capture_output=True, text=True).stdout
+    got = {tuple(map(int, line.split()[:3])): tuple(map(int, line.split()[3:]))
+           for line in out.splitlines()}
+    assert got[(-1, -1, 0)] == (1, 2, 16)    # the library's plan: two CTAs per row
+    assert got[(2, -1, 0)] == (1, 1, 8)      # two CTAs per SM forced: one CTA per row
+    assert got[(4, -1, 0)] == (1, 1, 4)
+    assert got[(1, -1, 0)] == (1, 2, 16)     # one CTA per SM forced: the cluster stays
+    assert got[(-1, 4, 0)] == (1, 4, 16)     # a cluster of four forced
+    assert got[(1, 8, 0)] == (1, 8, 16)
+    assert got[(2, 2, 0)][0] == 0            # both forced: no plan
+    assert got[(-1, 4, 1)] == (1, 1, 16)     # top-K: one CTA per row
+    assert got[(-1, 1, 0)] == (1, 1, 16)     # clusters forced off
