@@ -215,6 +215,14 @@ def test_launch_overrides_struct_layout_matches_header():
     assert ctypes.sizeof(ml.RlLaunchOverrides) == 64
 
 
+def test_every_launch_override_is_documented_in_the_header():
+    text = open(HEADER).read()
+    doc = text[text.index("Launch-plan overrides"):text.index("typedef struct {",
+                                                             text.index("Launch-plan overrides"))]
+    for name, _ in ml.RlLaunchOverrides._fields_:
+        assert re.search(r"\*\s+" + name + r"\s", doc), name
+
+
 def test_launch_overrides_are_validated_and_cleared(lib):
     o = ml.RlLaunchOverrides()
     assert lib.rl_launch_overrides_init(ctypes.byref(o)) == 0
