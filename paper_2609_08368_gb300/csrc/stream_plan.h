@@ -113,7 +113,7 @@ struct StreamPlan {
 // CTA per SM). With one CTA per row and per SM, 152 rows are live at once and
 // the second read of each row comes from L2 only while they fit in it; each
 // row of a cluster costs one exchange between its CTAs, which short slices
-// do not repay, and clusters of 4 or 8 leave some SMs idle. Measured on
+// do not repay. Measured on
 // GB300 (fractions of the copy peak, the glm recipe's rows with the
 // vocabulary shown; one CTA / two / four per row):
 //   bf16 400 KB 0.972 / 0.903, 448 KB 0.965 / 0.946, 512 KB 0.916 / 0.934 /
